@@ -1,0 +1,209 @@
+"""CPU oracle of the UltraMem memory-layer forward -- TEST INFRASTRUCTURE ONLY.
+
+Loads ``ultramem_oracle.c`` (plain fp64 C, OpenMP over tokens) through ctypes.
+Only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this package; the product path never does.
+
+Arrays are numpy: fp32 tensors as ``float32``, bf16 tensors as their raw
+``uint16`` bit patterns, the Tucker cores and (u, t) as ``float32``.  The
+paper's notation is kept: ``x, w_q, w_q_col, k_row, k_col, core, u, t, values,
+w_proj, perm`` (see ``ultramem_oracle.h`` for shapes and equations).
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "ultramem_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "_ultramem_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+F32, BF16 = 0, 1
+ACT_NONE, ACT_SOFTMAX = 0, 1
+
+
+class Config(C.Structure):
+    _fields_ = [(name, C.c_int32) for name in (
+        "d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out",
+        "topk", "topm", "has_proj", "share_query", "act", "dtype")] + [
+        ("shuffle_seed", C.c_uint64)]
+
+
+class Tensors(C.Structure):
+    _fields_ = [("x", C.c_void_p), ("w_q", C.c_void_p), ("w_q_col", C.c_void_p),
+                ("k_row", C.c_void_p), ("k_col", C.c_void_p),
+                ("core", C.c_void_p), ("u", C.c_void_p), ("t", C.c_void_p),
+                ("values", C.c_void_p), ("w_proj", C.c_void_p), ("perm", C.c_void_p)]
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle shared library in place (gcc, -O2, OpenMP)."""
+    if force or not os.path.exists(_LIB_PATH) or \
+            os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + ".%d.tmp" % os.getpid()
+        subprocess.check_call(["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared",
+                               "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = C.CDLL(build())
+            P = C.c_void_p
+            lib.uo_forward.argtypes = [P, P, C.c_int64, P, C.c_int64, P, P, P, C.c_int32]
+            lib.uo_lookup_reduce.argtypes = [P, P, C.c_int64, P, P, P, C.c_int32]
+            lib.uo_row_col_scores.argtypes = [P, P, C.c_int64, C.c_int32, P, P]
+            lib.uo_rank1.argtypes = [P, C.c_int32, P, P, P]
+            lib.uo_shuffle.argtypes = [P, P, C.c_int64]
+            lib.uo_shuffle.restype = C.c_int64
+            lib.uo_shuffle_params.argtypes = [C.c_uint64, C.c_uint64, P, P]
+            lib.uo_splitmix64.argtypes = [C.c_uint64]
+            lib.uo_splitmix64.restype = C.c_uint64
+            _lib = lib
+    return _lib
+
+
+_CFG_KEYS = ("d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out", "topk",
+             "topm", "has_proj", "share_query", "act", "dtype", "shuffle_seed")
+
+
+def make_config(cfg: dict) -> Config:
+    c = Config()
+    for k in _CFG_KEYS:
+        setattr(c, k, int(cfg[k]))
+    return c
+
+
+def keys_per_axis(cfg: dict) -> int:
+    s = int(round(cfg["expand_e"] ** 0.5))
+    return s * int(cfg["n"])
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data
+
+
+def _stored(a, dtype):
+    """Checks that a stored tensor has the storage type the config names."""
+    if a is None:
+        return None
+    want = np.uint16 if dtype == BF16 else np.float32
+    if a.dtype != want:
+        raise TypeError(f"oracle expects {want.__name__} storage, got {a.dtype}")
+    return np.ascontiguousarray(a)
+
+
+def _tensors(cfg: dict, t: dict):
+    dt = int(cfg["dtype"])
+    keep = {}
+    for k in ("x", "w_q", "w_q_col", "k_row", "k_col", "values", "w_proj"):
+        keep[k] = _stored(t.get(k), dt)
+    for k in ("core", "u", "t"):
+        a = t.get(k)
+        keep[k] = None if a is None else np.ascontiguousarray(a, dtype=np.float32)
+    p = t.get("perm")
+    keep["perm"] = None if p is None else np.ascontiguousarray(p, dtype=np.int64)
+    s = Tensors(*[_ptr(keep[k]) for k in ("x", "w_q", "w_q_col", "k_row", "k_col",
+                                          "core", "u", "t", "values", "w_proj", "perm")])
+    return s, keep
+
+
+def forward(cfg: dict, tensors: dict, B: int, tokens=None, threads: int = 0):
+    """Eq. 4-10 then Eq. 13-15 for the listed tokens (all B if None).
+
+    Returns ``(out [n, d_out] f64, idx [n, H, m] i64, w [n, H, m] f64)``."""
+    lib = _load()
+    c = make_config(cfg)
+    s, keep = _tensors(cfg, tensors)
+    tok = None if tokens is None else np.ascontiguousarray(tokens, dtype=np.int64)
+    n = B if tok is None else len(tok)
+    H, m = int(cfg["heads"]), int(cfg["topm"])
+    out = np.zeros((n, int(cfg["d_out"])), np.float64)
+    idx = np.zeros((n, H, m), np.int64)
+    w = np.zeros((n, H, m), np.float64)
+    st = lib.uo_forward(C.byref(c), C.byref(s), int(B), _ptr(tok), int(n),
+                        out.ctypes.data, idx.ctypes.data, w.ctypes.data, int(threads))
+    del keep
+    if st != 0:
+        raise ValueError(f"uo_forward failed with status {st}")
+    return out, idx, w
+
+
+def lookup_reduce(cfg: dict, tensors: dict, idx, w, threads: int = 0):
+    """Eq. 14-15 alone on given (virtual address, weight) pairs [n, H, m]."""
+    lib = _load()
+    c = make_config(cfg)
+    s, keep = _tensors(cfg, tensors)
+    idx = np.ascontiguousarray(idx, dtype=np.int64)
+    w = np.ascontiguousarray(w, dtype=np.float64)
+    n = idx.shape[0]
+    out = np.zeros((n, int(cfg["d_out"])), np.float64)
+    st = lib.uo_lookup_reduce(C.byref(c), C.byref(s), int(n), idx.ctypes.data,
+                              w.ctypes.data, out.ctypes.data, int(threads))
+    del keep
+    if st != 0:
+        raise ValueError(f"uo_lookup_reduce failed with status {st}")
+    return out
+
+
+def row_col_scores(cfg: dict, tensors: dict, b: int, h: int):
+    """Eq. 4 for token b, head h: ``(S_row [r, K], S_col [r, K])`` in fp64."""
+    lib = _load()
+    c = make_config(cfg)
+    s, keep = _tensors(cfg, tensors)
+    r, K = int(cfg["rank"]), keys_per_axis(cfg)
+    sr = np.zeros((r, K), np.float64)
+    sc = np.zeros((r, K), np.float64)
+    st = lib.uo_row_col_scores(C.byref(c), C.byref(s), int(b), int(h),
+                               sr.ctypes.data, sc.ctypes.data)
+    del keep
+    if st != 0:
+        raise ValueError(f"uo_row_col_scores failed with status {st}")
+    return sr, sc
+
+
+def rank1(core):
+    """Leading singular triplet ``(u, t, sigma)`` of one r x r core (Eq. 7)."""
+    lib = _load()
+    c = np.ascontiguousarray(core, dtype=np.float64)
+    r = c.shape[0]
+    u = np.zeros(r, np.float64)
+    t = np.zeros(r, np.float64)
+    sig = np.zeros(1, np.float64)
+    st = lib.uo_rank1(c.ctypes.data, r, u.ctypes.data, t.ctypes.data, sig.ctypes.data)
+    if st != 0:
+        raise ValueError(f"uo_rank1 failed with status {st}")
+    return u, t, float(sig[0])
+
+
+def shuffle(cfg: dict, v, perm=None):
+    """Eq. 14: shuffled virtual addresses for an array of addresses."""
+    lib = _load()
+    c = make_config(cfg)
+    p = None if perm is None else np.ascontiguousarray(perm, dtype=np.int64)
+    v = np.asarray(v, dtype=np.int64)
+    out = np.array([lib.uo_shuffle(C.byref(c), _ptr(p), int(e)) for e in v.ravel()],
+                   dtype=np.int64)
+    return out.reshape(v.shape)
+
+
+def shuffle_params(seed: int, m: int):
+    lib = _load()
+    a = C.c_uint64()
+    c = C.c_uint64()
+    lib.uo_shuffle_params(C.c_uint64(seed), C.c_uint64(m), C.byref(a), C.byref(c))
+    return a.value, c.value
+
+
+def splitmix64(state: int) -> int:
+    """First output of a SplitMix64 generator in the given state."""
+    return int(_load().uo_splitmix64(C.c_uint64(state)))

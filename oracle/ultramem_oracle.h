@@ -1,0 +1,114 @@
+/*
+ * ultramem_oracle.h -- the CPU oracle of the UltraMem memory-layer forward.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This is a plain, slow, fp64 statement of what the
+ * layer computes, written from "Ultra-Sparse Memory Network" (Huang et al.,
+ * ICLR 2025, arXiv 2411.12364).  Only the tests, the smoke check and the
+ * benchmark's CPU-baseline leg may load it.  It shares no code, header, table
+ * or helper with the CUDA library; neither includes or links the other.
+ *
+ * Every tensor is read in the precision it is stored in (fp32, or bf16 given
+ * as raw uint16 bit patterns) and widened exactly to double.  All arithmetic
+ * is fp64.  Where a floating-point score decides an index (the per-axis top-k
+ * and the final top-m), the decision is taken on the score rounded to fp32,
+ * the precision the GPU kernels decide in; ties go to the smaller index.
+ *
+ * Paper sections and equations cited below use the paper's own numbering:
+ *   Eq. 1   generic memory layer          s = sigma(K q),  o = V^T s
+ *   Eq. 2-3 product keys (PKM)            two-phase top-m, softmax pooling
+ *   Eq. 4   row/column scores             S_row = K_row q_row, S_col = K_col q_col
+ *   Eq. 5   Tucker grid score             S_grid = TopM(S_row^T C S_col)
+ *   Eq. 6-7 rank-1 approximation          C ~ u t^T (leading singular pair)
+ *   Eq. 8-9 per-axis pruning              I_TopM(u^T S_row), I_TopM(t^T S_col)
+ *   Eq. 10  exact score on the survivors  TopM(S~_row^T C S~_col)
+ *   Eq. 13  virtual blocks                V~_p = V W_p
+ *   Eq. 14  shuffle of virtual addresses  s^ = Shuffle(vec(S_grid))
+ *   Eq. 15  implicit value expansion      o = sum_p W_p^T (V^T s^_p)
+ */
+#ifndef ULTRAMEM_ORACLE_H
+#define ULTRAMEM_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum { UO_F32 = 0, UO_BF16 = 1 };          /* storage type of the big tensors */
+enum { UO_ACT_NONE = 0, UO_ACT_SOFTMAX = 1 }; /* Trick 1 removes the softmax   */
+
+typedef struct {
+    int32_t d_in;        /* D_i: width of the input hidden x                    */
+    int32_t d_k;         /* D_k: query/key width of one head, D_k % r == 0      */
+    int32_t heads;       /* H: key sets sharing one value table (Sec. 3.1)      */
+    int32_t rank;        /* r: Tucker rank (Eq. 5)                              */
+    int32_t n;           /* physical grid side; the table holds N = n*n rows    */
+    int32_t expand_e;    /* E: virtual expansion, a perfect square (Eq. 13)     */
+    int32_t d_v;         /* D_v: physical value width                           */
+    int32_t d_out;       /* D'_v: virtual value width = output width            */
+    int32_t topk;        /* k: survivors per axis (Eq. 8-9)                     */
+    int32_t topm;        /* m: values read per head (Eq. 10)                    */
+    int32_t has_proj;    /* 1: IVE projectors W_p present; 0 needs E == 1       */
+    int32_t share_query; /* 1: one query for both key sets (Trick 5)            */
+    int32_t act;         /* UO_ACT_NONE (Trick 1) or UO_ACT_SOFTMAX (PKM)       */
+    int32_t dtype;       /* UO_F32 or UO_BF16 for x, W_q, keys, V, W_p          */
+    uint64_t shuffle_seed; /* 0: identity shuffle; else the seeded bijection   */
+} uo_config;
+
+typedef struct {
+    const void *x;        /* [B][d_in]                                           */
+    const void *w_q;      /* [H*d_k][d_in]  q = W_q x, head h = rows h*d_k..     */
+    const void *w_q_col;  /* [H*d_k][d_in] column query when share_query == 0   */
+    const void *k_row;    /* [H][K][d_k], K = sqrt(E)*n keys per axis            */
+    const void *k_col;    /* [H][K][d_k]                                         */
+    const float *core;    /* [H][r][r] Tucker cores C_h, always fp32             */
+    const float *u;       /* [H][r] or NULL: leading left singular vectors       */
+    const float *t;       /* [H][r] or NULL: leading right singular vectors      */
+    const void *values;   /* [N][d_v] physical table V                           */
+    const void *w_proj;   /* [E][d_v][d_out] projectors W_p, or NULL             */
+    const int64_t *perm;  /* [E*N] explicit shuffle, or NULL for the seeded one  */
+} uo_tensors;
+
+/* Status codes. */
+enum { UO_OK = 0, UO_EINVAL = -1, UO_ENOMEM = -2 };
+
+/* Full forward (Sec. 3.2, Eq. 4-10 then Eq. 13-15) for the tokens listed in
+ * `tokens` (n_tokens entries, each in [0, B)); tokens == NULL means all B in
+ * order.  Outputs are indexed by position in that list:
+ *   out [n_tokens][d_out]   layer output o
+ *   idx [n_tokens][H][m]    virtual address v = i*K + j of each selected slot,
+ *                           ordered by (score desc, v asc); may be NULL
+ *   w   [n_tokens][H][m]    the weight applied to that slot; may be NULL
+ * n_threads <= 0 uses the OpenMP default. */
+int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
+               const int64_t *tokens, int64_t n_tokens,
+               double *out, int64_t *idx, double *w, int32_t n_threads);
+
+/* Eq. 14-15 alone: pool the given (virtual address, weight) pairs and project.
+ * idx/w are [n_tokens][H][m]; only values, w_proj and perm of `x` are read. */
+int uo_lookup_reduce(const uo_config *cfg, const uo_tensors *x, int64_t n_tokens,
+                     const int64_t *idx, const double *w, double *out,
+                     int32_t n_threads);
+
+/* Eq. 4 for one (token b, head h): s_row[r][K], s_col[r][K]. */
+int uo_row_col_scores(const uo_config *cfg, const uo_tensors *x, int64_t b,
+                      int32_t h, double *s_row, double *s_col);
+
+/* Leading singular triplet of an r x r matrix (row-major), Eq. 7 / Eq. 11.
+ * Sign rule: sum(u) > 0, or if that sum is exactly 0 the first non-zero
+ * entry of u is positive; t = C^T u / sigma.  Returns UO_OK. */
+int uo_rank1(const double *c, int32_t r, double *u, double *t, double *sigma);
+
+/* Eq. 14: the shuffled virtual address pi(v) for v in [0, E*N). */
+int64_t uo_shuffle(const uo_config *cfg, const int64_t *perm, int64_t v);
+
+/* The first output of a SplitMix64 generator whose state is `state`. */
+uint64_t uo_splitmix64(uint64_t state);
+
+/* The multiplier and offset of the seeded bijection pi(v) = (a v + c) mod M. */
+void uo_shuffle_params(uint64_t seed, uint64_t m, uint64_t *a, uint64_t *c);
+
+#ifdef __cplusplus
+}
+#endif
+#endif
