@@ -1,0 +1,389 @@
+"""Benchmark of the UltraMem layer forward on GB300.
+
+One step = one forward (S1-S9) of one decode batch of the named workload,
+inputs already resident in HBM.  Default: the decode-shaped layer (1024x1024
+physical grid, E=4, 2 heads, top-32, 64 tokens).  The L2 is flushed (256 MiB
+write) between timed steps, outside the timed events.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME --batch B]
+  python bench.py --impl reference ...      # the CPU oracle as the reference arm
+
+Prints one JSON line on rank 0.  Under torchrun each rank runs its own
+replica of the layer on its own token batches (no collective on the data
+path); the step time is the max over ranks and ``value`` counts all ranks'
+tokens.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "UltraMem layer tokens/s at decode batch; gather HBM GB/s as % of GB300 peak"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default=None)
+    ap.add_argument("--batch", type=int, default=None)
+    ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
+            int(os.environ.get("LOCAL_RANK", 0)))
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def algorithmic_bytes(cfg, B):
+    """Bytes each stage must move at least (paper's Sec. 4 memory-access model
+    with heads: the gather reads min(B*H*m, N) rows of D_v)."""
+    es = 4 if int(cfg["dtype"]) == 0 else 2
+    H, dk, din = cfg["heads"], cfg["d_k"], cfg["d_in"]
+    K = int(round(cfg["expand_e"] ** 0.5)) * cfg["n"]
+    A = 1 if cfg["share_query"] else 2
+    N = cfg["n"] ** 2
+    rows = min(B * H * cfg["topm"], N)
+    return {
+        "query": A * H * dk * din * es + B * din * es,
+        "score": 2 * H * K * dk * es,
+        "select": 0,
+        "gather": rows * cfg["d_v"] * es,
+        "project": (cfg["expand_e"] * cfg["d_v"] * cfg["d_out"] * es if cfg["has_proj"] else 0)
+        + B * cfg["d_out"] * es,
+    }
+
+
+def launches_per_forward(cfg):
+    return 4 + (2 if cfg["has_proj"] else 0)
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during timing."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index, enabled=True):
+        self.proc = None
+        self.path = None
+        self.gpu = gpu_index
+        if not enabled:
+            return
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, fl in rows for i, f in enumerate(fl)
+                          if f.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows),
+                "sm_max_mhz": max(r[1] for r in rows), "reasons": reasons,
+                "samples": len(rows)}
+
+
+def source_sha(path):
+    return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
+
+
+def ncu_traffic(kernel_stage, workload, batch):
+    """DRAM bytes per launch of a stage's kernel from the committed ncu
+    summary, or None if absent or taken on another version of the kernel."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        d = json.load(open(path))
+        e = d[kernel_stage]
+        src = os.path.join(ROOT, "paper_2411_12364_gb300", "csrc", e["source"])
+        if e["workload"] != workload or int(e["batch"]) != batch:
+            return None
+        if e["source_sha"] != source_sha(src):
+            return None
+        return float(e["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
+def cpu_baseline(cfg, weights_np, B, budget_s=12.0):
+    """The oracle, as it stands, on the host cores: whole batches of the
+    workload until about budget_s seconds of wall time have passed."""
+    import numpy as np
+    import oracle
+    from paper_2411_12364_gb300 import workloads
+    cores = len(os.sched_getaffinity(0))
+    done, t0, batches = 0, time.perf_counter(), 0
+    while True:
+        x = workloads.stored_numpy(workloads.make_tokens(cfg, B, 1000 + batches))
+        t = dict(weights_np, x=x)
+        oracle.forward(cfg, t, B, threads=cores)
+        done += B
+        batches += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s or batches >= 64:
+            break
+    return {"value": done / el, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{batches} batch(es) of {B} tokens of the same workload, "
+                      f"{el:.1f} s wall, fp64, OpenMP over tokens"}
+
+
+def numpy_weights(w):
+    from paper_2411_12364_gb300 import workloads
+    return {k: workloads.stored_numpy(v) for k, v in w.items()}
+
+
+def run_reference(args, cfg, B, wl):
+    """The reference arm: the CPU oracle timed on the host cores."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    import torch
+    from paper_2411_12364_gb300 import workloads
+    w = workloads.make_weights(cfg, device="cpu")
+    wn = numpy_weights(w)
+    import oracle
+    cores = len(os.sched_getaffinity(0))
+    sample = min(B, 8)      # tokens per step: a bounded slice of the batch
+    for i in range(args.warmup):
+        x = workloads.stored_numpy(workloads.make_tokens(cfg, sample, 2000 + i))
+        oracle.forward(cfg, dict(wn, x=x), sample, threads=cores)
+    times = []
+    for i in range(args.steps):
+        x = workloads.stored_numpy(workloads.make_tokens(cfg, sample, 3000 + i))
+        t0 = time.perf_counter()
+        oracle.forward(cfg, dict(wn, x=x), sample, threads=cores)
+        times.append(time.perf_counter() - t0)
+        if sum(times) > 120:
+            break
+    k = len(times)
+    ms = 1e3 * sum(times) / k
+    value = sample / (ms / 1e3)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": k, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": dict(workload=wl, batch=B, **_cfg_brief(cfg)),
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores,
+                             "kind": "oracle",
+                             "sample": f"{sample} of the {B} tokens of a batch per step"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def _cfg_brief(cfg):
+    keys = ("d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out", "topk", "topm")
+    d = {k: int(cfg[k]) for k in keys}
+    d["storage"] = "f32" if int(cfg["dtype"]) == 0 else "bf16"
+    return d
+
+
+def main():
+    args = parse()
+    from paper_2411_12364_gb300 import workloads
+    wl = args.workload or workloads.HEADLINE[0]
+    B = args.batch or (workloads.HEADLINE[1] if wl == workloads.HEADLINE[0]
+                       else workloads.CONFIGS[wl]["batches"][-1])
+    cfg = workloads.layer_config(wl)
+    if args.impl == "reference":
+        return run_reference(args, cfg, B, wl)
+
+    import torch
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    from paper_2411_12364_gb300.binding import UltraMemLayer
+
+    w = workloads.make_weights(cfg, device="cuda")
+    layer = UltraMemLayer(cfg, w, B)
+    NB = 8     # distinct token batches cycled through (per rank)
+    xs = [workloads.make_tokens(cfg, B, 100 * rank + i, device="cuda") for i in range(NB)]
+    out = torch.empty((B, cfg["d_out"]), dtype=layer.dtype, device="cuda")
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.Stream()
+
+    use_graph = not args.no_graph
+    graphs = []
+    with torch.cuda.stream(stream):
+        for i in range(3):
+            layer.forward(xs[0], out=out)
+        torch.cuda.synchronize()
+        if use_graph:
+            for i in range(NB):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    layer.forward(xs[i], out=out)
+                graphs.append(g)
+    torch.cuda.synchronize()
+
+    def step(i):
+        if use_graph:
+            graphs[i % NB].replay()
+        else:
+            layer.forward(xs[i % NB], out=out)
+
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            step(i)
+            flush.fill_(float(i))
+    torch.cuda.synchronize()
+
+    # ---- timed region ----------------------------------------------------
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
+    clocks = Clocks(local, enabled=not args.no_clocks)
+    time.sleep(0.3)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for i in range(K):
+            ev[i][0].record(stream)
+            step(i)
+            ev[i][1].record(stream)
+            flush.fill_(float(i))
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    total_ms = sum(a.elapsed_time(b) for a, b in ev)
+    ms = total_ms / K
+    if dist:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * B / (ms / 1e3)
+
+    # ---- per-stage device times on the same stream (direct launches) ----
+    layer.profile(True)
+    stage_ms = {}
+    with torch.cuda.stream(stream):
+        for i in range(K):
+            layer.forward(xs[i % NB], out=out)
+            torch.cuda.synchronize()
+            for k, v in layer.profile_read().items():
+                stage_ms.setdefault(k, []).append(v)
+            flush.fill_(float(i))
+    layer.profile(False)
+    stage_avg = {k: sum(v) / len(v) for k, v in stage_ms.items()}
+    alg = algorithmic_bytes(cfg, B)
+    peak, peak_kind = peaks()
+    dominant = max(stage_avg, key=stage_avg.get)
+    dom_bytes = alg[dominant]
+    src_of = {"query": "um_score.cu", "score": "um_score.cu", "select": "um_select.cu",
+              "gather": "um_gather.cu", "project": "um_gather.cu"}
+    roof = {"kernel": dominant, "bound": "hbm", "achieved": dom_bytes / (stage_avg[dominant] * 1e6),
+            "peak": peak, "unit": "GB/s", "peak_kind": peak_kind,
+            "traffic": ncu_traffic(dominant, wl, B), "algorithmic_bytes": dom_bytes,
+            "avg_ms": stage_avg[dominant]}
+    roof["frac"] = roof["achieved"] / peak
+    if dom_bytes == 0:
+        roof["bound"] = "alu"
+        roof["achieved"] = None
+        roof["frac"] = None
+    gms = stage_avg.get("gather")
+    gather = None
+    if gms:
+        gbs = alg["gather"] / (gms * 1e6)
+        gather = {"achieved_gbs": gbs, "ms": gms, "bytes": alg["gather"],
+                  "frac_of_measured": gbs / peak, "frac_of_nominal_8tbs": gbs / NOMINAL_HBM_GBS,
+                  "traffic": ncu_traffic("gather", wl, B)}
+
+    # ---- end to end through the public API with host buffers -------------
+    xh = [x.cpu().pin_memory() for x in xs]
+    oh = torch.empty((B, cfg["d_out"]), dtype=layer.dtype).pin_memory()
+    with torch.cuda.stream(stream):
+        for i in range(3):
+            layer.forward_host(xh[i % NB], oh)
+        e2e_t = []
+        for i in range(K):
+            t0 = time.perf_counter()
+            layer.forward_host(xh[i % NB], oh)
+            e2e_t.append(time.perf_counter() - t0)
+    e2e_s = sum(e2e_t) / len(e2e_t)
+    if dist:
+        t = torch.tensor([e2e_s], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    es = 4 if int(cfg["dtype"]) == 0 else 2
+    e2e = {"value": world * B / e2e_s, "unit": "tokens/s",
+           "h2d_bytes_per_step": B * cfg["d_in"] * es, "d2h_bytes_per_step": B * cfg["d_out"] * es,
+           "ms_per_step": e2e_s * 1e3}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(cfg, numpy_weights(w), B)
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+                "steps": K, "warmup": args.warmup, "ms_per_step": ms,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "f32", "data": "synthetic",
+                "config": dict(workload=wl, batch=B, **_cfg_brief(cfg),
+                               l2="flushed between steps (256 MiB write, outside timing)",
+                               cuda_graph=use_graph, parallelism=f"replicas x{world}"),
+                "roofline": roof, "gather": gather, "stages_ms": stage_avg,
+                "gpu_launches": K * launches_per_forward(cfg), "e2e": e2e,
+                "cpu_baseline": cpu, "clocks": clk}
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

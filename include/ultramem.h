@@ -1,0 +1,167 @@
+/*
+ * ultramem.h -- C ABI of the UltraMem memory-layer forward for GB300 (sm_103a).
+ *
+ * The layer is the one of "Ultra-Sparse Memory Network" (Huang et al., ICLR
+ * 2025, arXiv 2411.12364), Sec. 3.2, inference forward only:
+ *
+ *   S1  q = W_q x                                  query projection, shared by the
+ *                                                  row and column key sets (Trick 5)
+ *   S2  S_row = K_row q, S_col = K_col q           Eq. 4, keys reshaped r x K x (D_k/r)
+ *   S3  a = u^T S_row, b = t^T S_col               Eq. 6-7, (u, t) leading singular
+ *                                                  pair of the Tucker core C
+ *   S4  I = top-k(a), J = top-k(b)                 Eq. 8-9
+ *   S5  g(i,j) = S_row[:,i]^T C S_col[:,j]         Eq. 10, only on I x J
+ *   S6  top-m of g; weights = the raw scores       Eq. 10, Trick 1 (softmax removed)
+ *   S7  v' = Shuffle(v), p = v' / N, row = v' % N  Eq. 14, v = i*K + j
+ *   S8  acc[p] += w * V[row]                       Eq. 15, pooled per virtual block
+ *   S9  o = sum_p W_p^T acc[p]                     Eq. 13/15 (IVE) + Trick 6 output
+ *
+ * Shapes (all row-major and contiguous):
+ *   K = sqrt(E) * n keys per axis ("the key size is expanded by sqrt(E) times",
+ *   Sec. 3.2 IVE); N = n*n physical value rows; the virtual grid has K*K = E*N
+ *   slots.  Heads share the value table and their pooled rows are summed.
+ *
+ * Conventions for every entry point:
+ *   - Tensor pointers are DEVICE pointers unless a comment says HOST.  The
+ *     layer borrows the caller's weights for its whole lifetime and never
+ *     copies the value table; the caller keeps them alive and unchanged.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Calls that take a stream are asynchronous on it.
+ *   - Errors are returned as ultramem_status; nothing aborts, traps or throws.
+ *     ULTRAMEM_EINVAL means the call was rejected before anything launched.
+ *   - One layer handle must not be used by two calls at once (its workspace
+ *     is shared); different handles are independent.
+ */
+#ifndef ULTRAMEM_H
+#define ULTRAMEM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum ultramem_status {
+    ULTRAMEM_OK = 0,
+    ULTRAMEM_EINVAL = -1,   /* invalid config, size or pointer; nothing launched    */
+    ULTRAMEM_ENOMEM = -2,   /* a device or host allocation failed                    */
+    ULTRAMEM_ECUDA = -3,    /* a CUDA runtime call or kernel launch failed           */
+    ULTRAMEM_ETIMEOUT = -4, /* a bounded device-side wait gave up                    */
+    ULTRAMEM_EDEVICE = -5,  /* a kernel's own check recorded an error (bad index)    */
+    ULTRAMEM_ENODEV = -6    /* no CUDA device of compute capability 10.3             */
+} ultramem_status;
+
+enum { ULTRAMEM_F32 = 0, ULTRAMEM_BF16 = 1 };          /* storage of x, W_q, keys, V, W_p, out */
+enum { ULTRAMEM_ACT_NONE = 0, ULTRAMEM_ACT_SOFTMAX = 1 }; /* Trick 1 vs PKM's softmax (Eq. 3)  */
+
+/* Hyper-parameters of one layer, in the paper's notation. */
+typedef struct ultramem_config {
+    int32_t d_in;        /* D_i, width of x                                          */
+    int32_t d_k;         /* D_k, query/key width of one head; d_k % rank == 0        */
+    int32_t heads;       /* H, key sets that read the shared table (Sec. 3.1)        */
+    int32_t rank;        /* r, Tucker rank (Eq. 5), 1..8                              */
+    int32_t n;           /* physical grid side, N = n*n rows; K = sqrt(E)*n <= 49152  */
+    int32_t expand_e;    /* E, virtual expansion, a perfect square 1..16 (Eq. 13)    */
+    int32_t d_v;         /* D_v, physical value width, multiple of 8                  */
+    int32_t d_out;       /* D'_v, output width; == d_v when has_proj == 0             */
+    int32_t topk;        /* k, survivors per axis (Eq. 8-9), 1..min(K, 128)           */
+    int32_t topm;        /* m, slots read per head (Eq. 10), 1..min(k*k, 1024)        */
+    int32_t has_proj;    /* 1: projectors W_p present; 0 requires E == 1              */
+    int32_t share_query; /* 1: one query for both key sets (Trick 5); 0: W_q_col too  */
+    int32_t act;         /* ULTRAMEM_ACT_NONE or ULTRAMEM_ACT_SOFTMAX                 */
+    int32_t dtype;       /* ULTRAMEM_F32 or ULTRAMEM_BF16                              */
+    int32_t max_tokens;  /* largest B any later call may pass; sizes the workspace    */
+    int32_t reserved;    /* must be 0                                                 */
+    uint64_t shuffle_seed; /* Eq. 14 shuffle: 0 = identity, otherwise the seeded
+                              bijection pi(v) = (a v + c) mod E*N whose a and c come
+                              from the first two SplitMix64 outputs of the seed
+                              (a = 1 + o1 mod (E*N - 1) stepped up to gcd(a, E*N) = 1,
+                              c = o2 mod E*N); E*N must be < 2^32                     */
+} ultramem_config;
+
+/* The layer's parameters.  Device tensors are in the storage type cfg.dtype
+ * (fp32, or bf16 as 16-bit words) unless noted. */
+typedef struct ultramem_weights {
+    const void *w_q;       /* [H*D_k][D_i]; head h owns rows h*D_k..h*D_k+D_k-1       */
+    const void *w_q_col;   /* [H*D_k][D_i] column query when share_query == 0, else NULL */
+    const void *k_row;     /* [H][K][D_k]; rank chunk alpha = columns alpha*D_k/r..    */
+    const void *k_col;     /* [H][K][D_k]                                              */
+    const float *core;     /* HOST fp32 [H][r][r], Tucker cores C_h, copied at create  */
+    const float *u;        /* HOST fp32 [H][r] or NULL: leading left singular vectors  */
+    const float *t;        /* HOST fp32 [H][r] or NULL (both or neither); when NULL
+                              they are computed at create from the SVD of C_h with the
+                              sign rule sum(u) > 0 (first non-zero entry if the sum is 0) */
+    const void *values;    /* [N][D_v], physical table V; 16-byte aligned              */
+    const void *w_proj;    /* [E][D_v][D'_v] projectors W_p, or NULL when has_proj == 0 */
+    const uint32_t *perm;  /* [E*N] explicit shuffle v -> v', or NULL for the seeded one */
+} ultramem_weights;
+
+typedef struct ultramem_layer ultramem_layer;
+
+/* Validates cfg and weights, computes (u, t) if not given, derives the shuffle,
+ * allocates the workspace for cfg.max_tokens tokens on the current device and
+ * writes a new handle to *out.  Returns ULTRAMEM_EINVAL for an invalid config
+ * (including a core whose leading singular value is 0 when u, t are NULL),
+ * ULTRAMEM_ENOMEM if the workspace cannot be allocated, ULTRAMEM_ENODEV if the
+ * current device is not compute capability 10.3. */
+ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weights *w,
+                                ultramem_layer **out);
+
+/* Frees the workspace and the handle; borrowed weights are untouched.  NULL is
+ * a no-op.  Waits for work still queued on the layer's workspace. */
+void ultramem_destroy(ultramem_layer *layer);
+
+/* S1-S9 for B tokens: x [B][D_i] -> out [B][D'_v] (both cfg.dtype).  Optional
+ * outputs (NULL to skip): idx_out [B][H][m] int64 virtual addresses v = i*K + j,
+ * w_out [B][H][m] fp32 weights, each head's m slots ordered by (score desc,
+ * v asc).  0 <= B <= max_tokens (B == 0 launches nothing). */
+ultramem_status ultramem_forward(ultramem_layer *layer, const void *x, int32_t B,
+                                 void *out, int64_t *idx_out, float *w_out, void *stream);
+
+/* The same forward on HOST buffers: copies x to the device, runs the forward
+ * and copies out back, all on `stream`, and returns after the stream has
+ * finished.  Pinned host memory gives asynchronous copies; pageable works. */
+ultramem_status ultramem_forward_host(ultramem_layer *layer, const void *x_host, int32_t B,
+                                      void *out_host, void *stream);
+
+/* S1-S6 only (retrieval, Eq. 4-10): idx_out [B][H][m] int64 and w_out
+ * [B][H][m] fp32 as in ultramem_forward; both required. */
+ultramem_status ultramem_retrieve(ultramem_layer *layer, const void *x, int32_t B,
+                                  int64_t *idx_out, float *w_out, void *stream);
+
+/* S7-S9 only (the lookup-reduce of Eq. 14-15) on given slots: idx [B][H][m]
+ * int64 virtual addresses in [0, E*N), w [B][H][m] fp32 -> out [B][D'_v].  An
+ * address out of range is not read: the kernel records it and the next
+ * ultramem_check returns ULTRAMEM_EDEVICE. */
+ultramem_status ultramem_lookup_reduce(ultramem_layer *layer, const int64_t *idx,
+                                       const float *w, int32_t B, void *out, void *stream);
+
+/* Synchronises `stream`, then reads and clears the layer's device error word:
+ * ULTRAMEM_EDEVICE if a kernel recorded a bad index, ULTRAMEM_ETIMEOUT if a
+ * bounded wait gave up, ULTRAMEM_ECUDA if the stream reports an error. */
+ultramem_status ultramem_check(ultramem_layer *layer, void *stream);
+
+/* Leading singular triplet of one r x r core (HOST, row-major fp32) with the
+ * sign rule above (Eq. 7; the SVD of Eq. 11).  ULTRAMEM_EINVAL if sigma == 0. */
+ultramem_status ultramem_rank1(const float *core, int32_t r, float *u, float *t,
+                               float *sigma);
+
+/* Per-stage timing for profiling: while enabled, every forward records CUDA
+ * events between its kernels on its stream.  ultramem_profile_read fills
+ * ms[0..n) with the device time of each stage of the most recent forward
+ * (the caller synchronises first) and returns the number of stages;
+ * ultramem_stage_name names stage i.  Disabled by default. */
+ultramem_status ultramem_profile_enable(ultramem_layer *layer, int32_t enable);
+int32_t ultramem_profile_read(ultramem_layer *layer, float *ms, int32_t n);
+const char *ultramem_stage_name(int32_t i);
+
+/* Human-readable name of a status code. */
+const char *ultramem_status_string(ultramem_status s);
+
+/* ABI version, currently 1. */
+int32_t ultramem_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ULTRAMEM_H */

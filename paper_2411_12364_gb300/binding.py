@@ -1,0 +1,236 @@
+"""Thin Python binding of libultramem.so (include/ultramem.h).
+
+Argument marshalling only: torch tensors become device pointers and the
+current torch stream becomes the cudaStream_t; every step of the layer runs
+in the CUDA library.  There is no fallback: if the library cannot be built or
+loaded, or no GPU is present, the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EDEVICE, ENODEV = 0, -1, -2, -3, -4, -5, -6
+F32, BF16 = 0, 1
+ACT_NONE, ACT_SOFTMAX = 0, 1
+
+# every function include/ultramem.h declares
+EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
+           "ultramem_forward_host", "ultramem_retrieve", "ultramem_lookup_reduce",
+           "ultramem_check", "ultramem_rank1", "ultramem_profile_enable",
+           "ultramem_profile_read", "ultramem_stage_name", "ultramem_status_string",
+           "ultramem_version")
+
+
+class Config(C.Structure):
+    _fields_ = [(name, C.c_int32) for name in (
+        "d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out", "topk", "topm",
+        "has_proj", "share_query", "act", "dtype", "max_tokens", "reserved")] + [
+        ("shuffle_seed", C.c_uint64)]
+
+
+class Weights(C.Structure):
+    _fields_ = [("w_q", C.c_void_p), ("w_q_col", C.c_void_p), ("k_row", C.c_void_p),
+                ("k_col", C.c_void_p), ("core", C.c_void_p), ("u", C.c_void_p),
+                ("t", C.c_void_p), ("values", C.c_void_p), ("w_proj", C.c_void_p),
+                ("perm", C.c_void_p)]
+
+
+class UltraMemError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: {status_string(status)} ({status})")
+        self.status = status
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def load(path: str | None = None) -> C.CDLL:
+    """Builds (if needed) and loads the CUDA library."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = path or _build.build()
+        lib = C.CDLL(path)
+        P, I32, I64 = C.c_void_p, C.c_int32, C.c_int64
+        lib.ultramem_create.argtypes = [P, P, P]
+        lib.ultramem_create.restype = I32
+        lib.ultramem_destroy.argtypes = [P]
+        lib.ultramem_destroy.restype = None
+        lib.ultramem_forward.argtypes = [P, P, I32, P, P, P, P]
+        lib.ultramem_forward.restype = I32
+        lib.ultramem_forward_host.argtypes = [P, P, I32, P, P]
+        lib.ultramem_forward_host.restype = I32
+        lib.ultramem_retrieve.argtypes = [P, P, I32, P, P, P]
+        lib.ultramem_retrieve.restype = I32
+        lib.ultramem_lookup_reduce.argtypes = [P, P, P, I32, P, P]
+        lib.ultramem_lookup_reduce.restype = I32
+        lib.ultramem_check.argtypes = [P, P]
+        lib.ultramem_check.restype = I32
+        lib.ultramem_rank1.argtypes = [P, I32, P, P, P]
+        lib.ultramem_rank1.restype = I32
+        lib.ultramem_profile_enable.argtypes = [P, I32]
+        lib.ultramem_profile_enable.restype = I32
+        lib.ultramem_profile_read.argtypes = [P, P, I32]
+        lib.ultramem_profile_read.restype = I32
+        lib.ultramem_stage_name.argtypes = [I32]
+        lib.ultramem_stage_name.restype = C.c_char_p
+        lib.ultramem_status_string.argtypes = [I32]
+        lib.ultramem_status_string.restype = C.c_char_p
+        lib.ultramem_version.argtypes = []
+        lib.ultramem_version.restype = I32
+        _lib = lib
+        return lib
+
+
+def status_string(s: int) -> str:
+    return load().ultramem_status_string(int(s)).decode()
+
+
+def _check(status: int, what: str):
+    if status != OK:
+        raise UltraMemError(status, what)
+
+
+def rank1(core):
+    """Leading singular triplet (u, t, sigma) of one r x r core, Eq. 7."""
+    import numpy as np
+    c = np.ascontiguousarray(core, dtype=np.float32)
+    r = c.shape[0]
+    u = np.zeros(r, np.float32)
+    t = np.zeros(r, np.float32)
+    s = np.zeros(1, np.float32)
+    _check(load().ultramem_rank1(c.ctypes.data, r, u.ctypes.data, t.ctypes.data,
+                                 s.ctypes.data), "ultramem_rank1")
+    return u, t, float(s[0])
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def _stream():
+    return torch.cuda.current_stream().cuda_stream
+
+
+_CFG_KEYS = ("d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out", "topk",
+             "topm", "has_proj", "share_query", "act", "dtype")
+
+
+class UltraMemLayer:
+    """One UltraMem layer on the current CUDA device.
+
+    ``weights`` holds device tensors in the layer's storage type (``w_q``,
+    ``w_q_col``, ``k_row``, ``k_col``, ``values``, ``w_proj``), the cores
+    ``core`` [H, r, r] (any device, fp32) and optionally ``u``, ``t`` [H, r]
+    and an explicit shuffle ``perm`` (int32/uint32 device tensor).  The layer
+    keeps references to them for its lifetime."""
+
+    def __init__(self, cfg: dict, weights: dict, max_tokens: int):
+        if not torch.cuda.is_available():
+            raise RuntimeError("UltraMemLayer needs a CUDA device (GB300, sm_103a)")
+        self.lib = load()
+        self.cfg = dict(cfg)
+        c = Config()
+        for k in _CFG_KEYS:
+            setattr(c, k, int(cfg[k]))
+        c.max_tokens = int(max_tokens)
+        c.reserved = 0
+        c.shuffle_seed = int(cfg.get("shuffle_seed", 0))
+        self._c = c
+        dev_keys = ("w_q", "w_q_col", "k_row", "k_col", "values", "w_proj", "perm")
+        self._keep = {k: (None if weights.get(k) is None else weights[k].contiguous())
+                      for k in dev_keys}
+        for k, v in self._keep.items():
+            if v is not None and not v.is_cuda:
+                raise ValueError(f"{k} must be a CUDA tensor")
+        self._core = weights["core"].detach().to("cpu", torch.float32).contiguous()
+        u, t = weights.get("u"), weights.get("t")
+        self._u = None if u is None else torch.as_tensor(u).to("cpu", torch.float32).contiguous()
+        self._t = None if t is None else torch.as_tensor(t).to("cpu", torch.float32).contiguous()
+        w = Weights(_ptr(self._keep["w_q"]), _ptr(self._keep["w_q_col"]),
+                    _ptr(self._keep["k_row"]), _ptr(self._keep["k_col"]),
+                    self._core.data_ptr(), _ptr(self._u), _ptr(self._t),
+                    _ptr(self._keep["values"]), _ptr(self._keep["w_proj"]),
+                    _ptr(self._keep["perm"]))
+        h = C.c_void_p()
+        _check(self.lib.ultramem_create(C.byref(c), C.byref(w), C.byref(h)), "ultramem_create")
+        self._h = h
+        self.max_tokens = int(max_tokens)
+        self.dtype = torch.float32 if int(cfg["dtype"]) == F32 else torch.bfloat16
+
+    # -- calls ------------------------------------------------------------
+    def forward(self, x: torch.Tensor, out: torch.Tensor | None = None, with_slots=False):
+        """S1-S9.  Returns out [B, D'_v] (and idx [B,H,m] int64, w [B,H,m] fp32
+        when ``with_slots``)."""
+        x = x.contiguous()
+        B = x.shape[0]
+        if out is None:
+            out = torch.empty((B, int(self.cfg["d_out"])), dtype=self.dtype, device=x.device)
+        idx = w = None
+        if with_slots:
+            H, m = int(self.cfg["heads"]), int(self.cfg["topm"])
+            idx = torch.empty((B, H, m), dtype=torch.int64, device=x.device)
+            w = torch.empty((B, H, m), dtype=torch.float32, device=x.device)
+        _check(self.lib.ultramem_forward(self._h, x.data_ptr(), B, out.data_ptr(), _ptr(idx),
+                                         _ptr(w), _stream()), "ultramem_forward")
+        return (out, idx, w) if with_slots else out
+
+    def forward_host(self, x_host: torch.Tensor, out_host: torch.Tensor):
+        """The forward on host tensors (pinned for asynchronous copies)."""
+        _check(self.lib.ultramem_forward_host(self._h, x_host.data_ptr(), x_host.shape[0],
+                                              out_host.data_ptr(), _stream()),
+               "ultramem_forward_host")
+        return out_host
+
+    def retrieve(self, x: torch.Tensor):
+        """S1-S6: (idx [B,H,m] int64 virtual addresses, w [B,H,m] fp32)."""
+        x = x.contiguous()
+        B = x.shape[0]
+        H, m = int(self.cfg["heads"]), int(self.cfg["topm"])
+        idx = torch.empty((B, H, m), dtype=torch.int64, device=x.device)
+        w = torch.empty((B, H, m), dtype=torch.float32, device=x.device)
+        _check(self.lib.ultramem_retrieve(self._h, x.data_ptr(), B, idx.data_ptr(),
+                                          w.data_ptr(), _stream()), "ultramem_retrieve")
+        return idx, w
+
+    def lookup_reduce(self, idx: torch.Tensor, w: torch.Tensor):
+        """S7-S9 on given slots (Eq. 14-15)."""
+        idx = idx.contiguous().to(torch.int64)
+        w = w.contiguous().to(torch.float32)
+        B = idx.shape[0]
+        out = torch.empty((B, int(self.cfg["d_out"])), dtype=self.dtype, device=idx.device)
+        _check(self.lib.ultramem_lookup_reduce(self._h, idx.data_ptr(), w.data_ptr(), B,
+                                               out.data_ptr(), _stream()),
+               "ultramem_lookup_reduce")
+        return out
+
+    def check(self) -> int:
+        """Syncs the current stream and returns the device error status."""
+        return int(self.lib.ultramem_check(self._h, _stream()))
+
+    def profile(self, enable: bool = True):
+        _check(self.lib.ultramem_profile_enable(self._h, int(enable)), "profile_enable")
+
+    def profile_read(self) -> dict:
+        buf = (C.c_float * 8)()
+        n = self.lib.ultramem_profile_read(self._h, buf, 8)
+        return {self.lib.ultramem_stage_name(i).decode(): float(buf[i]) for i in range(n)}
+
+    def close(self):
+        if getattr(self, "_h", None):
+            self.lib.ultramem_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

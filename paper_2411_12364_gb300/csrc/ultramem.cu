@@ -1,0 +1,513 @@
+// ultramem.cu -- the C ABI declared in include/ultramem.h: validation, the
+// create-time SVD and shuffle parameters, workspace ownership, the launch
+// sequence of one forward, per-stage profiling and the device error word.
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <new>
+
+#include "um_internal.cuh"
+
+using um::Dims;
+using um::Ptrs;
+
+namespace {
+
+constexpr int kStages = 5;
+const char *const kStageNames[kStages] = {"query", "score", "select", "gather", "project"};
+
+struct Workspace {
+    float *q_part = nullptr, *s = nullptr, *sel_w = nullptr, *acc = nullptr,
+          *proj_part = nullptr;
+    int32_t *sel_row = nullptr, *sel_p = nullptr;
+    float *core = nullptr, *u = nullptr, *t = nullptr;
+    int *err = nullptr;
+    void *x_stage = nullptr, *out_stage = nullptr;
+};
+
+}  // namespace
+
+struct ultramem_layer {
+    ultramem_config cfg;
+    ultramem_weights w;
+    int device;
+    Dims base;           // every field but B, q_splits, p_splits
+    Workspace ws;
+    bool profiling = false;
+    bool profiled_once = false;
+    cudaEvent_t ev[kStages + 1] = {};
+};
+
+namespace {
+
+int64_t keys_per_axis(const ultramem_config &c) {
+    int s = (int)lround(sqrt((double)c.expand_e));
+    return (int64_t)s * c.n;
+}
+
+size_t elt_size(const ultramem_config &c) { return c.dtype == ULTRAMEM_BF16 ? 2 : 4; }
+
+// Split counts of the two split-K contractions for a given batch: enough CTAs
+// to cover the 152 SMs about twice, each split at least 64 deep.
+int query_splits(const ultramem_config &c, int B) {
+    int tiles = ((c.heads * c.d_k + 63) / 64) * ((B + 31) / 32) * (c.share_query ? 1 : 2);
+    int s = (304 + tiles - 1) / tiles;
+    int cap = c.d_in / 64 > 0 ? c.d_in / 64 : 1;
+    if (s > 8) s = 8;
+    if (s > cap) s = cap;
+    return s < 1 ? 1 : s;
+}
+
+int proj_splits(const ultramem_config &c, int B) {
+    if (!c.has_proj) return 1;
+    int tiles = ((c.d_out + 63) / 64) * ((B + 31) / 32);
+    int s = (304 + tiles - 1) / tiles;
+    int kd = c.expand_e * c.d_v;
+    int cap = kd / 64 > 0 ? kd / 64 : 1;
+    if (s > 8) s = 8;
+    if (s > cap) s = cap;
+    return s < 1 ? 1 : s;
+}
+
+ultramem_status validate(const ultramem_config *c, const ultramem_weights *w) {
+    if (!c || !w) return ULTRAMEM_EINVAL;
+    if (c->reserved != 0) return ULTRAMEM_EINVAL;
+    if (c->d_in <= 0 || c->d_k <= 0 || c->heads <= 0 || c->rank < 1 || c->rank > 8)
+        return ULTRAMEM_EINVAL;
+    if (c->d_k % c->rank) return ULTRAMEM_EINVAL;
+    if (c->n <= 0 || c->d_v <= 0 || c->d_v % 8) return ULTRAMEM_EINVAL;
+    int s = (int)lround(sqrt((double)c->expand_e));
+    if (c->expand_e < 1 || c->expand_e > 16 || s * s != c->expand_e) return ULTRAMEM_EINVAL;
+    int64_t K = keys_per_axis(*c);
+    if (K > 49152) return ULTRAMEM_EINVAL;
+    uint64_t M = (uint64_t)c->expand_e * (uint64_t)c->n * (uint64_t)c->n;
+    if (M >= (1ull << 32)) return ULTRAMEM_EINVAL;
+    if (c->topk < 1 || c->topk > 128 || c->topk > K) return ULTRAMEM_EINVAL;
+    if (c->topm < 1 || c->topm > 1024 || c->topm > c->topk * c->topk) return ULTRAMEM_EINVAL;
+    if (c->has_proj != 0 && c->has_proj != 1) return ULTRAMEM_EINVAL;
+    if (!c->has_proj && (c->expand_e != 1 || c->d_out != c->d_v)) return ULTRAMEM_EINVAL;
+    if (c->has_proj && c->d_out <= 0) return ULTRAMEM_EINVAL;
+    if (c->share_query != 0 && c->share_query != 1) return ULTRAMEM_EINVAL;
+    if (c->act != ULTRAMEM_ACT_NONE && c->act != ULTRAMEM_ACT_SOFTMAX) return ULTRAMEM_EINVAL;
+    if (c->dtype != ULTRAMEM_F32 && c->dtype != ULTRAMEM_BF16) return ULTRAMEM_EINVAL;
+    if (c->max_tokens < 1 || c->max_tokens > (1 << 20)) return ULTRAMEM_EINVAL;
+    if (!w->w_q || !w->k_row || !w->k_col || !w->core || !w->values) return ULTRAMEM_EINVAL;
+    if (!c->share_query && !w->w_q_col) return ULTRAMEM_EINVAL;
+    if (c->has_proj && !w->w_proj) return ULTRAMEM_EINVAL;
+    if ((w->u == nullptr) != (w->t == nullptr)) return ULTRAMEM_EINVAL;
+    if (((uintptr_t)w->values) % 16) return ULTRAMEM_EINVAL;
+    return ULTRAMEM_OK;
+}
+
+// Leading singular triplet by one-sided (Hestenes) Jacobi on the columns of
+// C: rotations orthogonalise the columns of U = C V; the column norms are the
+// singular values and V holds the right singular vectors.
+ultramem_status rank1_host(const double *c, int r, double *u, double *t, double *sigma) {
+    double U[64], Vm[64];
+    for (int i = 0; i < r * r; ++i) U[i] = c[i];
+    for (int i = 0; i < r; ++i)
+        for (int j = 0; j < r; ++j) Vm[i * r + j] = i == j ? 1.0 : 0.0;
+    for (int sweep = 0; sweep < 60; ++sweep) {
+        bool rotated = false;
+        for (int p = 0; p < r; ++p)
+            for (int q = p + 1; q < r; ++q) {
+                double al = 0, be = 0, ga = 0;
+                for (int i = 0; i < r; ++i) {
+                    al += U[i * r + p] * U[i * r + p];
+                    be += U[i * r + q] * U[i * r + q];
+                    ga += U[i * r + p] * U[i * r + q];
+                }
+                if (fabs(ga) <= 1e-15 * sqrt(al * be) || ga == 0.0) continue;
+                rotated = true;
+                double zeta = (be - al) / (2.0 * ga);
+                double tn = (zeta >= 0 ? 1.0 : -1.0) / (fabs(zeta) + sqrt(1.0 + zeta * zeta));
+                double cs = 1.0 / sqrt(1.0 + tn * tn), sn = cs * tn;
+                for (int i = 0; i < r; ++i) {
+                    double x = U[i * r + p], y = U[i * r + q];
+                    U[i * r + p] = cs * x - sn * y;
+                    U[i * r + q] = sn * x + cs * y;
+                    x = Vm[i * r + p];
+                    y = Vm[i * r + q];
+                    Vm[i * r + p] = cs * x - sn * y;
+                    Vm[i * r + q] = sn * x + cs * y;
+                }
+            }
+        if (!rotated) break;
+    }
+    int best = 0;
+    double bestn = -1;
+    for (int j = 0; j < r; ++j) {
+        double nn = 0;
+        for (int i = 0; i < r; ++i) nn += U[i * r + j] * U[i * r + j];
+        if (nn > bestn) { bestn = nn; best = j; }
+    }
+    double sg = sqrt(bestn);
+    if (!(sg > 0.0)) return ULTRAMEM_EINVAL;
+    for (int i = 0; i < r; ++i) u[i] = U[i * r + best] / sg;
+    double sum = 0;
+    for (int i = 0; i < r; ++i) sum += u[i];
+    bool flip = sum < 0;
+    if (sum == 0)
+        for (int i = 0; i < r; ++i)
+            if (u[i] != 0) { flip = u[i] < 0; break; }
+    if (flip)
+        for (int i = 0; i < r; ++i) u[i] = -u[i];
+    for (int j = 0; j < r; ++j) {   // t = C^T u / sigma
+        double a = 0;
+        for (int i = 0; i < r; ++i) a += c[i * r + j] * u[i];
+        t[j] = a / sg;
+    }
+    *sigma = sg;
+    return ULTRAMEM_OK;
+}
+
+uint64_t splitmix_out(uint64_t state) {   // SplitMix64 output function
+    uint64_t z = state + 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+void shuffle_params(uint64_t seed, uint64_t M, uint64_t *a, uint64_t *c) {
+    if (seed == 0 || M <= 1) { *a = 1; *c = 0; return; }
+    uint64_t o1 = splitmix_out(seed), o2 = splitmix_out(seed + 0x9E3779B97F4A7C15ull);
+    uint64_t x = 1 + o1 % (M - 1);
+    for (;;) {
+        uint64_t g = x, h = M;
+        while (h) { uint64_t r = g % h; g = h; h = r; }
+        if (g == 1) break;
+        x = x + 1 >= M ? 1 : x + 1;
+    }
+    *a = x;
+    *c = o2 % M;
+}
+
+template <typename T> cudaError_t dalloc(T **p, size_t n) {
+    if (n == 0) n = 1;
+    return cudaMalloc(reinterpret_cast<void **>(p), n * sizeof(T));
+}
+
+void free_workspace(Workspace &ws) {
+    void *ptrs[] = {ws.q_part, ws.s, ws.sel_w, ws.acc, ws.proj_part, ws.sel_row, ws.sel_p,
+                    ws.core, ws.u, ws.t, ws.err, ws.x_stage, ws.out_stage};
+    for (void *p : ptrs)
+        if (p) cudaFree(p);
+    ws = Workspace();
+}
+
+Ptrs make_ptrs(ultramem_layer *L) {
+    Ptrs p;
+    memset(&p, 0, sizeof p);
+    p.w_q = L->w.w_q;
+    p.w_q_col = L->w.w_q_col;
+    p.k_row = L->w.k_row;
+    p.k_col = L->w.k_col;
+    p.values = L->w.values;
+    p.w_proj = L->w.w_proj;
+    p.perm = L->w.perm;
+    p.core = L->ws.core;
+    p.u = L->ws.u;
+    p.t = L->ws.t;
+    p.q_part = L->ws.q_part;
+    p.s = L->ws.s;
+    p.sel_w = L->ws.sel_w;
+    p.acc = L->ws.acc;
+    p.proj_part = L->ws.proj_part;
+    p.sel_row = L->ws.sel_row;
+    p.sel_p = L->ws.sel_p;
+    p.err = L->ws.err;
+    return p;
+}
+
+Dims dims_for(const ultramem_layer *L, int B) {
+    Dims d = L->base;
+    d.B = B;
+    d.q_splits = query_splits(L->cfg, B);
+    d.p_splits = proj_splits(L->cfg, B);
+    return d;
+}
+
+ultramem_status from_cuda(cudaError_t e) {
+    if (e == cudaSuccess) return ULTRAMEM_OK;
+    if (e == cudaErrorMemoryAllocation) return ULTRAMEM_ENOMEM;
+    return ULTRAMEM_ECUDA;
+}
+
+void mark(ultramem_layer *L, int i, cudaStream_t st) {
+    if (L->profiling) cudaEventRecord(L->ev[i], st);
+}
+
+// S1..S6 (retrieval) then S7..S9; `retrieve_only` stops after S6.
+ultramem_status run(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
+                    bool retrieve_only) {
+    cudaError_t e;
+    mark(L, 0, st);
+    if ((e = um::launch_query(d, p, st)) != cudaSuccess) return from_cuda(e);
+    mark(L, 1, st);
+    if ((e = um::launch_score(d, p, st)) != cudaSuccess) return from_cuda(e);
+    mark(L, 2, st);
+    if ((e = um::launch_select(d, p, st)) != cudaSuccess) return from_cuda(e);
+    mark(L, 3, st);
+    if (retrieve_only) return ULTRAMEM_OK;
+    if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
+    mark(L, 4, st);
+    if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
+    mark(L, 5, st);
+    if (L->profiling) L->profiled_once = true;
+    return ULTRAMEM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t ultramem_version(void) { return 1; }
+
+const char *ultramem_status_string(ultramem_status s) {
+    switch (s) {
+    case ULTRAMEM_OK: return "ok";
+    case ULTRAMEM_EINVAL: return "invalid argument";
+    case ULTRAMEM_ENOMEM: return "out of memory";
+    case ULTRAMEM_ECUDA: return "CUDA error";
+    case ULTRAMEM_ETIMEOUT: return "device wait timed out";
+    case ULTRAMEM_EDEVICE: return "device-side check failed";
+    case ULTRAMEM_ENODEV: return "no compute capability 10.3 device";
+    }
+    return "unknown status";
+}
+
+const char *ultramem_stage_name(int32_t i) {
+    return (i >= 0 && i < kStages) ? kStageNames[i] : nullptr;
+}
+
+ultramem_status ultramem_rank1(const float *core, int32_t r, float *u, float *t,
+                               float *sigma) {
+    if (!core || !u || !t || !sigma || r < 1 || r > 8) return ULTRAMEM_EINVAL;
+    double c[64], uu[8], tt[8], sg;
+    for (int i = 0; i < r * r; ++i) c[i] = core[i];
+    ultramem_status s = rank1_host(c, r, uu, tt, &sg);
+    if (s != ULTRAMEM_OK) return s;
+    for (int i = 0; i < r; ++i) {
+        u[i] = (float)uu[i];
+        t[i] = (float)tt[i];
+    }
+    *sigma = (float)sg;
+    return ULTRAMEM_OK;
+}
+
+ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weights *w,
+                                ultramem_layer **out) {
+    if (!out) return ULTRAMEM_EINVAL;
+    *out = nullptr;
+    ultramem_status st = validate(cfg, w);
+    if (st != ULTRAMEM_OK) return st;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return ULTRAMEM_ENODEV;
+    int major = 0, minor = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    if (major != 10 || minor != 3) return ULTRAMEM_ENODEV;
+
+    const int H = cfg->heads, r = cfg->rank;
+    // (u, t) per head: given, or the SVD of each core (Eq. 7)
+    float *hu = (float *)malloc(sizeof(float) * H * r);
+    float *ht = (float *)malloc(sizeof(float) * H * r);
+    if (!hu || !ht) { free(hu); free(ht); return ULTRAMEM_ENOMEM; }
+    for (int h = 0; h < H; ++h) {
+        if (w->u) {
+            memcpy(hu + h * r, w->u + h * r, sizeof(float) * r);
+            memcpy(ht + h * r, w->t + h * r, sizeof(float) * r);
+        } else {
+            float sg;
+            if (ultramem_rank1(w->core + (size_t)h * r * r, r, hu + h * r, ht + h * r, &sg) !=
+                ULTRAMEM_OK) {
+                free(hu); free(ht);
+                return ULTRAMEM_EINVAL;
+            }
+        }
+    }
+
+    ultramem_layer *L = new (std::nothrow) ultramem_layer();
+    if (!L) { free(hu); free(ht); return ULTRAMEM_ENOMEM; }
+    L->cfg = *cfg;
+    L->w = *w;
+    L->device = dev;
+    Dims &d = L->base;
+    memset(&d, 0, sizeof d);
+    d.d_in = cfg->d_in;
+    d.d_k = cfg->d_k;
+    d.H = H;
+    d.r = r;
+    d.dk = cfg->d_k / r;
+    d.K = (int)keys_per_axis(*cfg);
+    d.N = (int64_t)cfg->n * cfg->n;
+    d.M = (uint64_t)cfg->expand_e * (uint64_t)d.N;
+    d.E = cfg->expand_e;
+    d.d_v = cfg->d_v;
+    d.d_out = cfg->d_out;
+    d.k = cfg->topk;
+    d.m = cfg->topm;
+    d.A = cfg->share_query ? 1 : 2;
+    d.act = cfg->act;
+    d.dtype = cfg->dtype;
+    d.has_proj = cfg->has_proj;
+    shuffle_params(cfg->shuffle_seed, d.M, &d.shuf_a, &d.shuf_c);
+
+    const size_t Bm = (size_t)cfg->max_tokens, HD = (size_t)H * cfg->d_k;
+    size_t qmax = 0, pmax = 0;
+    for (size_t B = 1; B <= Bm; B = (B < 32 ? B + 1 : B + 32)) {
+        size_t q = (size_t)query_splits(*cfg, (int)B) * B, pp = (size_t)proj_splits(*cfg, (int)B) * B;
+        if (q > qmax) qmax = q;
+        if (pp > pmax) pmax = pp;
+    }
+    {
+        size_t q = (size_t)query_splits(*cfg, (int)Bm) * Bm, pp = (size_t)proj_splits(*cfg, (int)Bm) * Bm;
+        if (q > qmax) qmax = q;
+        if (pp > pmax) pmax = pp;
+    }
+    Workspace &ws = L->ws;
+    cudaError_t e = cudaSuccess;
+    const size_t hm = Bm * H * cfg->topm;
+    if (e == cudaSuccess) e = dalloc(&ws.q_part, qmax * d.A * HD);
+    if (e == cudaSuccess) e = dalloc(&ws.s, Bm * H * 2 * (size_t)d.K * r);
+    if (e == cudaSuccess) e = dalloc(&ws.sel_w, hm);
+    if (e == cudaSuccess) e = dalloc(&ws.sel_row, hm);
+    if (e == cudaSuccess) e = dalloc(&ws.sel_p, hm);
+    if (e == cudaSuccess) e = dalloc(&ws.acc, cfg->has_proj ? Bm * d.E * d.d_v : 1);
+    if (e == cudaSuccess) e = dalloc(&ws.proj_part, cfg->has_proj ? pmax * d.d_out : 1);
+    if (e == cudaSuccess) e = dalloc(&ws.core, (size_t)H * r * r);
+    if (e == cudaSuccess) e = dalloc(&ws.u, (size_t)H * r);
+    if (e == cudaSuccess) e = dalloc(&ws.t, (size_t)H * r);
+    if (e == cudaSuccess) e = dalloc(&ws.err, 1);
+    if (e == cudaSuccess)
+        e = cudaMalloc(&ws.x_stage, Bm * cfg->d_in * elt_size(*cfg));
+    if (e == cudaSuccess)
+        e = cudaMalloc(&ws.out_stage, Bm * cfg->d_out * elt_size(*cfg));
+    if (e == cudaSuccess)
+        e = cudaMemcpy(ws.core, w->core, sizeof(float) * H * r * r, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(ws.u, hu, sizeof(float) * H * r, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(ws.t, ht, sizeof(float) * H * r, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemset(ws.err, 0, sizeof(int));
+    free(hu);
+    free(ht);
+    if (e == cudaSuccess) e = um::configure_select(d);
+    if (e == cudaSuccess) e = um::configure_gather(d);
+    if (e != cudaSuccess) {
+        free_workspace(ws);
+        delete L;
+        cudaGetLastError();
+        return from_cuda(e);
+    }
+    *out = L;
+    return ULTRAMEM_OK;
+}
+
+void ultramem_destroy(ultramem_layer *L) {
+    if (!L) return;
+    cudaDeviceSynchronize();
+    for (auto &ev : L->ev)
+        if (ev) cudaEventDestroy(ev);
+    free_workspace(L->ws);
+    delete L;
+}
+
+ultramem_status ultramem_forward(ultramem_layer *L, const void *x, int32_t B, void *out,
+                                 int64_t *idx_out, float *w_out, void *stream) {
+    if (!L || B < 0 || B > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (B == 0) return ULTRAMEM_OK;
+    if (!x || !out) return ULTRAMEM_EINVAL;
+    Dims d = dims_for(L, B);
+    Ptrs p = make_ptrs(L);
+    p.x = x;
+    p.out = out;
+    p.idx_out = idx_out;
+    p.w_out = w_out;
+    return run(L, d, p, (cudaStream_t)stream, false);
+}
+
+ultramem_status ultramem_retrieve(ultramem_layer *L, const void *x, int32_t B,
+                                  int64_t *idx_out, float *w_out, void *stream) {
+    if (!L || B < 0 || B > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (B == 0) return ULTRAMEM_OK;
+    if (!x || !idx_out || !w_out) return ULTRAMEM_EINVAL;
+    Dims d = dims_for(L, B);
+    Ptrs p = make_ptrs(L);
+    p.x = x;
+    p.idx_out = idx_out;
+    p.w_out = w_out;
+    return run(L, d, p, (cudaStream_t)stream, true);
+}
+
+ultramem_status ultramem_lookup_reduce(ultramem_layer *L, const int64_t *idx, const float *w,
+                                       int32_t B, void *out, void *stream) {
+    if (!L || B < 0 || B > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (B == 0) return ULTRAMEM_OK;
+    if (!idx || !w || !out) return ULTRAMEM_EINVAL;
+    Dims d = dims_for(L, B);
+    Ptrs p = make_ptrs(L);
+    p.idx_in = idx;
+    p.w_in = w;
+    p.out = out;
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e;
+    if ((e = um::launch_slots_from_addresses(d, p, st)) != cudaSuccess) return from_cuda(e);
+    if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
+    if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
+    return ULTRAMEM_OK;
+}
+
+ultramem_status ultramem_forward_host(ultramem_layer *L, const void *x_host, int32_t B,
+                                      void *out_host, void *stream) {
+    if (!L || B < 0 || B > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (B == 0) return ULTRAMEM_OK;
+    if (!x_host || !out_host) return ULTRAMEM_EINVAL;
+    cudaStream_t st = (cudaStream_t)stream;
+    const size_t es = elt_size(L->cfg);
+    cudaError_t e = cudaMemcpyAsync(L->ws.x_stage, x_host, (size_t)B * L->cfg.d_in * es,
+                                    cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return from_cuda(e);
+    ultramem_status s = ultramem_forward(L, L->ws.x_stage, B, L->ws.out_stage, nullptr,
+                                         nullptr, stream);
+    if (s != ULTRAMEM_OK) return s;
+    e = cudaMemcpyAsync(out_host, L->ws.out_stage, (size_t)B * L->cfg.d_out * es,
+                        cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return from_cuda(e);
+    return from_cuda(cudaStreamSynchronize(st));
+}
+
+ultramem_status ultramem_check(ultramem_layer *L, void *stream) {
+    if (!L) return ULTRAMEM_EINVAL;
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return ULTRAMEM_ECUDA;
+    int flags = 0;
+    if (cudaMemcpy(&flags, L->ws.err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+        return ULTRAMEM_ECUDA;
+    if (flags && cudaMemset(L->ws.err, 0, sizeof(int)) != cudaSuccess) return ULTRAMEM_ECUDA;
+    if (flags & um::kErrTimeout) return ULTRAMEM_ETIMEOUT;
+    if (flags & um::kErrBadIndex) return ULTRAMEM_EDEVICE;
+    return ULTRAMEM_OK;
+}
+
+ultramem_status ultramem_profile_enable(ultramem_layer *L, int32_t enable) {
+    if (!L) return ULTRAMEM_EINVAL;
+    if (enable && !L->ev[0])
+        for (auto &ev : L->ev)
+            if (cudaEventCreate(&ev) != cudaSuccess) return ULTRAMEM_ECUDA;
+    L->profiling = enable != 0;
+    L->profiled_once = false;
+    return ULTRAMEM_OK;
+}
+
+int32_t ultramem_profile_read(ultramem_layer *L, float *ms, int32_t n) {
+    if (!L || !ms || !L->profiled_once) return 0;
+    int cnt = n < kStages ? n : kStages;
+    for (int i = 0; i < cnt; ++i) {
+        float t = 0.f;
+        if (cudaEventElapsedTime(&t, L->ev[i], L->ev[i + 1]) != cudaSuccess) t = -1.f;
+        ms[i] = t;
+    }
+    return cnt;
+}
+
+}  // extern "C"

@@ -1,0 +1,184 @@
+// um_gather.cu -- S8 (weighted gather-sum grouped by virtual block, Eq. 15's
+// inner V^T s^_p) and S9 (the IVE projection o = sum_p W_p^T acc_p).
+//
+// Gather: one CTA per token.  Each warp takes a run of selected slots, issues
+// the 16-byte loads of all its rows before using any (memory-level
+// parallelism on the random rows of a multi-GB table), and accumulates
+// w * V[row] into its own fp32 copy of acc[E][D_v] in shared memory; the
+// warps' copies are summed at the end.  Row loads bypass L1 (read-only path).
+#include "um_internal.cuh"
+
+namespace um {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kUnroll = 4;   // rows in flight per warp
+
+__device__ __forceinline__ uint4 ld_stream(const void *ptr) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(ptr));
+    return v;
+}
+
+// add w * (8 bf16 or 4 fp32 packed in 16 bytes) into dst
+__device__ __forceinline__ void fma_vec(float *dst, uint4 v, float w, __nv_bfloat16) {
+    const uint32_t u[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        float lo = __uint_as_float(u[q] << 16), hi = __uint_as_float(u[q] & 0xffff0000u);
+        dst[2 * q] = fmaf(w, lo, dst[2 * q]);
+        dst[2 * q + 1] = fmaf(w, hi, dst[2 * q + 1]);
+    }
+}
+__device__ __forceinline__ void fma_vec(float *dst, uint4 v, float w, float) {
+    dst[0] = fmaf(w, __uint_as_float(v.x), dst[0]);
+    dst[1] = fmaf(w, __uint_as_float(v.y), dst[1]);
+    dst[2] = fmaf(w, __uint_as_float(v.z), dst[2]);
+    dst[3] = fmaf(w, __uint_as_float(v.w), dst[3]);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) gather_kernel(Dims d, Ptrs p) {
+    extern __shared__ __align__(16) float acc_w[];   // [kWarps][E][D_v]
+    const int b = blockIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int EDv = d.E * d.d_v;
+    float *mine = acc_w + (size_t)warp * EDv;
+    for (int i = lane; i < EDv; i += 32) mine[i] = 0.f;
+    __syncwarp();
+
+    constexpr int EPV = 16 / sizeof(T);   // elements per 16-byte vector
+    const int VPR = d.d_v / EPV;          // vectors per row
+    const int hm = d.H * d.m;
+    const int64_t base = (int64_t)b * hm;
+    const T *V = static_cast<const T *>(p.values);
+    for (int e0 = warp * kUnroll; e0 < hm; e0 += kWarps * kUnroll) {
+        int row[kUnroll], blk[kUnroll];
+        float w[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            int e = e0 + u;
+            bool ok = e < hm;
+            row[u] = ok ? p.sel_row[base + e] : 0;
+            blk[u] = ok ? p.sel_p[base + e] : 0;
+            w[u] = ok ? p.sel_w[base + e] : 0.f;
+        }
+        for (int vv = lane; vv < VPR; vv += 32) {
+            uint4 val[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u)
+                val[u] = (e0 + u < hm) ? ld_stream(V + (int64_t)row[u] * d.d_v + vv * EPV)
+                                       : make_uint4(0, 0, 0, 0);
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u)
+                if (e0 + u < hm) fma_vec(mine + blk[u] * d.d_v + vv * EPV, val[u], w[u], T());
+        }
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < EDv; i += kThreads) {
+        float s = 0.f;
+#pragma unroll
+        for (int wv = 0; wv < kWarps; ++wv) s += acc_w[(size_t)wv * EDv + i];
+        if (d.has_proj)
+            p.acc[(int64_t)b * EDv + i] = s;
+        else
+            static_cast<T *>(p.out)[(int64_t)b * d.d_v + i] = from_f<T>(s);
+    }
+}
+
+// proj_part[split][b][o] = sum over this split's slice of E*D_v of acc[b][c] W[c][o]
+// (W = the E projectors stacked: [E*D_v][D'_v]).  Tile 32 tokens x 64 outputs.
+template <typename T>
+__global__ void __launch_bounds__(kThreads) proj_kernel(Dims d, Ptrs p) {
+    const int Kd = d.E * d.d_v;
+    const int split = blockIdx.z;
+    const int chunk = (Kd + d.p_splits - 1) / d.p_splits;
+    const int kb = split * chunk, ke = min(Kd, kb + chunk);
+    const int o0 = blockIdx.x * 64, b0 = blockIdx.y * 32;
+    const T *W = static_cast<const T *>(p.w_proj);
+    __shared__ float as[32][33];   // [c][token]
+    __shared__ float ws[32][65];   // [c][output]
+    const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+    float acc[2][4] = {};
+    for (int k0 = kb; k0 < ke; k0 += 32) {
+        for (int e = tid; e < 32 * 32; e += kThreads) {
+            int bb = e / 32, kk = e % 32, b = b0 + bb, c = k0 + kk;
+            as[kk][bb] = (b < d.B && c < ke) ? p.acc[(int64_t)b * Kd + c] : 0.f;
+        }
+        for (int e = tid; e < 32 * 64; e += kThreads) {
+            int kk = e / 64, oo = e % 64, c = k0 + kk, o = o0 + oo;
+            ws[kk][oo] = (c < ke && o < d.d_out) ? to_f(W[(int64_t)c * d.d_out + o]) : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int kk = 0; kk < 32; ++kk) {
+            float a0 = as[kk][ty * 2], a1 = as[kk][ty * 2 + 1];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                float wv = ws[kk][tx * 4 + j];
+                acc[0][j] = fmaf(a0, wv, acc[0][j]);
+                acc[1][j] = fmaf(a1, wv, acc[1][j]);
+            }
+        }
+        __syncthreads();
+    }
+    for (int i = 0; i < 2; ++i)
+        for (int j = 0; j < 4; ++j) {
+            int b = b0 + ty * 2 + i, o = o0 + tx * 4 + j;
+            if (b < d.B && o < d.d_out)
+                p.proj_part[((int64_t)split * d.B + b) * d.d_out + o] = acc[i][j];
+        }
+}
+
+template <typename T>
+__global__ void proj_reduce_kernel(Dims d, Ptrs p) {
+    const int64_t total = (int64_t)d.B * d.d_out;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        float s = 0.f;
+        for (int sp = 0; sp < d.p_splits; ++sp) s += p.proj_part[(int64_t)sp * total + i];
+        static_cast<T *>(p.out)[i] = from_f<T>(s);
+    }
+}
+
+}  // namespace
+
+size_t gather_smem_bytes(const Dims &d) { return sizeof(float) * kWarps * d.E * d.d_v; }
+
+cudaError_t configure_gather(const Dims &d) {
+    cudaError_t e = cudaFuncSetAttribute(gather_kernel<float>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)gather_smem_bytes(d));
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(gather_kernel<__nv_bfloat16>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)gather_smem_bytes(d));
+}
+
+cudaError_t launch_gather(const Dims &d, const Ptrs &p, cudaStream_t st) {
+    if (d.dtype == ULTRAMEM_BF16)
+        gather_kernel<__nv_bfloat16><<<d.B, kThreads, gather_smem_bytes(d), st>>>(d, p);
+    else
+        gather_kernel<float><<<d.B, kThreads, gather_smem_bytes(d), st>>>(d, p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_proj(const Dims &d, const Ptrs &p, cudaStream_t st) {
+    dim3 grid((d.d_out + 63) / 64, (d.B + 31) / 32, d.p_splits);
+    int64_t total = (int64_t)d.B * d.d_out;
+    int rblocks = (int)((total + 255) / 256);
+    if (rblocks > 4096) rblocks = 4096;
+    if (d.dtype == ULTRAMEM_BF16) {
+        proj_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(d, p);
+        proj_reduce_kernel<__nv_bfloat16><<<rblocks, 256, 0, st>>>(d, p);
+    } else {
+        proj_kernel<float><<<grid, kThreads, 0, st>>>(d, p);
+        proj_reduce_kernel<float><<<rblocks, 256, 0, st>>>(d, p);
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace um

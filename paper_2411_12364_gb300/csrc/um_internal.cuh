@@ -1,0 +1,83 @@
+// um_internal.cuh -- shared declarations of the UltraMem CUDA library.
+//
+// Every kernel receives the layer's dimensions (Dims) and the device pointers
+// it touches (Ptrs) by value.  Workspace layouts (all fp32 unless noted):
+//   q_part   [q_splits][A][B][H*D_k]   split-K partial sums of q = W_q x
+//   s        [B][H][2][K][r]           S_row (axis 0) and S_col (axis 1), Eq. 4
+//   sel_row  [B][H][m] int32           physical row of each selected slot
+//   sel_p    [B][H][m] int32           virtual block p of each selected slot
+//   sel_w    [B][H][m]                 weight of each selected slot
+//   acc      [B][E*D_v]                per-block pooled rows, Eq. 15 inner sum
+//   proj_part[p_splits][B][D'_v]       split-K partial sums of the projection
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/ultramem.h"
+
+namespace um {
+
+constexpr int kErrBadIndex = 1;   // an address outside [0, E*N) was given
+constexpr int kErrTimeout = 2;    // a bounded wait gave up
+
+struct Dims {
+    int B;            // tokens in this call
+    int d_in, d_k, H, r, dk;  // dk = D_k / r
+    int K;            // keys per axis
+    int64_t N;        // physical rows
+    uint64_t M;       // virtual slots E*N
+    int E, d_v, d_out, k, m;
+    int A;            // 1 = shared query, 2 = separate column query
+    int act, dtype, has_proj;
+    uint64_t shuf_a, shuf_c;
+    int q_splits, p_splits;
+};
+
+struct Ptrs {
+    const void *x, *w_q, *w_q_col, *k_row, *k_col, *values, *w_proj;
+    const uint32_t *perm;
+    const float *core, *u, *t;   // library copies: [H][r][r], [H][r], [H][r]
+    float *q_part, *s, *sel_w, *acc, *proj_part;
+    int32_t *sel_row, *sel_p;
+    void *out;
+    int64_t *idx_out;
+    float *w_out;
+    const int64_t *idx_in;       // lookup_reduce input addresses
+    const float *w_in;           // lookup_reduce input weights
+    int *err;                    // device error word (bit flags above)
+};
+
+cudaError_t launch_query(const Dims &d, const Ptrs &p, cudaStream_t st);
+cudaError_t launch_score(const Dims &d, const Ptrs &p, cudaStream_t st);
+cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st);
+cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream_t st);
+cudaError_t launch_gather(const Dims &d, const Ptrs &p, cudaStream_t st);
+cudaError_t launch_proj(const Dims &d, const Ptrs &p, cudaStream_t st);
+
+// kernel attributes for large dynamic shared memory, set at layer creation
+cudaError_t configure_select(const Dims &d);
+cudaError_t configure_gather(const Dims &d);
+size_t select_smem_bytes(const Dims &d);
+size_t gather_smem_bytes(const Dims &d);
+
+// ---- small device helpers ------------------------------------------------
+
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) {
+    return __float2bfloat16_rn(v);
+}
+
+// The Eq. 14 shuffle: explicit table or the seeded affine bijection.
+__device__ __forceinline__ uint64_t shuffle_address(const Dims &d, const uint32_t *perm,
+                                                    uint64_t v) {
+    if (perm) return perm[v];
+    return (d.shuf_a * v + d.shuf_c) % d.M;   // M < 2^32 so a*v < 2^64
+}
+
+}  // namespace um

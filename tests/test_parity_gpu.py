@@ -1,0 +1,173 @@
+"""GPU parity: the CUDA library against the CPU oracle on the same seeded
+inputs, through the C ABI (ctypes binding).  Indices bit-exact up to the
+near-tie rule, weights and outputs within the stated tolerances."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2411_12364_gb300 import workloads
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(cfg, B, gpu_lib, tokens=None, max_tokens=None, batch_index=0, perm=None,
+         pass_svd=True):
+    from paper_2411_12364_gb300.binding import UltraMemLayer
+    w = workloads.make_weights(cfg, device="cuda")
+    if perm is not None:
+        w["perm"] = perm
+    x = workloads.make_tokens(cfg, B, batch_index, device="cuda")
+    t = parity.numpy_inputs(cfg, w, x)
+    if perm is not None:
+        t["perm"] = perm.cpu().numpy().astype(np.int64)
+    lw = dict(w)
+    if pass_svd:
+        lw["u"], lw["t"] = torch.from_numpy(t["u"]), torch.from_numpy(t["t"])
+    layer = UltraMemLayer(cfg, lw, max_tokens or B)
+    out, idx, wt = layer.forward(x, with_slots=True)
+    torch.cuda.synchronize()
+    assert layer.check() == 0
+    tokens = np.arange(B) if tokens is None else np.asarray(tokens)
+    o_out, o_idx, o_w = oracle.forward(cfg, t, B, tokens=tokens)
+    res = parity.compare(cfg, t, tokens, out.float().cpu().numpy(), idx.cpu().numpy(),
+                         wt.cpu().numpy(), o_out, o_idx, o_w)
+    return layer, (w, x, t), (out, idx, wt), res
+
+
+SMALL = [
+    dict(dtype=0),
+    dict(dtype=1),
+    dict(dtype=0, expand_e=1, has_proj=0, d_out=64, n=40),
+    dict(dtype=1, expand_e=9, n=11, d_out=72),
+    dict(dtype=0, rank=1, d_k=24),
+    dict(dtype=0, rank=3, d_k=48, heads=3),
+    dict(dtype=1, share_query=0),
+    dict(dtype=0, act=1),
+    dict(dtype=0, topk=48, topm=1),          # k = K: no pruning
+    dict(dtype=0, n=6, topk=5, topm=25),     # m = k*k
+    dict(dtype=1, heads=4, topk=16, topm=40, d_v=128, d_out=40),
+    dict(dtype=0, shuffle_seed=0),
+]
+
+
+@pytest.mark.parametrize("B", [1, 7, 37, 70])
+@pytest.mark.parametrize("over", SMALL, ids=[str(i) for i in range(len(SMALL))])
+def test_small_layers(over, B, gpu_lib):
+    cfg = workloads.small_config(**over)
+    _run(cfg, B, gpu_lib)
+
+
+def test_tiny_fp32_workload(gpu_lib):
+    cfg = workloads.layer_config("tiny_fp32")
+    _run(cfg, 16, gpu_lib)
+
+
+def test_decode_1m_workload(gpu_lib):
+    cfg = workloads.layer_config("decode_1m")
+    _run(cfg, 64, gpu_lib)
+
+
+@pytest.mark.parametrize("B", [1, 8, 32, 128])
+def test_mid_4m_workload(B, gpu_lib):
+    cfg = workloads.layer_config("mid_4m")
+    _run(cfg, B, gpu_lib)
+
+
+@pytest.mark.parametrize("B", [1, 64, 256])
+def test_large_20m_workload(B, gpu_lib):
+    cfg = workloads.layer_config("large_20m")
+    _run(cfg, B, gpu_lib)
+
+
+def test_prefill_16k_sampled(gpu_lib):
+    """All 16384 tokens run on the GPU; a seeded sample of 384 (including the
+    first and last tile's tokens) is checked against the oracle."""
+    cfg = workloads.layer_config("prefill_16k")
+    rng = np.random.default_rng(4)
+    sample = np.unique(np.concatenate([np.arange(8), np.arange(16384 - 8, 16384),
+                                       rng.choice(16384, 368, replace=False)]))
+    _run(cfg, 16384, gpu_lib, tokens=sample)
+
+
+def test_lookup_reduce_on_oracle_slots(gpu_lib):
+    """S7-S9 alone: the GPU pools the oracle's own (v, w) like the oracle."""
+    from paper_2411_12364_gb300.binding import UltraMemLayer
+    cfg = workloads.layer_config("decode_1m")
+    w = workloads.make_weights(cfg, device="cuda")
+    x = workloads.make_tokens(cfg, 16, device="cuda")
+    t = parity.numpy_inputs(cfg, w, x)
+    layer = UltraMemLayer(cfg, dict(w, u=torch.from_numpy(t["u"]), t=torch.from_numpy(t["t"])), 16)
+    o_out, o_idx, o_w = oracle.forward(cfg, t, 16)
+    out = layer.lookup_reduce(torch.from_numpy(o_idx).cuda(),
+                              torch.from_numpy(o_w.astype(np.float32)).cuda())
+    ref = oracle.lookup_reduce(cfg, t, o_idx, o_w.astype(np.float32).astype(np.float64))
+    got = out.float().cpu().numpy()
+    err = np.abs(got - ref).max(1) / np.abs(ref).max(1)
+    assert err.max() <= parity.out_tol(cfg)
+    assert layer.check() == 0
+
+
+def test_retrieve_and_host_forward_agree_with_forward(gpu_lib):
+    cfg = workloads.small_config(dtype=1)
+    layer, (w, x, t), (out, idx, wt), _ = _run(cfg, 33, gpu_lib)
+    i2, w2 = layer.retrieve(x)
+    assert torch.equal(i2, idx) and torch.equal(w2, wt)
+    xh = x.cpu().pin_memory()
+    oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    layer.forward_host(xh, oh)
+    assert torch.equal(oh, out.cpu())
+
+
+def test_forward_is_deterministic(gpu_lib):
+    cfg = workloads.small_config(dtype=1, heads=3)
+    layer, (w, x, t), (out, idx, wt), _ = _run(cfg, 70, gpu_lib)
+    for _ in range(3):
+        o2, i2, w2 = layer.forward(x, with_slots=True)
+        assert torch.equal(o2, out) and torch.equal(i2, idx) and torch.equal(w2, wt)
+
+
+def test_library_svd_and_explicit_perm(gpu_lib):
+    """(u, t) computed by the library at create, and an explicit shuffle
+    table, both give the oracle's result."""
+    cfg = workloads.small_config(dtype=0, n=10)
+    M = cfg["expand_e"] * cfg["n"] ** 2
+    perm = torch.from_numpy(np.random.default_rng(3).permutation(M).astype(np.int32)).cuda()
+    _run(cfg, 20, gpu_lib, perm=perm, pass_svd=False)
+
+
+def test_workspace_reuse_across_batch_sizes(gpu_lib):
+    """One handle sized for 70 tokens serves smaller batches too."""
+    cfg = workloads.small_config(dtype=1)
+    layer, (w, x, t), (out, idx, wt), _ = _run(cfg, 70, gpu_lib)
+    for B in (1, 5, 32, 64):
+        o2, i2, w2 = layer.forward(x[:B].contiguous(), with_slots=True)
+        assert torch.equal(i2, idx[:B])
+        assert torch.equal(o2, out[:B])
+
+
+def test_bad_address_is_reported_not_read(gpu_lib):
+    """An out-of-range virtual address given to lookup_reduce is skipped by
+    the kernel's own bounds check and reported by ultramem_check."""
+    from paper_2411_12364_gb300 import binding
+    cfg = workloads.small_config(dtype=1)
+    layer, (w, x, t), (out, idx, wt), _ = _run(cfg, 4, gpu_lib)
+    bad = idx.clone()
+    bad[1, 0, 0] = cfg["expand_e"] * cfg["n"] ** 2 + 5
+    bad[2, 1, 3] = -1
+    layer.lookup_reduce(bad, wt)
+    assert layer.check() == binding.EDEVICE
+    assert layer.check() == 0   # the error word is cleared by the read
+
+
+def test_batch_limits(gpu_lib):
+    from paper_2411_12364_gb300 import binding
+    cfg = workloads.small_config(dtype=1)
+    layer, (w, x, t), _, _ = _run(cfg, 8, gpu_lib)
+    lib = binding.load()
+    st = lib.ultramem_forward(layer._h, x.data_ptr(), 0, None, None, None, None)
+    assert st == binding.OK
+    big = torch.zeros((9, cfg["d_in"]), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(binding.UltraMemError):
+        layer.forward(big)
