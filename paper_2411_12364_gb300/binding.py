@@ -24,7 +24,7 @@ EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
            "ultramem_forward_host", "ultramem_retrieve", "ultramem_lookup_reduce",
            "ultramem_check", "ultramem_rank1", "ultramem_profile_enable",
            "ultramem_profile_read", "ultramem_stage_name", "ultramem_status_string",
-           "ultramem_version")
+           "ultramem_last_error", "ultramem_version")
 
 
 class Config(C.Structure):
@@ -43,7 +43,12 @@ class Weights(C.Structure):
 
 class UltraMemError(RuntimeError):
     def __init__(self, status: int, what: str):
-        super().__init__(f"{what}: {status_string(status)} ({status})")
+        msg = f"{what}: {status_string(status)} ({status})"
+        if status in (ECUDA, ENOMEM):
+            detail = load().ultramem_last_error().decode()
+            if detail:
+                msg += f" [{detail}]"
+        super().__init__(msg)
         self.status = status
 
 
@@ -84,6 +89,8 @@ def load(path: str | None = None) -> C.CDLL:
         lib.ultramem_stage_name.restype = C.c_char_p
         lib.ultramem_status_string.argtypes = [I32]
         lib.ultramem_status_string.restype = C.c_char_p
+        lib.ultramem_last_error.argtypes = []
+        lib.ultramem_last_error.restype = C.c_char_p
         lib.ultramem_version.argtypes = []
         lib.ultramem_version.restype = I32
         _lib = lib

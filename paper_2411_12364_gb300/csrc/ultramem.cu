@@ -2,6 +2,7 @@
 // create-time SVD and shuffle parameters, workspace ownership, the launch
 // sequence of one forward, per-stage profiling and the device error word.
 #include <math.h>
+#include <stdio.h>
 #include <stdlib.h>
 #include <string.h>
 
@@ -24,6 +25,7 @@ struct Workspace {
     float *core = nullptr, *u = nullptr, *t = nullptr;
     int *err = nullptr;
     void *x_stage = nullptr, *out_stage = nullptr;
+    __nv_bfloat16 *qs = nullptr, *acc_bf = nullptr, *w_pt = nullptr;   // tensor path
 };
 
 }  // namespace
@@ -34,6 +36,8 @@ struct ultramem_layer {
     int device;
     Dims base;           // every field but B, q_splits, p_splits
     Workspace ws;
+    bool tc = false;     // bf16 tensor-core path (tcgen05) for S1, S2, S9
+    um::TcMaps maps;     // weight descriptors of the tensor path
     bool profiling = false;
     bool profiled_once = false;
     cudaEvent_t ev[kStages + 1] = {};
@@ -59,6 +63,24 @@ int query_splits(const ultramem_config &c, int B) {
     return s < 1 ? 1 : s;
 }
 
+// Tensor path: split D_i so that about 128 CTAs stream W_q.
+int tc_query_splits(const ultramem_config &c, int B) {
+    int m_tiles = (c.heads * c.d_k + 127) / 128;
+    int nt = um::tc_n_tile(B, 1);
+    int n_tiles = (B + nt - 1) / nt;
+    int kb = (c.d_in + 63) / 64;
+    int s = (128 + m_tiles * n_tiles - 1) / (m_tiles * n_tiles);
+    if (s > kb) s = kb;
+    return s < 1 ? 1 : s;
+}
+
+// The tensor path needs bf16 storage, rank chunks of whole 16-wide MMA
+// steps, at most 4 chunks (TMEM columns) and 16-byte rows for TMA.
+bool tc_eligible(const ultramem_config &c) {
+    return c.dtype == ULTRAMEM_BF16 && (c.d_k / c.rank) % 16 == 0 && c.rank <= 4 &&
+           c.d_in % 8 == 0 && (c.expand_e * c.d_v) % 8 == 0 && c.d_k % 8 == 0;
+}
+
 int proj_splits(const ultramem_config &c, int B) {
     if (!c.has_proj) return 1;
     int tiles = ((c.d_out + 63) / 64) * ((B + 31) / 32);
@@ -80,7 +102,7 @@ ultramem_status validate(const ultramem_config *c, const ultramem_weights *w) {
     int s = (int)lround(sqrt((double)c->expand_e));
     if (c->expand_e < 1 || c->expand_e > 16 || s * s != c->expand_e) return ULTRAMEM_EINVAL;
     int64_t K = keys_per_axis(*c);
-    if (K > 49152) return ULTRAMEM_EINVAL;
+    if (K > 40960) return ULTRAMEM_EINVAL;
     uint64_t M = (uint64_t)c->expand_e * (uint64_t)c->n * (uint64_t)c->n;
     if (M >= (1ull << 32)) return ULTRAMEM_EINVAL;
     if (c->topk < 1 || c->topk > 128 || c->topk > K) return ULTRAMEM_EINVAL;
@@ -189,8 +211,10 @@ template <typename T> cudaError_t dalloc(T **p, size_t n) {
 }
 
 void free_workspace(Workspace &ws) {
-    void *ptrs[] = {ws.q_part, ws.s, ws.sel_w, ws.acc, ws.proj_part, ws.sel_row, ws.sel_p,
-                    ws.core, ws.u, ws.t, ws.err, ws.x_stage, ws.out_stage};
+    void *ptrs[] = {ws.q_part, ws.s,    ws.sel_w,   ws.acc,       ws.proj_part,
+                    ws.sel_row, ws.sel_p, ws.core,   ws.u,         ws.t,
+                    ws.err,    ws.x_stage, ws.out_stage, ws.qs,     ws.acc_bf,
+                    ws.w_pt};
     for (void *p : ptrs)
         if (p) cudaFree(p);
     ws = Workspace();
@@ -223,24 +247,36 @@ Ptrs make_ptrs(ultramem_layer *L) {
 Dims dims_for(const ultramem_layer *L, int B) {
     Dims d = L->base;
     d.B = B;
-    d.q_splits = query_splits(L->cfg, B);
+    d.q_splits = L->tc ? tc_query_splits(L->cfg, B) : query_splits(L->cfg, B);
     d.p_splits = proj_splits(L->cfg, B);
     return d;
 }
 
+thread_local char g_last_error[256] = "";
+
 ultramem_status from_cuda(cudaError_t e) {
     if (e == cudaSuccess) return ULTRAMEM_OK;
+    snprintf(g_last_error, sizeof g_last_error, "%s: %s", cudaGetErrorName(e),
+             cudaGetErrorString(e));
     if (e == cudaErrorMemoryAllocation) return ULTRAMEM_ENOMEM;
     return ULTRAMEM_ECUDA;
 }
 
+// Stage events; under stream capture they must be external event nodes so
+// that every replay of the graph records them.
 void mark(ultramem_layer *L, int i, cudaStream_t st) {
-    if (L->profiling) cudaEventRecord(L->ev[i], st);
+    if (!L->profiling) return;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    cudaStreamIsCapturing(st, &cs);
+    if (cs == cudaStreamCaptureStatusActive)
+        cudaEventRecordWithFlags(L->ev[i], st, cudaEventRecordExternal);
+    else
+        cudaEventRecord(L->ev[i], st);
 }
 
 // S1..S6 (retrieval) then S7..S9; `retrieve_only` stops after S6.
-ultramem_status run(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
-                    bool retrieve_only) {
+ultramem_status run_cuda_core(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
+                              bool retrieve_only) {
     cudaError_t e;
     mark(L, 0, st);
     if ((e = um::launch_query(d, p, st)) != cudaSuccess) return from_cuda(e);
@@ -258,11 +294,54 @@ ultramem_status run(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
     return ULTRAMEM_OK;
 }
 
+// The bf16 path: S1, S2 and S9 on tcgen05 tensor cores, S3-S8 as above.
+ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
+                           bool retrieve_only) {
+    const ultramem_config &c = L->cfg;
+    um::TcMaps mp = L->maps;
+    const int Bmax = c.max_tokens;
+    const int nt1 = um::tc_n_tile(d.B, 1), ntr = um::tc_n_tile(d.B, d.r);
+    if (!um::tc_encode(&mp.x, p.x, (uint64_t)c.d_in, (uint64_t)d.B, 1, (uint32_t)nt1, 2))
+        return ULTRAMEM_EINVAL;   // x must be 16-byte aligned
+    if (!um::tc_encode(&mp.qs, L->ws.qs, 3ull * c.d_k, (uint64_t)Bmax, (uint64_t)d.A * d.H,
+                       (uint32_t)ntr, 3) ||
+        !um::tc_encode(&mp.acc, L->ws.acc_bf, (uint64_t)d.E * d.d_v, (uint64_t)Bmax, 1,
+                       (uint32_t)nt1, 2))
+        return ULTRAMEM_ECUDA;
+    p.acc_bf = c.has_proj ? L->ws.acc_bf : nullptr;
+    cudaError_t e;
+    mark(L, 0, st);
+    if ((e = um::launch_query_tc(d, p, mp, d.q_splits, st)) != cudaSuccess) return from_cuda(e);
+    if ((e = um::launch_qsplit(d, p, L->ws.qs, d.q_splits, Bmax, st)) != cudaSuccess)
+        return from_cuda(e);
+    mark(L, 1, st);
+    if ((e = um::launch_score_tc(d, p, mp, st)) != cudaSuccess) return from_cuda(e);
+    mark(L, 2, st);
+    if ((e = um::launch_select(d, p, st)) != cudaSuccess) return from_cuda(e);
+    mark(L, 3, st);
+    if (retrieve_only) return ULTRAMEM_OK;
+    if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
+    mark(L, 4, st);
+    if (d.has_proj && (e = um::launch_proj_tc(d, p, mp, st)) != cudaSuccess) return from_cuda(e);
+    mark(L, 5, st);
+    if (L->profiling) L->profiled_once = true;
+    return ULTRAMEM_OK;
+}
+
+ultramem_status run(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
+                    bool retrieve_only) {
+    cudaGetLastError();   // a stale error from unrelated work is not ours to report
+    return L->tc ? run_tensor(L, d, p, st, retrieve_only)
+                 : run_cuda_core(L, d, p, st, retrieve_only);
+}
+
 }  // namespace
 
 extern "C" {
 
 int32_t ultramem_version(void) { return 1; }
+
+const char *ultramem_last_error(void) { return g_last_error; }
 
 const char *ultramem_status_string(ultramem_status s) {
     switch (s) {
@@ -356,15 +435,15 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
 
     const size_t Bm = (size_t)cfg->max_tokens, HD = (size_t)H * cfg->d_k;
     size_t qmax = 0, pmax = 0;
-    for (size_t B = 1; B <= Bm; B = (B < 32 ? B + 1 : B + 32)) {
-        size_t q = (size_t)query_splits(*cfg, (int)B) * B, pp = (size_t)proj_splits(*cfg, (int)B) * B;
+    L->tc = tc_eligible(*cfg) && um::tc_init();
+    for (size_t B = 1; B <= Bm; B = (B < 256 ? B + 1 : B + 16)) {
+        size_t q = (size_t)query_splits(*cfg, (int)B) * B;
+        size_t qt = (size_t)tc_query_splits(*cfg, (int)B) * B;
+        size_t pp = (size_t)proj_splits(*cfg, (int)B) * B;
         if (q > qmax) qmax = q;
+        if (qt > qmax) qmax = qt;
         if (pp > pmax) pmax = pp;
-    }
-    {
-        size_t q = (size_t)query_splits(*cfg, (int)Bm) * Bm, pp = (size_t)proj_splits(*cfg, (int)Bm) * Bm;
-        if (q > qmax) qmax = q;
-        if (pp > pmax) pmax = pp;
+        if (B + 16 > Bm && B < Bm && B >= 256) B = Bm - 16;   // visit Bm itself
     }
     Workspace &ws = L->ws;
     cudaError_t e = cudaSuccess;
@@ -391,6 +470,36 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     if (e == cudaSuccess) e = cudaMemset(ws.err, 0, sizeof(int));
     free(hu);
     free(ht);
+    const size_t kd = (size_t)d.E * d.d_v;
+    if (e == cudaSuccess && L->tc) {
+        // tensor path: split queries, bf16 acc, K-major copy of the projectors
+        e = dalloc(&ws.qs, (size_t)d.A * H * Bm * 3 * cfg->d_k);
+        if (e == cudaSuccess) e = cudaMemset(ws.qs, 0, sizeof(__nv_bfloat16) * d.A * H * Bm * 3 * cfg->d_k);
+        if (e == cudaSuccess) e = dalloc(&ws.acc_bf, Bm * kd);
+        if (e == cudaSuccess) e = cudaMemset(ws.acc_bf, 0, sizeof(__nv_bfloat16) * Bm * kd);
+        if (e == cudaSuccess && cfg->has_proj) {
+            e = dalloc(&ws.w_pt, kd * cfg->d_out);
+            if (e == cudaSuccess) e = um::launch_transpose_bf16(w->w_proj, ws.w_pt, (int)kd, cfg->d_out, 0);
+            if (e == cudaSuccess) e = cudaDeviceSynchronize();
+        }
+        if (e == cudaSuccess) e = um::configure_tc();
+        bool ok = e == cudaSuccess;
+        const uint64_t HD = (uint64_t)H * cfg->d_k;
+        ok = ok && um::tc_encode(&L->maps.w_q, w->w_q, cfg->d_in, HD, 1, 128, 2);
+        ok = ok && um::tc_encode(&L->maps.w_q_col, cfg->share_query ? w->w_q : w->w_q_col,
+                                 cfg->d_in, HD, 1, 128, 2);
+        ok = ok && um::tc_encode(&L->maps.k_row, w->k_row, cfg->d_k, d.K, H, 128, 3);
+        ok = ok && um::tc_encode(&L->maps.k_col, w->k_col, cfg->d_k, d.K, H, 128, 3);
+        if (cfg->has_proj)
+            ok = ok && um::tc_encode(&L->maps.w_pt, ws.w_pt, kd, cfg->d_out, 1, 128, 2);
+        else
+            L->maps.w_pt = L->maps.w_q;
+        if (e == cudaSuccess && !ok) {
+            free_workspace(ws);
+            delete L;
+            return ULTRAMEM_EINVAL;   // a weight is not 16-byte aligned
+        }
+    }
     if (e == cudaSuccess) e = um::configure_select(d);
     if (e == cudaSuccess) e = um::configure_gather(d);
     if (e != cudaSuccess) {
@@ -451,6 +560,7 @@ ultramem_status ultramem_lookup_reduce(ultramem_layer *L, const int64_t *idx, co
     p.out = out;
     cudaStream_t st = (cudaStream_t)stream;
     cudaError_t e;
+    cudaGetLastError();
     if ((e = um::launch_slots_from_addresses(d, p, st)) != cudaSuccess) return from_cuda(e);
     if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
     if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
@@ -464,6 +574,7 @@ ultramem_status ultramem_forward_host(ultramem_layer *L, const void *x_host, int
     if (!x_host || !out_host) return ULTRAMEM_EINVAL;
     cudaStream_t st = (cudaStream_t)stream;
     const size_t es = elt_size(L->cfg);
+    cudaGetLastError();
     cudaError_t e = cudaMemcpyAsync(L->ws.x_stage, x_host, (size_t)B * L->cfg.d_in * es,
                                     cudaMemcpyHostToDevice, st);
     if (e != cudaSuccess) return from_cuda(e);
@@ -504,7 +615,10 @@ int32_t ultramem_profile_read(ultramem_layer *L, float *ms, int32_t n) {
     int cnt = n < kStages ? n : kStages;
     for (int i = 0; i < cnt; ++i) {
         float t = 0.f;
-        if (cudaEventElapsedTime(&t, L->ev[i], L->ev[i + 1]) != cudaSuccess) t = -1.f;
+        if (cudaEventElapsedTime(&t, L->ev[i], L->ev[i + 1]) != cudaSuccess) {
+            cudaGetLastError();
+            t = -1.f;
+        }
         ms[i] = t;
     }
     return cnt;

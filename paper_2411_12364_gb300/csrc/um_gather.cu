@@ -13,7 +13,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kUnroll = 4;   // rows in flight per warp
+constexpr int kUnroll = 8;   // rows in flight per warp
 
 __device__ __forceinline__ uint4 ld_stream(const void *ptr) {
     uint4 v;
@@ -82,7 +82,9 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Dims d, Ptrs p) {
         float s = 0.f;
 #pragma unroll
         for (int wv = 0; wv < kWarps; ++wv) s += acc_w[(size_t)wv * EDv + i];
-        if (d.has_proj)
+        if (p.acc_bf)
+            p.acc_bf[(int64_t)b * EDv + i] = __float2bfloat16_rn(s);
+        else if (d.has_proj)
             p.acc[(int64_t)b * EDv + i] = s;
         else
             static_cast<T *>(p.out)[(int64_t)b * d.d_v + i] = from_f<T>(s);

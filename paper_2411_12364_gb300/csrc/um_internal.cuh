@@ -11,6 +11,7 @@
 //   proj_part[p_splits][B][D'_v]       split-K partial sums of the projection
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -44,10 +45,32 @@ struct Ptrs {
     void *out;
     int64_t *idx_out;
     float *w_out;
+    __nv_bfloat16 *acc_bf;       // tensor path: acc rounded to bf16 [B][E*D_v]
     const int64_t *idx_in;       // lookup_reduce input addresses
     const float *w_in;           // lookup_reduce input weights
     int *err;                    // device error word (bit flags above)
 };
+
+// TMA descriptors of the tensor-core path: weights (encoded at create) and
+// the per-call operands (token batch x, split queries qs, pooled acc).
+struct TcMaps {
+    CUtensorMap w_q, w_q_col, k_row, k_col, w_pt;
+    CUtensorMap x, qs, acc;
+};
+
+bool tc_init();
+bool tc_encode(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid, uint64_t outer,
+               uint32_t box_rows, int rank);
+int tc_n_tile(int B, int n_acc);
+cudaError_t configure_tc();
+cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int splits,
+                            cudaStream_t st);
+cudaError_t launch_qsplit(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, int splits, int Bmax,
+                          cudaStream_t st);
+cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st);
+cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st);
+cudaError_t launch_transpose_bf16(const void *src, void *dst, int rows, int cols,
+                                  cudaStream_t st);
 
 cudaError_t launch_query(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_score(const Dims &d, const Ptrs &p, cudaStream_t st);

@@ -1,11 +1,19 @@
 // um_select.cu -- S3..S7 for one (token, head) per CTA, in shared memory:
 //   rank-1 scores a = u^T S_row, b = t^T S_col          (Eq. 6-7)
-//   top-k of each axis by radix select                  (Eq. 8-9)
+//   top-k of each axis                                  (Eq. 8-9)
 //   exact Tucker score g on the k*k survivors           (Eq. 10)
 //   top-m of g, ordered by (score desc, v asc)          (Eq. 10)
 //   weights (raw scores, or PKM's softmax), shuffle     (Trick 1, Eq. 3, Eq. 14)
 // No K*K grid is ever formed.  Scores are compared as order-preserving 32-bit
 // keys of their fp32 values; ties go to the smaller index.
+//
+// Top-k of n keys (topk_positions): each thread takes the maximum of its
+// strided share of the keys; tau = the kk-th largest of those 256 maxima is
+// a lower bound of the kk-th largest key for any input (kk threads each own
+// a key >= tau).  Keys > tau are gathered, plus -- only when fewer than kk
+// keys exceed tau -- the first ties at tau in position order; these
+// candidates (typically one to three times kk) are ranked exactly.  If more
+// than kCap keys exceed tau, a radix select over all n keys is used instead.
 #include "um_internal.cuh"
 
 namespace um {
@@ -13,6 +21,8 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
+constexpr int kCap = 2048;       // candidate capacity of the threshold path
+constexpr int kMaxOut = 1024;    // largest k or m
 
 struct SelShared {
     int hist[256];
@@ -20,6 +30,13 @@ struct SelShared {
     int digit;
     int remaining;
     float scalar;
+    uint32_t vt[kThreads];
+    uint32_t cand_key[kCap];
+    int cand_pos[kCap];
+    uint32_t win_key[kMaxOut];
+    int win_pos[kMaxOut];
+    int n_gt;
+    uint32_t tau;
 };
 
 // fp32 -> uint32 whose unsigned order is the float order (-0 folded into +0).
@@ -33,7 +50,7 @@ __device__ __forceinline__ float ord2f(uint32_t o) {
 }
 
 // Exclusive prefix sum of one int per thread over the block; also syncs.
-__device__ int block_exclusive_scan(int v, SelShared &sh, int *total) {
+__device__ int block_exclusive_scan(int v, SelShared &sh) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     int incl = v;
 #pragma unroll
@@ -43,14 +60,9 @@ __device__ int block_exclusive_scan(int v, SelShared &sh, int *total) {
     }
     if (lane == 31) sh.warp_tot[warp] = incl;
     __syncthreads();
-    int before = 0, all = 0;
-    for (int w = 0; w < kWarps; ++w) {
-        int t = sh.warp_tot[w];
-        if (w < warp) before += t;
-        all += t;
-    }
+    int before = 0;
+    for (int w = 0; w < warp; ++w) before += sh.warp_tot[w];
     __syncthreads();
-    if (total) *total = all;
     return before + incl - v;
 }
 
@@ -106,58 +118,109 @@ __device__ uint32_t select_kth_largest(const uint32_t *key, int n, int kk, SelSh
     return prefix;
 }
 
-// Writes to out[], in increasing position order, every i < n with key > T
-// and the first need_eq positions with key == T (at most cap entries).
-__device__ void ordered_select(const uint32_t *key, int n, uint32_t T, int need_eq, int *out,
-                               int cap, SelShared &sh) {
+// Appends to sh.cand_*[base..] the first `need` positions (in position
+// order) with key == T, using contiguous per-thread ranges.
+__device__ void gather_ties_in_order(const uint32_t *key, int n, uint32_t T, int need, int base,
+                                     SelShared &sh) {
     const int per = (n + kThreads - 1) / kThreads;
     const int beg = min(n, (int)threadIdx.x * per), end = min(n, beg + per);
     int eq = 0;
     for (int i = beg; i < end; ++i) eq += key[i] == T;
-    const int eq_before = block_exclusive_scan(eq, sh, nullptr);
-    int take = 0;
-    for (int i = beg, e = eq_before; i < end; ++i) {
-        uint32_t v = key[i];
-        if (v > T) ++take;
-        else if (v == T) take += (e++ < need_eq);
-    }
-    int o = block_exclusive_scan(take, sh, nullptr);
-    for (int i = beg, e = eq_before; i < end; ++i) {
-        uint32_t v = key[i];
-        bool sel = v > T;
-        if (v == T) sel = (e++ < need_eq);
-        if (sel && o < cap) out[o] = i;
-        o += sel;
-    }
+    int e = block_exclusive_scan(eq, sh);
+    for (int i = beg; i < end && e < need; ++i)
+        if (key[i] == T) {
+            sh.cand_key[base + e] = T;
+            sh.cand_pos[base + e] = i;
+            ++e;
+        }
     __syncthreads();
 }
 
-// Ascending bitonic sort of P (a power of two) 64-bit words in shared memory.
-__device__ void bitonic_sort(unsigned long long *a, int P) {
-    for (int size = 2; size <= P; size <<= 1)
-        for (int stride = size >> 1; stride > 0; stride >>= 1) {
-            for (int i = threadIdx.x; i < P / 2; i += kThreads) {
-                int lo = 2 * i - (i & (stride - 1));
-                int hi = lo + stride;
-                bool up = ((lo & size) == 0);
-                unsigned long long x = a[lo], y = a[hi];
-                if ((x > y) == up) { a[lo] = y; a[hi] = x; }
-            }
-            __syncthreads();
-        }
-}
+enum { kOrderByPosition = 0, kOrderByScore = 1 };
 
-__device__ __forceinline__ int pow2_at_least(int m) {
-    int P = 1;
-    while (P < m) P <<= 1;
-    return P;
+// Positions of the kk largest keys of key[0..n) (ties: smaller position
+// first).  Leaves them in sh.win_pos / sh.win_key ordered by (key desc,
+// position asc); with kOrderByPosition, also writes the positions in
+// increasing order to out[0..kk).
+__device__ void topk_positions(const uint32_t *key, int n, int kk, int *out, int order,
+                               SelShared &sh) {
+    // tau = kk-th largest per-thread maximum (0 when fewer than kk threads own
+    // a key, which makes every key a candidate)
+    uint32_t vmax = 0;
+    for (int i = threadIdx.x; i < n; i += kThreads) vmax = max(vmax, key[i]);
+    sh.vt[threadIdx.x] = vmax;
+    if (threadIdx.x == 0) { sh.n_gt = 0; sh.tau = 0; }
+    __syncthreads();
+    {
+        int rank = 0;
+        for (int t = 0; t < kThreads; ++t) {
+            uint32_t o = sh.vt[t];
+            rank += (o > vmax) || (o == vmax && t < (int)threadIdx.x);
+        }
+        if (rank == kk - 1) sh.tau = vmax;
+    }
+    __syncthreads();
+    const uint32_t tau = sh.tau;
+    for (int i = threadIdx.x; i < n; i += kThreads) {
+        uint32_t v = key[i];
+        if (v > tau) {
+            int slot = atomicAdd(&sh.n_gt, 1);
+            if (slot < kCap) { sh.cand_key[slot] = v; sh.cand_pos[slot] = i; }
+        }
+    }
+    __syncthreads();
+    int c = sh.n_gt;
+    if (c > kCap) {
+        int need_eq;
+        uint32_t T = select_kth_largest(key, n, kk, sh, &need_eq);
+        // every key > T, then the first need_eq ties at T
+        if (threadIdx.x == 0) sh.n_gt = 0;
+        __syncthreads();
+        for (int i = threadIdx.x; i < n; i += kThreads) {
+            uint32_t v = key[i];
+            if (v > T) {
+                int slot = atomicAdd(&sh.n_gt, 1);
+                sh.cand_key[slot] = v;   // fewer than kk <= kCap of them
+                sh.cand_pos[slot] = i;
+            }
+        }
+        __syncthreads();
+        gather_ties_in_order(key, n, T, need_eq, kk - need_eq, sh);
+        c = kk;
+    } else if (c < kk) {
+        gather_ties_in_order(key, n, tau, kk - c, c, sh);
+        c = kk;
+    }
+    // exact rank of every candidate by (key desc, position asc)
+    for (int e = threadIdx.x; e < c; e += kThreads) {
+        const uint32_t ke = sh.cand_key[e];
+        const int pe = sh.cand_pos[e];
+        int rank = 0;
+        for (int f = 0; f < c; ++f) {
+            uint32_t kf = sh.cand_key[f];
+            rank += (kf > ke) || (kf == ke && sh.cand_pos[f] < pe);
+        }
+        if (rank < kk) {
+            sh.win_key[rank] = ke;
+            sh.win_pos[rank] = pe;
+        }
+    }
+    __syncthreads();
+    if (order == kOrderByPosition) {
+        for (int e = threadIdx.x; e < kk; e += kThreads) {
+            const int pe = sh.win_pos[e];
+            int r = 0;
+            for (int f = 0; f < kk; ++f) r += sh.win_pos[f] < pe;
+            out[r] = pe;
+        }
+        __syncthreads();
+    }
 }
 
 struct SelLayout {
     uint32_t *key;
-    int *sel_i, *sel_j, *win;
+    int *sel_i, *sel_j;
     float *srow, *scol, *R;
-    unsigned long long *sortbuf;
 };
 
 __device__ SelLayout carve(const Dims &d, unsigned char *base) {
@@ -166,15 +229,10 @@ __device__ SelLayout carve(const Dims &d, unsigned char *base) {
     size_t off = 0;
     L.key = reinterpret_cast<uint32_t *>(base + off);
     off += sizeof(uint32_t) * nkey;
-    off = (off + 15) & ~size_t(15);
-    L.sortbuf = reinterpret_cast<unsigned long long *>(base + off);
-    off += sizeof(unsigned long long) * pow2_at_least(d.m);
     L.sel_i = reinterpret_cast<int *>(base + off);
     off += sizeof(int) * d.k;
     L.sel_j = reinterpret_cast<int *>(base + off);
     off += sizeof(int) * d.k;
-    L.win = reinterpret_cast<int *>(base + off);
-    off += sizeof(int) * d.m;
     L.srow = reinterpret_cast<float *>(base + off);
     off += sizeof(float) * d.k * d.r;
     L.scol = reinterpret_cast<float *>(base + off);
@@ -191,7 +249,7 @@ __global__ void __launch_bounds__(kThreads) select_kernel(Dims d, Ptrs p) {
     const int r = d.r, K = d.K, k = d.k, m = d.m;
     const float *C = p.core + (int64_t)h * r * r;
 
-    // Eq. 6-9 per axis: rank-1 score, top-k, survivors in increasing index
+    // Eq. 6-9 per axis: rank-1 score, top-k; survivors in increasing index
     for (int axis = 0; axis < 2; ++axis) {
         const float *coef = (axis == 0 ? p.u : p.t) + (int64_t)h * r;
         const float *S = p.s + (((int64_t)b * d.H + h) * 2 + axis) * (int64_t)K * r;
@@ -201,10 +259,8 @@ __global__ void __launch_bounds__(kThreads) select_kernel(Dims d, Ptrs p) {
             L.key[i] = f2ord(a);
         }
         __syncthreads();
-        int need_eq;
-        uint32_t T = select_kth_largest(L.key, K, k, sh, &need_eq);
         int *sel = axis == 0 ? L.sel_i : L.sel_j;
-        ordered_select(L.key, K, T, need_eq, sel, k, sh);
+        topk_positions(L.key, K, k, sel, kOrderByPosition, sh);
         float *keep = axis == 0 ? L.srow : L.scol;
         for (int e = threadIdx.x; e < k * r; e += kThreads)
             keep[e] = S[(int64_t)sel[e / r] * r + (e % r)];
@@ -225,42 +281,29 @@ __global__ void __launch_bounds__(kThreads) select_kernel(Dims d, Ptrs p) {
         int ii = c / k, jj = c - ii * k;
         float g = 0.f;
         for (int be = 0; be < r; ++be) g = fmaf(L.R[ii * r + be], L.scol[jj * r + be], g);
-        L.key[c] = f2ord(g);   // candidate c = ii*k + jj: increasing c is increasing v
+        L.key[c] = f2ord(g);   // I and J ascending: increasing c is increasing v
     }
     __syncthreads();
-    int need_eq;
-    uint32_t T = select_kth_largest(L.key, k2, m, sh, &need_eq);
-    ordered_select(L.key, k2, T, need_eq, L.win, m, sh);
-
-    // order the m winners by (score desc, v asc)
-    const int P = pow2_at_least(m);
-    for (int e = threadIdx.x; e < P; e += kThreads)
-        L.sortbuf[e] = e < m ? ((unsigned long long)(~L.key[L.win[e]]) << 32) |
-                                   (unsigned)L.win[e]
-                             : ~0ull;
-    __syncthreads();
-    bitonic_sort(L.sortbuf, P);
+    topk_positions(L.key, k2, m, nullptr, kOrderByScore, sh);
 
     // PKM's softmax over the m selected scores (Eq. 3); Trick 1 skips it
+    const float gmax = ord2f(sh.win_key[0]);
     if (d.act == ULTRAMEM_ACT_SOFTMAX) {
         if (threadIdx.x < 32) {
-            float gmax = ord2f(L.key[(int)(L.sortbuf[0] & 0xffffffffu)]);
             float z = 0.f;
-            for (int e = threadIdx.x; e < m; e += 32)
-                z += __expf(ord2f(L.key[(int)(L.sortbuf[e] & 0xffffffffu)]) - gmax);
+            for (int e = threadIdx.x; e < m; e += 32) z += __expf(ord2f(sh.win_key[e]) - gmax);
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(0xffffffffu, z, off);
             if (threadIdx.x == 0) sh.scalar = z;
         }
         __syncthreads();
     }
-    const float gmax = ord2f(L.key[(int)(L.sortbuf[0] & 0xffffffffu)]);
     const int64_t base = ((int64_t)b * d.H + h) * m;
     for (int e = threadIdx.x; e < m; e += kThreads) {
-        int c = (int)(L.sortbuf[e] & 0xffffffffu);
+        int c = sh.win_pos[e];
         int ii = c / k, jj = c - ii * k;
         uint64_t v = (uint64_t)L.sel_i[ii] * (uint64_t)K + (uint64_t)L.sel_j[jj];
-        float g = ord2f(L.key[c]);
+        float g = ord2f(sh.win_key[e]);
         float w = d.act == ULTRAMEM_ACT_SOFTMAX ? __expf(g - gmax) / sh.scalar : g;
         uint64_t vs = shuffle_address(d, p.perm, v);   // Eq. 14
         uint64_t pb = vs / (uint64_t)d.N;
@@ -298,13 +341,7 @@ __global__ void slots_kernel(Dims d, Ptrs p) {
 
 size_t select_smem_bytes(const Dims &d) {
     size_t nkey = (size_t)(d.K > d.k * d.k ? d.K : d.k * d.k);
-    size_t P = 1;
-    while ((int)P < d.m) P <<= 1;
-    size_t off = sizeof(uint32_t) * nkey;
-    off = (off + 15) & ~size_t(15);
-    off += sizeof(unsigned long long) * P;
-    off += sizeof(int) * (2 * d.k + d.m);
-    off += sizeof(float) * 3 * d.k * d.r;
+    size_t off = sizeof(uint32_t) * nkey + sizeof(int) * 2 * d.k + sizeof(float) * 3 * d.k * d.r;
     return (off + 15) & ~size_t(15);
 }
 

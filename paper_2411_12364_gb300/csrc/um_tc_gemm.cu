@@ -1,0 +1,443 @@
+// um_tc_gemm.cu -- the three dense contractions of the layer on tcgen05
+// tensor cores (bf16 storage mode):
+//   S1  q_part = W_q x            M = H*D_k outputs, N = tokens, K = D_i (split-K)
+//   S2  S_alpha = K_chunk q_chunk M = keys, N = tokens, K = D_k in r chunks (Eq. 4)
+//   S9  out = W_p^T acc           M = D'_v outputs, N = tokens, K = E*D_v (Eq. 15)
+// Weights fill the 128-row M side ("swap AB"), so a decode batch of B tokens
+// is the N side of one MMA (N = B rounded up to 16).
+//
+// q is an fp32 result; the scores must be as exact as fp32 because they pick
+// indices, so q enters S2 as three bf16 terms q = q1 + q2 + q3 (each the bf16
+// rounding of what the previous terms leave, residual <= 2^-24 |q|) and each
+// key tile is multiplied by all three, accumulating in fp32.  Keys are bf16
+// and enter exactly.
+//
+// One CTA (4 warps) computes one 128 x N tile: warp 0 lane 0 issues the TMA
+// loads of a 4-stage ring, warp 1 lane 0 issues the MMAs, and all four warps
+// then read TMEM (row i = lane i) for the epilogue.  Every mbarrier wait is
+// bounded; a timeout sets the layer's error word.
+#include <cudaTypedefs.h>
+
+#include "um_internal.cuh"
+#include "um_tc.cuh"
+
+namespace um {
+namespace {
+
+using namespace tc;
+
+constexpr int kThreads = 128;
+constexpr int kMaxStages = 4;
+constexpr int kMaxAcc = 4;
+constexpr size_t kSmemBudget = 225 * 1024;   // leaves room for static smem
+
+struct Tile {
+    int m0, n0;        // first A row, first B row of the tile
+    int a_sel;         // which A map (0/1)
+    int a_z, b_z;      // third coordinate of 3-D maps (-1: 2-D map)
+    int kb0, nkb;      // K blocks [kb0, kb0 + nkb)
+};
+
+__host__ __device__ inline size_t stage_bytes_of(int nsplit, int n_tile) {
+    return kTileABytes + (size_t)nsplit * n_tile * 128;
+}
+
+// As many ring stages as fit (at most 4, never more than the K blocks).
+inline int stages_for(int nsplit, int n_tile, int nkb) {
+    int s = (int)((kSmemBudget - 1024) / stage_bytes_of(nsplit, n_tile));
+    if (s > kMaxStages) s = kMaxStages;
+    if (s > nkb) s = nkb;
+    return s < 1 ? 1 : s;
+}
+
+template <int NSPLIT, class Op>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0,
+                   const __grid_constant__ CUtensorMap mapA1,
+                   const __grid_constant__ CUtensorMap mapB, Op op) {
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full[kMaxStages], empty[kMaxStages], accbar;
+    __shared__ uint32_t tmem_slot;
+    uint8_t *ring = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const Tile t = op.tile();
+    const int n_tile = op.n_tile;
+    const uint32_t b_bytes = (uint32_t)n_tile * 128;
+    const uint32_t stage_bytes = kTileABytes + NSPLIT * b_bytes;
+    const uint32_t ncols = tmem_cols_for((uint32_t)(op.n_acc * n_tile));
+    const CUtensorMap *mapA = t.a_sel ? &mapA1 : &mapA0;
+    const int kStages = op.stages;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(&accbar, 1);
+        fence_mbar_init();
+        prefetch_tensormap(mapA);
+        prefetch_tensormap(&mapB);
+    }
+    if (warp == 0) tmem_alloc(&tmem_slot, ncols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        // producer: TMA loads of A (128 x 64) and NSPLIT B tiles (N x 64)
+        int it = 0;
+        for (; it < t.nkb; ++it) {
+            const int s = it % kStages;
+            if (it >= kStages && !mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
+                atomicOr(op.err, kErrTimeout);
+                break;
+            }
+            uint8_t *sa = ring + (size_t)s * stage_bytes;
+            mbar_arrive_expect_tx(&full[s], stage_bytes);
+            const int kx = (t.kb0 + it) * kBlockK;
+            if (t.a_z >= 0) tma_load_3d(sa, mapA, &full[s], kx, t.m0, t.a_z);
+            else tma_load_2d(sa, mapA, &full[s], kx, t.m0);
+#pragma unroll
+            for (int j = 0; j < NSPLIT; ++j) {
+                uint8_t *sb = sa + kTileABytes + j * b_bytes;
+                const int bx = j * op.b_split_stride + kx;
+                if (t.b_z >= 0) tma_load_3d(sb, &mapB, &full[s], bx, t.n0, t.b_z);
+                else tma_load_2d(sb, &mapB, &full[s], bx, t.n0);
+            }
+        }
+        // loads still in flight (only after a timeout) land before exit
+        for (int j = (it > kStages ? it - kStages : 0); j < it; ++j)
+            mbar_wait(&full[j % kStages], (j / kStages) & 1);
+    } else if (warp == 1 && lane == 0) {
+        // MMA issuer
+        const uint32_t idesc = idesc_bf16_f32(kTileM, n_tile);
+        uint32_t started = 0;
+        for (int it = 0; it < t.nkb; ++it) {
+            const int s = it % kStages;
+            if (!mbar_wait(&full[s], (it / kStages) & 1)) {
+                atomicOr(op.err, kErrTimeout);
+                break;
+            }
+            tc_fence_after();
+            const uint32_t sa = smem_u32(ring + (size_t)s * stage_bytes);
+#pragma unroll
+            for (int k16 = 0; k16 < kBlockK / 16; ++k16) {
+                const int kg = (t.kb0 + it) * kBlockK + k16 * 16;
+                int acc = kg / op.acc_chunk;
+                if (acc >= op.n_acc) acc = op.n_acc - 1;
+                const uint32_t dt = tmem + (uint32_t)(acc * n_tile);
+                const uint64_t ad = desc_k_sw128(sa + k16 * 32);
+#pragma unroll
+                for (int j = 0; j < NSPLIT; ++j) {
+                    const uint64_t bd = desc_k_sw128(sa + kTileABytes + j * b_bytes + k16 * 32);
+                    mma_bf16(dt, ad, bd, idesc, (started >> acc) & 1u);
+                    started |= 1u << acc;
+                }
+            }
+            mma_commit(&empty[s]);   // frees the stage once these MMAs are done
+        }
+        mma_commit(&accbar);
+    }
+    __syncwarp();
+    if (!mbar_wait(&accbar, 0)) atomicOr(op.err, kErrTimeout);
+    tc_fence_after();
+
+    // epilogue: thread = tile row (TMEM lane), 16 columns at a time
+    const int row = warp * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+    for (int c = 0; c < n_tile; c += 16) {
+        float v[kMaxAcc][16];
+#pragma unroll
+        for (int a = 0; a < kMaxAcc; ++a)
+            if (a < op.n_acc) tmem_ld16(lane_base + (uint32_t)(a * n_tile + c), v[a]);
+        op.store(t, row, c, v);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, ncols);
+}
+
+// ---- S1: query projection, split over D_i --------------------------------
+struct QueryOp {
+    int n_tile, stages, n_acc, acc_chunk, b_split_stride;
+    int *err;
+    int B, HD, A, a, splits, kb_total;
+    float *q_part;   // [splits][A][B][HD]
+    __device__ Tile tile() const {
+        Tile t;
+        t.m0 = blockIdx.x * kTileM;
+        t.n0 = blockIdx.y * n_tile;
+        t.a_sel = 0;
+        t.a_z = -1;
+        t.b_z = -1;
+        const int split = blockIdx.z;
+        const int per = (kb_total + splits - 1) / splits;
+        t.kb0 = split * per;
+        t.nkb = max(0, min(kb_total, t.kb0 + per) - t.kb0);
+        return t;
+    }
+    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
+        const int m = t.m0 + row;
+        if (m >= HD) return;
+        const int split = blockIdx.z;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int n = t.n0 + c + j;
+            if (n < B) q_part[(((int64_t)split * A + a) * B + n) * HD + m] = t.nkb ? v[0][j] : 0.f;
+        }
+    }
+};
+
+// ---- S2: row/column scores, one accumulator per rank chunk ------------------
+struct ScoreOp {
+    int n_tile, stages, n_acc, acc_chunk, b_split_stride;
+    int *err;
+    int B, H, K, r, A, kb_total;
+    float *s;   // [B][H][2][K][r]
+    __device__ Tile tile() const {
+        Tile t;
+        const int h = blockIdx.z >> 1, axis = blockIdx.z & 1;
+        t.m0 = blockIdx.x * kTileM;
+        t.n0 = blockIdx.y * n_tile;
+        t.a_sel = axis;
+        t.a_z = h;
+        t.b_z = (A == 2 && axis == 1 ? H : 0) + h;
+        t.kb0 = 0;
+        t.nkb = kb_total;
+        return t;
+    }
+    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
+        const int i = t.m0 + row;
+        if (i >= K) return;
+        const int h = blockIdx.z >> 1, axis = blockIdx.z & 1;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int n = t.n0 + c + j;
+            if (n >= B) break;
+            float *dst = s + ((((int64_t)n * H + h) * 2 + axis) * K + i) * r;
+            if (r == 2) {
+                *reinterpret_cast<float2 *>(dst) = make_float2(v[0][j], v[1][j]);
+            } else {
+                for (int a = 0; a < r; ++a) dst[a] = v[a][j];
+            }
+        }
+    }
+};
+
+// ---- S9: IVE projection --------------------------------------------------
+struct ProjOp {
+    int n_tile, stages, n_acc, acc_chunk, b_split_stride;
+    int *err;
+    int B, d_out, kb_total;
+    __nv_bfloat16 *out;   // [B][d_out]
+    __device__ Tile tile() const {
+        Tile t;
+        t.m0 = blockIdx.x * kTileM;
+        t.n0 = blockIdx.y * n_tile;
+        t.a_sel = 0;
+        t.a_z = -1;
+        t.b_z = -1;
+        t.kb0 = 0;
+        t.nkb = kb_total;
+        return t;
+    }
+    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
+        const int o = t.m0 + row;
+        if (o >= d_out) return;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int n = t.n0 + c + j;
+            if (n < B) out[(int64_t)n * d_out + o] = __float2bfloat16_rn(v[0][j]);
+        }
+    }
+};
+
+// ---- q = sum of split partials, then the three-term bf16 split -------------
+// qs layout: [A*H][Bmax][3][D_k] (token rows of 3*D_k), the B operand of S2.
+__global__ void qsplit_kernel(Dims d, const float *__restrict__ q_part,
+                              __nv_bfloat16 *__restrict__ qs, int splits, int Bmax) {
+    const int HD = d.H * d.d_k;
+    const int64_t total = (int64_t)d.A * d.B * HD;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int o = (int)(e % HD);
+        const int64_t ab = e / HD;
+        const int b = (int)(ab % d.B), a = (int)(ab / d.B);
+        float q = 0.f;
+        for (int s = 0; s < splits; ++s) q += q_part[(((int64_t)s * d.A + a) * d.B + b) * HD + o];
+        const __nv_bfloat16 q1 = __float2bfloat16_rn(q);
+        const float r1 = q - __bfloat162float(q1);
+        const __nv_bfloat16 q2 = __float2bfloat16_rn(r1);
+        const float r2 = r1 - __bfloat162float(q2);
+        const __nv_bfloat16 q3 = __float2bfloat16_rn(r2);
+        const int h = o / d.d_k, c = o % d.d_k;
+        __nv_bfloat16 *dst = qs + (((int64_t)(a * d.H + h) * Bmax + b) * 3) * d.d_k + c;
+        dst[0] = q1;
+        dst[d.d_k] = q2;
+        dst[2 * d.d_k] = q3;
+    }
+}
+
+// dst[c][r] = src[r][c] for a rows x cols bf16 matrix (32 x 32 tiles)
+__global__ void transpose_kernel(const __nv_bfloat16 *__restrict__ src,
+                                 __nv_bfloat16 *__restrict__ dst, int rows, int cols) {
+    __shared__ __nv_bfloat16 tile[32][33];
+    const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int r = r0 + i, c = c0 + threadIdx.x;
+        if (r < rows && c < cols) tile[i][threadIdx.x] = src[(int64_t)r * cols + c];
+    }
+    __syncthreads();
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int c = c0 + i, r = r0 + threadIdx.x;
+        if (r < rows && c < cols) dst[(int64_t)c * rows + r] = tile[threadIdx.x][i];
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+}  // namespace
+
+cudaError_t launch_transpose_bf16(const void *src, void *dst, int rows, int cols,
+                                  cudaStream_t st) {
+    dim3 grid((cols + 31) / 32, (rows + 31) / 32);
+    transpose_kernel<<<grid, dim3(32, 8), 0, st>>>(static_cast<const __nv_bfloat16 *>(src),
+                                                   static_cast<__nv_bfloat16 *>(dst), rows, cols);
+    return cudaGetLastError();
+}
+
+// ---- host side ---------------------------------------------------------------
+
+bool tc_init() {
+    if (g_encode) return true;
+    cudaDriverEntryPointQueryResult q;
+    void *fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn) {
+        cudaGetLastError();
+        return false;
+    }
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    return true;
+}
+
+// bf16 tensor [outer][mid][inner] with inner contiguous, as a rank-2 map
+// (inner, mid) or rank-3 map (inner, mid, outer); box = 64 x box_rows (x 1),
+// 128-byte swizzle, zero fill out of bounds.
+bool tc_encode(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid,
+               uint64_t outer, uint32_t box_rows, int rank) {
+    if (!g_encode || ((uintptr_t)base & 15) || (inner * 2) % 16) return false;
+    cuuint64_t dims[3] = {inner, mid, outer};
+    cuuint64_t strides[2] = {inner * 2, inner * 2 * mid};
+    cuuint32_t box[3] = {(cuuint32_t)kBlockK, box_rows, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank,
+                          const_cast<void *>(base), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+int tc_n_tile(int B, int n_acc) {
+    int cap = 256 / n_acc;          // n_acc * N <= 512 TMEM columns, N <= 256
+    if (cap > 256) cap = 256;
+    int n = ((B + 15) / 16) * 16;
+    return n < cap ? n : cap;
+}
+
+template <int NSPLIT, class Op>
+static cudaError_t launch_gemm(dim3 grid, const CUtensorMap &a0, const CUtensorMap &a1,
+                               const CUtensorMap &b, Op op, int nkb, cudaStream_t st) {
+    op.stages = stages_for(NSPLIT, op.n_tile, nkb);
+    const size_t smem = 1024 + (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile);
+    tc_gemm_kernel<NSPLIT, Op><<<grid, kThreads, smem, st>>>(a0, a1, b, op);
+    return cudaGetLastError();
+}
+
+template <int NSPLIT, class Op> static cudaError_t allow_smem() {
+    return cudaFuncSetAttribute(tc_gemm_kernel<NSPLIT, Op>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBudget);
+}
+
+cudaError_t configure_tc() {
+    cudaError_t e = allow_smem<1, QueryOp>();
+    if (e == cudaSuccess) e = allow_smem<3, ScoreOp>();
+    if (e == cudaSuccess) e = allow_smem<1, ProjOp>();
+    return e;
+}
+
+cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int splits,
+                            cudaStream_t st) {
+    const int HD = d.H * d.d_k;
+    const int n_tile = tc_n_tile(d.B, 1);
+    const int kb_total = (d.d_in + kBlockK - 1) / kBlockK;
+    for (int a = 0; a < d.A; ++a) {
+        QueryOp op;
+        op.n_tile = n_tile;
+        op.n_acc = 1;
+        op.acc_chunk = 1 << 30;
+        op.b_split_stride = 0;
+        op.err = p.err;
+        op.B = d.B;
+        op.HD = HD;
+        op.A = d.A;
+        op.a = a;
+        op.splits = splits;
+        op.kb_total = kb_total;
+        op.q_part = p.q_part;
+        dim3 grid((HD + kTileM - 1) / kTileM, (d.B + n_tile - 1) / n_tile, splits);
+        const int per = (kb_total + splits - 1) / splits;
+        cudaError_t e =
+            launch_gemm<1>(grid, a == 0 ? mp.w_q : mp.w_q_col, mp.w_q, mp.x, op, per, st);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+cudaError_t launch_qsplit(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, int splits, int Bmax,
+                          cudaStream_t st) {
+    const int64_t total = (int64_t)d.A * d.B * d.H * d.d_k;
+    int blocks = (int)((total + 255) / 256);
+    if (blocks > 2048) blocks = 2048;
+    qsplit_kernel<<<blocks, 256, 0, st>>>(d, p.q_part, qs, splits, Bmax);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
+    ScoreOp op;
+    op.n_tile = tc_n_tile(d.B, d.r);
+    op.n_acc = d.r;
+    op.acc_chunk = d.dk;
+    op.b_split_stride = d.d_k;
+    op.err = p.err;
+    op.B = d.B;
+    op.H = d.H;
+    op.K = d.K;
+    op.r = d.r;
+    op.A = d.A;
+    op.kb_total = (d.d_k + kBlockK - 1) / kBlockK;
+    op.s = p.s;
+    dim3 grid((d.K + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 2 * d.H);
+    return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs, op, op.kb_total, st);
+}
+
+cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
+    ProjOp op;
+    op.n_tile = tc_n_tile(d.B, 1);
+    op.n_acc = 1;
+    op.acc_chunk = 1 << 30;
+    op.b_split_stride = 0;
+    op.err = p.err;
+    op.B = d.B;
+    op.d_out = d.d_out;
+    op.kb_total = (d.E * d.d_v + kBlockK - 1) / kBlockK;
+    op.out = static_cast<__nv_bfloat16 *>(p.out);
+    dim3 grid((d.d_out + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 1);
+    return launch_gemm<1>(grid, mp.w_pt, mp.w_pt, mp.acc, op, op.kb_total, st);
+}
+
+}  // namespace um
