@@ -60,7 +60,7 @@ typedef struct ultramem_config {
     int32_t d_k;         /* D_k, query/key width of one head; d_k % rank == 0        */
     int32_t heads;       /* H, key sets that read the shared table (Sec. 3.1)        */
     int32_t rank;        /* r, Tucker rank (Eq. 5), 1..8                              */
-    int32_t n;           /* physical grid side, N = n*n rows; K = sqrt(E)*n <= 40960  */
+    int32_t n;           /* physical grid side, N = n*n rows; K = sqrt(E)*n <= 20480  */
     int32_t expand_e;    /* E, virtual expansion, a perfect square 1..16 (Eq. 13)    */
     int32_t d_v;         /* D_v, physical value width, multiple of 8                  */
     int32_t d_out;       /* D'_v, output width; == d_v when has_proj == 0             */

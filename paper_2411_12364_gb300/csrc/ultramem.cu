@@ -19,8 +19,8 @@ constexpr int kStages = 5;
 const char *const kStageNames[kStages] = {"query", "score", "select", "gather", "project"};
 
 struct Workspace {
-    float *q_part = nullptr, *s = nullptr, *sel_w = nullptr, *acc = nullptr,
-          *proj_part = nullptr;
+    float *q_part = nullptr, *sel_w = nullptr, *acc = nullptr, *proj_part = nullptr;
+    uint32_t *akey = nullptr;
     int32_t *sel_row = nullptr, *sel_p = nullptr;
     float *core = nullptr, *u = nullptr, *t = nullptr;
     int *err = nullptr;
@@ -102,7 +102,7 @@ ultramem_status validate(const ultramem_config *c, const ultramem_weights *w) {
     int s = (int)lround(sqrt((double)c->expand_e));
     if (c->expand_e < 1 || c->expand_e > 16 || s * s != c->expand_e) return ULTRAMEM_EINVAL;
     int64_t K = keys_per_axis(*c);
-    if (K > 40960) return ULTRAMEM_EINVAL;
+    if (K > 20480) return ULTRAMEM_EINVAL;
     uint64_t M = (uint64_t)c->expand_e * (uint64_t)c->n * (uint64_t)c->n;
     if (M >= (1ull << 32)) return ULTRAMEM_EINVAL;
     if (c->topk < 1 || c->topk > 128 || c->topk > K) return ULTRAMEM_EINVAL;
@@ -211,7 +211,7 @@ template <typename T> cudaError_t dalloc(T **p, size_t n) {
 }
 
 void free_workspace(Workspace &ws) {
-    void *ptrs[] = {ws.q_part, ws.s,    ws.sel_w,   ws.acc,       ws.proj_part,
+    void *ptrs[] = {ws.q_part, ws.akey, ws.sel_w,   ws.acc,       ws.proj_part,
                     ws.sel_row, ws.sel_p, ws.core,   ws.u,         ws.t,
                     ws.err,    ws.x_stage, ws.out_stage, ws.qs,     ws.acc_bf,
                     ws.w_pt};
@@ -234,7 +234,7 @@ Ptrs make_ptrs(ultramem_layer *L) {
     p.u = L->ws.u;
     p.t = L->ws.t;
     p.q_part = L->ws.q_part;
-    p.s = L->ws.s;
+    p.akey = L->ws.akey;
     p.sel_w = L->ws.sel_w;
     p.acc = L->ws.acc;
     p.proj_part = L->ws.proj_part;
@@ -449,7 +449,7 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     cudaError_t e = cudaSuccess;
     const size_t hm = Bm * H * cfg->topm;
     if (e == cudaSuccess) e = dalloc(&ws.q_part, qmax * d.A * HD);
-    if (e == cudaSuccess) e = dalloc(&ws.s, Bm * H * 2 * (size_t)d.K * r);
+    if (e == cudaSuccess) e = dalloc(&ws.akey, Bm * H * 2 * (size_t)d.K);
     if (e == cudaSuccess) e = dalloc(&ws.sel_w, hm);
     if (e == cudaSuccess) e = dalloc(&ws.sel_row, hm);
     if (e == cudaSuccess) e = dalloc(&ws.sel_p, hm);

@@ -1,11 +1,14 @@
 // um_gather.cu -- S8 (weighted gather-sum grouped by virtual block, Eq. 15's
-// inner V^T s^_p) and S9 (the IVE projection o = sum_p W_p^T acc_p).
+// inner V^T s^_p) and S9 on CUDA cores (the IVE projection o = sum_p W_p^T
+// acc_p, used for fp32 storage).
 //
-// Gather: one CTA per token.  Each warp takes a run of selected slots, issues
-// the 16-byte loads of all its rows before using any (memory-level
-// parallelism on the random rows of a multi-GB table), and accumulates
-// w * V[row] into its own fp32 copy of acc[E][D_v] in shared memory; the
-// warps' copies are summed at the end.  Row loads bypass L1 (read-only path).
+// Gather: one CTA per token.  Each warp takes a run of selected slots and
+// issues the 16-byte loads of all its rows before using any (memory-level
+// parallelism on random rows of a multi-GB table); a lane owns 16 bytes of
+// every row.  With E <= 4 blocks each lane keeps its accumulators acc[p][..]
+// in registers (the row's block p selects which, branch-free); larger E
+// accumulate into a per-warp copy in shared memory.  The warps' partial sums
+// are added at the end.  Row loads bypass L1 (read-only path).
 #include "um_internal.cuh"
 
 namespace um {
@@ -40,6 +43,94 @@ __device__ __forceinline__ void fma_vec(float *dst, uint4 v, float w, float) {
     dst[3] = fmaf(w, __uint_as_float(v.w), dst[3]);
 }
 
+template <typename T>
+__device__ __forceinline__ void unpack(uint4 v, float (&f)[16 / sizeof(T)]);
+template <>
+__device__ __forceinline__ void unpack<__nv_bfloat16>(uint4 v, float (&f)[8]) {
+    const uint32_t u[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        f[2 * q] = __uint_as_float(u[q] << 16);
+        f[2 * q + 1] = __uint_as_float(u[q] & 0xffff0000u);
+    }
+}
+template <>
+__device__ __forceinline__ void unpack<float>(uint4 v, float (&f)[4]) {
+    f[0] = __uint_as_float(v.x);
+    f[1] = __uint_as_float(v.y);
+    f[2] = __uint_as_float(v.z);
+    f[3] = __uint_as_float(v.w);
+}
+
+// Register-accumulating gather for E <= EMAX blocks and rows of at most
+// 32 vectors (one 16-byte vector per lane).
+template <typename T, int EMAX>
+__global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
+    extern __shared__ __align__(16) float red[];   // [kWarps][E][D_v]
+    constexpr int EPV = 16 / sizeof(T);
+    const int b = blockIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int EDv = d.E * d.d_v;
+    const int VPR = d.d_v / EPV;          // vectors per row, <= 32 here
+    const bool active = lane < VPR;
+    const int hm = d.H * d.m;
+    const int64_t base = (int64_t)b * hm;
+    const T *V = static_cast<const T *>(p.values);
+    float acc[EMAX][EPV];
+#pragma unroll
+    for (int q = 0; q < EMAX; ++q)
+#pragma unroll
+        for (int c = 0; c < EPV; ++c) acc[q][c] = 0.f;
+
+    for (int e0 = warp * kUnroll; e0 < hm; e0 += kWarps * kUnroll) {
+        uint4 val[kUnroll];
+        int blk[kUnroll];
+        float w[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const int e = e0 + u;
+            const bool ok = e < hm;
+            const int row = ok ? p.sel_row[base + e] : 0;
+            blk[u] = ok ? p.sel_p[base + e] : -1;
+            w[u] = ok ? p.sel_w[base + e] : 0.f;
+            val[u] = (ok && active) ? ld_stream(V + (int64_t)row * d.d_v + lane * EPV)
+                                    : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            float f[EPV];
+            unpack<T>(val[u], f);
+#pragma unroll
+            for (int q = 0; q < EMAX; ++q) {
+                const float wq = blk[u] == q ? w[u] : 0.f;   // branch-free block select
+#pragma unroll
+                for (int c = 0; c < EPV; ++c) acc[q][c] = fmaf(wq, f[c], acc[q][c]);
+            }
+        }
+    }
+    // sum the warps' partial accumulators
+    if (active)
+#pragma unroll
+        for (int q = 0; q < EMAX; ++q)
+            if (q < d.E)
+#pragma unroll
+                for (int c = 0; c < EPV; ++c)
+                    red[(size_t)warp * EDv + q * d.d_v + lane * EPV + c] = acc[q][c];
+    __syncthreads();
+    for (int i = threadIdx.x; i < EDv; i += kThreads) {
+        float s = 0.f;
+#pragma unroll
+        for (int wv = 0; wv < kWarps; ++wv) s += red[(size_t)wv * EDv + i];
+        if (p.acc_bf)
+            p.acc_bf[(int64_t)b * EDv + i] = __float2bfloat16_rn(s);
+        else if (d.has_proj)
+            p.acc[(int64_t)b * EDv + i] = s;
+        else
+            static_cast<T *>(p.out)[(int64_t)b * d.d_v + i] = from_f<T>(s);
+    }
+}
+
+// Shared-memory-accumulating gather for any E and row width.
 template <typename T>
 __global__ void __launch_bounds__(kThreads) gather_kernel(Dims d, Ptrs p) {
     extern __shared__ __align__(16) float acc_w[];   // [kWarps][E][D_v]
@@ -150,21 +241,38 @@ __global__ void proj_reduce_kernel(Dims d, Ptrs p) {
 
 size_t gather_smem_bytes(const Dims &d) { return sizeof(float) * kWarps * d.E * d.d_v; }
 
+template <typename K> static cudaError_t allow(K kern, size_t bytes) {
+    return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
 cudaError_t configure_gather(const Dims &d) {
-    cudaError_t e = cudaFuncSetAttribute(gather_kernel<float>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)gather_smem_bytes(d));
-    if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(gather_kernel<__nv_bfloat16>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)gather_smem_bytes(d));
+    const size_t bytes = gather_smem_bytes(d);
+    cudaError_t e = allow(gather_kernel<float>, bytes);
+    if (e == cudaSuccess) e = allow(gather_kernel<__nv_bfloat16>, bytes);
+    if (e == cudaSuccess) e = allow(gather_reg_kernel<float, 1>, bytes);
+    if (e == cudaSuccess) e = allow(gather_reg_kernel<float, 4>, bytes);
+    if (e == cudaSuccess) e = allow(gather_reg_kernel<__nv_bfloat16, 1>, bytes);
+    if (e == cudaSuccess) e = allow(gather_reg_kernel<__nv_bfloat16, 4>, bytes);
+    return e;
+}
+
+template <typename T>
+static void launch_gather_t(const Dims &d, const Ptrs &p, cudaStream_t st) {
+    const size_t bytes = gather_smem_bytes(d);
+    const bool fits_lanes = d.d_v / (16 / (int)sizeof(T)) <= 32;
+    if (fits_lanes && d.E == 1)
+        gather_reg_kernel<T, 1><<<d.B, kThreads, bytes, st>>>(d, p);
+    else if (fits_lanes && d.E <= 4)
+        gather_reg_kernel<T, 4><<<d.B, kThreads, bytes, st>>>(d, p);
+    else
+        gather_kernel<T><<<d.B, kThreads, bytes, st>>>(d, p);
 }
 
 cudaError_t launch_gather(const Dims &d, const Ptrs &p, cudaStream_t st) {
     if (d.dtype == ULTRAMEM_BF16)
-        gather_kernel<__nv_bfloat16><<<d.B, kThreads, gather_smem_bytes(d), st>>>(d, p);
+        launch_gather_t<__nv_bfloat16>(d, p, st);
     else
-        gather_kernel<float><<<d.B, kThreads, gather_smem_bytes(d), st>>>(d, p);
+        launch_gather_t<float>(d, p, st);
     return cudaGetLastError();
 }
 

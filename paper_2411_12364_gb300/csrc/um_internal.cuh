@@ -3,7 +3,8 @@
 // Every kernel receives the layer's dimensions (Dims) and the device pointers
 // it touches (Ptrs) by value.  Workspace layouts (all fp32 unless noted):
 //   q_part   [q_splits][A][B][H*D_k]   split-K partial sums of q = W_q x
-//   s        [B][H][2][K][r]           S_row (axis 0) and S_col (axis 1), Eq. 4
+//   akey     [B][H][2][K] uint32       order-preserving key of the rank-1 score
+//                                      u^T S_row (axis 0) / t^T S_col (axis 1), Eq. 6
 //   sel_row  [B][H][m] int32           physical row of each selected slot
 //   sel_p    [B][H][m] int32           virtual block p of each selected slot
 //   sel_w    [B][H][m]                 weight of each selected slot
@@ -40,7 +41,8 @@ struct Ptrs {
     const void *x, *w_q, *w_q_col, *k_row, *k_col, *values, *w_proj;
     const uint32_t *perm;
     const float *core, *u, *t;   // library copies: [H][r][r], [H][r], [H][r]
-    float *q_part, *s, *sel_w, *acc, *proj_part;
+    float *q_part, *sel_w, *acc, *proj_part;
+    uint32_t *akey;
     int32_t *sel_row, *sel_p;
     void *out;
     int64_t *idx_out;
@@ -94,6 +96,16 @@ template <typename T> __device__ __forceinline__ T from_f(float v);
 template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
 template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) {
     return __float2bfloat16_rn(v);
+}
+
+// fp32 -> uint32 whose unsigned order is the float order (-0 folded into +0).
+__device__ __forceinline__ uint32_t f2ord(float f) {
+    uint32_t u = __float_as_uint(f + 0.0f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float ord2f(uint32_t o) {
+    uint32_t u = (o & 0x80000000u) ? (o & 0x7fffffffu) : ~o;
+    return __uint_as_float(u);
 }
 
 // The Eq. 14 shuffle: explicit table or the seeded affine bijection.

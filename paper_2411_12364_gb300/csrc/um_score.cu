@@ -1,7 +1,7 @@
-// um_score.cu -- query projection (S1) and row/column scores (S2, Eq. 4) on
-// CUDA cores in fp32.  Both are small contractions at decode batch sizes; the
-// query projection is split over D_i so that enough CTAs stream W_q, and the
-// partial sums are added when the score kernel loads the query.
+// um_score.cu -- query projection (S1) and row/column scores (S2-S3, Eq. 4
+// and 6) on CUDA cores in fp32, the path of fp32 storage.  The query
+// projection is split over D_i so that enough CTAs stream W_q; the partial
+// sums are added when the score kernel loads the query.
 #include "um_internal.cuh"
 
 namespace um {
@@ -55,21 +55,26 @@ __global__ void __launch_bounds__(kThreads) query_kernel(Dims d, Ptrs p) {
         }
 }
 
-// s[b][h][axis][i][alpha] = sum_{c < dk} key[h][i][alpha*dk + c] * q[b][h][alpha*dk + c]
-// Tile: 64 keys x 32 tokens; each thread owns 4 keys x 2 tokens, one rank
-// chunk alpha at a time (Eq. 4 with the r x K x (D_k/r) reshape).
+// For each rank chunk alpha, S_alpha[b][i] = sum_{c < dk} key[h][i][alpha*dk + c]
+// * q[b][h][alpha*dk + c] (Eq. 4 with the r x K x (D_k/r) reshape); the chunk
+// scores are folded into the rank-1 score a = sum_alpha coef[alpha] S_alpha
+// (coef = u for row keys, t for column keys, Eq. 6-7) and its
+// order-preserving key is stored: akey[b][h][axis][i].
+// Tile: 64 keys x 32 tokens; each thread owns 4 keys x 2 tokens.
 template <typename T>
 __global__ void __launch_bounds__(kThreads) score_kernel(Dims d, Ptrs p) {
     const int h = blockIdx.z >> 1, axis = blockIdx.z & 1;
     const int a = (axis == 1 && d.A == 2) ? 1 : 0;
     const T *keys = static_cast<const T *>(axis == 0 ? p.k_row : p.k_col) +
                     (int64_t)h * d.K * d.d_k;
+    const float *coef = (axis == 0 ? p.u : p.t) + (int64_t)h * d.r;
     const int i0 = blockIdx.x * 64, b0 = blockIdx.y * 32;
     const int HD = d.H * d.d_k;
 
     __shared__ float ks[32][65];  // [c][key]
     __shared__ float qs[32][33];  // [c][token]
     const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+    float folded[4][2] = {};
     for (int al = 0; al < d.r; ++al) {
         float acc[4][2] = {};
         for (int c0 = 0; c0 < d.dk; c0 += 32) {
@@ -101,13 +106,17 @@ __global__ void __launch_bounds__(kThreads) score_kernel(Dims d, Ptrs p) {
             }
             __syncthreads();
         }
+        const float cf = coef[al];
         for (int j = 0; j < 4; ++j)
-            for (int t = 0; t < 2; ++t) {
-                int i = i0 + tx * 4 + j, b = b0 + ty * 2 + t;
-                if (i < d.K && b < d.B)
-                    p.s[((((int64_t)b * d.H + h) * 2 + axis) * d.K + i) * d.r + al] = acc[j][t];
-            }
+            for (int t = 0; t < 2; ++t)
+                folded[j][t] = al == 0 ? cf * acc[j][t] : fmaf(cf, acc[j][t], folded[j][t]);
     }
+    for (int j = 0; j < 4; ++j)
+        for (int t = 0; t < 2; ++t) {
+            int i = i0 + tx * 4 + j, b = b0 + ty * 2 + t;
+            if (i < d.K && b < d.B)
+                p.akey[(((int64_t)b * d.H + h) * 2 + axis) * d.K + i] = f2ord(folded[j][t]);
+        }
 }
 
 }  // namespace

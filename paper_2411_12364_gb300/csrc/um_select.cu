@@ -1,19 +1,26 @@
-// um_select.cu -- S3..S7 for one (token, head) per CTA, in shared memory:
-//   rank-1 scores a = u^T S_row, b = t^T S_col          (Eq. 6-7)
-//   top-k of each axis                                  (Eq. 8-9)
-//   exact Tucker score g on the k*k survivors           (Eq. 10)
+// um_select.cu -- S4..S7 for one (token, head) per CTA:
+//   top-k of each axis on the rank-1 score keys         (Eq. 8-9)
+//   exact chunk scores S_alpha of the 2k survivors      (Eq. 4)
+//   exact Tucker score g on the k*k survivor pairs      (Eq. 10)
 //   top-m of g, ordered by (score desc, v asc)          (Eq. 10)
 //   weights (raw scores, or PKM's softmax), shuffle     (Trick 1, Eq. 3, Eq. 14)
-// No K*K grid is ever formed.  Scores are compared as order-preserving 32-bit
-// keys of their fp32 values; ties go to the smaller index.
+// No K*K grid is ever formed.  The scoring kernel leaves, per key, the
+// order-preserving 32-bit key of its fp32 rank-1 score; the exact chunk
+// scores of the k survivors of each axis are recomputed here from q and the
+// key rows.  Ties go to the smaller index.
 //
-// Top-k of n keys (topk_positions): each thread takes the maximum of its
-// strided share of the keys; tau = the kk-th largest of those 256 maxima is
-// a lower bound of the kk-th largest key for any input (kk threads each own
-// a key >= tau).  Keys > tau are gathered, plus -- only when fewer than kk
-// keys exceed tau -- the first ties at tau in position order; these
-// candidates (typically one to three times kk) are ranked exactly.  If more
-// than kCap keys exceed tau, a radix select over all n keys is used instead.
+// Top-k of n keys, in two stages.  Candidates (whole block): each thread
+// takes the maximum of its strided share of the keys; each warp takes the
+// j-th largest of its 32 lane maxima (j = ceil(k / 8), a register bitonic
+// sort) and tau is the smallest of the 8 warp values.  Every warp owns at
+// least j keys >= tau, so at least k keys are >= tau whatever the input:
+// every key of the top k is >= tau.  Each warp appends its keys >= tau to its
+// own region (ballot, no atomics); when more than 2k survive, the same bound
+// is taken again over the survivors.  Order (one warp): the candidates, as
+// 64-bit composites (key, ~position) whose descending order is key
+// descending then position ascending, are sorted in registers by a bitonic
+// network (shuffles across lanes, swaps across registers).  Rare inputs with
+// too many candidates (heavy ties) take an exact radix select instead.
 #include "um_internal.cuh"
 
 namespace um {
@@ -21,32 +28,63 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kCap = 2048;       // candidate capacity of the threshold path
-constexpr int kMaxOut = 1024;    // largest k or m
+constexpr int kRegion = 128;               // candidates per warp region
+constexpr int kCap = kWarps * kRegion;     // 1024 per selection
+constexpr int kMaxK = 128;
+constexpr int kMaxM = 1024;
+constexpr unsigned kFull = 0xffffffffu;
+
+typedef unsigned long long u64;
 
 struct SelShared {
+    u64 cand[2][kCap];      // per selection: kWarps regions of kRegion (or one flat list)
+    u64 fwin[kMaxM];        // final winners by rank
+    int wcnt[2][kWarps];    // region fill counts
+    uint32_t vt[2][kWarps];
     int hist[256];
     int warp_tot[kWarps];
-    int digit;
-    int remaining;
+    int digit, remaining;
     float scalar;
-    uint32_t vt[kThreads];
-    uint32_t cand_key[kCap];
-    int cand_pos[kCap];
-    uint32_t win_key[kMaxOut];
-    int win_pos[kMaxOut];
-    int n_gt;
-    uint32_t tau;
 };
 
-// fp32 -> uint32 whose unsigned order is the float order (-0 folded into +0).
-__device__ __forceinline__ uint32_t f2ord(float f) {
-    uint32_t u = __float_as_uint(f + 0.0f);
-    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+__device__ __forceinline__ u64 comp_of(uint32_t key, uint32_t pos) {
+    return ((u64)key << 32) | (u64)(~pos);
 }
-__device__ __forceinline__ float ord2f(uint32_t o) {
-    uint32_t u = (o & 0x80000000u) ? (o & 0x7fffffffu) : ~o;
-    return __uint_as_float(u);
+__device__ __forceinline__ uint32_t key_of(u64 c) { return (uint32_t)(c >> 32); }
+__device__ __forceinline__ uint32_t pos_of(u64 c) { return ~(uint32_t)c; }
+
+template <typename T>
+__device__ __forceinline__ void unpack16(uint4 v, float (&f)[16 / sizeof(T)]);
+template <>
+__device__ __forceinline__ void unpack16<__nv_bfloat16>(uint4 v, float (&f)[8]) {
+    const uint32_t u[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        f[2 * q] = __uint_as_float(u[q] << 16);
+        f[2 * q + 1] = __uint_as_float(u[q] & 0xffff0000u);
+    }
+}
+template <>
+__device__ __forceinline__ void unpack16<float>(uint4 v, float (&f)[4]) {
+    f[0] = __uint_as_float(v.x);
+    f[1] = __uint_as_float(v.y);
+    f[2] = __uint_as_float(v.z);
+    f[3] = __uint_as_float(v.w);
+}
+
+// j-th largest (1-based, j <= 32) of one value per lane: descending bitonic
+// sort across the warp.
+__device__ __forceinline__ uint32_t warp_jth_largest(uint32_t v, int j) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int blk = 2; blk <= 32; blk <<= 1)
+#pragma unroll
+        for (int st = blk >> 1; st > 0; st >>= 1) {
+            const uint32_t o = __shfl_xor_sync(kFull, v, st);
+            const bool keep_max = ((lane & st) == 0) == ((lane & blk) == 0);
+            v = keep_max ? max(v, o) : min(v, o);
+        }
+    return __shfl_sync(kFull, v, j - 1);
 }
 
 // Exclusive prefix sum of one int per thread over the block; also syncs.
@@ -55,7 +93,7 @@ __device__ int block_exclusive_scan(int v, SelShared &sh) {
     int incl = v;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
-        int y = __shfl_up_sync(0xffffffffu, incl, off);
+        int y = __shfl_up_sync(kFull, incl, off);
         if (lane >= off) incl += y;
     }
     if (lane == 31) sh.warp_tot[warp] = incl;
@@ -92,7 +130,7 @@ __device__ uint32_t select_kth_largest(const uint32_t *key, int n, int kk, SelSh
             int incl = s;
 #pragma unroll
             for (int off = 1; off < 32; off <<= 1) {
-                int y = __shfl_up_sync(0xffffffffu, incl, off);
+                int y = __shfl_up_sync(kFull, incl, off);
                 if (lane >= off) incl += y;
             }
             int before = incl - s;
@@ -118,117 +156,349 @@ __device__ uint32_t select_kth_largest(const uint32_t *key, int n, int kk, SelSh
     return prefix;
 }
 
-// Appends to sh.cand_*[base..] the first `need` positions (in position
-// order) with key == T, using contiguous per-thread ranges.
-__device__ void gather_ties_in_order(const uint32_t *key, int n, uint32_t T, int need, int base,
-                                     SelShared &sh) {
+// Exact fallback for selection s: a flat list of exactly kk candidates (every
+// key > T, then the first ties at T in position order) in cand[s], counted
+// in region 0.  Kept out of line: it only runs when a region overflows.
+__device__ __noinline__ void radix_fallback(const uint32_t *key, int n, int kk, int s,
+                                            SelShared &sh) {
+    int need_eq;
+    const uint32_t T = select_kth_largest(key, n, kk, sh, &need_eq);
+    const int n_gt = kk - need_eq;
     const int per = (n + kThreads - 1) / kThreads;
     const int beg = min(n, (int)threadIdx.x * per), end = min(n, beg + per);
-    int eq = 0;
-    for (int i = beg; i < end; ++i) eq += key[i] == T;
+    int gt = 0, eq = 0;
+    for (int i = beg; i < end; ++i) {
+        gt += key[i] > T;
+        eq += key[i] == T;
+    }
+    int o = block_exclusive_scan(gt, sh);
     int e = block_exclusive_scan(eq, sh);
-    for (int i = beg; i < end && e < need; ++i)
-        if (key[i] == T) {
-            sh.cand_key[base + e] = T;
-            sh.cand_pos[base + e] = i;
-            ++e;
-        }
+    for (int i = beg; i < end; ++i) {
+        const uint32_t v = key[i];
+        if (v > T) sh.cand[s][o++] = comp_of(v, (uint32_t)i);
+        else if (v == T && e < need_eq) sh.cand[s][n_gt + e++] = comp_of(v, (uint32_t)i);
+        else if (v == T) ++e;
+    }
+    if (threadIdx.x < kWarps) sh.wcnt[s][threadIdx.x] = threadIdx.x == 0 ? kk : 0;
     __syncthreads();
 }
 
-enum { kOrderByPosition = 0, kOrderByScore = 1 };
+// Tightens selection s: the same bound over the survivors of each region.
+__device__ void tighten(int s, int kk, SelShared &sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    constexpr int kPer = kRegion / 32;
+    const int mycnt = sh.wcnt[s][warp];
+    u64 mine[kPer];
+    uint32_t vm = 0;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+        const int f = lane + 32 * q;
+        mine[q] = f < mycnt ? sh.cand[s][warp * kRegion + f] : 0ull;
+        vm = max(vm, key_of(mine[q]));
+    }
+    const int j = (kk + kWarps - 1) / kWarps;
+    const uint32_t tw = j <= 32 ? warp_jth_largest(vm, j) : 0u;
+    if (lane == 0) sh.vt[s][warp] = tw;
+    __syncthreads();
+    uint32_t tau = sh.vt[s][0];
+    for (int w = 1; w < kWarps; ++w) tau = min(tau, sh.vt[s][w]);
+    u64 *region = sh.cand[s] + warp * kRegion;
+    int cnt = 0;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+        const bool pr = lane + 32 * q < mycnt && key_of(mine[q]) >= tau;
+        const unsigned bal = __ballot_sync(kFull, pr);
+        if (pr) region[cnt + __popc(bal & ((1u << lane) - 1u))] = mine[q];
+        cnt += __popc(bal);
+    }
+    __syncthreads();   // everyone has read wcnt before it changes
+    if (lane == 0) sh.wcnt[s][warp] = cnt;
+    __syncthreads();
+}
 
-// Positions of the kk largest keys of key[0..n) (ties: smaller position
-// first).  Leaves them in sh.win_pos / sh.win_key ordered by (key desc,
-// position asc); with kOrderByPosition, also writes the positions in
-// increasing order to out[0..kk).
-__device__ void topk_positions(const uint32_t *key, int n, int kk, int *out, int order,
-                               SelShared &sh) {
-    // tau = kk-th largest per-thread maximum (0 when fewer than kk threads own
-    // a key, which makes every key a candidate)
-    uint32_t vmax = 0;
-    for (int i = threadIdx.x; i < n; i += kThreads) vmax = max(vmax, key[i]);
-    sh.vt[threadIdx.x] = vmax;
-    if (threadIdx.x == 0) { sh.n_gt = 0; sh.tau = 0; }
-    __syncthreads();
-    {
-        int rank = 0;
-        for (int t = 0; t < kThreads; ++t) {
-            uint32_t o = sh.vt[t];
-            rank += (o > vmax) || (o == vmax && t < (int)threadIdx.x);
-        }
-        if (rank == kk - 1) sh.tau = vmax;
+// Candidates of ns (1 or 2) selections of n keys each, key[s][0..n), for
+// their top kk: thresholds, per-warp compaction, tightening or the radix
+// fallback.  Leaves them in sh.cand[s] (kWarps regions counted by
+// sh.wcnt[s][w], or a flat list in region 0 when sh.wcnt[s][0] > kRegion).
+// vmax[s] is this thread's maximum over its strided share of key[s].  Every
+// thread of the block calls it; it ends with a barrier.
+__device__ void select_candidates(const uint32_t *key0, const uint32_t *key1, int ns, int n,
+                                  int kk, uint32_t vmax0, uint32_t vmax1, SelShared &sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int j = (kk + kWarps - 1) / kWarps;
+#pragma unroll 1
+    for (int s = 0; s < ns; ++s) {
+        const uint32_t tw = j <= 32 ? warp_jth_largest(s ? vmax1 : vmax0, j) : 0u;
+        if (lane == 0) sh.vt[s][warp] = tw;
     }
     __syncthreads();
-    const uint32_t tau = sh.tau;
-    for (int i = threadIdx.x; i < n; i += kThreads) {
-        uint32_t v = key[i];
-        if (v > tau) {
-            int slot = atomicAdd(&sh.n_gt, 1);
-            if (slot < kCap) { sh.cand_key[slot] = v; sh.cand_pos[slot] = i; }
+    // each warp appends its keys >= tau to its own region
+#pragma unroll 1
+    for (int s = 0; s < ns; ++s) {
+        const uint32_t *key = s ? key1 : key0;
+        uint32_t tau = sh.vt[s][0];
+        for (int w = 1; w < kWarps; ++w) tau = min(tau, sh.vt[s][w]);
+        u64 *region = sh.cand[s] + warp * kRegion;
+        int cnt = 0;
+        for (int b0 = warp * 32; b0 < n; b0 += kThreads) {
+            const int i = b0 + lane;
+            const uint32_t v = i < n ? key[i] : 0u;
+            const bool pr = i < n && v >= tau;
+            const unsigned bal = __ballot_sync(kFull, pr);
+            const int slot = cnt + __popc(bal & ((1u << lane) - 1u));
+            if (pr && slot < kRegion) region[slot] = comp_of(v, (uint32_t)i);
+            cnt += __popc(bal);
         }
+        if (lane == 0) sh.wcnt[s][warp] = cnt;
     }
     __syncthreads();
-    int c = sh.n_gt;
-    if (c > kCap) {
-        int need_eq;
-        uint32_t T = select_kth_largest(key, n, kk, sh, &need_eq);
-        // every key > T, then the first need_eq ties at T
-        if (threadIdx.x == 0) sh.n_gt = 0;
+#pragma unroll 1
+    for (int s = 0; s < ns; ++s) {
+        int total = 0;
+        bool over = false;
+        for (int w = 0; w < kWarps; ++w) {
+            total += sh.wcnt[s][w];
+            over |= sh.wcnt[s][w] > kRegion;
+        }
         __syncthreads();
-        for (int i = threadIdx.x; i < n; i += kThreads) {
-            uint32_t v = key[i];
-            if (v > T) {
-                int slot = atomicAdd(&sh.n_gt, 1);
-                sh.cand_key[slot] = v;   // fewer than kk <= kCap of them
-                sh.cand_pos[slot] = i;
+        if (!over && total > 2 * kk) {
+            tighten(s, kk, sh);
+            total = 0;
+            for (int w = 0; w < kWarps; ++w) total += sh.wcnt[s][w];
+            __syncthreads();
+            over = total > 8 * 32 && kk <= 8 * 32;   // too many to sort in registers
+        }
+        if (over) radix_fallback(s ? key1 : key0, n, kk, s, sh);   // rare, exact
+    }
+}
+
+__device__ __forceinline__ int candidate_count(int s, const SelShared &sh) {
+    if (sh.wcnt[s][0] > kRegion) return sh.wcnt[s][0];   // flat list
+    int total = 0;
+    for (int w = 0; w < kWarps; ++w) total += sh.wcnt[s][w];
+    return total;
+}
+
+// Descending bitonic sort of 32*R values held as v[q] on lane l = element
+// q*32 + l: shuffles for strides below 32, register swaps above.
+template <int R>
+__device__ __forceinline__ void warp_sort_desc(u64 (&v)[R]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll 1
+    for (int size = 2; size <= 32 * R; size <<= 1) {
+#pragma unroll 1
+        for (int j = size >> 1; j > 0; j >>= 1) {
+            if (j < 32) {
+#pragma unroll
+                for (int q = 0; q < R; ++q) {
+                    const u64 o = __shfl_xor_sync(kFull, v[q], j);
+                    const int e = q * 32 + lane;
+                    const bool keep_max = ((e & j) == 0) == ((e & size) == 0);
+                    v[q] = keep_max ? (v[q] > o ? v[q] : o) : (v[q] < o ? v[q] : o);
+                }
+            } else {
+                const int jq = j >> 5;
+#pragma unroll
+                for (int m = 1; m < R; m <<= 1) {
+                    if (jq != m) continue;
+#pragma unroll
+                    for (int q = 0; q < R; ++q) {
+                        if (q & m) continue;
+                        const bool desc = ((q * 32 + lane) & size) == 0;
+                        const u64 a = v[q], b = v[q | m];
+                        const bool sw = desc ? (a < b) : (a > b);
+                        v[q] = sw ? b : a;
+                        v[q | m] = sw ? a : b;
+                    }
+                }
             }
         }
-        __syncthreads();
-        gather_ties_in_order(key, n, T, need_eq, kk - need_eq, sh);
-        c = kk;
-    } else if (c < kk) {
-        gather_ties_in_order(key, n, tau, kk - c, c, sh);
-        c = kk;
     }
-    // exact rank of every candidate by (key desc, position asc)
-    for (int e = threadIdx.x; e < c; e += kThreads) {
-        const uint32_t ke = sh.cand_key[e];
-        const int pe = sh.cand_pos[e];
-        int rank = 0;
-        for (int f = 0; f < c; ++f) {
-            uint32_t kf = sh.cand_key[f];
-            rank += (kf > ke) || (kf == ke && sh.cand_pos[f] < pe);
+}
+
+// One warp: the candidates of selection s (at most 32*R) sorted descending
+// into v; element e = q*32 + lane, zero-padded.
+template <int R>
+__device__ __forceinline__ void warp_gather_sorted(int s, const SelShared &sh, u64 (&v)[R]) {
+    const int lane = threadIdx.x & 31;
+    const bool flat = sh.wcnt[s][0] > kRegion;
+    int pref[kWarps + 1];
+    pref[0] = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w)
+        pref[w + 1] = pref[w] + (flat ? (w == 0 ? sh.wcnt[s][0] : 0) : sh.wcnt[s][w]);
+#pragma unroll
+    for (int q = 0; q < R; ++q) {
+        const int f = q * 32 + lane;
+        u64 val = 0ull;
+        if (f < pref[kWarps]) {
+            int w = 0, before = 0;
+#pragma unroll
+            for (int x = 1; x < kWarps; ++x)
+                if (f >= pref[x]) { w = x; before = pref[x]; }
+            val = sh.cand[s][(flat ? 0 : w * kRegion) + f - before];
         }
-        if (rank < kk) {
-            sh.win_key[rank] = ke;
-            sh.win_pos[rank] = pe;
+        v[q] = val;
+    }
+    warp_sort_desc<R>(v);
+}
+
+// Block-level exact ranks of selection s's candidates (any count up to
+// kCap) into win[rank] for rank < kk; each warp ranks its own region's
+// entries against all entries (a flat list is split w, w+8, ... over warps).
+__device__ void block_rank(int s, int kk, u64 *win, SelShared &sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const bool flat = sh.wcnt[s][0] > kRegion;
+    const int mine_n = flat ? (sh.wcnt[s][0] + kWarps - 1 - warp) / kWarps : sh.wcnt[s][warp];
+    for (int q = lane; q < mine_n; q += 32) {
+        const u64 ce = sh.cand[s][flat ? warp + q * kWarps : warp * kRegion + q];
+        int before = 0;
+#pragma unroll 1
+        for (int w = 0; w < (flat ? 1 : kWarps); ++w) {
+            const u64 *reg = sh.cand[s] + w * kRegion;
+            const int cw = sh.wcnt[s][w];
+            int f = 0;
+            for (; f + 4 <= cw; f += 4) {
+                const u64 a0 = reg[f], a1 = reg[f + 1], a2 = reg[f + 2], a3 = reg[f + 3];
+                before += (a0 > ce) + (a1 > ce) + (a2 > ce) + (a3 > ce);
+            }
+            for (; f < cw; ++f) before += reg[f] > ce;
         }
+        if (before < kk) win[before] = ce;
+    }
+}
+
+// Final top-m: candidates sorted by one warp when they fit its registers,
+// else ranked by the whole block; win[rank] for rank < kk.  Ends with a
+// barrier.
+__device__ void finish_top(int s, int kk, u64 *win, SelShared &sh) {
+    const int c = candidate_count(s, sh);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (c <= 256) {
+        if (warp == 0) {
+            if (c <= 64) {
+                u64 v[2];
+                warp_gather_sorted<2>(s, sh, v);
+#pragma unroll
+                for (int q = 0; q < 2; ++q)
+                    if (q * 32 + lane < kk) win[q * 32 + lane] = v[q];
+            } else if (c <= 128) {
+                u64 v[4];
+                warp_gather_sorted<4>(s, sh, v);
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    if (q * 32 + lane < kk) win[q * 32 + lane] = v[q];
+            } else {
+                u64 v[8];
+                warp_gather_sorted<8>(s, sh, v);
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    if (q * 32 + lane < kk) win[q * 32 + lane] = v[q];
+            }
+        }
+    } else {
+        block_rank(s, kk, win, sh);
     }
     __syncthreads();
-    if (order == kOrderByPosition) {
-        for (int e = threadIdx.x; e < kk; e += kThreads) {
-            const int pe = sh.win_pos[e];
-            int r = 0;
-            for (int f = 0; f < kk; ++f) r += sh.win_pos[f] < pe;
-            out[r] = pe;
+}
+
+// Exact chunk scores of one key row against q (fp32 in shared memory):
+// out[alpha] = sum_{c < dk} row[alpha*dk + c] * q[alpha*dk + c]  (Eq. 4).
+// 16-byte loads, up to 8 in flight, when the row and chunks are aligned.
+template <typename T>
+__device__ void row_scores(const T *row, const float *q, const Dims &d, float *out) {
+    constexpr int EPV = 16 / sizeof(T);
+    const int dk = d.dk;
+    const bool vec = d.d_k % EPV == 0 && dk % EPV == 0 && ((uintptr_t)row & 15) == 0;
+#pragma unroll 1
+    for (int al = 0; al < d.r; ++al) {
+        const int c0 = al * dk;
+        float acc = 0.f;
+        if (vec) {
+            const uint4 *rv = reinterpret_cast<const uint4 *>(row + c0);
+            const int nv = dk / EPV;
+#pragma unroll 1
+            for (int v0 = 0; v0 < nv; v0 += 8) {
+                uint4 buf[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u)
+                    buf[u] = v0 + u < nv ? rv[v0 + u] : make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    if (v0 + u >= nv) break;
+                    float f[EPV];
+                    unpack16<T>(buf[u], f);
+                    const float *qq = q + c0 + (v0 + u) * EPV;
+#pragma unroll
+                    for (int e = 0; e < EPV; ++e) acc = fmaf(f[e], qq[e], acc);
+                }
+            }
+        } else {
+#pragma unroll 4
+            for (int c = 0; c < dk; ++c) acc = fmaf(to_f(row[c0 + c]), q[c0 + c], acc);
         }
-        __syncthreads();
+        out[al] = acc;
     }
+}
+
+// One warp per axis: the top-k of the axis' candidates, in increasing key
+// index (so that enumerating I x J row-major is increasing v = i*K + j), and
+// each survivor's exact chunk scores, one lane per survivor.
+template <typename T, int R>
+__device__ void finish_axis(const Dims &d, const Ptrs &p, int h, int axis, const float *qv,
+                            const SelShared &sh, int *sel, float *S_out) {
+    const int lane = threadIdx.x & 31;
+    const int k = d.k;
+    u64 v[R];
+    warp_gather_sorted<R>(axis, sh, v);
+    u64 pk[R];   // winners keyed by ~position: descending order = increasing index
+#pragma unroll
+    for (int q = 0; q < R; ++q)
+        pk[q] = q * 32 + lane < k ? (u64)(uint32_t)(~pos_of(v[q])) : 0ull;
+    warp_sort_desc<R>(pk);
+    const T *keys = static_cast<const T *>(axis == 0 ? p.k_row : p.k_col);
+#pragma unroll
+    for (int q = 0; q < R; ++q) {
+        const int e = q * 32 + lane;
+        if (e < k) {
+            const uint32_t pos = ~(uint32_t)pk[q];
+            sel[e] = (int)pos;
+            row_scores<T>(keys + ((int64_t)h * d.K + pos) * d.d_k, qv + axis * d.d_k, d,
+                          S_out + e * d.r);
+        }
+    }
+}
+
+template <typename T>
+__device__ void finish_axes(const Dims &d, const Ptrs &p, int h, const float *qv,
+                            const SelShared &sh, int *sel_i, int *sel_j, float *srow,
+                            float *scol) {
+    const int warp = threadIdx.x >> 5;
+    if (warp >= 2) return;
+    const int c = candidate_count(warp, sh);   // <= 256 (see select_candidates)
+    int *sel = warp == 0 ? sel_i : sel_j;
+    float *So = warp == 0 ? srow : scol;
+    if (c <= 64) finish_axis<T, 2>(d, p, h, warp, qv, sh, sel, So);
+    else if (c <= 128) finish_axis<T, 4>(d, p, h, warp, qv, sh, sel, So);
+    else finish_axis<T, 8>(d, p, h, warp, qv, sh, sel, So);
 }
 
 struct SelLayout {
-    uint32_t *key;
+    uint32_t *key0, *key1;
+    float *qv;          // [2][D_k] row and column query of this (token, head)
     int *sel_i, *sel_j;
     float *srow, *scol, *R;
 };
 
 __device__ SelLayout carve(const Dims &d, unsigned char *base) {
     SelLayout L;
-    const int nkey = max(d.K, d.k * d.k);
     size_t off = 0;
-    L.key = reinterpret_cast<uint32_t *>(base + off);
-    off += sizeof(uint32_t) * nkey;
+    L.key0 = reinterpret_cast<uint32_t *>(base + off);
+    off += sizeof(uint32_t) * max(d.K, d.k * d.k);
+    L.key1 = reinterpret_cast<uint32_t *>(base + off);
+    off += sizeof(uint32_t) * d.K;
+    L.qv = reinterpret_cast<float *>(base + off);
+    off += sizeof(float) * 2 * d.d_k;
     L.sel_i = reinterpret_cast<int *>(base + off);
     off += sizeof(int) * d.k;
     L.sel_j = reinterpret_cast<int *>(base + off);
@@ -241,6 +511,7 @@ __device__ SelLayout carve(const Dims &d, unsigned char *base) {
     return L;
 }
 
+template <typename T>
 __global__ void __launch_bounds__(kThreads) select_kernel(Dims d, Ptrs p) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ SelShared sh;
@@ -248,24 +519,50 @@ __global__ void __launch_bounds__(kThreads) select_kernel(Dims d, Ptrs p) {
     SelLayout L = carve(d, smem_raw);
     const int r = d.r, K = d.K, k = d.k, m = d.m;
     const float *C = p.core + (int64_t)h * r * r;
+    const uint32_t *A0 = p.akey + (((int64_t)b * d.H + h) * 2) * (int64_t)K;
+    const uint32_t *A1 = A0 + K;
 
-    // Eq. 6-9 per axis: rank-1 score, top-k; survivors in increasing index
-    for (int axis = 0; axis < 2; ++axis) {
-        const float *coef = (axis == 0 ? p.u : p.t) + (int64_t)h * r;
-        const float *S = p.s + (((int64_t)b * d.H + h) * 2 + axis) * (int64_t)K * r;
-        for (int i = threadIdx.x; i < K; i += kThreads) {
-            float a = 0.f;
-            for (int al = 0; al < r; ++al) a = fmaf(coef[al], S[(int64_t)i * r + al], a);
-            L.key[i] = f2ord(a);
+    // rank-1 score keys of both axes (Eq. 6-7, from the scoring kernel) and
+    // the row/column query of this (token, head), summed over its D_i splits
+    uint32_t vm0 = 0, vm1 = 0;
+    for (int i0 = threadIdx.x; i0 < K; i0 += 4 * kThreads) {
+        uint32_t a[4], c2[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int i = i0 + q * kThreads;
+            a[q] = i < K ? A0[i] : 0u;
+            c2[q] = i < K ? A1[i] : 0u;
         }
-        __syncthreads();
-        int *sel = axis == 0 ? L.sel_i : L.sel_j;
-        topk_positions(L.key, K, k, sel, kOrderByPosition, sh);
-        float *keep = axis == 0 ? L.srow : L.scol;
-        for (int e = threadIdx.x; e < k * r; e += kThreads)
-            keep[e] = S[(int64_t)sel[e / r] * r + (e % r)];
-        __syncthreads();
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int i = i0 + q * kThreads;
+            if (i < K) {
+                L.key0[i] = a[q];
+                L.key1[i] = c2[q];
+                vm0 = max(vm0, a[q]);
+                vm1 = max(vm1, c2[q]);
+            }
+        }
     }
+    {
+        const int HD = d.H * d.d_k;
+        for (int e = threadIdx.x; e < 2 * d.d_k; e += kThreads) {
+            const int axis = e / d.d_k, c = e % d.d_k;
+            const int a = (axis == 1 && d.A == 2) ? 1 : 0;
+            const float *src = p.q_part + ((int64_t)a * d.B + b) * HD + h * d.d_k + c;
+            const int64_t split_stride = (int64_t)d.A * d.B * HD;
+            float q = 0.f;
+            for (int s = 0; s < d.q_splits; ++s) q += src[s * split_stride];
+            L.qv[e] = q;
+        }
+    }
+    // (the first barrier of select_candidates orders these shared-memory writes)
+
+    // Eq. 8-9: top-k of both axes
+    select_candidates(L.key0, L.key1, 2, K, k, vm0, vm1, sh);
+    // survivors in increasing index, with their exact chunk scores (Eq. 4)
+    finish_axes<T>(d, p, h, L.qv, sh, L.sel_i, L.sel_j, L.srow, L.scol);
+    __syncthreads();
 
     // Eq. 10: g(i,j) = sum_ab S_row[a,i] C[a,b] S_col[b,j] on I x J, as
     // R[i][b] = sum_a S_row[a,i] C[a,b] then g = sum_b R[i][b] S_col[b,j].
@@ -277,36 +574,44 @@ __global__ void __launch_bounds__(kThreads) select_kernel(Dims d, Ptrs p) {
     }
     __syncthreads();
     const int k2 = k * k;
+    uint32_t vmg = 0;
+    const int dii = kThreads / k, djj = kThreads % k;   // (ii, jj) step per c += kThreads
+    int ii = threadIdx.x / k, jj = threadIdx.x % k;
     for (int c = threadIdx.x; c < k2; c += kThreads) {
-        int ii = c / k, jj = c - ii * k;
         float g = 0.f;
         for (int be = 0; be < r; ++be) g = fmaf(L.R[ii * r + be], L.scol[jj * r + be], g);
-        L.key[c] = f2ord(g);   // I and J ascending: increasing c is increasing v
+        const uint32_t kg = f2ord(g);
+        L.key0[c] = kg;
+        vmg = max(vmg, kg);
+        ii += dii;
+        jj += djj;
+        if (jj >= k) { jj -= k; ++ii; }
     }
-    __syncthreads();
-    topk_positions(L.key, k2, m, nullptr, kOrderByScore, sh);
+    select_candidates(L.key0, nullptr, 1, k2, m, vmg, 0u, sh);
+    finish_top(0, m, sh.fwin, sh);
 
     // PKM's softmax over the m selected scores (Eq. 3); Trick 1 skips it
-    const float gmax = ord2f(sh.win_key[0]);
+    const float gmax = ord2f(key_of(sh.fwin[0]));
     if (d.act == ULTRAMEM_ACT_SOFTMAX) {
         if (threadIdx.x < 32) {
             float z = 0.f;
-            for (int e = threadIdx.x; e < m; e += 32) z += __expf(ord2f(sh.win_key[e]) - gmax);
+            for (int e = threadIdx.x; e < m; e += 32) z += __expf(ord2f(key_of(sh.fwin[e])) - gmax);
 #pragma unroll
-            for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(0xffffffffu, z, off);
+            for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(kFull, z, off);
             if (threadIdx.x == 0) sh.scalar = z;
         }
         __syncthreads();
     }
     const int64_t base = ((int64_t)b * d.H + h) * m;
     for (int e = threadIdx.x; e < m; e += kThreads) {
-        int c = sh.win_pos[e];
-        int ii = c / k, jj = c - ii * k;
-        uint64_t v = (uint64_t)L.sel_i[ii] * (uint64_t)K + (uint64_t)L.sel_j[jj];
-        float g = ord2f(sh.win_key[e]);
-        float w = d.act == ULTRAMEM_ACT_SOFTMAX ? __expf(g - gmax) / sh.scalar : g;
-        uint64_t vs = shuffle_address(d, p.perm, v);   // Eq. 14
-        uint64_t pb = vs / (uint64_t)d.N;
+        const u64 wc = sh.fwin[e];
+        const int c = (int)pos_of(wc);
+        const int ii = c / k, jj = c - ii * k;
+        const uint64_t v = (uint64_t)L.sel_i[ii] * (uint64_t)K + (uint64_t)L.sel_j[jj];
+        const float g = ord2f(key_of(wc));
+        const float w = d.act == ULTRAMEM_ACT_SOFTMAX ? __expf(g - gmax) / sh.scalar : g;
+        const uint64_t vs = shuffle_address(d, p.perm, v);   // Eq. 14
+        const uint64_t pb = vs / (uint64_t)d.N;
         p.sel_row[base + e] = (int32_t)(vs - pb * (uint64_t)d.N);
         p.sel_p[base + e] = (int32_t)pb;
         p.sel_w[base + e] = w;
@@ -340,13 +645,17 @@ __global__ void slots_kernel(Dims d, Ptrs p) {
 }  // namespace
 
 size_t select_smem_bytes(const Dims &d) {
-    size_t nkey = (size_t)(d.K > d.k * d.k ? d.K : d.k * d.k);
-    size_t off = sizeof(uint32_t) * nkey + sizeof(int) * 2 * d.k + sizeof(float) * 3 * d.k * d.r;
+    size_t nkey0 = (size_t)(d.K > d.k * d.k ? d.K : d.k * d.k);
+    size_t off = sizeof(uint32_t) * (nkey0 + d.K) + sizeof(float) * 2 * d.d_k +
+                 sizeof(int) * 2 * d.k + sizeof(float) * 3 * d.k * d.r;
     return (off + 15) & ~size_t(15);
 }
 
 cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st) {
-    select_kernel<<<d.B * d.H, kThreads, select_smem_bytes(d), st>>>(d, p);
+    if (d.dtype == ULTRAMEM_BF16)
+        select_kernel<__nv_bfloat16><<<d.B * d.H, kThreads, select_smem_bytes(d), st>>>(d, p);
+    else
+        select_kernel<float><<<d.B * d.H, kThreads, select_smem_bytes(d), st>>>(d, p);
     return cudaGetLastError();
 }
 
@@ -360,8 +669,12 @@ cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream
 }
 
 cudaError_t configure_select(const Dims &d) {
-    return cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)select_smem_bytes(d));
+    const int bytes = (int)select_smem_bytes(d);
+    cudaError_t e = cudaFuncSetAttribute(select_kernel<float>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(select_kernel<__nv_bfloat16>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
 }  // namespace um

@@ -192,37 +192,44 @@ struct QueryOp {
 };
 
 // ---- S2: row/column scores, one accumulator per rank chunk ------------------
+// The epilogue folds the r chunk scores into the rank-1 score (Eq. 6-7),
+// a = sum_alpha coef[alpha] S_alpha with coef = u (row keys) or t (column
+// keys), and stores its order-preserving 32-bit key.
+template <int R>
 struct ScoreOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
-    int B, H, K, r, A, kb_total;
-    float *s;   // [B][H][2][K][r]
+    int B, H, K, A, kb_total;
+    const float *u, *t;   // [H][R]
+    uint32_t *akey;       // [B][H][2][K]
     __device__ Tile tile() const {
-        Tile t;
+        Tile tl;
         const int h = blockIdx.z >> 1, axis = blockIdx.z & 1;
-        t.m0 = blockIdx.x * kTileM;
-        t.n0 = blockIdx.y * n_tile;
-        t.a_sel = axis;
-        t.a_z = h;
-        t.b_z = (A == 2 && axis == 1 ? H : 0) + h;
-        t.kb0 = 0;
-        t.nkb = kb_total;
-        return t;
+        tl.m0 = blockIdx.x * kTileM;
+        tl.n0 = blockIdx.y * n_tile;
+        tl.a_sel = axis;
+        tl.a_z = h;
+        tl.b_z = (A == 2 && axis == 1 ? H : 0) + h;
+        tl.kb0 = 0;
+        tl.nkb = kb_total;
+        return tl;
     }
-    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
-        const int i = t.m0 + row;
+    __device__ void store(const Tile &tl, int row, int c, float (&v)[kMaxAcc][16]) const {
+        const int i = tl.m0 + row;
         if (i >= K) return;
         const int h = blockIdx.z >> 1, axis = blockIdx.z & 1;
+        const float *coef = (axis == 0 ? u : t) + h * R;
+        float cf[R];
+#pragma unroll
+        for (int a = 0; a < R; ++a) cf[a] = coef[a];
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
-            const int n = t.n0 + c + j;
+            const int n = tl.n0 + c + j;
             if (n >= B) break;
-            float *dst = s + ((((int64_t)n * H + h) * 2 + axis) * K + i) * r;
-            if (r == 2) {
-                *reinterpret_cast<float2 *>(dst) = make_float2(v[0][j], v[1][j]);
-            } else {
-                for (int a = 0; a < r; ++a) dst[a] = v[a][j];
-            }
+            float a = cf[0] * v[0][j];
+#pragma unroll
+            for (int al = 1; al < R; ++al) a = fmaf(cf[al], v[al][j], a);
+            akey[(((int64_t)n * H + h) * 2 + axis) * K + i] = f2ord(a);
         }
     }
 };
@@ -365,7 +372,10 @@ template <int NSPLIT, class Op> static cudaError_t allow_smem() {
 
 cudaError_t configure_tc() {
     cudaError_t e = allow_smem<1, QueryOp>();
-    if (e == cudaSuccess) e = allow_smem<3, ScoreOp>();
+    if (e == cudaSuccess) e = allow_smem<3, ScoreOp<1>>();
+    if (e == cudaSuccess) e = allow_smem<3, ScoreOp<2>>();
+    if (e == cudaSuccess) e = allow_smem<3, ScoreOp<3>>();
+    if (e == cudaSuccess) e = allow_smem<3, ScoreOp<4>>();
     if (e == cudaSuccess) e = allow_smem<1, ProjOp>();
     return e;
 }
@@ -407,22 +417,34 @@ cudaError_t launch_qsplit(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, int s
     return cudaGetLastError();
 }
 
-cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
-    ScoreOp op;
-    op.n_tile = tc_n_tile(d.B, d.r);
-    op.n_acc = d.r;
+template <int R>
+static cudaError_t launch_score_r(const Dims &d, const Ptrs &p, const TcMaps &mp,
+                                  cudaStream_t st) {
+    ScoreOp<R> op;
+    op.n_tile = tc_n_tile(d.B, R);
+    op.n_acc = R;
     op.acc_chunk = d.dk;
     op.b_split_stride = d.d_k;
     op.err = p.err;
     op.B = d.B;
     op.H = d.H;
     op.K = d.K;
-    op.r = d.r;
     op.A = d.A;
     op.kb_total = (d.d_k + kBlockK - 1) / kBlockK;
-    op.s = p.s;
+    op.u = p.u;
+    op.t = p.t;
+    op.akey = p.akey;
     dim3 grid((d.K + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 2 * d.H);
     return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs, op, op.kb_total, st);
+}
+
+cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
+    switch (d.r) {
+    case 1: return launch_score_r<1>(d, p, mp, st);
+    case 2: return launch_score_r<2>(d, p, mp, st);
+    case 3: return launch_score_r<3>(d, p, mp, st);
+    default: return launch_score_r<4>(d, p, mp, st);
+    }
 }
 
 cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
