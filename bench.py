@@ -81,6 +81,19 @@ def algorithmic_bytes(cfg, B):
     }
 
 
+def aggregate_step(ms, batch, dist=None, device="cpu"):
+    """The slowest rank's step time and the whole-job tokens/s (every rank
+    processes its own batch of `batch` tokens)."""
+    world = 1
+    if dist is not None and dist.is_available() and dist.is_initialized():
+        import torch
+        world = dist.get_world_size()
+        t = torch.tensor([ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return ms, world * batch / (ms / 1e3)
+
+
 def launches_per_forward(cfg):
     return 4 + (2 if cfg["has_proj"] else 0)
 
@@ -302,12 +315,7 @@ def main():
         dist.barrier()
     clk = clocks.stop()
     total_ms = sum(a.elapsed_time(b) for a, b in ev)
-    ms = total_ms / K
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * B / (ms / 1e3)
+    ms, value = aggregate_step(total_ms / K, B, dist, device="cuda")
 
     # ---- per-stage device times: the forward with the layer's stage events
     # captured in a graph too, so the events see the kernels back to back ----
@@ -371,15 +379,11 @@ def main():
             t0 = time.perf_counter()
             layer.forward_host(xh[i % NB], oh)
             e2e_t.append(time.perf_counter() - t0)
-    e2e_s = sum(e2e_t) / len(e2e_t)
-    if dist:
-        t = torch.tensor([e2e_s], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_ms, e2e_value = aggregate_step(1e3 * sum(e2e_t) / len(e2e_t), B, dist, device="cuda")
     es = 4 if int(cfg["dtype"]) == 0 else 2
-    e2e = {"value": world * B / e2e_s, "unit": "tokens/s",
+    e2e = {"value": e2e_value, "unit": "tokens/s",
            "h2d_bytes_per_step": B * cfg["d_in"] * es, "d2h_bytes_per_step": B * cfg["d_out"] * es,
-           "ms_per_step": e2e_s * 1e3}
+           "ms_per_step": e2e_ms}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
