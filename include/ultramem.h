@@ -136,6 +136,29 @@ ultramem_status ultramem_retrieve(ultramem_layer *layer, const void *x, int32_t 
 ultramem_status ultramem_lookup_reduce(ultramem_layer *layer, const int64_t *idx,
                                        const float *w, int32_t B, void *out, void *stream);
 
+/* The lookup-reduce of ultramem_lookup_reduce (S7-S9) without a layer handle
+ * and without allocating anything.  The paper has no counterpart: this entry
+ * point exists for callers that cannot call cudaMalloc or create a layer -- a
+ * host that owns the device allocator, runs inside a fixed memory budget, or
+ * must not risk an allocation blocking or failing at this point.  Its scratch
+ * is one 8 MiB array of static device memory that every GPU loading the
+ * library holds until the process exits; a batch whose scratch would exceed
+ * it is rejected with ULTRAMEM_EINVAL.  cfg: d_k, rank, topk, max_tokens are
+ * ignored; heads, topm, n, expand_e, d_v, d_out, has_proj, dtype and
+ * shuffle_seed are used as in ultramem_create.  values [N][D_v] and w_proj
+ * [E][D_v][D'_v] as in ultramem_weights (w_proj may be NULL when has_proj is
+ * 0), perm optional; idx [B][H][m] int64 and w [B][H][m] fp32 as in
+ * ultramem_lookup_reduce; out [B][D'_v].  Out-of-range addresses are skipped
+ * (weight 0).  Asynchronous on `stream`.  The first call on a device looks up
+ * the array's device address and sets a kernel attribute; make that first
+ * call before any stream capture.  Every call shares the one array, so calls
+ * that overlap on the GPU (other streams, other host threads) race and must
+ * be ordered by the caller. */
+ultramem_status ultramem_lookup_reduce_noalloc(const ultramem_config *cfg, const void *values,
+                                               const void *w_proj, const uint32_t *perm,
+                                               const int64_t *idx, const float *w, int32_t B,
+                                               void *out, void *stream);
+
 /* Synchronises `stream`, then reads and clears the layer's device error word:
  * ULTRAMEM_EDEVICE if a kernel recorded a bad index, ULTRAMEM_ETIMEOUT if a
  * bounded wait gave up, ULTRAMEM_ECUDA if the stream reports an error. */

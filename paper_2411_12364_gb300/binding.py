@@ -24,7 +24,7 @@ EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
            "ultramem_forward_host", "ultramem_retrieve", "ultramem_lookup_reduce",
            "ultramem_check", "ultramem_rank1", "ultramem_profile_enable",
            "ultramem_profile_read", "ultramem_stage_name", "ultramem_status_string",
-           "ultramem_last_error", "ultramem_version")
+           "ultramem_last_error", "ultramem_version", "ultramem_lookup_reduce_noalloc")
 
 
 class Config(C.Structure):
@@ -89,6 +89,8 @@ def load(path: str | None = None) -> C.CDLL:
         lib.ultramem_stage_name.restype = C.c_char_p
         lib.ultramem_status_string.argtypes = [I32]
         lib.ultramem_status_string.restype = C.c_char_p
+        lib.ultramem_lookup_reduce_noalloc.argtypes = [P, P, P, P, P, P, I32, P, P]
+        lib.ultramem_lookup_reduce_noalloc.restype = I32
         lib.ultramem_last_error.argtypes = []
         lib.ultramem_last_error.restype = C.c_char_p
         lib.ultramem_version.argtypes = []

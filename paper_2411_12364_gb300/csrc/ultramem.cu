@@ -625,3 +625,11 @@ int32_t ultramem_profile_read(ultramem_layer *L, float *ms, int32_t n) {
 }
 
 }  // extern "C"
+
+namespace um {
+// The seeded shuffle's multiplier and offset, for entry points defined in
+// other translation units.
+void host_shuffle_params(uint64_t seed, uint64_t M, uint64_t *a, uint64_t *c) {
+    shuffle_params(seed, M, a, c);
+}
+}  // namespace um
