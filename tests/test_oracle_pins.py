@@ -81,7 +81,7 @@ def _positive_layer(cfg, B, rank1_core):
 
 @pytest.mark.parametrize("rank", [1, 2, 4])
 def test_rank1_core_two_phase_is_exact(rank):
-    """Spec invariant: with C = sigma u t^T and positive scores, the
+    """Invariant of the method: with C = sigma u t^T and positive scores, the
     grid score is sigma*a_i*b_j, monotone in both factors, so the two-phase
     top-m (Eq. 8-10 with k = m) equals brute force over all K*K slots."""
     cfg = _f32_cfg(rank=rank, d_k=8, topk=6, topm=6, n=8)
@@ -95,7 +95,7 @@ def test_rank1_core_two_phase_is_exact(rank):
 
 
 def test_rank_one_reduces_to_product_key_memory():
-    """Spec invariant: at r = 1 the core is a positive scalar c and
+    """Invariant of the method: at r = 1 the core is a positive scalar c and
     g(i,j) = c*S_row[i]*S_col[j]; with positive scores log g = log c +
     log S_row[i] + log S_col[j], the additive product-key score of PKM
     (Eq. 2), whose two-phase top-m is exact.  PKM's retrieval is computed
@@ -148,7 +148,7 @@ def test_general_core_selection_invariants():
 
 
 def test_explicit_virtual_table_equals_implicit():
-    """Spec invariant: materialising V~_p = V W_p (Eq. 13), scattering
+    """Invariant of the method: materialising V~_p = V W_p (Eq. 13), scattering
     the weights at the shuffled addresses (Eq. 14) and taking V~^T s^ gives
     the implicit sum_p W_p^T (V^T s^_p) of Eq. 15."""
     cfg = _f32_cfg(n=6, expand_e=4, d_v=8, d_out=11, topk=5, topm=7, heads=3)
@@ -181,7 +181,7 @@ def test_no_expansion_is_plain_weighted_pooling():
 
 
 def test_softmax_weights_sum_to_one():
-    """Spec invariant: with PKM's softmax (Eq. 3) the m weights of a
+    """Invariant of the method: with PKM's softmax (Eq. 3) the m weights of a
     head are positive, sum to 1 and keep the score order; without it
     (Trick 1) they are the raw scores."""
     cfg = _f32_cfg(act=1, topm=7)
