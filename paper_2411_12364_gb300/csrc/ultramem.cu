@@ -74,6 +74,23 @@ int tc_query_splits(const ultramem_config &c, int B) {
     return s < 1 ? 1 : s;
 }
 
+// Tensor path: split E*D_v so that about 128 CTAs stream W_p, with the fp32
+// partial sums held to at most twice the projector's bytes.
+int tc_proj_splits(const ultramem_config &c, int B) {
+    if (!c.has_proj) return 1;
+    int m_tiles = (c.d_out + 127) / 128;
+    int nt = um::tc_n_tile(B, 1);
+    int n_tiles = (B + nt - 1) / nt;
+    int kd = c.expand_e * c.d_v;
+    int kb = (kd + 63) / 64;
+    int s = (128 + m_tiles * n_tiles - 1) / (m_tiles * n_tiles);
+    int cap = kd / B;
+    if (s > 8) s = 8;
+    if (s > kb) s = kb;
+    if (s > cap) s = cap;
+    return s < 1 ? 1 : s;
+}
+
 // The tensor path needs bf16 storage, rank chunks of whole 16-wide MMA
 // steps, at most 4 chunks (TMEM columns) and 16-byte rows for TMA.
 bool tc_eligible(const ultramem_config &c) {
@@ -248,7 +265,7 @@ Dims dims_for(const ultramem_layer *L, int B) {
     Dims d = L->base;
     d.B = B;
     d.q_splits = L->tc ? tc_query_splits(L->cfg, B) : query_splits(L->cfg, B);
-    d.p_splits = proj_splits(L->cfg, B);
+    d.p_splits = L->tc ? tc_proj_splits(L->cfg, B) : proj_splits(L->cfg, B);
     return d;
 }
 
@@ -440,9 +457,11 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
         size_t q = (size_t)query_splits(*cfg, (int)B) * B;
         size_t qt = (size_t)tc_query_splits(*cfg, (int)B) * B;
         size_t pp = (size_t)proj_splits(*cfg, (int)B) * B;
+        size_t pt = (size_t)tc_proj_splits(*cfg, (int)B) * B;
         if (q > qmax) qmax = q;
         if (qt > qmax) qmax = qt;
         if (pp > pmax) pmax = pp;
+        if (pt > pmax) pmax = pt;
         if (B + 16 > Bm && B < Bm && B >= 256) B = Bm - 16;   // visit Bm itself
     }
     Workspace &ws = L->ws;

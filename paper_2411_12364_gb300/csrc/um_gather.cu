@@ -276,6 +276,18 @@ cudaError_t launch_gather(const Dims &d, const Ptrs &p, cudaStream_t st) {
     return cudaGetLastError();
 }
 
+// out = the sum of the p_splits partial projections, in split order
+cudaError_t launch_proj_reduce(const Dims &d, const Ptrs &p, cudaStream_t st) {
+    int64_t total = (int64_t)d.B * d.d_out;
+    int rblocks = (int)((total + 255) / 256);
+    if (rblocks > 4096) rblocks = 4096;
+    if (d.dtype == ULTRAMEM_BF16)
+        proj_reduce_kernel<__nv_bfloat16><<<rblocks, 256, 0, st>>>(d, p);
+    else
+        proj_reduce_kernel<float><<<rblocks, 256, 0, st>>>(d, p);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_proj(const Dims &d, const Ptrs &p, cudaStream_t st) {
     dim3 grid((d.d_out + 63) / 64, (d.B + 31) / 32, d.p_splits);
     int64_t total = (int64_t)d.B * d.d_out;

@@ -80,6 +80,7 @@ cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_gather(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_proj(const Dims &d, const Ptrs &p, cudaStream_t st);
+cudaError_t launch_proj_reduce(const Dims &d, const Ptrs &p, cudaStream_t st);
 
 // kernel attributes for large dynamic shared memory, set at layer creation
 cudaError_t configure_select(const Dims &d);

@@ -20,17 +20,12 @@ namespace tc {
 constexpr int kBlockK = 64;                  // bf16 elements per 128-byte row
 constexpr int kTileM = 128;
 constexpr uint32_t kTileABytes = kTileM * kBlockK * 2;   // 16 KiB
-constexpr uint64_t kWaitLimitNs = 1000000000ull;          // 1 s per wait
+constexpr long long kWaitLimitCycles = 2000000000ll;      // ~1 s per wait at ~2 GHz
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return (uint32_t)__cvta_generic_to_shared(p);
 }
 
-__device__ __forceinline__ uint64_t globaltimer() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
 
 // ---- mbarrier ------------------------------------------------------------
 
@@ -61,13 +56,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Waits for the phase of `parity` to complete; gives up after kWaitLimitNs
-// and returns false (the caller records the timeout and unwinds).
+// Waits for the phase of `parity` to complete; gives up after
+// kWaitLimitCycles of this SM's clock and returns false (the caller records
+// the timeout and unwinds).  The SM cycle counter is cheap to read, so a
+// completed phase is noticed at once.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
     if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t deadline = globaltimer() + kWaitLimitNs;
+    const long long start = clock64();
     while (!mbar_try_wait(bar, parity))
-        if (globaltimer() > deadline) return false;
+        if (clock64() - start > kWaitLimitCycles) return false;
     return true;
 }
 
@@ -132,6 +129,26 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 32 lanes x 32 bits, 32 consecutive columns per thread; no wait (the caller
+// issues tmem_ld_wait once for a batch of loads)
+__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32"
+        " {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_ld_wait() {
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
 // ---- MMA -------------------------------------------------------------------

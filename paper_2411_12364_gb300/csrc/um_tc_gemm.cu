@@ -15,7 +15,7 @@
 // One CTA (4 warps) computes one 128 x N tile: warp 0 lane 0 issues the TMA
 // loads of a 4-stage ring, warp 1 lane 0 issues the MMAs, and all four warps
 // then read TMEM (row i = lane i) for the epilogue.  Every mbarrier wait is
-// bounded; a timeout sets the layer's error word.
+// bounded (~1 s); a timeout sets the layer's error word.
 #include <cudaTypedefs.h>
 
 #include "um_internal.cuh"
@@ -86,7 +86,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
 
-    if (warp == 0 && lane == 0) {
+    // Roles: lane 0 of warp 0 produces, lane 0 of warp 1 issues the MMAs; the
+    // other lanes of those warps wait at __syncwarp (not spinning on the
+    // accumulator barrier, which would steal the role lane's issue slots).
+    if (warp == 0) {
+      if (lane == 0) {
         // producer: TMA loads of A (128 x 64) and NSPLIT B tiles (N x 64)
         int it = 0;
         for (; it < t.nkb; ++it) {
@@ -111,10 +115,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         // loads still in flight (only after a timeout) land before exit
         for (int j = (it > kStages ? it - kStages : 0); j < it; ++j)
             mbar_wait(&full[j % kStages], (j / kStages) & 1);
-    } else if (warp == 1 && lane == 0) {
-        // MMA issuer
+      }
+      __syncwarp();
+    } else if (warp == 1) {
+      if (lane == 0) {
+        // MMA issuer.  Descriptors are built once per stage and advanced by
+        // 32 bytes (2 in the >>4 address field) per 16-wide K step; the
+        // accumulator of each step follows its rank chunk without division.
         const uint32_t idesc = idesc_bf16_f32(kTileM, n_tile);
         uint32_t started = 0;
+        int acc = (t.kb0 * kBlockK) / op.acc_chunk;
+        int next_chunk = (acc + 1) * op.acc_chunk;   // K index where acc advances
         for (int it = 0; it < t.nkb; ++it) {
             const int s = it % kStages;
             if (!mbar_wait(&full[s], (it / kStages) & 1)) {
@@ -123,37 +134,54 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
             const uint32_t sa = smem_u32(ring + (size_t)s * stage_bytes);
+            const uint64_t ad0 = desc_k_sw128(sa);
+            uint64_t bd0[NSPLIT];
+#pragma unroll
+            for (int j = 0; j < NSPLIT; ++j) bd0[j] = desc_k_sw128(sa + kTileABytes + j * b_bytes);
 #pragma unroll
             for (int k16 = 0; k16 < kBlockK / 16; ++k16) {
                 const int kg = (t.kb0 + it) * kBlockK + k16 * 16;
-                int acc = kg / op.acc_chunk;
-                if (acc >= op.n_acc) acc = op.n_acc - 1;
+                while (kg >= next_chunk && acc < op.n_acc - 1) {
+                    ++acc;
+                    next_chunk += op.acc_chunk;
+                }
                 const uint32_t dt = tmem + (uint32_t)(acc * n_tile);
-                const uint64_t ad = desc_k_sw128(sa + k16 * 32);
+                const uint32_t acc_bit = 1u << acc;
 #pragma unroll
                 for (int j = 0; j < NSPLIT; ++j) {
-                    const uint64_t bd = desc_k_sw128(sa + kTileABytes + j * b_bytes + k16 * 32);
-                    mma_bf16(dt, ad, bd, idesc, (started >> acc) & 1u);
-                    started |= 1u << acc;
+                    mma_bf16(dt, ad0 + 2 * k16, bd0[j] + 2 * k16, idesc, started & acc_bit);
+                    started |= acc_bit;
                 }
             }
             mma_commit(&empty[s]);   // frees the stage once these MMAs are done
         }
         mma_commit(&accbar);
+      }
+      __syncwarp();
     }
-    __syncwarp();
     if (!mbar_wait(&accbar, 0)) atomicOr(op.err, kErrTimeout);
     tc_fence_after();
 
-    // epilogue: thread = tile row (TMEM lane), 16 columns at a time
+    // epilogue: thread = tile row (TMEM lane); each chunk of 16 columns of
+    // every accumulator is read with one wait per 32 columns
     const int row = warp * 32 + lane;
     const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
-    for (int c = 0; c < n_tile; c += 16) {
-        float v[kMaxAcc][16];
+    for (int c0 = 0; c0 < n_tile; c0 += 32) {
+        uint32_t r[kMaxAcc][32];
 #pragma unroll
         for (int a = 0; a < kMaxAcc; ++a)
-            if (a < op.n_acc) tmem_ld16(lane_base + (uint32_t)(a * n_tile + c), v[a]);
-        op.store(t, row, c, v);
+            if (a < op.n_acc) tmem_ld32_nowait(lane_base + (uint32_t)(a * n_tile + c0), r[a]);
+        tmem_ld_wait();
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            if (c0 + half * 16 >= n_tile) break;
+            float v[kMaxAcc][16];
+#pragma unroll
+            for (int a = 0; a < kMaxAcc; ++a)
+#pragma unroll
+                for (int i = 0; i < 16; ++i) v[a][i] = __uint_as_float(r[a][half * 16 + i]);
+            op.store(t, row, c0 + half * 16, v);
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -234,12 +262,16 @@ struct ScoreOp {
     }
 };
 
-// ---- S9: IVE projection --------------------------------------------------
+// ---- S9: IVE projection, split over E*D_v --------------------------------
+// With one split the tile is written as bf16 output; with several, each
+// split writes fp32 partial sums part[split][n][o] that a second kernel adds
+// in split order.
 struct ProjOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
-    int B, d_out, kb_total;
+    int B, d_out, kb_total, splits;
     __nv_bfloat16 *out;   // [B][d_out]
+    float *part;          // [splits][B][d_out]
     __device__ Tile tile() const {
         Tile t;
         t.m0 = blockIdx.x * kTileM;
@@ -247,8 +279,9 @@ struct ProjOp {
         t.a_sel = 0;
         t.a_z = -1;
         t.b_z = -1;
-        t.kb0 = 0;
-        t.nkb = kb_total;
+        const int per = (kb_total + splits - 1) / splits;
+        t.kb0 = blockIdx.z * per;
+        t.nkb = max(0, min(kb_total, t.kb0 + per) - t.kb0);
         return t;
     }
     __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
@@ -257,7 +290,11 @@ struct ProjOp {
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
             const int n = t.n0 + c + j;
-            if (n < B) out[(int64_t)n * d_out + o] = __float2bfloat16_rn(v[0][j]);
+            if (n >= B) break;
+            if (splits == 1)
+                out[(int64_t)n * d_out + o] = __float2bfloat16_rn(v[0][j]);
+            else
+                part[((int64_t)blockIdx.z * B + n) * d_out + o] = t.nkb ? v[0][j] : 0.f;
         }
     }
 };
@@ -457,9 +494,14 @@ cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaS
     op.B = d.B;
     op.d_out = d.d_out;
     op.kb_total = (d.E * d.d_v + kBlockK - 1) / kBlockK;
+    op.splits = d.p_splits;
     op.out = static_cast<__nv_bfloat16 *>(p.out);
-    dim3 grid((d.d_out + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 1);
-    return launch_gemm<1>(grid, mp.w_pt, mp.w_pt, mp.acc, op, op.kb_total, st);
+    op.part = p.proj_part;
+    dim3 grid((d.d_out + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, op.splits);
+    const int per = (op.kb_total + op.splits - 1) / op.splits;
+    cudaError_t e = launch_gemm<1>(grid, mp.w_pt, mp.w_pt, mp.acc, op, per, st);
+    if (e == cudaSuccess && op.splits > 1) e = launch_proj_reduce(d, p, st);
+    return e;
 }
 
 }  // namespace um
