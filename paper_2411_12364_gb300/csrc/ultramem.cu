@@ -334,7 +334,9 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     mark(L, 1, st);
     if ((e = um::launch_score_tc(d, p, mp, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 2, st);
-    if ((e = um::launch_select(d, p, st)) != cudaSuccess) return from_cuda(e);
+    Dims ds = d;
+    ds.q_splits = 1;   // qsplit left the summed query in split 0
+    if ((e = um::launch_select(ds, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 3, st);
     if (retrieve_only) return ULTRAMEM_OK;
     if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
@@ -449,6 +451,7 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     d.dtype = cfg->dtype;
     d.has_proj = cfg->has_proj;
     shuffle_params(cfg->shuffle_seed, d.M, &d.shuf_a, &d.shuf_c);
+    d.shuf_mu = um::barrett_mu(d.M);
 
     const size_t Bm = (size_t)cfg->max_tokens, HD = (size_t)H * cfg->d_k;
     size_t qmax = 0, pmax = 0;

@@ -2,7 +2,8 @@
 //
 // Every kernel receives the layer's dimensions (Dims) and the device pointers
 // it touches (Ptrs) by value.  Workspace layouts (all fp32 unless noted):
-//   q_part   [q_splits][A][B][H*D_k]   split-K partial sums of q = W_q x
+//   q_part   [q_splits][A][B][H*D_k]   split-K partial sums of q = W_q x (the
+//                                      tensor path sums them into split 0)
 //   akey     [B][H][2][K] uint32       order-preserving key of the rank-1 score
 //                                      u^T S_row (axis 0) / t^T S_col (axis 1), Eq. 6
 //   sel_row  [B][H][m] int32           physical row of each selected slot
@@ -34,6 +35,7 @@ struct Dims {
     int A;            // 1 = shared query, 2 = separate column query
     int act, dtype, has_proj;
     uint64_t shuf_a, shuf_c;
+    uint64_t shuf_mu;  // floor((2^64 - 1) / M), the Barrett constant of M
     int q_splits, p_splits;
 };
 
@@ -109,11 +111,22 @@ __device__ __forceinline__ float ord2f(uint32_t o) {
     return __uint_as_float(u);
 }
 
-// The Eq. 14 shuffle: explicit table or the seeded affine bijection.
+// Barrett's constant for reduction modulo M (P. Barrett, CRYPTO '86).
+inline uint64_t barrett_mu(uint64_t M) { return M ? ~0ull / M : 0; }
+
+// The Eq. 14 shuffle: explicit table or the seeded affine bijection
+// (a v + c) mod M.  M < 2^32 and a, c, v < M, so a v + c < 2^64.  The
+// remainder uses Barrett's reduction: with mu = floor((2^64 - 1) / M) the
+// quotient estimate floor(x mu / 2^64) is at most 2 below floor(x / M), so
+// at most two corrections make it exact.
 __device__ __forceinline__ uint64_t shuffle_address(const Dims &d, const uint32_t *perm,
                                                     uint64_t v) {
     if (perm) return perm[v];
-    return (d.shuf_a * v + d.shuf_c) % d.M;   // M < 2^32 so a*v < 2^64
+    const uint64_t x = d.shuf_a * v + d.shuf_c;
+    uint64_t r = x - __umul64hi(x, d.shuf_mu) * d.M;
+    if (r >= d.M) r -= d.M;
+    if (r >= d.M) r -= d.M;
+    return r;
 }
 
 }  // namespace um

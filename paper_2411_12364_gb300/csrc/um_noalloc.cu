@@ -87,6 +87,7 @@ extern "C" ultramem_status ultramem_lookup_reduce_noalloc(const ultramem_config 
     const int kd = d.E * d.d_v;
     d.p_splits = c.has_proj ? splits_for(B, d.d_out, kd) : 1;
     um::host_shuffle_params(c.shuffle_seed, M, &d.shuf_a, &d.shuf_c);
+    d.shuf_mu = um::barrett_mu(M);
 
     // scratch layout: error word | rows | blocks | weights | acc | partials
     const size_t slots = (size_t)B * d.H * d.m;

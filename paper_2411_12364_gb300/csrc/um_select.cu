@@ -9,18 +9,19 @@
 // scores of the k survivors of each axis are recomputed here from q and the
 // key rows.  Ties go to the smaller index.
 //
-// Top-k of n keys, in two stages.  Candidates (whole block): each thread
-// takes the maximum of its strided share of the keys; each warp takes the
-// j-th largest of its 32 lane maxima (j = ceil(k / 8), a register bitonic
-// sort) and tau is the smallest of the 8 warp values.  Every warp owns at
-// least j keys >= tau, so at least k keys are >= tau whatever the input:
-// every key of the top k is >= tau.  Each warp appends its keys >= tau to its
-// own region (ballot, no atomics); when more than 2k survive, the same bound
-// is taken again over the survivors.  Order (one warp): the candidates, as
-// 64-bit composites (key, ~position) whose descending order is key
-// descending then position ascending, are sorted in registers by a bitonic
-// network (shuffles across lanes, swaps across registers).  Rare inputs with
-// too many candidates (heavy ties) take an exact radix select instead.
+// Top-k of n keys, in two stages.  Candidates: each thread takes the maximum
+// of its share of the keys; each warp takes the j-th largest of its 32 lane
+// maxima (j = ceil(k / 8), a register bitonic network) and tau is the
+// smallest of the 8 warp values.  Every warp owns at least j keys >= tau, so
+// at least k keys are >= tau whatever the input: every key of the top k is
+// >= tau.  The keys >= tau are appended to one flat list per selection
+// (ballot, one shared atomic per warp).  When the list is long the same
+// bound is taken again over it; when it overflows (heavy ties) an exact radix
+// select replaces it.  Order: the candidates are 64-bit composites (key,
+// ~position) whose descending order is key descending then position
+// ascending; the rank of each is the number of candidates above it, counted
+// in parallel (a group of lanes per candidate), and the ones ranked below k
+// are the winners, in rank order.
 #include "um_internal.cuh"
 
 namespace um {
@@ -28,18 +29,28 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kRegion = 128;               // candidates per warp region
-constexpr int kCap = kWarps * kRegion;     // 1024 per selection
+constexpr int kCap = 1024;                 // candidates per selection
+constexpr int kPerThread = kCap / kThreads;
 constexpr int kMaxK = 128;
 constexpr int kMaxM = 1024;
+constexpr int kMaxR = 8;
+constexpr int kRankSort = 256;             // longer lists are tightened first
 constexpr unsigned kFull = 0xffffffffu;
+
+// counter slots of SelShared::cnt
+constexpr int kCntAxis = 0;      // +s: first pass of axis s
+constexpr int kCntAxisT = 2;     // +s: tightened axis s
+constexpr int kCntTop = 4;       // final top-m
+constexpr int kCntTopT = 5;      // tightened final top-m
 
 typedef unsigned long long u64;
 
 struct SelShared {
-    u64 cand[2][kCap];      // per selection: kWarps regions of kRegion (or one flat list)
-    u64 fwin[kMaxM];        // final winners by rank
-    int wcnt[2][kWarps];    // region fill counts
+    __align__(16) u64 cand[2][kCap];   // flat candidate lists, one per selection
+    __align__(16) u64 win[2][kMaxK];   // axis winners by rank
+    __align__(16) u64 fwin[kMaxM];     // final winners by rank
+    float core[kMaxR * kMaxR];         // C of this head
+    int cnt[8];                        // list lengths (may exceed kCap: overflow)
     uint32_t vt[2][kWarps];
     int hist[256];
     int warp_tot[kWarps];
@@ -52,6 +63,9 @@ __device__ __forceinline__ u64 comp_of(uint32_t key, uint32_t pos) {
 }
 __device__ __forceinline__ uint32_t key_of(u64 c) { return (uint32_t)(c >> 32); }
 __device__ __forceinline__ uint32_t pos_of(u64 c) { return ~(uint32_t)c; }
+__device__ __forceinline__ uint32_t max4(uint4 v) {
+    return max(max(v.x, v.y), max(v.z, v.w));
+}
 
 template <typename T>
 __device__ __forceinline__ void unpack16(uint4 v, float (&f)[16 / sizeof(T)]);
@@ -72,19 +86,43 @@ __device__ __forceinline__ void unpack16<float>(uint4 v, float (&f)[4]) {
     f[3] = __uint_as_float(v.w);
 }
 
-// j-th largest (1-based, j <= 32) of one value per lane: descending bitonic
-// sort across the warp.
-__device__ __forceinline__ uint32_t warp_jth_largest(uint32_t v, int j) {
+// Descending bitonic network across the warp on two independent values per
+// lane; returns the j-th largest (1-based, j <= 32) of each.
+__device__ __forceinline__ void warp_jth_largest2(uint32_t a, uint32_t b, int j, uint32_t *ja,
+                                                  uint32_t *jb) {
     const int lane = threadIdx.x & 31;
 #pragma unroll
     for (int blk = 2; blk <= 32; blk <<= 1)
 #pragma unroll
         for (int st = blk >> 1; st > 0; st >>= 1) {
-            const uint32_t o = __shfl_xor_sync(kFull, v, st);
+            const uint32_t oa = __shfl_xor_sync(kFull, a, st);
+            const uint32_t ob = __shfl_xor_sync(kFull, b, st);
             const bool keep_max = ((lane & st) == 0) == ((lane & blk) == 0);
-            v = keep_max ? max(v, o) : min(v, o);
+            a = keep_max ? max(a, oa) : min(a, oa);
+            b = keep_max ? max(b, ob) : min(b, ob);
         }
-    return __shfl_sync(kFull, v, j - 1);
+    *ja = __shfl_sync(kFull, a, j - 1);
+    *jb = __shfl_sync(kFull, b, j - 1);
+}
+
+// Each warp's bound for a top-kk selection from its lanes' maxima (vm0, vm1
+// for two selections) into sh.vt[s][warp].  No barrier.
+__device__ __forceinline__ void warp_bounds(uint32_t vm0, uint32_t vm1, int kk, SelShared &sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int j = (kk + kWarps - 1) / kWarps;
+    uint32_t t0 = 0u, t1 = 0u;
+    if (j <= 32) warp_jth_largest2(vm0, vm1, j, &t0, &t1);
+    if (lane == 0) {
+        sh.vt[0][warp] = t0;
+        sh.vt[1][warp] = t1;
+    }
+}
+
+__device__ __forceinline__ uint32_t block_bound(int s, const SelShared &sh) {
+    uint32_t tau = sh.vt[s][0];
+#pragma unroll
+    for (int w = 1; w < kWarps; ++w) tau = min(tau, sh.vt[s][w]);
+    return tau;
 }
 
 // Exclusive prefix sum of one int per thread over the block; also syncs.
@@ -156,10 +194,10 @@ __device__ uint32_t select_kth_largest(const uint32_t *key, int n, int kk, SelSh
     return prefix;
 }
 
-// Exact fallback for selection s: a flat list of exactly kk candidates (every
-// key > T, then the first ties at T in position order) in cand[s], counted
-// in region 0.  Kept out of line: it only runs when a region overflows.
-__device__ __noinline__ void radix_fallback(const uint32_t *key, int n, int kk, int s,
+// Exact replacement of an overflowed list: exactly kk candidates (every key
+// > T, then the first ties at T in position order) into cand[s], length in
+// cnt[slot].  Out of line: it only runs on heavy ties.
+__device__ __noinline__ void radix_fallback(const uint32_t *key, int n, int kk, int s, int slot,
                                             SelShared &sh) {
     int need_eq;
     const uint32_t T = select_kth_largest(key, n, kk, sh, &need_eq);
@@ -179,416 +217,414 @@ __device__ __noinline__ void radix_fallback(const uint32_t *key, int n, int kk, 
         else if (v == T && e < need_eq) sh.cand[s][n_gt + e++] = comp_of(v, (uint32_t)i);
         else if (v == T) ++e;
     }
-    if (threadIdx.x < kWarps) sh.wcnt[s][threadIdx.x] = threadIdx.x == 0 ? kk : 0;
+    if (threadIdx.x == 0) sh.cnt[slot] = kk;
     __syncthreads();
 }
 
-// Tightens selection s: the same bound over the survivors of each region.
-__device__ void tighten(int s, int kk, SelShared &sh) {
+// Appends the lanes' composites with pr set to list (length counter *cnt):
+// one shared atomic per warp.  Entries past kCap are dropped (the counter
+// still counts them, which marks the overflow).
+__device__ __forceinline__ void warp_append(bool pr, u64 comp, u64 *list, int *cnt) {
+    const int lane = threadIdx.x & 31;
+    const unsigned bal = __ballot_sync(kFull, pr);
+    if (bal == 0u) return;
+    int base = 0;
+    if (lane == 0) base = atomicAdd(cnt, __popc(bal));
+    base = __shfl_sync(kFull, base, 0);
+    const int slot = base + __popc(bal & ((1u << lane) - 1u));
+    if (pr && slot < kCap) list[slot] = comp;
+}
+
+// Appends key[i] >= tau_s (i < n) of NS selections to their lists.  Each
+// warp handles 32-key batches in a strided share, 8 batches per round with
+// one atomic per selection and round.
+template <int NS>
+__device__ void compact(const uint32_t *key0, const uint32_t *key1, int n, uint32_t tau0,
+                        uint32_t tau1, SelShared &sh, int slot0, int slot1) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    constexpr int kPer = kRegion / 32;
-    const int mycnt = sh.wcnt[s][warp];
-    u64 mine[kPer];
+    constexpr int kB = 8;
+#pragma unroll 1
+    for (int c0 = warp * 32 + lane; c0 - lane < n; c0 += kB * kThreads) {
+#pragma unroll
+        for (int s = 0; s < NS; ++s) {
+            const uint32_t *key = s ? key1 : key0;
+            const uint32_t tau = s ? tau1 : tau0;
+            uint32_t v[kB];
+            unsigned bal[kB];
+            int tot = 0;
+#pragma unroll
+            for (int u = 0; u < kB; ++u) {
+                const int i = c0 + u * kThreads;
+                v[u] = i < n ? key[i] : 0u;
+                bal[u] = __ballot_sync(kFull, i < n && v[u] >= tau);
+                tot += __popc(bal[u]);
+            }
+            if (tot == 0) continue;
+            int base = 0;
+            if (lane == 0) base = atomicAdd(&sh.cnt[s ? slot1 : slot0], tot);
+            base = __shfl_sync(kFull, base, 0);
+            u64 *list = sh.cand[s];
+#pragma unroll
+            for (int u = 0; u < kB; ++u) {
+                const int slot = base + __popc(bal[u] & ((1u << lane) - 1u));
+                if (((bal[u] >> lane) & 1u) && slot < kCap)
+                    list[slot] = comp_of(v[u], (uint32_t)(c0 + u * kThreads));
+                base += __popc(bal[u]);
+            }
+        }
+    }
+}
+
+// The same bound taken again over list s (c entries, c <= kCap); the
+// survivors replace the list, length in cnt[slot_out].  Whole block; ends
+// with a barrier.
+__device__ void tighten(int s, int c, int kk, int slot_out, SelShared &sh) {
+    u64 mine[kPerThread];
     uint32_t vm = 0;
 #pragma unroll
-    for (int q = 0; q < kPer; ++q) {
-        const int f = lane + 32 * q;
-        mine[q] = f < mycnt ? sh.cand[s][warp * kRegion + f] : 0ull;
+    for (int q = 0; q < kPerThread; ++q) {
+        const int f = threadIdx.x + q * kThreads;
+        mine[q] = f < c ? sh.cand[s][f] : 0ull;
         vm = max(vm, key_of(mine[q]));
     }
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int j = (kk + kWarps - 1) / kWarps;
-    const uint32_t tw = j <= 32 ? warp_jth_largest(vm, j) : 0u;
+    uint32_t tw = 0u, unused;
+    if (j <= 32) warp_jth_largest2(vm, 0u, j, &tw, &unused);
     if (lane == 0) sh.vt[s][warp] = tw;
-    __syncthreads();
-    uint32_t tau = sh.vt[s][0];
-    for (int w = 1; w < kWarps; ++w) tau = min(tau, sh.vt[s][w]);
-    u64 *region = sh.cand[s] + warp * kRegion;
-    int cnt = 0;
+    __syncthreads();   // also: every list entry has been read
+    const uint32_t tau = block_bound(s, sh);
 #pragma unroll
-    for (int q = 0; q < kPer; ++q) {
-        const bool pr = lane + 32 * q < mycnt && key_of(mine[q]) >= tau;
-        const unsigned bal = __ballot_sync(kFull, pr);
-        if (pr) region[cnt + __popc(bal & ((1u << lane) - 1u))] = mine[q];
-        cnt += __popc(bal);
-    }
-    __syncthreads();   // everyone has read wcnt before it changes
-    if (lane == 0) sh.wcnt[s][warp] = cnt;
-    __syncthreads();
-}
-
-// Candidates of ns (1 or 2) selections of n keys each, key[s][0..n), for
-// their top kk: thresholds, per-warp compaction, tightening or the radix
-// fallback.  Leaves them in sh.cand[s] (kWarps regions counted by
-// sh.wcnt[s][w], or a flat list in region 0 when sh.wcnt[s][0] > kRegion).
-// vmax[s] is this thread's maximum over its strided share of key[s].  Every
-// thread of the block calls it; it ends with a barrier.
-__device__ void select_candidates(const uint32_t *key0, const uint32_t *key1, int ns, int n,
-                                  int kk, uint32_t vmax0, uint32_t vmax1, SelShared &sh) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int j = (kk + kWarps - 1) / kWarps;
-#pragma unroll 1
-    for (int s = 0; s < ns; ++s) {
-        const uint32_t tw = j <= 32 ? warp_jth_largest(s ? vmax1 : vmax0, j) : 0u;
-        if (lane == 0) sh.vt[s][warp] = tw;
-    }
-    __syncthreads();
-    // each warp appends its keys >= tau to its own region
-#pragma unroll 1
-    for (int s = 0; s < ns; ++s) {
-        const uint32_t *key = s ? key1 : key0;
-        uint32_t tau = sh.vt[s][0];
-        for (int w = 1; w < kWarps; ++w) tau = min(tau, sh.vt[s][w]);
-        u64 *region = sh.cand[s] + warp * kRegion;
-        int cnt = 0;
-        for (int b0 = warp * 32; b0 < n; b0 += kThreads) {
-            const int i = b0 + lane;
-            const uint32_t v = i < n ? key[i] : 0u;
-            const bool pr = i < n && v >= tau;
-            const unsigned bal = __ballot_sync(kFull, pr);
-            const int slot = cnt + __popc(bal & ((1u << lane) - 1u));
-            if (pr && slot < kRegion) region[slot] = comp_of(v, (uint32_t)i);
-            cnt += __popc(bal);
-        }
-        if (lane == 0) sh.wcnt[s][warp] = cnt;
-    }
-    __syncthreads();
-#pragma unroll 1
-    for (int s = 0; s < ns; ++s) {
-        int total = 0;
-        bool over = false;
-        for (int w = 0; w < kWarps; ++w) {
-            total += sh.wcnt[s][w];
-            over |= sh.wcnt[s][w] > kRegion;
-        }
-        __syncthreads();
-        if (!over && total > 2 * kk) {
-            tighten(s, kk, sh);
-            total = 0;
-            for (int w = 0; w < kWarps; ++w) total += sh.wcnt[s][w];
-            __syncthreads();
-            over = total > 8 * 32 && kk <= 8 * 32;   // too many to sort in registers
-        }
-        if (over) radix_fallback(s ? key1 : key0, n, kk, s, sh);   // rare, exact
-    }
-}
-
-__device__ __forceinline__ int candidate_count(int s, const SelShared &sh) {
-    if (sh.wcnt[s][0] > kRegion) return sh.wcnt[s][0];   // flat list
-    int total = 0;
-    for (int w = 0; w < kWarps; ++w) total += sh.wcnt[s][w];
-    return total;
-}
-
-// Descending bitonic sort of 32*R values held as v[q] on lane l = element
-// q*32 + l: shuffles for strides below 32, register swaps above.
-template <int R>
-__device__ __forceinline__ void warp_sort_desc(u64 (&v)[R]) {
-    const int lane = threadIdx.x & 31;
-#pragma unroll 1
-    for (int size = 2; size <= 32 * R; size <<= 1) {
-#pragma unroll 1
-        for (int j = size >> 1; j > 0; j >>= 1) {
-            if (j < 32) {
-#pragma unroll
-                for (int q = 0; q < R; ++q) {
-                    const u64 o = __shfl_xor_sync(kFull, v[q], j);
-                    const int e = q * 32 + lane;
-                    const bool keep_max = ((e & j) == 0) == ((e & size) == 0);
-                    v[q] = keep_max ? (v[q] > o ? v[q] : o) : (v[q] < o ? v[q] : o);
-                }
-            } else {
-                const int jq = j >> 5;
-#pragma unroll
-                for (int m = 1; m < R; m <<= 1) {
-                    if (jq != m) continue;
-#pragma unroll
-                    for (int q = 0; q < R; ++q) {
-                        if (q & m) continue;
-                        const bool desc = ((q * 32 + lane) & size) == 0;
-                        const u64 a = v[q], b = v[q | m];
-                        const bool sw = desc ? (a < b) : (a > b);
-                        v[q] = sw ? b : a;
-                        v[q | m] = sw ? a : b;
-                    }
-                }
-            }
-        }
-    }
-}
-
-// One warp: the candidates of selection s (at most 32*R) sorted descending
-// into v; element e = q*32 + lane, zero-padded.
-template <int R>
-__device__ __forceinline__ void warp_gather_sorted(int s, const SelShared &sh, u64 (&v)[R]) {
-    const int lane = threadIdx.x & 31;
-    const bool flat = sh.wcnt[s][0] > kRegion;
-    int pref[kWarps + 1];
-    pref[0] = 0;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w)
-        pref[w + 1] = pref[w] + (flat ? (w == 0 ? sh.wcnt[s][0] : 0) : sh.wcnt[s][w]);
-#pragma unroll
-    for (int q = 0; q < R; ++q) {
-        const int f = q * 32 + lane;
-        u64 val = 0ull;
-        if (f < pref[kWarps]) {
-            int w = 0, before = 0;
-#pragma unroll
-            for (int x = 1; x < kWarps; ++x)
-                if (f >= pref[x]) { w = x; before = pref[x]; }
-            val = sh.cand[s][(flat ? 0 : w * kRegion) + f - before];
-        }
-        v[q] = val;
-    }
-    warp_sort_desc<R>(v);
-}
-
-// Block-level exact ranks of selection s's candidates (any count up to
-// kCap) into win[rank] for rank < kk; each warp ranks its own region's
-// entries against all entries (a flat list is split w, w+8, ... over warps).
-__device__ void block_rank(int s, int kk, u64 *win, SelShared &sh) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const bool flat = sh.wcnt[s][0] > kRegion;
-    const int mine_n = flat ? (sh.wcnt[s][0] + kWarps - 1 - warp) / kWarps : sh.wcnt[s][warp];
-    for (int q = lane; q < mine_n; q += 32) {
-        const u64 ce = sh.cand[s][flat ? warp + q * kWarps : warp * kRegion + q];
-        int before = 0;
-#pragma unroll 1
-        for (int w = 0; w < (flat ? 1 : kWarps); ++w) {
-            const u64 *reg = sh.cand[s] + w * kRegion;
-            const int cw = sh.wcnt[s][w];
-            int f = 0;
-            for (; f + 4 <= cw; f += 4) {
-                const u64 a0 = reg[f], a1 = reg[f + 1], a2 = reg[f + 2], a3 = reg[f + 3];
-                before += (a0 > ce) + (a1 > ce) + (a2 > ce) + (a3 > ce);
-            }
-            for (; f < cw; ++f) before += reg[f] > ce;
-        }
-        if (before < kk) win[before] = ce;
-    }
-}
-
-// Final top-m: candidates sorted by one warp when they fit its registers,
-// else ranked by the whole block; win[rank] for rank < kk.  Ends with a
-// barrier.
-__device__ void finish_top(int s, int kk, u64 *win, SelShared &sh) {
-    const int c = candidate_count(s, sh);
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    if (c <= 256) {
-        if (warp == 0) {
-            if (c <= 64) {
-                u64 v[2];
-                warp_gather_sorted<2>(s, sh, v);
-#pragma unroll
-                for (int q = 0; q < 2; ++q)
-                    if (q * 32 + lane < kk) win[q * 32 + lane] = v[q];
-            } else if (c <= 128) {
-                u64 v[4];
-                warp_gather_sorted<4>(s, sh, v);
-#pragma unroll
-                for (int q = 0; q < 4; ++q)
-                    if (q * 32 + lane < kk) win[q * 32 + lane] = v[q];
-            } else {
-                u64 v[8];
-                warp_gather_sorted<8>(s, sh, v);
-#pragma unroll
-                for (int q = 0; q < 8; ++q)
-                    if (q * 32 + lane < kk) win[q * 32 + lane] = v[q];
-            }
-        }
-    } else {
-        block_rank(s, kk, win, sh);
+    for (int q = 0; q < kPerThread; ++q) {
+        const bool pr = threadIdx.x + q * kThreads < c && key_of(mine[q]) >= tau;
+        warp_append(pr, mine[q], sh.cand[s], &sh.cnt[slot_out]);
     }
     __syncthreads();
 }
 
-// Exact chunk scores of one key row against q (fp32 in shared memory):
-// out[alpha] = sum_{c < dk} row[alpha*dk + c] * q[alpha*dk + c]  (Eq. 4).
-// 16-byte loads, up to 8 in flight, when the row and chunks are aligned.
-template <typename T>
-__device__ void row_scores(const T *row, const float *q, const Dims &d, float *out) {
-    constexpr int EPV = 16 / sizeof(T);
-    const int dk = d.dk;
-    const bool vec = d.d_k % EPV == 0 && dk % EPV == 0 && ((uintptr_t)row & 15) == 0;
-#pragma unroll 1
-    for (int al = 0; al < d.r; ++al) {
-        const int c0 = al * dk;
-        float acc = 0.f;
-        if (vec) {
-            const uint4 *rv = reinterpret_cast<const uint4 *>(row + c0);
-            const int nv = dk / EPV;
-#pragma unroll 1
-            for (int v0 = 0; v0 < nv; v0 += 8) {
-                uint4 buf[8];
-#pragma unroll
-                for (int u = 0; u < 8; ++u)
-                    buf[u] = v0 + u < nv ? rv[v0 + u] : make_uint4(0, 0, 0, 0);
-#pragma unroll
-                for (int u = 0; u < 8; ++u) {
-                    if (v0 + u >= nv) break;
-                    float f[EPV];
-                    unpack16<T>(buf[u], f);
-                    const float *qq = q + c0 + (v0 + u) * EPV;
-#pragma unroll
-                    for (int e = 0; e < EPV; ++e) acc = fmaf(f[e], qq[e], acc);
-                }
-            }
-        } else {
-#pragma unroll 4
-            for (int c = 0; c < dk; ++c) acc = fmaf(to_f(row[c0 + c]), q[c0 + c], acc);
-        }
-        out[al] = acc;
+// Length of list s once it can be ranked: the radix select replaces an
+// overflowed list, a long one is tightened.  Uniform; may sync.
+__device__ int settle(int s, const uint32_t *key, int n, int kk, int slot, int slot_t,
+                      SelShared &sh) {
+    const int c = sh.cnt[slot];
+    if (c > kCap) {
+        radix_fallback(key, n, kk, s, slot, sh);
+        return kk;
     }
+    if (c > kRankSort && c > 2 * kk) {
+        tighten(s, c, kk, slot_t, sh);
+        return sh.cnt[slot_t];
+    }
+    return c;
 }
 
-// One warp per axis: the top-k of the axis' candidates, in increasing key
-// index (so that enumerating I x J row-major is increasing v = i*K + j), and
-// each survivor's exact chunk scores, one lane per survivor.
-template <typename T, int R>
-__device__ void finish_axis(const Dims &d, const Ptrs &p, int h, int axis, const float *qv,
-                            const SelShared &sh, int *sel, float *S_out) {
-    const int lane = threadIdx.x & 31;
-    const int k = d.k;
-    u64 v[R];
-    warp_gather_sorted<R>(axis, sh, v);
-    u64 pk[R];   // winners keyed by ~position: descending order = increasing index
-#pragma unroll
-    for (int q = 0; q < R; ++q)
-        pk[q] = q * 32 + lane < k ? (u64)(uint32_t)(~pos_of(v[q])) : 0ull;
-    warp_sort_desc<R>(pk);
-    const T *keys = static_cast<const T *>(axis == 0 ? p.k_row : p.k_col);
-#pragma unroll
-    for (int q = 0; q < R; ++q) {
-        const int e = q * 32 + lane;
-        if (e < k) {
-            const uint32_t pos = ~(uint32_t)pk[q];
-            sel[e] = (int)pos;
-            row_scores<T>(keys + ((int64_t)h * d.K + pos) * d.d_k, qv + axis * d.d_k, d,
-                          S_out + e * d.r);
+// Ranks of the c entries of list (threads [0, nt) of the selection, nt a
+// power of two, tid the thread's index among them): a group of G lanes per
+// entry counts the entries above it; entries of rank < kk go to win[rank].
+__device__ __forceinline__ void rank_list(const u64 *list, int c, int kk, u64 *win, int tid,
+                                          int nt) {
+    int G = 1;
+    while (G < 32 && 2 * G * c <= nt) G <<= 1;
+    const int sub = tid & (G - 1), slots = nt / G;
+    const int span = (((c + G - 1) / G) + 7) & ~7;
+    const int lo = min(c, sub * span), hi = min(c, lo + span);
+    const ulonglong2 *l2 = reinterpret_cast<const ulonglong2 *>(list);
+#pragma unroll 1
+    for (int f0 = 0; f0 < c; f0 += slots) {
+        const int f = f0 + tid / G;
+        const u64 me = f < c ? list[f] : ~0ull;
+        int before = 0, g = lo;
+#pragma unroll 1
+        for (; g + 8 <= hi; g += 8) {
+            const ulonglong2 a = l2[g / 2], b = l2[g / 2 + 1], x = l2[g / 2 + 2],
+                             y = l2[g / 2 + 3];
+            before += (a.x > me) + (a.y > me) + (b.x > me) + (b.y > me) + (x.x > me) +
+                      (x.y > me) + (y.x > me) + (y.y > me);
         }
+        for (; g < hi; ++g) before += list[g] > me;
+        for (int off = G >> 1; off > 0; off >>= 1) before += __shfl_xor_sync(kFull, before, off);
+        if (sub == 0 && f < c && before < kk) win[before] = me;
     }
-}
-
-template <typename T>
-__device__ void finish_axes(const Dims &d, const Ptrs &p, int h, const float *qv,
-                            const SelShared &sh, int *sel_i, int *sel_j, float *srow,
-                            float *scol) {
-    const int warp = threadIdx.x >> 5;
-    if (warp >= 2) return;
-    const int c = candidate_count(warp, sh);   // <= 256 (see select_candidates)
-    int *sel = warp == 0 ? sel_i : sel_j;
-    float *So = warp == 0 ? srow : scol;
-    if (c <= 64) finish_axis<T, 2>(d, p, h, warp, qv, sh, sel, So);
-    else if (c <= 128) finish_axis<T, 4>(d, p, h, warp, qv, sh, sel, So);
-    else finish_axis<T, 8>(d, p, h, warp, qv, sh, sel, So);
 }
 
 struct SelLayout {
-    uint32_t *key0, *key1;
     float *qv;          // [2][D_k] row and column query of this (token, head)
-    int *sel_i, *sel_j;
-    float *srow, *scol, *R;
+    uint32_t *key0;     // [max(K, k*k)] axis-0 keys, then the g keys
+    uint32_t *key1;     // [K] axis-1 keys
+    int *sel_i, *sel_j; // [k] surviving rows / columns in increasing index
+    float *R, *scol;    // [k][r] R = S_row^T C and S_col of the survivors
 };
 
-__device__ SelLayout carve(const Dims &d, unsigned char *base) {
-    SelLayout L;
+// Dynamic shared memory layout; every section starts on 16 bytes.
+struct SelOffsets {
+    size_t qv, key0, key1, sel_i, sel_j, R, scol, total;
+};
+__host__ __device__ inline SelOffsets sel_offsets(const Dims &d) {
+    auto up = [](size_t x) { return (x + 15) & ~size_t(15); };
+    SelOffsets o;
     size_t off = 0;
-    L.key0 = reinterpret_cast<uint32_t *>(base + off);
-    off += sizeof(uint32_t) * max(d.K, d.k * d.k);
-    L.key1 = reinterpret_cast<uint32_t *>(base + off);
-    off += sizeof(uint32_t) * d.K;
-    L.qv = reinterpret_cast<float *>(base + off);
-    off += sizeof(float) * 2 * d.d_k;
-    L.sel_i = reinterpret_cast<int *>(base + off);
-    off += sizeof(int) * d.k;
-    L.sel_j = reinterpret_cast<int *>(base + off);
-    off += sizeof(int) * d.k;
-    L.srow = reinterpret_cast<float *>(base + off);
-    off += sizeof(float) * d.k * d.r;
-    L.scol = reinterpret_cast<float *>(base + off);
-    off += sizeof(float) * d.k * d.r;
-    L.R = reinterpret_cast<float *>(base + off);
+    o.qv = off;    off = up(off + sizeof(float) * 2 * d.d_k);
+    o.key0 = off;  off = up(off + sizeof(uint32_t) * (d.K > d.k * d.k ? d.K : d.k * d.k));
+    o.key1 = off;  off = up(off + sizeof(uint32_t) * d.K);
+    o.sel_i = off; off = up(off + sizeof(int) * d.k);
+    o.sel_j = off; off = up(off + sizeof(int) * d.k);
+    o.R = off;     off = up(off + sizeof(float) * d.k * d.r);
+    o.scol = off;  off = up(off + sizeof(float) * d.k * d.r);
+    o.total = off;
+    return o;
+}
+
+__device__ SelLayout carve(const Dims &d, unsigned char *base) {
+    const SelOffsets o = sel_offsets(d);
+    SelLayout L;
+    L.qv = reinterpret_cast<float *>(base + o.qv);
+    L.key0 = reinterpret_cast<uint32_t *>(base + o.key0);
+    L.key1 = reinterpret_cast<uint32_t *>(base + o.key1);
+    L.sel_i = reinterpret_cast<int *>(base + o.sel_i);
+    L.sel_j = reinterpret_cast<int *>(base + o.sel_j);
+    L.R = reinterpret_cast<float *>(base + o.R);
+    L.scol = reinterpret_cast<float *>(base + o.scol);
     return L;
 }
 
-template <typename T>
-__global__ void __launch_bounds__(kThreads) select_kernel(Dims d, Ptrs p) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    __shared__ SelShared sh;
-    const int b = blockIdx.x / d.H, h = blockIdx.x % d.H;
-    SelLayout L = carve(d, smem_raw);
-    const int r = d.r, K = d.K, k = d.k, m = d.m;
-    const float *C = p.core + (int64_t)h * r * r;
-    const uint32_t *A0 = p.akey + (((int64_t)b * d.H + h) * 2) * (int64_t)K;
-    const uint32_t *A1 = A0 + K;
-
-    // rank-1 score keys of both axes (Eq. 6-7, from the scoring kernel) and
-    // the row/column query of this (token, head), summed over its D_i splits
-    uint32_t vm0 = 0, vm1 = 0;
-    for (int i0 = threadIdx.x; i0 < K; i0 += 4 * kThreads) {
-        uint32_t a[4], c2[4];
+// Loads the rank-1 score keys of both axes (Eq. 6-7, written by the scoring
+// kernel) into shared memory and returns this thread's maxima; all loads of
+// a round are issued before any store.
+__device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1, int K,
+                                          const SelLayout &L, uint32_t *vm0, uint32_t *vm1) {
+    uint32_t m0 = 0, m1 = 0;
+    if ((K & 3) == 0) {
+        const uint4 *V0 = reinterpret_cast<const uint4 *>(A0);
+        const uint4 *V1 = reinterpret_cast<const uint4 *>(A1);
+        uint4 *S0 = reinterpret_cast<uint4 *>(L.key0), *S1 = reinterpret_cast<uint4 *>(L.key1);
+        const int nv = K >> 2;
+#pragma unroll 1
+        for (int v0 = threadIdx.x; v0 < nv; v0 += 4 * kThreads) {
+            uint4 a[4], c[4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int i = i0 + q * kThreads;
-            a[q] = i < K ? A0[i] : 0u;
-            c2[q] = i < K ? A1[i] : 0u;
+            for (int q = 0; q < 4; ++q) {
+                const int i = v0 + q * kThreads;
+                a[q] = i < nv ? V0[i] : make_uint4(0, 0, 0, 0);
+                c[q] = i < nv ? V1[i] : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int i = v0 + q * kThreads;
+                if (i < nv) {
+                    S0[i] = a[q];
+                    S1[i] = c[q];
+                }
+                m0 = max(m0, max4(a[q]));
+                m1 = max(m1, max4(c[q]));
+            }
         }
+    } else {
+#pragma unroll 1
+        for (int i0 = threadIdx.x; i0 < K; i0 += 4 * kThreads) {
+            uint32_t a[4], c[4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int i = i0 + q * kThreads;
-            if (i < K) {
-                L.key0[i] = a[q];
-                L.key1[i] = c2[q];
-                vm0 = max(vm0, a[q]);
-                vm1 = max(vm1, c2[q]);
+            for (int q = 0; q < 4; ++q) {
+                const int i = i0 + q * kThreads;
+                a[q] = i < K ? A0[i] : 0u;
+                c[q] = i < K ? A1[i] : 0u;
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int i = i0 + q * kThreads;
+                if (i < K) {
+                    L.key0[i] = a[q];
+                    L.key1[i] = c[q];
+                }
+                m0 = max(m0, a[q]);
+                m1 = max(m1, c[q]);
             }
         }
     }
-    {
-        const int HD = d.H * d.d_k;
-        for (int e = threadIdx.x; e < 2 * d.d_k; e += kThreads) {
-            const int axis = e / d.d_k, c = e % d.d_k;
-            const int a = (axis == 1 && d.A == 2) ? 1 : 0;
-            const float *src = p.q_part + ((int64_t)a * d.B + b) * HD + h * d.d_k + c;
-            const int64_t split_stride = (int64_t)d.A * d.B * HD;
-            float q = 0.f;
-            for (int s = 0; s < d.q_splits; ++s) q += src[s * split_stride];
-            L.qv[e] = q;
+    *vm0 = m0;
+    *vm1 = m1;
+}
+
+// The 2k axis survivors, one group of G lanes each: the survivor's place in
+// increasing key index (so that enumerating I x J row-major is increasing
+// v = i*K + j), and its exact chunk scores S_alpha (Eq. 4) from 16-byte
+// loads of its key row split over the group.  Row survivors store
+// R[i][b] = sum_a S_row[a,i] C[a,b], column survivors S_col[j][b].
+template <typename T>
+__device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLayout &L,
+                               const SelShared &sh) {
+    constexpr int EPV = 16 / sizeof(T);
+    const int k = d.k, r = d.r, dk = d.dk, D = d.d_k;
+    int G = 1;
+    while (G < 32 && 2 * k * G * 2 <= kThreads) G <<= 1;
+    const int lane = threadIdx.x & 31, sub = lane & (G - 1);
+    const int sv = threadIdx.x / G;   // 2k * G <= kThreads: one pass
+    const bool active = sv < 2 * k;
+    const int s = active && sv >= k ? 1 : 0;
+    const int qi = active ? sv - s * k : 0;
+    const uint32_t pos = active ? pos_of(sh.win[s][qi]) : 0u;
+
+    int ord = 0;
+    if (active)
+        for (int g = sub; g < k; g += G) ord += pos_of(sh.win[s][g]) < pos;
+    for (int off = G >> 1; off > 0; off >>= 1) ord += __shfl_xor_sync(kFull, ord, off);
+
+    const T *row = static_cast<const T *>(s ? p.k_col : p.k_row) + ((int64_t)h * d.K + pos) * D;
+    const float *q = L.qv + s * D;
+    float S[kMaxR];
+#pragma unroll
+    for (int a = 0; a < kMaxR; ++a) S[a] = 0.f;
+    const bool vec = D % EPV == 0 && dk % EPV == 0 && ((uintptr_t)row & 15) == 0;
+    if (vec) {
+        // vector u of the row (EPV elements) belongs to chunk u*EPV / dk
+        const uint4 *rv = reinterpret_cast<const uint4 *>(row);
+        const int nvec = D / EPV;
+#pragma unroll 1
+        for (int u0 = sub; u0 < nvec; u0 += 8 * G) {
+            uint4 buf[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int iv = u0 + u * G;
+                buf[u] = active && iv < nvec ? rv[iv] : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int iv = u0 + u * G;
+                if (iv < nvec) {
+                    float f[EPV];
+                    unpack16<T>(buf[u], f);
+                    // q + iv*EPV is 16-byte aligned: qv is, and D % EPV == 0
+                    const float4 *qq = reinterpret_cast<const float4 *>(q + iv * EPV);
+                    float pv = 0.f;
+#pragma unroll
+                    for (int e4 = 0; e4 < EPV / 4; ++e4) {
+                        const float4 q4 = qq[e4];
+                        pv = fmaf(f[4 * e4], q4.x, pv);
+                        pv = fmaf(f[4 * e4 + 1], q4.y, pv);
+                        pv = fmaf(f[4 * e4 + 2], q4.z, pv);
+                        pv = fmaf(f[4 * e4 + 3], q4.w, pv);
+                    }
+                    const int al = iv * EPV / dk;
+#pragma unroll
+                    for (int a = 0; a < kMaxR; ++a) S[a] += a == al ? pv : 0.f;
+                }
+            }
+        }
+    } else {
+#pragma unroll
+        for (int a = 0; a < kMaxR; ++a) {
+            if (a < r && active) {
+                float acc = 0.f;
+                for (int c = a * dk + sub; c < (a + 1) * dk; c += G)
+                    acc = fmaf(to_f(row[c]), q[c], acc);
+                S[a] = acc;
+            }
         }
     }
-    // (the first barrier of select_candidates orders these shared-memory writes)
+#pragma unroll
+    for (int a = 0; a < kMaxR; ++a) {
+        if (a < r)
+            for (int off = G >> 1; off > 0; off >>= 1) S[a] += __shfl_xor_sync(kFull, S[a], off);
+    }
+    if (active && sub == 0) {
+        if (s == 0) {
+            L.sel_i[ord] = (int)pos;
+#pragma unroll
+            for (int b = 0; b < kMaxR; ++b) {
+                if (b < r) {
+                    float acc = 0.f;
+#pragma unroll
+                    for (int a = 0; a < kMaxR; ++a)
+                        if (a < r) acc = fmaf(S[a], sh.core[a * r + b], acc);
+                    L.R[ord * r + b] = acc;
+                }
+            }
+        } else {
+            L.sel_j[ord] = (int)pos;
+#pragma unroll
+            for (int b = 0; b < kMaxR; ++b)
+                if (b < r) L.scol[ord * r + b] = S[b];
+        }
+    }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    __shared__ SelShared sh;
+    const int b = blockIdx.x / d.H, h = blockIdx.x % d.H;
+    const SelLayout L = carve(d, smem_raw);
+    const int r = d.r, K = d.K, k = d.k, m = d.m;
+    const uint32_t *A0 = p.akey + (((int64_t)b * d.H + h) * 2) * (int64_t)K;
+    const uint32_t *A1 = A0 + K;
+
+    if (threadIdx.x < 8) sh.cnt[threadIdx.x] = 0;
+    // C of this head and the row/column query of this (token, head), summed
+    // over its D_i splits: loaded before the keys, stored after them
+    const float core_e = threadIdx.x < r * r ? p.core[(int64_t)h * r * r + threadIdx.x] : 0.f;
+    const int HD = d.H * d.d_k;
+    const int64_t split_stride = (int64_t)d.A * d.B * HD;
+    auto q_src = [&](int e) {
+        const int axis = e / d.d_k, c = e - axis * d.d_k;
+        const int a = (axis == 1 && d.A == 2) ? 1 : 0;
+        return p.q_part + ((int64_t)a * d.B + b) * HD + h * d.d_k + c;
+    };
+    auto q_of = [&](int e) {
+        const float *src = q_src(e);
+        float q = 0.f;
+        for (int s = 0; s < d.q_splits; ++s) q += src[s * split_stride];
+        return q;
+    };
+    const bool one_split = d.q_splits == 1;
+    float q0 = 0.f;
+    if (threadIdx.x < 2 * d.d_k) q0 = one_split ? *q_src(threadIdx.x) : q_of(threadIdx.x);
+    uint32_t vm0, vm1;
+    load_keys(A0, A1, K, L, &vm0, &vm1);
+    if (threadIdx.x < r * r) sh.core[threadIdx.x] = core_e;
+    if (threadIdx.x < 2 * d.d_k) L.qv[threadIdx.x] = q0;
+    for (int e = threadIdx.x + kThreads; e < 2 * d.d_k; e += kThreads) L.qv[e] = q_of(e);
 
     // Eq. 8-9: top-k of both axes
-    select_candidates(L.key0, L.key1, 2, K, k, vm0, vm1, sh);
-    // survivors in increasing index, with their exact chunk scores (Eq. 4)
-    finish_axes<T>(d, p, h, L.qv, sh, L.sel_i, L.sel_j, L.srow, L.scol);
+    warp_bounds(vm0, vm1, k, sh);
+    __syncthreads();
+    compact<2>(L.key0, L.key1, K, block_bound(0, sh), block_bound(1, sh), sh, kCntAxis,
+               kCntAxis + 1);
+    __syncthreads();
+    const int c0 = settle(0, L.key0, K, k, kCntAxis, kCntAxisT, sh);
+    const int c1 = settle(1, L.key1, K, k, kCntAxis + 1, kCntAxisT + 1, sh);
+    {
+        const int s = threadIdx.x >= kThreads / 2;
+        rank_list(sh.cand[s], s ? c1 : c0, k, sh.win[s], threadIdx.x & (kThreads / 2 - 1),
+                  kThreads / 2);
+    }
+    __syncthreads();
+    // survivors in increasing index with their exact chunk scores (Eq. 4)
+    axis_survivors<T>(d, p, h, L, sh);
     __syncthreads();
 
-    // Eq. 10: g(i,j) = sum_ab S_row[a,i] C[a,b] S_col[b,j] on I x J, as
-    // R[i][b] = sum_a S_row[a,i] C[a,b] then g = sum_b R[i][b] S_col[b,j].
-    for (int e = threadIdx.x; e < k * r; e += kThreads) {
-        int ii = e / r, be = e % r;
-        float acc = 0.f;
-        for (int al = 0; al < r; ++al) acc = fmaf(L.srow[ii * r + al], C[al * r + be], acc);
-        L.R[e] = acc;
-    }
-    __syncthreads();
+    // Eq. 10: g(i,j) = sum_b R[i][b] S_col[b,j] on I x J, R = S_row^T C
     const int k2 = k * k;
     uint32_t vmg = 0;
-    const int dii = kThreads / k, djj = kThreads % k;   // (ii, jj) step per c += kThreads
-    int ii = threadIdx.x / k, jj = threadIdx.x % k;
-    for (int c = threadIdx.x; c < k2; c += kThreads) {
-        float g = 0.f;
-        for (int be = 0; be < r; ++be) g = fmaf(L.R[ii * r + be], L.scol[jj * r + be], g);
-        const uint32_t kg = f2ord(g);
-        L.key0[c] = kg;
-        vmg = max(vmg, kg);
-        ii += dii;
-        jj += djj;
-        if (jj >= k) { jj -= k; ++ii; }
+    {
+        const int dii = kThreads / k, djj = kThreads % k;   // (ii, jj) step per c += kThreads
+        int ii = threadIdx.x / k, jj = threadIdx.x % k;
+        for (int c = threadIdx.x; c < k2; c += kThreads) {
+            float g = 0.f;
+            for (int be = 0; be < r; ++be) g = fmaf(L.R[ii * r + be], L.scol[jj * r + be], g);
+            const uint32_t kg = f2ord(g);
+            L.key0[c] = kg;
+            vmg = max(vmg, kg);
+            ii += dii;
+            jj += djj;
+            if (jj >= k) { jj -= k; ++ii; }
+        }
     }
-    select_candidates(L.key0, nullptr, 1, k2, m, vmg, 0u, sh);
-    finish_top(0, m, sh.fwin, sh);
+    warp_bounds(vmg, 0u, m, sh);
+    __syncthreads();
+    compact<1>(L.key0, nullptr, k2, block_bound(0, sh), 0u, sh, kCntTop, kCntTop);
+    __syncthreads();
+    const int cf = settle(0, L.key0, k2, m, kCntTop, kCntTopT, sh);
+    rank_list(sh.cand[0], cf, m, sh.fwin, threadIdx.x, kThreads);
+    __syncthreads();
 
     // PKM's softmax over the m selected scores (Eq. 3); Trick 1 skips it
     const float gmax = ord2f(key_of(sh.fwin[0]));
@@ -603,6 +639,7 @@ __global__ void __launch_bounds__(kThreads) select_kernel(Dims d, Ptrs p) {
         __syncthreads();
     }
     const int64_t base = ((int64_t)b * d.H + h) * m;
+    const uint32_t N = (uint32_t)d.N;
     for (int e = threadIdx.x; e < m; e += kThreads) {
         const u64 wc = sh.fwin[e];
         const int c = (int)pos_of(wc);
@@ -610,9 +647,9 @@ __global__ void __launch_bounds__(kThreads) select_kernel(Dims d, Ptrs p) {
         const uint64_t v = (uint64_t)L.sel_i[ii] * (uint64_t)K + (uint64_t)L.sel_j[jj];
         const float g = ord2f(key_of(wc));
         const float w = d.act == ULTRAMEM_ACT_SOFTMAX ? __expf(g - gmax) / sh.scalar : g;
-        const uint64_t vs = shuffle_address(d, p.perm, v);   // Eq. 14
-        const uint64_t pb = vs / (uint64_t)d.N;
-        p.sel_row[base + e] = (int32_t)(vs - pb * (uint64_t)d.N);
+        const uint32_t vs = (uint32_t)shuffle_address(d, p.perm, v);   // Eq. 14, < M < 2^32
+        const uint32_t pb = vs / N;
+        p.sel_row[base + e] = (int32_t)(vs - pb * N);
         p.sel_p[base + e] = (int32_t)pb;
         p.sel_w[base + e] = w;
         if (p.idx_out) p.idx_out[base + e] = (int64_t)v;
@@ -644,12 +681,7 @@ __global__ void slots_kernel(Dims d, Ptrs p) {
 
 }  // namespace
 
-size_t select_smem_bytes(const Dims &d) {
-    size_t nkey0 = (size_t)(d.K > d.k * d.k ? d.K : d.k * d.k);
-    size_t off = sizeof(uint32_t) * (nkey0 + d.K) + sizeof(float) * 2 * d.d_k +
-                 sizeof(int) * 2 * d.k + sizeof(float) * 3 * d.k * d.r;
-    return (off + 15) & ~size_t(15);
-}
+size_t select_smem_bytes(const Dims &d) { return sel_offsets(d).total; }
 
 cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st) {
     if (d.dtype == ULTRAMEM_BF16)

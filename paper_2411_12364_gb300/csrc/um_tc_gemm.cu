@@ -300,9 +300,11 @@ struct ProjOp {
 };
 
 // ---- q = sum of split partials, then the three-term bf16 split -------------
+// The fp32 sum is also written back over split 0, so that later stages read
+// one partial.
 // qs layout: [A*H][Bmax][3][D_k] (token rows of 3*D_k), the B operand of S2.
-__global__ void qsplit_kernel(Dims d, const float *__restrict__ q_part,
-                              __nv_bfloat16 *__restrict__ qs, int splits, int Bmax) {
+__global__ void qsplit_kernel(Dims d, float *q_part, __nv_bfloat16 *__restrict__ qs,
+                              int splits, int Bmax) {
     const int HD = d.H * d.d_k;
     const int64_t total = (int64_t)d.A * d.B * HD;
     for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
@@ -312,6 +314,7 @@ __global__ void qsplit_kernel(Dims d, const float *__restrict__ q_part,
         const int b = (int)(ab % d.B), a = (int)(ab / d.B);
         float q = 0.f;
         for (int s = 0; s < splits; ++s) q += q_part[(((int64_t)s * d.A + a) * d.B + b) * HD + o];
+        if (splits > 1) q_part[e] = q;   // the summed query replaces split 0 (same thread)
         const __nv_bfloat16 q1 = __float2bfloat16_rn(q);
         const float r1 = q - __bfloat162float(q1);
         const __nv_bfloat16 q2 = __float2bfloat16_rn(r1);
