@@ -64,17 +64,21 @@ def peaks():
 
 def algorithmic_bytes(cfg, B):
     """Bytes each stage must move at least (paper's Sec. 4 memory-access model
-    with heads: the gather reads min(B*H*m, N) rows of D_v)."""
+    with heads: the gather reads min(B*H*m, N) rows of D_v).  The selection
+    reads, per (token, head), the rank-1 score keys of both axes (2 K x 4 B),
+    the query (A D_k x 4 B) and the key rows of the 2k survivors
+    (2 k D_k x es), and writes m slots (row, block, weight: 12 B)."""
     es = 4 if int(cfg["dtype"]) == 0 else 2
     H, dk, din = cfg["heads"], cfg["d_k"], cfg["d_in"]
     K = int(round(cfg["expand_e"] ** 0.5)) * cfg["n"]
     A = 1 if cfg["share_query"] else 2
     N = cfg["n"] ** 2
-    rows = min(B * H * cfg["topm"], N)
+    k, m = cfg["topk"], cfg["topm"]
+    rows = min(B * H * m, N)
     return {
         "query": A * H * dk * din * es + B * din * es,
         "score": 2 * H * K * dk * es,
-        "select": 0,
+        "select": B * H * (2 * K * 4 + A * dk * 4 + 2 * k * dk * es + m * 12),
         "gather": rows * cfg["d_v"] * es,
         "project": (cfg["expand_e"] * cfg["d_v"] * cfg["d_out"] * es if cfg["has_proj"] else 0)
         + B * cfg["d_out"] * es,
@@ -92,10 +96,6 @@ def aggregate_step(ms, batch, dist=None, device="cpu"):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
     return ms, world * batch / (ms / 1e3)
-
-
-def launches_per_forward(cfg):
-    return 4 + (2 if cfg["has_proj"] else 0)
 
 
 class Clocks:
@@ -275,6 +275,7 @@ def main():
         for i in range(3):
             layer.forward(xs[0], out=out)
         torch.cuda.synchronize()
+        launches = layer.last_launches()   # kernels per forward (and per graph replay)
         if use_graph:
             for i in range(NB):
                 g = torch.cuda.CUDAGraph()
@@ -349,17 +350,11 @@ def main():
     peak, peak_kind = peaks()
     dominant = max(stage_avg, key=stage_avg.get)
     dom_bytes = alg[dominant]
-    src_of = {"query": "um_score.cu", "score": "um_score.cu", "select": "um_select.cu",
-              "gather": "um_gather.cu", "project": "um_gather.cu"}
     roof = {"kernel": dominant, "bound": "hbm", "achieved": dom_bytes / (stage_avg[dominant] * 1e6),
             "peak": peak, "unit": "GB/s", "peak_kind": peak_kind,
             "traffic": ncu_traffic(dominant, wl, B), "algorithmic_bytes": dom_bytes,
             "avg_ms": stage_avg[dominant]}
     roof["frac"] = roof["achieved"] / peak
-    if dom_bytes == 0:
-        roof["bound"] = "alu"
-        roof["achieved"] = None
-        roof["frac"] = None
     gms = stage_avg.get("gather")
     gather = None
     if gms:
@@ -393,12 +388,12 @@ def main():
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
                 "steps": K, "warmup": args.warmup, "ms_per_step": ms,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-                "dtype": "f32", "data": "synthetic",
-                "config": dict(workload=wl, batch=B, **_cfg_brief(cfg),
+                "dtype": "bf16" if int(cfg["dtype"]) else "f32", "data": "synthetic",
+                "config": dict(workload=wl, batch=B, **_cfg_brief(cfg), accumulate="f32",
                                l2="flushed between steps (256 MiB write, outside timing)",
                                cuda_graph=use_graph, parallelism=f"replicas x{world}"),
                 "roofline": roof, "gather": gather, "stages_ms": stage_avg,
-                "gpu_launches": K * launches_per_forward(cfg), "e2e": e2e,
+                "gpu_launches": K * launches, "e2e": e2e,
                 "cpu_baseline": cpu, "clocks": clk}
         print(json.dumps(line), flush=True)
     if dist:

@@ -178,6 +178,12 @@ ultramem_status ultramem_profile_enable(ultramem_layer *layer, int32_t enable);
 int32_t ultramem_profile_read(ultramem_layer *layer, float *ms, int32_t n);
 const char *ultramem_stage_name(int32_t i);
 
+/* Number of CUDA kernels the most recent successful ultramem_forward,
+ * ultramem_forward_host, ultramem_retrieve or ultramem_lookup_reduce call on
+ * this layer launched (a CUDA graph captured from a call launches the same
+ * kernels on every replay); 0 before the first call or for a NULL layer. */
+int32_t ultramem_last_launches(const ultramem_layer *layer);
+
 /* Text of the last CUDA error behind an ULTRAMEM_ECUDA or ULTRAMEM_ENOMEM
  * returned on the calling thread ("" if none). */
 const char *ultramem_last_error(void);

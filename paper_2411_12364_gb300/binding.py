@@ -24,7 +24,8 @@ EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
            "ultramem_forward_host", "ultramem_retrieve", "ultramem_lookup_reduce",
            "ultramem_check", "ultramem_rank1", "ultramem_profile_enable",
            "ultramem_profile_read", "ultramem_stage_name", "ultramem_status_string",
-           "ultramem_last_error", "ultramem_version", "ultramem_lookup_reduce_noalloc")
+           "ultramem_last_error", "ultramem_version", "ultramem_lookup_reduce_noalloc",
+           "ultramem_last_launches")
 
 
 class Config(C.Structure):
@@ -91,6 +92,8 @@ def load(path: str | None = None) -> C.CDLL:
         lib.ultramem_status_string.restype = C.c_char_p
         lib.ultramem_lookup_reduce_noalloc.argtypes = [P, P, P, P, P, P, I32, P, P]
         lib.ultramem_lookup_reduce_noalloc.restype = I32
+        lib.ultramem_last_launches.argtypes = [P]
+        lib.ultramem_last_launches.restype = I32
         lib.ultramem_last_error.argtypes = []
         lib.ultramem_last_error.restype = C.c_char_p
         lib.ultramem_version.argtypes = []
@@ -224,6 +227,10 @@ class UltraMemLayer:
     def check(self) -> int:
         """Syncs the current stream and returns the device error status."""
         return int(self.lib.ultramem_check(self._h, _stream()))
+
+    def last_launches(self) -> int:
+        """Kernels launched by the most recent successful call on this layer."""
+        return int(self.lib.ultramem_last_launches(self._h))
 
     def profile(self, enable: bool = True):
         _check(self.lib.ultramem_profile_enable(self._h, int(enable)), "profile_enable")

@@ -41,6 +41,7 @@ struct ultramem_layer {
     bool profiling = false;
     bool profiled_once = false;
     cudaEvent_t ev[kStages + 1] = {};
+    int launches = 0;    // kernels launched by the most recent successful call
 };
 
 namespace {
@@ -63,32 +64,28 @@ int query_splits(const ultramem_config &c, int B) {
     return s < 1 ? 1 : s;
 }
 
-// Tensor path: split D_i so that about 128 CTAs stream W_q.
-int tc_query_splits(const ultramem_config &c, int B) {
-    int m_tiles = (c.heads * c.d_k + 127) / 128;
+// Tensor path split-K: about `target` CTAs stream the weight, at most one
+// portable cluster (8) per tile, whole K blocks.
+int tc_splits(int m_rows, int B, int kdim, int target) {
+    int m_tiles = (m_rows + 127) / 128;
     int nt = um::tc_n_tile(B, 1);
     int n_tiles = (B + nt - 1) / nt;
-    int kb = (c.d_in + 63) / 64;
-    int s = (128 + m_tiles * n_tiles - 1) / (m_tiles * n_tiles);
+    int kb = (kdim + 63) / 64;
+    int s = (target + m_tiles * n_tiles - 1) / (m_tiles * n_tiles);
+    if (s > 8) s = 8;
     if (s > kb) s = kb;
     return s < 1 ? 1 : s;
 }
-
-// Tensor path: split E*D_v so that about 128 CTAs stream W_p, with the fp32
-// partial sums held to at most twice the projector's bytes.
+// Measured on GB300 (per forward, graphs of back-to-back forwards): the
+// query projection is fastest with the most splits; the IVE projection, whose
+// fp32 partials grow with the batch, with about 64 CTAs below 256 tokens and
+// unsplit from 256 tokens on.
+int tc_query_splits(const ultramem_config &c, int B) {
+    return tc_splits(c.heads * c.d_k, B, c.d_in, 128);
+}
 int tc_proj_splits(const ultramem_config &c, int B) {
-    if (!c.has_proj) return 1;
-    int m_tiles = (c.d_out + 127) / 128;
-    int nt = um::tc_n_tile(B, 1);
-    int n_tiles = (B + nt - 1) / nt;
-    int kd = c.expand_e * c.d_v;
-    int kb = (kd + 63) / 64;
-    int s = (128 + m_tiles * n_tiles - 1) / (m_tiles * n_tiles);
-    int cap = kd / B;
-    if (s > 8) s = 8;
-    if (s > kb) s = kb;
-    if (s > cap) s = cap;
-    return s < 1 ? 1 : s;
+    if (!c.has_proj || B >= 256) return 1;
+    return tc_splits(c.d_out, B, c.expand_e * c.d_v, 64);
 }
 
 // The tensor path needs bf16 storage, rank chunks of whole 16-wide MMA
@@ -293,7 +290,7 @@ void mark(ultramem_layer *L, int i, cudaStream_t st) {
 
 // S1..S6 (retrieval) then S7..S9; `retrieve_only` stops after S6.
 ultramem_status run_cuda_core(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
-                              bool retrieve_only) {
+                              bool retrieve_only, int *launches) {
     cudaError_t e;
     mark(L, 0, st);
     if ((e = um::launch_query(d, p, st)) != cudaSuccess) return from_cuda(e);
@@ -302,18 +299,20 @@ ultramem_status run_cuda_core(ultramem_layer *L, const Dims &d, Ptrs p, cudaStre
     mark(L, 2, st);
     if ((e = um::launch_select(d, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 3, st);
+    *launches = 3;
     if (retrieve_only) return ULTRAMEM_OK;
     if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 4, st);
     if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 5, st);
+    *launches = 4 + (d.has_proj ? 2 : 0);   // the projection and its split-K reduce
     if (L->profiling) L->profiled_once = true;
     return ULTRAMEM_OK;
 }
 
 // The bf16 path: S1, S2 and S9 on tcgen05 tensor cores, S3-S8 as above.
 ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
-                           bool retrieve_only) {
+                           bool retrieve_only, int *launches) {
     const ultramem_config &c = L->cfg;
     um::TcMaps mp = L->maps;
     const int Bmax = c.max_tokens;
@@ -328,21 +327,28 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     p.acc_bf = c.has_proj ? L->ws.acc_bf : nullptr;
     cudaError_t e;
     mark(L, 0, st);
-    if ((e = um::launch_query_tc(d, p, mp, d.q_splits, st)) != cudaSuccess) return from_cuda(e);
-    if ((e = um::launch_qsplit(d, p, L->ws.qs, d.q_splits, Bmax, st)) != cudaSuccess)
+    // Every kernel after the query projection is a programmatic dependent
+    // launch of its predecessor (not while profiling: the stage events sit
+    // between the kernels).  The query projection itself waits for all
+    // earlier work on the stream.
+    Dims dd = d;
+    dd.pdl = L->profiling ? 0 : 1;
+    if ((e = um::launch_query_tc(d, p, mp, d.q_splits, L->ws.qs, Bmax, st)) != cudaSuccess)
         return from_cuda(e);
     mark(L, 1, st);
-    if ((e = um::launch_score_tc(d, p, mp, st)) != cudaSuccess) return from_cuda(e);
+    if ((e = um::launch_score_tc(dd, p, mp, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 2, st);
-    Dims ds = d;
-    ds.q_splits = 1;   // qsplit left the summed query in split 0
+    Dims ds = dd;
+    ds.q_splits = 1;   // the query projection wrote the summed query
     if ((e = um::launch_select(ds, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 3, st);
+    *launches = d.A + 2;   // one query projection per query
     if (retrieve_only) return ULTRAMEM_OK;
-    if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
+    if ((e = um::launch_gather(dd, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 4, st);
-    if (d.has_proj && (e = um::launch_proj_tc(d, p, mp, st)) != cudaSuccess) return from_cuda(e);
+    if (d.has_proj && (e = um::launch_proj_tc(dd, p, mp, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 5, st);
+    *launches = d.A + 3 + (d.has_proj ? 1 : 0);
     if (L->profiling) L->profiled_once = true;
     return ULTRAMEM_OK;
 }
@@ -350,8 +356,11 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
 ultramem_status run(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
                     bool retrieve_only) {
     cudaGetLastError();   // a stale error from unrelated work is not ours to report
-    return L->tc ? run_tensor(L, d, p, st, retrieve_only)
-                 : run_cuda_core(L, d, p, st, retrieve_only);
+    int n = 0;
+    const ultramem_status s = L->tc ? run_tensor(L, d, p, st, retrieve_only, &n)
+                                    : run_cuda_core(L, d, p, st, retrieve_only, &n);
+    if (s == ULTRAMEM_OK) L->launches = n;
+    return s;
 }
 
 }  // namespace
@@ -586,6 +595,7 @@ ultramem_status ultramem_lookup_reduce(ultramem_layer *L, const int64_t *idx, co
     if ((e = um::launch_slots_from_addresses(d, p, st)) != cudaSuccess) return from_cuda(e);
     if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
     if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
+    L->launches = 2 + (d.has_proj ? 2 : 0);
     return ULTRAMEM_OK;
 }
 
@@ -631,6 +641,8 @@ ultramem_status ultramem_profile_enable(ultramem_layer *L, int32_t enable) {
     L->profiled_once = false;
     return ULTRAMEM_OK;
 }
+
+int32_t ultramem_last_launches(const ultramem_layer *L) { return L ? L->launches : 0; }
 
 int32_t ultramem_profile_read(ultramem_layer *L, float *ms, int32_t n) {
     if (!L || !ms || !L->profiled_once) return 0;

@@ -76,6 +76,8 @@ __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
     const int hm = d.H * d.m;
     const int64_t base = (int64_t)b * hm;
     const T *V = static_cast<const T *>(p.values);
+    pdl_wait();
+    pdl_trigger();
     float acc[EMAX][EPV];
 #pragma unroll
     for (int q = 0; q < EMAX; ++q)
@@ -137,6 +139,8 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Dims d, Ptrs p) {
     const int b = blockIdx.x;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int EDv = d.E * d.d_v;
+    pdl_wait();
+    pdl_trigger();
     float *mine = acc_w + (size_t)warp * EDv;
     for (int i = lane; i < EDv; i += 32) mine[i] = 0.f;
     __syncwarp();
@@ -228,6 +232,8 @@ __global__ void __launch_bounds__(kThreads) proj_kernel(Dims d, Ptrs p) {
 
 template <typename T>
 __global__ void proj_reduce_kernel(Dims d, Ptrs p) {
+    pdl_wait();
+    pdl_trigger();
     const int64_t total = (int64_t)d.B * d.d_out;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -257,35 +263,19 @@ cudaError_t configure_gather(const Dims &d) {
 }
 
 template <typename T>
-static void launch_gather_t(const Dims &d, const Ptrs &p, cudaStream_t st) {
+static cudaError_t launch_gather_t(const Dims &d, const Ptrs &p, cudaStream_t st) {
     const size_t bytes = gather_smem_bytes(d);
     const bool fits_lanes = d.d_v / (16 / (int)sizeof(T)) <= 32;
     if (fits_lanes && d.E == 1)
-        gather_reg_kernel<T, 1><<<d.B, kThreads, bytes, st>>>(d, p);
-    else if (fits_lanes && d.E <= 4)
-        gather_reg_kernel<T, 4><<<d.B, kThreads, bytes, st>>>(d, p);
-    else
-        gather_kernel<T><<<d.B, kThreads, bytes, st>>>(d, p);
+        return launch_kernel(d.pdl, gather_reg_kernel<T, 1>, d.B, kThreads, bytes, st, d, p);
+    if (fits_lanes && d.E <= 4)
+        return launch_kernel(d.pdl, gather_reg_kernel<T, 4>, d.B, kThreads, bytes, st, d, p);
+    return launch_kernel(d.pdl, gather_kernel<T>, d.B, kThreads, bytes, st, d, p);
 }
 
 cudaError_t launch_gather(const Dims &d, const Ptrs &p, cudaStream_t st) {
-    if (d.dtype == ULTRAMEM_BF16)
-        launch_gather_t<__nv_bfloat16>(d, p, st);
-    else
-        launch_gather_t<float>(d, p, st);
-    return cudaGetLastError();
-}
-
-// out = the sum of the p_splits partial projections, in split order
-cudaError_t launch_proj_reduce(const Dims &d, const Ptrs &p, cudaStream_t st) {
-    int64_t total = (int64_t)d.B * d.d_out;
-    int rblocks = (int)((total + 255) / 256);
-    if (rblocks > 4096) rblocks = 4096;
-    if (d.dtype == ULTRAMEM_BF16)
-        proj_reduce_kernel<__nv_bfloat16><<<rblocks, 256, 0, st>>>(d, p);
-    else
-        proj_reduce_kernel<float><<<rblocks, 256, 0, st>>>(d, p);
-    return cudaGetLastError();
+    if (d.dtype == ULTRAMEM_BF16) return launch_gather_t<__nv_bfloat16>(d, p, st);
+    return launch_gather_t<float>(d, p, st);
 }
 
 cudaError_t launch_proj(const Dims &d, const Ptrs &p, cudaStream_t st) {

@@ -3,7 +3,7 @@
 // Every kernel receives the layer's dimensions (Dims) and the device pointers
 // it touches (Ptrs) by value.  Workspace layouts (all fp32 unless noted):
 //   q_part   [q_splits][A][B][H*D_k]   split-K partial sums of q = W_q x (the
-//                                      tensor path sums them into split 0)
+//                                      tensor path leaves the sum in split 0)
 //   akey     [B][H][2][K] uint32       order-preserving key of the rank-1 score
 //                                      u^T S_row (axis 0) / t^T S_col (axis 1), Eq. 6
 //   sel_row  [B][H][m] int32           physical row of each selected slot
@@ -37,6 +37,8 @@ struct Dims {
     uint64_t shuf_a, shuf_c;
     uint64_t shuf_mu;  // floor((2^64 - 1) / M), the Barrett constant of M
     int q_splits, p_splits;
+    int pdl;           // host side: launch as a programmatic dependent of the
+                       // previous kernel on the stream
 };
 
 struct Ptrs {
@@ -68,9 +70,7 @@ bool tc_encode(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid,
 int tc_n_tile(int B, int n_acc);
 cudaError_t configure_tc();
 cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int splits,
-                            cudaStream_t st);
-cudaError_t launch_qsplit(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, int splits, int Bmax,
-                          cudaStream_t st);
+                            __nv_bfloat16 *qs, int Bmax, cudaStream_t st);
 cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st);
 cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st);
 cudaError_t launch_transpose_bf16(const void *src, void *dst, int rows, int cols,
@@ -82,13 +82,63 @@ cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_gather(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_proj(const Dims &d, const Ptrs &p, cudaStream_t st);
-cudaError_t launch_proj_reduce(const Dims &d, const Ptrs &p, cudaStream_t st);
 
 // kernel attributes for large dynamic shared memory, set at layer creation
 cudaError_t configure_select(const Dims &d);
 cudaError_t configure_gather(const Dims &d);
 size_t select_smem_bytes(const Dims &d);
 size_t gather_smem_bytes(const Dims &d);
+
+// ---- programmatic dependent launch ----------------------------------------
+// A kernel launched with programmatic stream serialization may start while
+// the previous kernel on the stream still runs.  Every kernel of the library
+// calls pdl_wait() before it touches memory that an earlier kernel writes or
+// reads (the wait returns once the previous grid has completed and its
+// memory is visible; since every kernel waits before it completes, that
+// covers all earlier kernels), and pdl_trigger() once its own resources are
+// held, to let the next kernel's CTAs be scheduled.  Both are no-ops for a
+// kernel launched without the attribute.  Before the wait a kernel reads
+// weights only.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Launches kernel<<<grid, block, smem, st>>>(args...), as a programmatic
+// dependent launch when `pdl`, in clusters of 1 x 1 x cluster_z CTAs when
+// cluster_z > 1.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(bool pdl, unsigned cluster_z, void (*kernel)(KArgs...), dim3 grid,
+                          dim3 block, size_t smem, cudaStream_t st, Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    unsigned n = 0;
+    if (pdl) {
+        attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    if (cluster_z > 1) {
+        attr[n].id = cudaLaunchAttributeClusterDimension;
+        attr[n].val.clusterDim.x = 1;
+        attr[n].val.clusterDim.y = 1;
+        attr[n].val.clusterDim.z = cluster_z;
+        ++n;
+    }
+    cfg.attrs = attr;
+    cfg.numAttrs = n;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(bool pdl, void (*kernel)(KArgs...), dim3 grid, dim3 block,
+                          size_t smem, cudaStream_t st, Args &&...args) {
+    return launch_kernel(pdl, 1u, kernel, grid, block, smem, st, static_cast<Args &&>(args)...);
+}
 
 // ---- small device helpers ------------------------------------------------
 

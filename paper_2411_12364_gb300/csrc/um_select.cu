@@ -9,12 +9,12 @@
 // scores of the k survivors of each axis are recomputed here from q and the
 // key rows.  Ties go to the smaller index.
 //
-// Top-k of n keys, in two stages.  Candidates: each thread takes the maximum
-// of its share of the keys; each warp takes the j-th largest of its 32 lane
-// maxima (j = ceil(k / 8), a register bitonic network) and tau is the
-// smallest of the 8 warp values.  Every warp owns at least j keys >= tau, so
-// at least k keys are >= tau whatever the input: every key of the top k is
-// >= tau.  The keys >= tau are appended to one flat list per selection
+// Top-k of n keys, in two stages.  Candidates: each thread keeps the two
+// largest of its share of the keys; each warp takes the j-th largest of its
+// lanes' 64 values (j = ceil(k / 8): j rounds of a warp max that removes one
+// instance) and tau is the smallest of the 8 warp values.  Every warp owns at
+// least j keys >= tau, so at least k keys are >= tau whatever the input:
+// every key of the top k is >= tau.  The keys >= tau are appended to one flat list per selection
 // (ballot, one shared atomic per warp).  When the list is long the same
 // bound is taken again over it; when it overflows (heavy ties) an exact radix
 // select replaces it.  Order: the candidates are 64-bit composites (key,
@@ -63,9 +63,6 @@ __device__ __forceinline__ u64 comp_of(uint32_t key, uint32_t pos) {
 }
 __device__ __forceinline__ uint32_t key_of(u64 c) { return (uint32_t)(c >> 32); }
 __device__ __forceinline__ uint32_t pos_of(u64 c) { return ~(uint32_t)c; }
-__device__ __forceinline__ uint32_t max4(uint4 v) {
-    return max(max(v.x, v.y), max(v.z, v.w));
-}
 
 template <typename T>
 __device__ __forceinline__ void unpack16(uint4 v, float (&f)[16 / sizeof(T)]);
@@ -86,32 +83,38 @@ __device__ __forceinline__ void unpack16<float>(uint4 v, float (&f)[4]) {
     f[3] = __uint_as_float(v.w);
 }
 
-// Descending bitonic network across the warp on two independent values per
-// lane; returns the j-th largest (1-based, j <= 32) of each.
-__device__ __forceinline__ void warp_jth_largest2(uint32_t a, uint32_t b, int j, uint32_t *ja,
-                                                  uint32_t *jb) {
-    const int lane = threadIdx.x & 31;
-#pragma unroll
-    for (int blk = 2; blk <= 32; blk <<= 1)
-#pragma unroll
-        for (int st = blk >> 1; st > 0; st >>= 1) {
-            const uint32_t oa = __shfl_xor_sync(kFull, a, st);
-            const uint32_t ob = __shfl_xor_sync(kFull, b, st);
-            const bool keep_max = ((lane & st) == 0) == ((lane & blk) == 0);
-            a = keep_max ? max(a, oa) : min(a, oa);
-            b = keep_max ? max(b, ob) : min(b, ob);
-        }
-    *ja = __shfl_sync(kFull, a, j - 1);
-    *jb = __shfl_sync(kFull, b, j - 1);
+// Inserts v into a lane's two largest values m1 >= m2.
+__device__ __forceinline__ void top2(uint32_t v, uint32_t &m1, uint32_t &m2) {
+    m2 = max(m2, min(v, m1));
+    m1 = max(m1, v);
 }
 
-// Each warp's bound for a top-kk selection from its lanes' maxima (vm0, vm1
-// for two selections) into sh.vt[s][warp].  No barrier.
-__device__ __forceinline__ void warp_bounds(uint32_t vm0, uint32_t vm1, int kk, SelShared &sh) {
+// The j-th largest (1 <= j <= 32) of the warp's 64 values {m1, m2}: j rounds
+// of a warp maximum, each removing one instance (the lowest lane holding it).
+__device__ __forceinline__ uint32_t warp_jth_top2(uint32_t m1, uint32_t m2, int j) {
+    const int lane = threadIdx.x & 31;
+    uint32_t t = 0u;
+#pragma unroll 1
+    for (int r = 0; r < j; ++r) {
+        t = __reduce_max_sync(kFull, m1);
+        const unsigned bal = __ballot_sync(kFull, m1 == t);
+        if (lane == __ffs(bal) - 1) {
+            m1 = m2;
+            m2 = 0u;
+        }
+    }
+    return t;
+}
+
+// Each warp's bound for a top-kk selection into sh.vt[s][warp] from its
+// lanes' two largest keys (a0 >= a1 of selection 0, b0 >= b1 of selection 1).
+// No barrier.
+__device__ __forceinline__ void warp_bounds(uint32_t a0, uint32_t a1, uint32_t b0, uint32_t b1,
+                                            int ns, int kk, SelShared &sh) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int j = (kk + kWarps - 1) / kWarps;
-    uint32_t t0 = 0u, t1 = 0u;
-    if (j <= 32) warp_jth_largest2(vm0, vm1, j, &t0, &t1);
+    const uint32_t t0 = j <= 32 ? warp_jth_top2(a0, a1, j) : 0u;
+    const uint32_t t1 = ns > 1 && j <= 32 ? warp_jth_top2(b0, b1, j) : 0u;
     if (lane == 0) {
         sh.vt[0][warp] = t0;
         sh.vt[1][warp] = t1;
@@ -280,17 +283,16 @@ __device__ void compact(const uint32_t *key0, const uint32_t *key1, int n, uint3
 // with a barrier.
 __device__ void tighten(int s, int c, int kk, int slot_out, SelShared &sh) {
     u64 mine[kPerThread];
-    uint32_t vm = 0;
+    uint32_t m1 = 0u, m2 = 0u;
 #pragma unroll
     for (int q = 0; q < kPerThread; ++q) {
         const int f = threadIdx.x + q * kThreads;
         mine[q] = f < c ? sh.cand[s][f] : 0ull;
-        vm = max(vm, key_of(mine[q]));
+        top2(key_of(mine[q]), m1, m2);
     }
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int j = (kk + kWarps - 1) / kWarps;
-    uint32_t tw = 0u, unused;
-    if (j <= 32) warp_jth_largest2(vm, 0u, j, &tw, &unused);
+    const uint32_t tw = j <= 32 ? warp_jth_top2(m1, m2, j) : 0u;
     if (lane == 0) sh.vt[s][warp] = tw;
     __syncthreads();   // also: every list entry has been read
     const uint32_t tau = block_bound(s, sh);
@@ -347,6 +349,12 @@ __device__ __forceinline__ void rank_list(const u64 *list, int c, int kk, u64 *w
     }
 }
 
+// Prefetch of [ptr, ptr + bytes) into L2, one 128-byte line per request.
+__device__ __forceinline__ void prefetch_l2(const void *ptr, uint32_t bytes) {
+    const char *c = static_cast<const char *>(ptr);
+    for (uint32_t o = 0; o < bytes; o += 128) asm volatile("prefetch.global.L2 [%0];" ::"l"(c + o));
+}
+
 struct SelLayout {
     float *qv;          // [2][D_k] row and column query of this (token, head)
     uint32_t *key0;     // [max(K, k*k)] axis-0 keys, then the g keys
@@ -388,11 +396,12 @@ __device__ SelLayout carve(const Dims &d, unsigned char *base) {
 }
 
 // Loads the rank-1 score keys of both axes (Eq. 6-7, written by the scoring
-// kernel) into shared memory and returns this thread's maxima; all loads of
-// a round are issued before any store.
+// kernel) into shared memory and returns this thread's two largest of each
+// axis (padding reads as 0, below every key); all loads of a round are
+// issued before any store.
 __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1, int K,
-                                          const SelLayout &L, uint32_t *vm0, uint32_t *vm1) {
-    uint32_t m0 = 0, m1 = 0;
+                                          const SelLayout &L, uint32_t (&top)[2][2]) {
+    uint32_t a1 = 0u, a2 = 0u, b1 = 0u, b2 = 0u;
     if ((K & 3) == 0) {
         const uint4 *V0 = reinterpret_cast<const uint4 *>(A0);
         const uint4 *V1 = reinterpret_cast<const uint4 *>(A1);
@@ -414,8 +423,14 @@ __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1
                     S0[i] = a[q];
                     S1[i] = c[q];
                 }
-                m0 = max(m0, max4(a[q]));
-                m1 = max(m1, max4(c[q]));
+                top2(a[q].x, a1, a2);
+                top2(a[q].y, a1, a2);
+                top2(a[q].z, a1, a2);
+                top2(a[q].w, a1, a2);
+                top2(c[q].x, b1, b2);
+                top2(c[q].y, b1, b2);
+                top2(c[q].z, b1, b2);
+                top2(c[q].w, b1, b2);
             }
         }
     } else {
@@ -435,13 +450,15 @@ __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1
                     L.key0[i] = a[q];
                     L.key1[i] = c[q];
                 }
-                m0 = max(m0, a[q]);
-                m1 = max(m1, c[q]);
+                top2(a[q], a1, a2);
+                top2(c[q], b1, b2);
             }
         }
     }
-    *vm0 = m0;
-    *vm1 = m1;
+    top[0][0] = a1;
+    top[0][1] = a2;
+    top[1][0] = b1;
+    top[1][1] = b2;
 }
 
 // The 2k axis survivors, one group of G lanes each: the survivor's place in
@@ -558,9 +575,12 @@ __global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
     const uint32_t *A1 = A0 + K;
 
     if (threadIdx.x < 8) sh.cnt[threadIdx.x] = 0;
-    // C of this head and the row/column query of this (token, head), summed
-    // over its D_i splits: loaded before the keys, stored after them
+    // C of this head (a weight: read before the dependency wait) and the
+    // row/column query of this (token, head), summed over its D_i splits:
+    // loaded before the keys, stored after them
     const float core_e = threadIdx.x < r * r ? p.core[(int64_t)h * r * r + threadIdx.x] : 0.f;
+    pdl_wait();
+    pdl_trigger();
     const int HD = d.H * d.d_k;
     const int64_t split_stride = (int64_t)d.A * d.B * HD;
     auto q_src = [&](int e) {
@@ -577,14 +597,14 @@ __global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
     const bool one_split = d.q_splits == 1;
     float q0 = 0.f;
     if (threadIdx.x < 2 * d.d_k) q0 = one_split ? *q_src(threadIdx.x) : q_of(threadIdx.x);
-    uint32_t vm0, vm1;
-    load_keys(A0, A1, K, L, &vm0, &vm1);
+    uint32_t top[2][2];
+    load_keys(A0, A1, K, L, top);
     if (threadIdx.x < r * r) sh.core[threadIdx.x] = core_e;
     if (threadIdx.x < 2 * d.d_k) L.qv[threadIdx.x] = q0;
     for (int e = threadIdx.x + kThreads; e < 2 * d.d_k; e += kThreads) L.qv[e] = q_of(e);
 
     // Eq. 8-9: top-k of both axes
-    warp_bounds(vm0, vm1, k, sh);
+    warp_bounds(top[0][0], top[0][1], top[1][0], top[1][1], 2, k, sh);
     __syncthreads();
     compact<2>(L.key0, L.key1, K, block_bound(0, sh), block_bound(1, sh), sh, kCntAxis,
                kCntAxis + 1);
@@ -603,7 +623,7 @@ __global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
 
     // Eq. 10: g(i,j) = sum_b R[i][b] S_col[b,j] on I x J, R = S_row^T C
     const int k2 = k * k;
-    uint32_t vmg = 0;
+    uint32_t g1 = 0u, g2 = 0u;
     {
         const int dii = kThreads / k, djj = kThreads % k;   // (ii, jj) step per c += kThreads
         int ii = threadIdx.x / k, jj = threadIdx.x % k;
@@ -612,13 +632,13 @@ __global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
             for (int be = 0; be < r; ++be) g = fmaf(L.R[ii * r + be], L.scol[jj * r + be], g);
             const uint32_t kg = f2ord(g);
             L.key0[c] = kg;
-            vmg = max(vmg, kg);
+            top2(kg, g1, g2);
             ii += dii;
             jj += djj;
             if (jj >= k) { jj -= k; ++ii; }
         }
     }
-    warp_bounds(vmg, 0u, m, sh);
+    warp_bounds(g1, g2, 0u, 0u, 1, m, sh);
     __syncthreads();
     compact<1>(L.key0, nullptr, k2, block_bound(0, sh), 0u, sh, kCntTop, kCntTop);
     __syncthreads();
@@ -640,6 +660,7 @@ __global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
     }
     const int64_t base = ((int64_t)b * d.H + h) * m;
     const uint32_t N = (uint32_t)d.N;
+    const uint32_t row_bytes = (uint32_t)d.d_v * (d.dtype == ULTRAMEM_BF16 ? 2u : 4u);
     for (int e = threadIdx.x; e < m; e += kThreads) {
         const u64 wc = sh.fwin[e];
         const int c = (int)pos_of(wc);
@@ -649,7 +670,11 @@ __global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
         const float w = d.act == ULTRAMEM_ACT_SOFTMAX ? __expf(g - gmax) / sh.scalar : g;
         const uint32_t vs = (uint32_t)shuffle_address(d, p.perm, v);   // Eq. 14, < M < 2^32
         const uint32_t pb = vs / N;
-        p.sel_row[base + e] = (int32_t)(vs - pb * N);
+        const uint32_t prow = vs - pb * N;
+        // the gather will read this value row: start moving it into L2
+        prefetch_l2(static_cast<const unsigned char *>(p.values) + (size_t)prow * row_bytes,
+                    row_bytes);
+        p.sel_row[base + e] = (int32_t)prow;
         p.sel_p[base + e] = (int32_t)pb;
         p.sel_w[base + e] = w;
         if (p.idx_out) p.idx_out[base + e] = (int64_t)v;
@@ -684,11 +709,11 @@ __global__ void slots_kernel(Dims d, Ptrs p) {
 size_t select_smem_bytes(const Dims &d) { return sel_offsets(d).total; }
 
 cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st) {
+    const size_t smem = select_smem_bytes(d);
     if (d.dtype == ULTRAMEM_BF16)
-        select_kernel<__nv_bfloat16><<<d.B * d.H, kThreads, select_smem_bytes(d), st>>>(d, p);
-    else
-        select_kernel<float><<<d.B * d.H, kThreads, select_smem_bytes(d), st>>>(d, p);
-    return cudaGetLastError();
+        return launch_kernel(d.pdl, select_kernel<__nv_bfloat16>, d.B * d.H, kThreads, smem, st,
+                             d, p);
+    return launch_kernel(d.pdl, select_kernel<float>, d.B * d.H, kThreads, smem, st, d, p);
 }
 
 cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream_t st) {

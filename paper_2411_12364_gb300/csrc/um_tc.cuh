@@ -192,6 +192,22 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar) {
         : "memory");
 }
 
+// ---- thread-block cluster ---------------------------------------------------
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// all threads of every CTA of the cluster; memory writes before it (shared
+// or global) are visible to reads after it anywhere in the cluster
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile(
+        "barrier.cluster.arrive.release.aligned;\n\t"
+        "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 __host__ __device__ constexpr uint32_t tmem_cols_for(uint32_t n) {
     uint32_t c = 32;
     while (c < n) c <<= 1;

@@ -12,10 +12,20 @@
 // key tile is multiplied by all three, accumulating in fp32.  Keys are bf16
 // and enter exactly.
 //
-// One CTA (4 warps) computes one 128 x N tile: warp 0 lane 0 issues the TMA
-// loads of a 4-stage ring, warp 1 lane 0 issues the MMAs, and all four warps
-// then read TMEM (row i = lane i) for the epilogue.  Every mbarrier wait is
+// One CTA (8 warps) computes one 128 x N tile: warp 0 lane 0 issues the TMA
+// loads of a 4-stage ring, warp 1 lane 0 issues the MMAs, and all eight warps
+// then read TMEM for the epilogue (row i = lane i; warps w and w + 4 share a
+// lane quarter and take alternate 32-column chunks).  Every mbarrier wait is
 // bounded (~1 s); a timeout sets the layer's error word.
+//
+// Split-K (S1 and S9 at small batches, so that enough SMs stream the
+// weights): the S CTAs of one tile form a thread-block cluster, used as a
+// barrier that all of them are guaranteed to reach together.  Each writes
+// its fp32 partial tile to a global (L2-resident) buffer; after the cluster
+// barrier (release / acquire) each CTA adds a slice of the tile's columns
+// over the S partials in split order (deterministic) and writes the result.
+// (Reading the partials from the peers' shared memory instead measured
+// several times slower on GB300.)
 #include <cudaTypedefs.h>
 
 #include "um_internal.cuh"
@@ -26,9 +36,10 @@ namespace {
 
 using namespace tc;
 
-constexpr int kThreads = 128;
+constexpr int kThreads = 256;
 constexpr int kMaxStages = 4;
 constexpr int kMaxAcc = 4;
+constexpr int kMaxSplits = 8;                // split-K CTAs per tile: one portable cluster
 constexpr size_t kSmemBudget = 225 * 1024;   // leaves room for static smem
 
 struct Tile {
@@ -66,7 +77,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n_tile = op.n_tile;
     const uint32_t b_bytes = (uint32_t)n_tile * 128;
     const uint32_t stage_bytes = kTileABytes + NSPLIT * b_bytes;
-    const uint32_t ncols = tmem_cols_for((uint32_t)(op.n_acc * n_tile));
+    // the epilogue reads 32 columns at a time: cover the last such read
+    const uint32_t ncols =
+        tmem_cols_for((uint32_t)((op.n_acc - 1) * n_tile + ((n_tile - 1) / 32) * 32 + 32));
     const CUtensorMap *mapA = t.a_sel ? &mapA1 : &mapA0;
     const int kStages = op.stages;
 
@@ -80,11 +93,44 @@ __global__ void __launch_bounds__(kThreads, 1)
         prefetch_tensormap(mapA);
         prefetch_tensormap(&mapB);
     }
+    __syncthreads();
+
+    // The A operand is a weight: the first ring stages of it are requested
+    // before the dependency wait, so that under programmatic dependent
+    // launch they stream while the previous kernel finishes.  Each stage's
+    // barrier expects its A and B bytes; B follows after the wait.
+    const int pre = min(kStages, t.nkb);
+    auto load_a = [&](int it) {
+        const int s = it % kStages;
+        uint8_t *sa = ring + (size_t)s * stage_bytes;
+        mbar_arrive_expect_tx(&full[s], stage_bytes);
+        const int kx = (t.kb0 + it) * kBlockK;
+        if (t.a_z >= 0) tma_load_3d(sa, mapA, &full[s], kx, t.m0, t.a_z);
+        else tma_load_2d(sa, mapA, &full[s], kx, t.m0);
+    };
+    auto load_b = [&](int it) {
+        const int s = it % kStages;
+        uint8_t *sa = ring + (size_t)s * stage_bytes;
+        const int kx = (t.kb0 + it) * kBlockK;
+#pragma unroll
+        for (int j = 0; j < NSPLIT; ++j) {
+            uint8_t *sb = sa + kTileABytes + j * b_bytes;
+            const int bx = j * op.b_split_stride + kx;
+            if (t.b_z >= 0) tma_load_3d(sb, &mapB, &full[s], bx, t.n0, t.b_z);
+            else tma_load_2d(sb, &mapB, &full[s], bx, t.n0);
+        }
+    };
+    if (threadIdx.x == 0)
+        for (int it = 0; it < pre; ++it) load_a(it);
+    pdl_wait();
+    // TMEM is taken only after the wait: a kernel that waits never holds
+    // columns that a CTA of an earlier kernel could still be waiting for
     if (warp == 0) tmem_alloc(&tmem_slot, ncols);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
+    pdl_trigger();
 
     // Roles: lane 0 of warp 0 produces, lane 0 of warp 1 issues the MMAs; the
     // other lanes of those warps wait at __syncwarp (not spinning on the
@@ -92,25 +138,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
       if (lane == 0) {
         // producer: TMA loads of A (128 x 64) and NSPLIT B tiles (N x 64)
-        int it = 0;
+        for (int it = 0; it < pre; ++it) load_b(it);
+        int it = pre;
         for (; it < t.nkb; ++it) {
             const int s = it % kStages;
-            if (it >= kStages && !mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
+            if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
                 atomicOr(op.err, kErrTimeout);
                 break;
             }
-            uint8_t *sa = ring + (size_t)s * stage_bytes;
-            mbar_arrive_expect_tx(&full[s], stage_bytes);
-            const int kx = (t.kb0 + it) * kBlockK;
-            if (t.a_z >= 0) tma_load_3d(sa, mapA, &full[s], kx, t.m0, t.a_z);
-            else tma_load_2d(sa, mapA, &full[s], kx, t.m0);
-#pragma unroll
-            for (int j = 0; j < NSPLIT; ++j) {
-                uint8_t *sb = sa + kTileABytes + j * b_bytes;
-                const int bx = j * op.b_split_stride + kx;
-                if (t.b_z >= 0) tma_load_3d(sb, &mapB, &full[s], bx, t.n0, t.b_z);
-                else tma_load_2d(sb, &mapB, &full[s], bx, t.n0);
-            }
+            load_a(it);
+            load_b(it);
         }
         // loads still in flight (only after a timeout) land before exit
         for (int j = (it > kStages ? it - kStages : 0); j < it; ++j)
@@ -162,11 +199,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!mbar_wait(&accbar, 0)) atomicOr(op.err, kErrTimeout);
     tc_fence_after();
 
-    // epilogue: thread = tile row (TMEM lane); each chunk of 16 columns of
-    // every accumulator is read with one wait per 32 columns
-    const int row = warp * 32 + lane;
-    const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
-    for (int c0 = 0; c0 < n_tile; c0 += 32) {
+    // epilogue: thread = tile row (TMEM lane); warp halves take alternate
+    // 32-column chunks, read with one wait for every accumulator.
+    constexpr int kGroups = kThreads / 128;   // warps sharing each TMEM lane quarter
+    const int quad = warp & 3, whalf = warp >> 2;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
+    const int S = op.cluster_splits();
+    for (int c0 = whalf * 32; c0 < n_tile; c0 += 32 * kGroups) {
         uint32_t r[kMaxAcc][32];
 #pragma unroll
         for (int a = 0; a < kMaxAcc; ++a)
@@ -180,20 +220,49 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int a = 0; a < kMaxAcc; ++a)
 #pragma unroll
                 for (int i = 0; i < 16; ++i) v[a][i] = __uint_as_float(r[a][half * 16 + i]);
-            op.store(t, row, c0 + half * 16, v);
+            if (S > 1) op.store_partial(t, row, c0 + half * 16, v);
+            else op.store(t, row, c0 + half * 16, v);
         }
     }
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, ncols);
+    if (S > 1) {
+        cluster_sync();   // every partial of the tile is written and visible
+        // this CTA's columns (a multiple of 4 per warp group), split between
+        // the groups of warps
+        const int per = (((n_tile + S - 1) / S) + 4 * kGroups - 1) & ~(4 * kGroups - 1);
+        const int nb = (int)cluster_ctarank() * per + whalf * (per / kGroups);
+        const int ne = min(n_tile, nb + per / kGroups);
+        for (int n = nb; n < ne; n += 4) {
+            float part[4][kMaxSplits];
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+#pragma unroll
+                for (int q = 0; q < kMaxSplits; ++q)
+                    part[e][q] = q < S ? op.load_partial(t, q, row, n + e) : 0.f;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                float sum = 0.f;
+#pragma unroll
+                for (int q = 0; q < kMaxSplits; ++q)
+                    if (q < S) sum += part[e][q];
+                op.store_sum(t, row, n + e, sum);
+            }
+        }
+    }
 }
 
 // ---- S1: query projection, split over D_i --------------------------------
+// q = W_q x is written in fp32 (q_part, split 0) for the selection and as
+// the three bf16 terms of the scoring contraction (qs).
 struct QueryOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
-    int B, HD, A, a, splits, kb_total;
-    float *q_part;   // [splits][A][B][HD]
+    int B, HD, A, a, splits, kb_total, H, d_k, Bmax;
+    float *q_part;        // [splits][A][B][HD]; the result is split 0
+    __nv_bfloat16 *qs;    // [A*H][Bmax][3][D_k]
+    __device__ int cluster_splits() const { return splits; }
     __device__ Tile tile() const {
         Tile t;
         t.m0 = blockIdx.x * kTileM;
@@ -207,15 +276,45 @@ struct QueryOp {
         t.nkb = max(0, min(kb_total, t.kb0 + per) - t.kb0);
         return t;
     }
+    __device__ void put(int m, int n, float q) const {
+        q_part[((int64_t)a * B + n) * HD + m] = q;
+        const __nv_bfloat16 q1 = __float2bfloat16_rn(q);
+        const float r1 = q - __bfloat162float(q1);
+        const __nv_bfloat16 q2 = __float2bfloat16_rn(r1);
+        const float r2 = r1 - __bfloat162float(q2);
+        const __nv_bfloat16 q3 = __float2bfloat16_rn(r2);
+        const int h = m / d_k, c = m - h * d_k;
+        __nv_bfloat16 *dst = qs + (((int64_t)(a * H + h) * Bmax + n) * 3) * d_k + c;
+        dst[0] = q1;
+        dst[d_k] = q2;
+        dst[2 * d_k] = q3;
+    }
     __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
         const int m = t.m0 + row;
         if (m >= HD) return;
-        const int split = blockIdx.z;
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
             const int n = t.n0 + c + j;
-            if (n < B) q_part[(((int64_t)split * A + a) * B + n) * HD + m] = t.nkb ? v[0][j] : 0.f;
+            if (n < B) put(m, n, t.nkb ? v[0][j] : 0.f);
         }
+    }
+    __device__ void store_sum(const Tile &t, int row, int c, float q) const {
+        const int m = t.m0 + row, n = t.n0 + c;
+        if (m < HD && n < B) put(m, n, q);
+    }
+    // split-K partials: q_part[split][a][n][m] (the sum later replaces split 0)
+    __device__ void store_partial(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
+        const int m = t.m0 + row;
+        if (m >= HD) return;
+        float *dst = q_part + (((int64_t)blockIdx.z * A + a) * B + t.n0 + c) * HD + m;
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+            if (t.n0 + c + j < B) dst[(int64_t)j * HD] = t.nkb ? v[0][j] : 0.f;
+    }
+    __device__ float load_partial(const Tile &t, int split, int row, int c) const {
+        const int m = t.m0 + row, n = t.n0 + c;
+        if (m >= HD || n >= B) return 0.f;
+        return __ldcg(q_part + (((int64_t)split * A + a) * B + n) * HD + m);
     }
 };
 
@@ -230,6 +329,10 @@ struct ScoreOp {
     int B, H, K, A, kb_total;
     const float *u, *t;   // [H][R]
     uint32_t *akey;       // [B][H][2][K]
+    __device__ int cluster_splits() const { return 1; }
+    __device__ void store_sum(const Tile &, int, int, float) const {}
+    __device__ void store_partial(const Tile &, int, int, float (&)[kMaxAcc][16]) const {}
+    __device__ float load_partial(const Tile &, int, int, int) const { return 0.f; }
     __device__ Tile tile() const {
         Tile tl;
         const int h = blockIdx.z >> 1, axis = blockIdx.z & 1;
@@ -250,28 +353,42 @@ struct ScoreOp {
         float cf[R];
 #pragma unroll
         for (int a = 0; a < R; ++a) cf[a] = coef[a];
+        const int n0 = tl.n0 + c;
+        const int64_t tok_stride = (int64_t)H * 2 * K;   // akey elements per token
+        uint32_t *dst = akey + ((int64_t)n0 * H + h) * 2 * K + (int64_t)axis * K + i;
+        const int nj = min(16, B - n0);
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
-            const int n = tl.n0 + c + j;
-            if (n >= B) break;
+            if (j >= nj) break;
             float a = cf[0] * v[0][j];
 #pragma unroll
             for (int al = 1; al < R; ++al) a = fmaf(cf[al], v[al][j], a);
-            akey[(((int64_t)n * H + h) * 2 + axis) * K + i] = f2ord(a);
+            dst[j * tok_stride] = f2ord(a);
         }
     }
 };
 
 // ---- S9: IVE projection, split over E*D_v --------------------------------
-// With one split the tile is written as bf16 output; with several, each
-// split writes fp32 partial sums part[split][n][o] that a second kernel adds
-// in split order.
 struct ProjOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
     int B, d_out, kb_total, splits;
     __nv_bfloat16 *out;   // [B][d_out]
-    float *part;          // [splits][B][d_out]
+    float *part;          // [splits][B][d_out] split-K partials
+    __device__ int cluster_splits() const { return splits; }
+    __device__ void store_partial(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
+        const int o = t.m0 + row;
+        if (o >= d_out) return;
+        float *dst = part + ((int64_t)blockIdx.z * B + t.n0 + c) * d_out + o;
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+            if (t.n0 + c + j < B) dst[(int64_t)j * d_out] = t.nkb ? v[0][j] : 0.f;
+    }
+    __device__ float load_partial(const Tile &t, int split, int row, int c) const {
+        const int o = t.m0 + row, n = t.n0 + c;
+        if (o >= d_out || n >= B) return 0.f;
+        return __ldcg(part + ((int64_t)split * B + n) * d_out + o);
+    }
     __device__ Tile tile() const {
         Tile t;
         t.m0 = blockIdx.x * kTileM;
@@ -291,42 +408,14 @@ struct ProjOp {
         for (int j = 0; j < 16; ++j) {
             const int n = t.n0 + c + j;
             if (n >= B) break;
-            if (splits == 1)
-                out[(int64_t)n * d_out + o] = __float2bfloat16_rn(v[0][j]);
-            else
-                part[((int64_t)blockIdx.z * B + n) * d_out + o] = t.nkb ? v[0][j] : 0.f;
+            out[(int64_t)n * d_out + o] = __float2bfloat16_rn(t.nkb ? v[0][j] : 0.f);
         }
     }
-};
-
-// ---- q = sum of split partials, then the three-term bf16 split -------------
-// The fp32 sum is also written back over split 0, so that later stages read
-// one partial.
-// qs layout: [A*H][Bmax][3][D_k] (token rows of 3*D_k), the B operand of S2.
-__global__ void qsplit_kernel(Dims d, float *q_part, __nv_bfloat16 *__restrict__ qs,
-                              int splits, int Bmax) {
-    const int HD = d.H * d.d_k;
-    const int64_t total = (int64_t)d.A * d.B * HD;
-    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
-         e += (int64_t)gridDim.x * blockDim.x) {
-        const int o = (int)(e % HD);
-        const int64_t ab = e / HD;
-        const int b = (int)(ab % d.B), a = (int)(ab / d.B);
-        float q = 0.f;
-        for (int s = 0; s < splits; ++s) q += q_part[(((int64_t)s * d.A + a) * d.B + b) * HD + o];
-        if (splits > 1) q_part[e] = q;   // the summed query replaces split 0 (same thread)
-        const __nv_bfloat16 q1 = __float2bfloat16_rn(q);
-        const float r1 = q - __bfloat162float(q1);
-        const __nv_bfloat16 q2 = __float2bfloat16_rn(r1);
-        const float r2 = r1 - __bfloat162float(q2);
-        const __nv_bfloat16 q3 = __float2bfloat16_rn(r2);
-        const int h = o / d.d_k, c = o % d.d_k;
-        __nv_bfloat16 *dst = qs + (((int64_t)(a * d.H + h) * Bmax + b) * 3) * d.d_k + c;
-        dst[0] = q1;
-        dst[d.d_k] = q2;
-        dst[2 * d.d_k] = q3;
+    __device__ void store_sum(const Tile &t, int row, int c, float v) const {
+        const int o = t.m0 + row, n = t.n0 + c;
+        if (o < d_out && n < B) out[(int64_t)n * d_out + o] = __float2bfloat16_rn(v);
     }
-}
+};
 
 // dst[c][r] = src[r][c] for a rows x cols bf16 matrix (32 x 32 tiles)
 __global__ void transpose_kernel(const __nv_bfloat16 *__restrict__ src,
@@ -396,13 +485,16 @@ int tc_n_tile(int B, int n_acc) {
     return n < cap ? n : cap;
 }
 
+// grid.z = the split count, which is also the cluster's z extent when > 1
 template <int NSPLIT, class Op>
 static cudaError_t launch_gemm(dim3 grid, const CUtensorMap &a0, const CUtensorMap &a1,
-                               const CUtensorMap &b, Op op, int nkb, cudaStream_t st) {
+                               const CUtensorMap &b, Op op, int nkb, bool pdl,
+                               cudaStream_t st) {
     op.stages = stages_for(NSPLIT, op.n_tile, nkb);
-    const size_t smem = 1024 + (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile);
-    tc_gemm_kernel<NSPLIT, Op><<<grid, kThreads, smem, st>>>(a0, a1, b, op);
-    return cudaGetLastError();
+    size_t ring = (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile);
+    const size_t smem = 1024 + ring;
+    return launch_kernel(pdl, grid.z > 1 ? grid.z : 1u, tc_gemm_kernel<NSPLIT, Op>, grid,
+                         kThreads, smem, st, a0, a1, b, op);
 }
 
 template <int NSPLIT, class Op> static cudaError_t allow_smem() {
@@ -421,10 +513,11 @@ cudaError_t configure_tc() {
 }
 
 cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int splits,
-                            cudaStream_t st) {
+                            __nv_bfloat16 *qs, int Bmax, cudaStream_t st) {
     const int HD = d.H * d.d_k;
     const int n_tile = tc_n_tile(d.B, 1);
     const int kb_total = (d.d_in + kBlockK - 1) / kBlockK;
+    if (splits > kMaxSplits) return cudaErrorInvalidValue;
     for (int a = 0; a < d.A; ++a) {
         QueryOp op;
         op.n_tile = n_tile;
@@ -438,23 +531,18 @@ cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int 
         op.a = a;
         op.splits = splits;
         op.kb_total = kb_total;
+        op.H = d.H;
+        op.d_k = d.d_k;
+        op.Bmax = Bmax;
         op.q_part = p.q_part;
+        op.qs = qs;
         dim3 grid((HD + kTileM - 1) / kTileM, (d.B + n_tile - 1) / n_tile, splits);
         const int per = (kb_total + splits - 1) / splits;
-        cudaError_t e =
-            launch_gemm<1>(grid, a == 0 ? mp.w_q : mp.w_q_col, mp.w_q, mp.x, op, per, st);
+        cudaError_t e = launch_gemm<1>(grid, a == 0 ? mp.w_q : mp.w_q_col, mp.w_q, mp.x, op, per,
+                                       false, st);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
-}
-
-cudaError_t launch_qsplit(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, int splits, int Bmax,
-                          cudaStream_t st) {
-    const int64_t total = (int64_t)d.A * d.B * d.H * d.d_k;
-    int blocks = (int)((total + 255) / 256);
-    if (blocks > 2048) blocks = 2048;
-    qsplit_kernel<<<blocks, 256, 0, st>>>(d, p.q_part, qs, splits, Bmax);
-    return cudaGetLastError();
 }
 
 template <int R>
@@ -475,7 +563,7 @@ static cudaError_t launch_score_r(const Dims &d, const Ptrs &p, const TcMaps &mp
     op.t = p.t;
     op.akey = p.akey;
     dim3 grid((d.K + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 2 * d.H);
-    return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs, op, op.kb_total, st);
+    return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs, op, op.kb_total, d.pdl, st);
 }
 
 cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
@@ -488,6 +576,7 @@ cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cuda
 }
 
 cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
+    if (d.p_splits > kMaxSplits) return cudaErrorInvalidValue;
     ProjOp op;
     op.n_tile = tc_n_tile(d.B, 1);
     op.n_acc = 1;
@@ -502,9 +591,7 @@ cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaS
     op.part = p.proj_part;
     dim3 grid((d.d_out + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, op.splits);
     const int per = (op.kb_total + op.splits - 1) / op.splits;
-    cudaError_t e = launch_gemm<1>(grid, mp.w_pt, mp.w_pt, mp.acc, op, per, st);
-    if (e == cudaSuccess && op.splits > 1) e = launch_proj_reduce(d, p, st);
-    return e;
+    return launch_gemm<1>(grid, mp.w_pt, mp.w_pt, mp.acc, op, per, d.pdl, st);
 }
 
 }  // namespace um

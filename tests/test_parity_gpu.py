@@ -171,3 +171,73 @@ def test_batch_limits(gpu_lib):
     big = torch.zeros((9, cfg["d_in"]), dtype=torch.bfloat16, device="cuda")
     with pytest.raises(binding.UltraMemError):
         layer.forward(big)
+
+
+def _tied_weights(cfg, rows_tied):
+    """Weights whose first `rows_tied` keys of each axis are one and the same
+    row, so that their rank-1 and exact scores tie exactly."""
+    w = workloads.make_weights(cfg, device="cuda")
+    for name in ("k_row", "k_col"):
+        k = w[name].clone()
+        k[:, :rows_tied, :] = k[:, :1, :]
+        w[name] = k
+    return w
+
+
+def _run_weights(cfg, w, B, gpu_lib):
+    from paper_2411_12364_gb300.binding import UltraMemLayer
+    x = workloads.make_tokens(cfg, B, 0, device="cuda")
+    t = parity.numpy_inputs(cfg, w, x)
+    layer = UltraMemLayer(cfg, dict(w, u=torch.from_numpy(t["u"]), t=torch.from_numpy(t["t"])), B)
+    out, idx, wt = layer.forward(x, with_slots=True)
+    torch.cuda.synchronize()
+    assert layer.check() == 0
+    o_out, o_idx, o_w = oracle.forward(cfg, t, B)
+    parity.compare(cfg, t, np.arange(B), out.float().cpu().numpy(), idx.cpu().numpy(),
+                   wt.cpu().numpy(), o_out, o_idx, o_w)
+    return idx
+
+
+@pytest.mark.parametrize("dtype", [0, 1])
+def test_all_keys_tied(dtype, gpu_lib):
+    """Every key of both axes is the same row: all K = 1200 rank-1 scores tie
+    (more candidates than a list holds, so the exact radix select runs), and
+    all k*k = 1600 Tucker scores tie too.  Ties go to the smaller index: the
+    slots are the first m pairs of rows 0..k-1 x columns 0..k-1."""
+    cfg = workloads.small_config(dtype=dtype, n=600, topk=40, topm=64)
+    K = workloads.keys_per_axis(cfg)
+    w = _tied_weights(cfg, K)
+    idx = _run_weights(cfg, w, 9, gpu_lib).cpu().numpy()
+    k, m = cfg["topk"], cfg["topm"]
+    pairs = np.array([i * K + j for i in range(k) for j in range(k)])[:m]
+    assert (np.sort(idx, axis=-1) == np.sort(pairs)).all()
+
+
+@pytest.mark.parametrize("dtype", [0, 1])
+def test_many_keys_tied(dtype, gpu_lib):
+    """500 of the 1200 keys of each axis tie: for tokens whose tied score is
+    at the top, the candidate list is long but fits (it is tightened before
+    ranking); the others cut through or below the tie."""
+    cfg = workloads.small_config(dtype=dtype, n=600, topk=40, topm=64)
+    _run_weights(cfg, _tied_weights(cfg, 500), 37, gpu_lib)
+
+
+def test_last_launches_counts_each_call(gpu_lib):
+    """The library's kernel count per call: the tensor path runs one query
+    projection per query, score and select (retrieve), then gather and the
+    projection (split-K reduced inside its clusters); the CUDA-core path adds
+    a reduce after each split-K contraction's partials; lookup_reduce runs
+    slots, gather, projection and reduce."""
+    cfg = workloads.small_config(dtype=1)
+    layer, (w, x, t), (out, idx, wt), _ = _run(cfg, 16, gpu_lib)
+    assert layer.last_launches() == 5
+    layer.retrieve(x)
+    assert layer.last_launches() == 3
+    layer.lookup_reduce(idx, wt)
+    assert layer.last_launches() == 4
+    cfg2 = workloads.small_config(dtype=1, share_query=0)
+    layer2, *_ = _run(cfg2, 16, gpu_lib)
+    assert layer2.last_launches() == 6
+    cfg32 = workloads.small_config(dtype=0)
+    layer32, *_ = _run(cfg32, 16, gpu_lib)
+    assert layer32.last_launches() == 6
