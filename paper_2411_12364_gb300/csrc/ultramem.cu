@@ -64,6 +64,14 @@ int query_splits(const ultramem_config &c, int B) {
     return s < 1 ? 1 : s;
 }
 
+// Batches up to this many tokens run the query projection (S1) on CUDA
+// cores (16 weight rows x 8 tokens per CTA, no split-K); larger ones, and
+// the IVE projection at every batch, on tcgen05.  Measured on GB300: at 64
+// tokens the CUDA-core query takes 3.3 us against 8.5 us for the split-K
+// tensor-core one; at 128 tokens (and for the projection, whose weight rows
+// it re-reads once per 8 tokens) it is slower.
+constexpr int kSmallQueryBatch = 64;
+
 // Tensor path split-K: about `target` CTAs stream the weight, at most one
 // portable cluster (8) per tile, whole K blocks.
 int tc_splits(int m_rows, int B, int kdim, int target) {
@@ -333,7 +341,9 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     // earlier work on the stream.
     Dims dd = d;
     dd.pdl = L->profiling ? 0 : 1;
-    if ((e = um::launch_query_tc(d, p, mp, d.q_splits, L->ws.qs, Bmax, st)) != cudaSuccess)
+    const bool small = d.B <= kSmallQueryBatch;
+    if ((e = small ? um::launch_query_small(d, p, L->ws.qs, Bmax, st)
+                   : um::launch_query_tc(d, p, mp, d.q_splits, L->ws.qs, Bmax, st)) != cudaSuccess)
         return from_cuda(e);
     mark(L, 1, st);
     if ((e = um::launch_score_tc(dd, p, mp, st)) != cudaSuccess) return from_cuda(e);
@@ -514,6 +524,7 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
             if (e == cudaSuccess) e = cudaDeviceSynchronize();
         }
         if (e == cudaSuccess) e = um::configure_tc();
+        if (e == cudaSuccess) e = um::configure_small();
         bool ok = e == cudaSuccess;
         const uint64_t HD = (uint64_t)H * cfg->d_k;
         ok = ok && um::tc_encode(&L->maps.w_q, w->w_q, cfg->d_in, HD, 1, 128, 2);

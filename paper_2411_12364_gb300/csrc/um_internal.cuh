@@ -72,6 +72,10 @@ cudaError_t configure_tc();
 cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int splits,
                             __nv_bfloat16 *qs, int Bmax, cudaStream_t st);
 cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st);
+// small batches: S1 on CUDA cores, 16 weight rows x 8 tokens per CTA
+cudaError_t configure_small();
+cudaError_t launch_query_small(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, int Bmax,
+                               cudaStream_t st);
 cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st);
 cudaError_t launch_transpose_bf16(const void *src, void *dst, int rows, int cols,
                                   cudaStream_t st);

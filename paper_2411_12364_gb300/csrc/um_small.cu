@@ -1,0 +1,196 @@
+// um_small.cu -- the query projection (S1) for small token batches, on CUDA
+// cores.
+//
+// At decode batches the contraction is a few hundred KB of weights times a
+// handful of tokens.  The tensor-core kernel needs 128 weight rows
+// per CTA, which leaves too few CTAs to stream the weights unless K is split,
+// and the split-K reduction then dominates.  Here a CTA takes 16 weight rows
+// x 8 tokens: its operand rows (bf16, K contiguous) arrive by 1-D bulk
+// copies (TMA) into shared memory in one round trip, 256 threads compute the
+// 128 dot products (2 x 2 outputs per thread over one of 8 interleaved
+// K-slices, then a fixed 3-step shuffle sum: deterministic), and the
+// epilogue writes the result in place.  No partial sums leave the CTA.
+//
+//   Y[n][o] = sum_d x[n][d] W_q[o][d]  -> q (fp32) and its 3-term bf16 split
+// (The tile re-reads each weight row once per 8 tokens, so from about 128
+// tokens on, and for the larger IVE projector, the tensor-core kernel wins.)
+#include "um_internal.cuh"
+#include "um_tc.cuh"
+
+namespace um {
+namespace {
+
+using namespace tc;
+
+constexpr int kThreads = 256;
+constexpr int kRows = 16;        // weight rows per CTA
+constexpr int kToks = 8;         // tokens per CTA
+constexpr int kChunk = 2048;     // K elements staged per round (4 KB per row)
+constexpr int kSlices = 8;       // interleaved K slices per output block
+
+struct SmallArgs {
+    const __nv_bfloat16 *W;      // [O][Kd]
+    const __nv_bfloat16 *X;      // [N][Kd]
+    int O, N, Kd;
+    int *err;
+    // S1 epilogue
+    float *q;                    // [A][B][HD] at a * B * HD (split 0 of q_part)
+    __nv_bfloat16 *qs;           // [A*H][Bmax][3][D_k] at a * H * Bmax * 3 * D_k
+    int d_k, Bmax;
+};
+
+struct QueryEp {
+    __device__ static void put(const SmallArgs &g, int o, int n, float v) {
+        g.q[(int64_t)n * g.O + o] = v;
+        const __nv_bfloat16 q1 = __float2bfloat16_rn(v);
+        const float r1 = v - __bfloat162float(q1);
+        const __nv_bfloat16 q2 = __float2bfloat16_rn(r1);
+        const float r2 = r1 - __bfloat162float(q2);
+        const __nv_bfloat16 q3 = __float2bfloat16_rn(r2);
+        const int h = o / g.d_k, c = o - h * g.d_k;
+        __nv_bfloat16 *dst = g.qs + (((int64_t)h * g.Bmax + n) * 3) * g.d_k + c;
+        dst[0] = q1;
+        dst[g.d_k] = q2;
+        dst[2 * g.d_k] = q3;
+    }
+};
+
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes,
+                                         uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void bf16x8(uint4 v, float (&f)[8]) {
+    const uint32_t u[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        f[2 * q] = __uint_as_float(u[q] << 16);
+        f[2 * q + 1] = __uint_as_float(u[q] & 0xffff0000u);
+    }
+}
+
+template <class Ep>
+__global__ void __launch_bounds__(kThreads) small_gemm_kernel(SmallArgs g) {
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    __shared__ __align__(8) uint64_t bar;
+    const int stride = min(kChunk, g.Kd);                                // elements per staged row
+    __nv_bfloat16 *Ws = reinterpret_cast<__nv_bfloat16 *>(smem_raw);   // [kRows][stride]
+    __nv_bfloat16 *Xs = Ws + kRows * stride;                             // [kToks][stride]
+    const int o0 = blockIdx.x * kRows, n0 = blockIdx.y * kToks;
+    const int nrows = min(kRows, g.O - o0), ntoks = min(kToks, g.N - n0);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int blk = warp * 4 + (lane >> 3), s = lane & 7;
+    const int r0 = 2 * (blk & 7), t0 = 2 * (blk >> 3);   // 8 row pairs x 4 token pairs
+
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    float acc[2][2] = {};
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int k0 = 0; k0 < g.Kd; k0 += kChunk) {
+        const int kc = min(kChunk, g.Kd - k0);
+        const uint32_t row_bytes = (uint32_t)kc * 2;
+        if (threadIdx.x == 0) {
+            // weights first (no dependency), the tokens after the wait
+            mbar_arrive_expect_tx(&bar, row_bytes * (uint32_t)(nrows + ntoks));
+            for (int r = 0; r < nrows; ++r)
+                bulk_g2s(Ws + r * stride, g.W + (int64_t)(o0 + r) * g.Kd + k0, row_bytes, &bar);
+        }
+        if (k0 == 0) pdl_wait();
+        if (threadIdx.x == 0)
+            for (int t = 0; t < ntoks; ++t)
+                bulk_g2s(Xs + t * stride, g.X + (int64_t)(n0 + t) * g.Kd + k0, row_bytes, &bar);
+        const bool timed_out = !mbar_wait(&bar, phase);
+        if (__syncthreads_or(timed_out)) {   // block-uniform
+            // give the copies in flight one more bounded wait before the
+            // shared memory is released, then stop
+            if (threadIdx.x == 0) atomicOr(g.err, kErrTimeout);
+            mbar_wait(&bar, phase);
+            ok = false;
+            break;
+        }
+        phase ^= 1;
+        {
+            // rows/tokens past the edge read whatever the buffer holds; their
+            // results are never written
+            const __nv_bfloat16 *w0 = Ws + r0 * stride, *w1 = w0 + stride;
+            const __nv_bfloat16 *x0 = Xs + t0 * stride, *x1 = x0 + stride;
+#pragma unroll 4
+            for (int kk = s * 8; kk < kc; kk += kSlices * 8) {
+                float a0[8], a1[8], b0[8], b1[8];
+                bf16x8(*reinterpret_cast<const uint4 *>(w0 + kk), a0);
+                bf16x8(*reinterpret_cast<const uint4 *>(w1 + kk), a1);
+                bf16x8(*reinterpret_cast<const uint4 *>(x0 + kk), b0);
+                bf16x8(*reinterpret_cast<const uint4 *>(x1 + kk), b1);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    acc[0][0] = fmaf(a0[e], b0[e], acc[0][0]);
+                    acc[0][1] = fmaf(a0[e], b1[e], acc[0][1]);
+                    acc[1][0] = fmaf(a1[e], b0[e], acc[1][0]);
+                    acc[1][1] = fmaf(a1[e], b1[e], acc[1][1]);
+                }
+            }
+        }
+        __syncthreads();   // the buffers are refilled by the next round
+    }
+    pdl_trigger();
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+        for (int j = 0; j < 2; ++j)
+#pragma unroll
+            for (int off = 1; off < kSlices; off <<= 1)
+                acc[i][j] += __shfl_xor_sync(0xffffffffu, acc[i][j], off);
+    if (s == 0 && ok) {
+#pragma unroll
+        for (int i = 0; i < 2; ++i)
+#pragma unroll
+            for (int j = 0; j < 2; ++j)
+                if (r0 + i < nrows && t0 + j < ntoks) Ep::put(g, o0 + r0 + i, n0 + t0 + j, acc[i][j]);
+    }
+}
+
+constexpr size_t kSmem = (size_t)(kRows + kToks) * kChunk * 2;   // 96 KB at most
+
+template <class Ep>
+cudaError_t launch_small(const SmallArgs &g, bool pdl, cudaStream_t st) {
+    dim3 grid((g.O + kRows - 1) / kRows, (g.N + kToks - 1) / kToks);
+    const size_t smem = (size_t)(kRows + kToks) * (g.Kd < kChunk ? g.Kd : kChunk) * 2;
+    return launch_kernel(pdl, small_gemm_kernel<Ep>, grid, kThreads, smem, st, g);
+}
+
+}  // namespace
+
+cudaError_t configure_small() {
+    return cudaFuncSetAttribute(small_gemm_kernel<QueryEp>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+}
+
+cudaError_t launch_query_small(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, int Bmax,
+                               cudaStream_t st) {
+    const int HD = d.H * d.d_k;
+    for (int a = 0; a < d.A; ++a) {
+        SmallArgs g = {};
+        g.W = static_cast<const __nv_bfloat16 *>(a == 0 ? p.w_q : p.w_q_col);
+        g.X = static_cast<const __nv_bfloat16 *>(p.x);
+        g.O = HD;
+        g.N = d.B;
+        g.Kd = d.d_in;
+        g.err = p.err;
+        g.q = p.q_part + (int64_t)a * d.B * HD;
+        g.qs = qs + (int64_t)a * d.H * Bmax * 3 * d.d_k;
+        g.d_k = d.d_k;
+        g.Bmax = Bmax;
+        cudaError_t e = launch_small<QueryEp>(g, false, st);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+}  // namespace um
