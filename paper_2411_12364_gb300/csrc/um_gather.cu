@@ -2,13 +2,18 @@
 // inner V^T s^_p) and S9 on CUDA cores (the IVE projection o = sum_p W_p^T
 // acc_p, used for fp32 storage).
 //
-// Gather: one CTA per token.  Each warp takes a run of selected slots and
-// issues the 16-byte loads of all its rows before using any (memory-level
-// parallelism on random rows of a multi-GB table); a lane owns 16 bytes of
-// every row.  With E <= 4 blocks each lane keeps its accumulators acc[p][..]
-// in registers (the row's block p selects which, branch-free); larger E
-// accumulate into a per-warp copy in shared memory.  The warps' partial sums
-// are added at the end.  Row loads bypass L1 (read-only path).
+// Gather, one CTA per token.  Random 512-byte rows of a multi-GB table reach
+// the HBM copy rate only with many rows in flight per SM (measured on GB300:
+// about 6.8 TB/s from 32 warps per SM with 8 rows each), so the main kernel
+// keeps few registers per thread:
+//   * the token's H*m slots are bucketed by virtual block p with a stable
+//     counting sort in shared memory (ballots per block, a scan over warps);
+//   * each warp serves one block, so a lane owns 16 bytes of every row and
+//     8 fp32 accumulators, and issues 8 row loads before using any;
+//   * 16 warps per CTA, two CTAs per SM; the warps of a block are summed in a
+//     fixed order at the end (deterministic).
+// Wider rows or more slots take the per-lane multi-block kernels below.  Row
+// loads bypass L1 (read-only path).
 #include "um_internal.cuh"
 
 namespace um {
@@ -63,7 +68,10 @@ __device__ __forceinline__ void unpack<float>(uint4 v, float (&f)[4]) {
 }
 
 // Register-accumulating gather for E <= EMAX blocks and rows of at most
-// 32 vectors (one 16-byte vector per lane).
+// 32 vectors (one 16-byte vector per lane).  Each warp takes a contiguous
+// run of the token's H*m slots; their (row, block, weight) are loaded once,
+// one slot per lane, and broadcast by shuffle; 8 value loads per warp are
+// in flight together.
 template <typename T, int EMAX>
 __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
     extern __shared__ __align__(16) float red[];   // [kWarps][E][D_v]
@@ -75,7 +83,9 @@ __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
     const bool active = lane < VPR;
     const int hm = d.H * d.m;
     const int64_t base = (int64_t)b * hm;
-    const T *V = static_cast<const T *>(p.values);
+    const T *V = static_cast<const T *>(p.values) + lane * EPV;
+    const int per_warp = (hm + kWarps - 1) / kWarps;
+    const int e_begin = min(hm, warp * per_warp), e_end = min(hm, e_begin + per_warp);
     pdl_wait();
     pdl_trigger();
     float acc[EMAX][EPV];
@@ -84,29 +94,37 @@ __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
 #pragma unroll
         for (int c = 0; c < EPV; ++c) acc[q][c] = 0.f;
 
-    for (int e0 = warp * kUnroll; e0 < hm; e0 += kWarps * kUnroll) {
-        uint4 val[kUnroll];
-        int blk[kUnroll];
-        float w[kUnroll];
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-            const int e = e0 + u;
-            const bool ok = e < hm;
-            const int row = ok ? p.sel_row[base + e] : 0;
-            blk[u] = ok ? p.sel_p[base + e] : -1;
-            w[u] = ok ? p.sel_w[base + e] : 0.f;
-            val[u] = (ok && active) ? ld_stream(V + (int64_t)row * d.d_v + lane * EPV)
-                                    : make_uint4(0, 0, 0, 0);
+    for (int c0 = e_begin; c0 < e_end; c0 += 32) {
+        const int n = min(32, e_end - c0);
+        int row_l = 0, blk_l = -1;
+        float w_l = 0.f;
+        if (lane < n) {
+            row_l = p.sel_row[base + c0 + lane];
+            blk_l = p.sel_p[base + c0 + lane];
+            w_l = p.sel_w[base + c0 + lane];
         }
+        for (int j0 = 0; j0 < n; j0 += kUnroll) {
+            uint4 val[kUnroll];
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-            float f[EPV];
-            unpack<T>(val[u], f);
+            for (int u = 0; u < kUnroll; ++u) {
+                const int j = j0 + u;
+                const int row = __shfl_sync(0xffffffffu, row_l, j & 31);
+                val[u] = (j < n && active) ? ld_stream(V + (int64_t)row * d.d_v)
+                                           : make_uint4(0, 0, 0, 0);
+            }
 #pragma unroll
-            for (int q = 0; q < EMAX; ++q) {
-                const float wq = blk[u] == q ? w[u] : 0.f;   // branch-free block select
+            for (int u = 0; u < kUnroll; ++u) {
+                const int j = j0 + u;
+                const int blk = __shfl_sync(0xffffffffu, blk_l, j & 31);
+                const float w = j < n ? __shfl_sync(0xffffffffu, w_l, j & 31) : 0.f;
+                float f[EPV];
+                unpack<T>(val[u], f);
 #pragma unroll
-                for (int c = 0; c < EPV; ++c) acc[q][c] = fmaf(wq, f[c], acc[q][c]);
+                for (int q = 0; q < EMAX; ++q) {
+                    const float wq = blk == q ? w : 0.f;   // branch-free block select
+#pragma unroll
+                    for (int c = 0; c < EPV; ++c) acc[q][c] = fmaf(wq, f[c], acc[q][c]);
+                }
             }
         }
     }
@@ -129,6 +147,124 @@ __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
             p.acc[(int64_t)b * EDv + i] = s;
         else
             static_cast<T *>(p.out)[(int64_t)b * d.d_v + i] = from_f<T>(s);
+    }
+}
+
+constexpr int kBMaxE = 16;
+
+size_t bucket_smem_bytes(const Dims &d, int warps) {
+    const int hm = d.H * d.m;
+    return sizeof(int) * 2 * (size_t)hm + sizeof(float) * (size_t)warps * d.d_v;
+}
+
+// THREADS = 512 (2 CTAs per SM) for batches up to about two CTAs per SM,
+// where each token's latency matters; 256 (4 CTAs per SM) for longer
+// grids, where CTAs in their bucketing or reduction phase overlap others'
+// loads (measured: 6.5 TB/s over 2.15 GB at 16384 tokens, against 5.4 with
+// 512).
+template <typename T, int THREADS>
+__global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(Dims d, Ptrs p) {
+    constexpr int kBThreads = THREADS, kBWarps = THREADS / 32;
+    extern __shared__ __align__(16) unsigned char gsm[];
+    __shared__ int wcnt[kBWarps][kBMaxE];   // per warp and block: count, then offset
+    __shared__ int tot[kBMaxE], start[kBMaxE];
+    constexpr int EPV = 16 / sizeof(T);
+    const int b = blockIdx.x, E = d.E, hm = d.H * d.m, Dv = d.d_v;
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int64_t base = (int64_t)b * hm;
+    float *red = reinterpret_cast<float *>(gsm);                 // [kBWarps][D_v]
+    int *row_s = reinterpret_cast<int *>(red + kBWarps * Dv);    // [hm] bucketed rows
+    float *w_s = reinterpret_cast<float *>(row_s + hm);          // [hm] their weights
+    pdl_wait();
+    pdl_trigger();
+
+    // stable counting sort of the slots by block (slot order kept within a block)
+    int row = 0, blk = -1;
+    float w = 0.f;
+    if (t < hm) {
+        row = p.sel_row[base + t];
+        blk = p.sel_p[base + t];
+        w = p.sel_w[base + t];
+        if (blk < 0 || blk >= E) blk = -1;   // not a slot of this layer: skipped
+    }
+    int rank = 0;
+    for (int q = 0; q < E; ++q) {
+        const unsigned m = __ballot_sync(0xffffffffu, blk == q);
+        if (blk == q) rank = __popc(m & ((1u << lane) - 1u));
+        if (lane == 0) wcnt[warp][q] = __popc(m);
+    }
+    __syncthreads();
+    if (t < E) {
+        int run = 0;
+        for (int wv = 0; wv < kBWarps; ++wv) {
+            const int c = wcnt[wv][t];
+            wcnt[wv][t] = run;
+            run += c;
+        }
+        tot[t] = run;
+    }
+    __syncthreads();
+    if (t == 0) {
+        int run = 0;
+        for (int q = 0; q < E; ++q) {
+            start[q] = run;
+            run += tot[q];
+        }
+    }
+    __syncthreads();
+    if (blk >= 0) {
+        const int pos = start[blk] + wcnt[warp][blk] + rank;
+        row_s[pos] = row;
+        w_s[pos] = w;
+    }
+    __syncthreads();
+
+    // warps [q*wpb, (q+1)*wpb) serve block q, each a contiguous share
+    const int wpb = kBWarps / E;
+    const int q = warp / wpb, sub = warp - q * wpb;
+    const bool active = lane * EPV < Dv;
+    const T *V = static_cast<const T *>(p.values) + lane * EPV;
+    float acc[EPV];
+#pragma unroll
+    for (int c = 0; c < EPV; ++c) acc[c] = 0.f;
+    if (q < E) {
+        const int n = tot[q], per = (n + wpb - 1) / wpb;
+        const int lo = start[q] + min(n, sub * per), hi = start[q] + min(n, (sub + 1) * per);
+        for (int j0 = lo; j0 < hi; j0 += kUnroll) {
+            uint4 val[kUnroll];
+            float wu[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int j = j0 + u;
+                const bool ok = j < hi;
+                wu[u] = ok ? w_s[j] : 0.f;
+                val[u] = (ok && active) ? ld_stream(V + (int64_t)row_s[j] * Dv)
+                                        : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                float f[EPV];
+                unpack<T>(val[u], f);
+#pragma unroll
+                for (int c = 0; c < EPV; ++c) acc[c] = fmaf(wu[u], f[c], acc[c]);
+            }
+        }
+        if (active)
+#pragma unroll
+            for (int c = 0; c < EPV; ++c) red[warp * Dv + lane * EPV + c] = acc[c];
+    }
+    __syncthreads();
+    const int EDv = E * Dv;
+    for (int i = t; i < EDv; i += kBThreads) {
+        const int qq = i / Dv, c = i - qq * Dv;
+        float sum = 0.f;
+        for (int sb = 0; sb < wpb; ++sb) sum += red[(qq * wpb + sb) * Dv + c];
+        if (p.acc_bf)
+            p.acc_bf[(int64_t)b * EDv + i] = __float2bfloat16_rn(sum);
+        else if (d.has_proj)
+            p.acc[(int64_t)b * EDv + i] = sum;
+        else
+            static_cast<T *>(p.out)[(int64_t)b * Dv + i] = from_f<T>(sum);
     }
 }
 
@@ -259,6 +395,12 @@ cudaError_t configure_gather(const Dims &d) {
     if (e == cudaSuccess) e = allow(gather_reg_kernel<float, 4>, bytes);
     if (e == cudaSuccess) e = allow(gather_reg_kernel<__nv_bfloat16, 1>, bytes);
     if (e == cudaSuccess) e = allow(gather_reg_kernel<__nv_bfloat16, 4>, bytes);
+    if (e == cudaSuccess) e = allow(gather_bucket_kernel<float, 512>, bucket_smem_bytes(d, 16));
+    if (e == cudaSuccess)
+        e = allow(gather_bucket_kernel<__nv_bfloat16, 512>, bucket_smem_bytes(d, 16));
+    if (e == cudaSuccess) e = allow(gather_bucket_kernel<float, 256>, bucket_smem_bytes(d, 8));
+    if (e == cudaSuccess)
+        e = allow(gather_bucket_kernel<__nv_bfloat16, 256>, bucket_smem_bytes(d, 8));
     return e;
 }
 
@@ -266,6 +408,14 @@ template <typename T>
 static cudaError_t launch_gather_t(const Dims &d, const Ptrs &p, cudaStream_t st) {
     const size_t bytes = gather_smem_bytes(d);
     const bool fits_lanes = d.d_v / (16 / (int)sizeof(T)) <= 32;
+    if (fits_lanes && d.d_v % (16 / (int)sizeof(T)) == 0 && d.E <= kBMaxE) {
+        if (d.B <= 2 * 152 && d.H * d.m <= 512)
+            return launch_kernel(d.pdl, gather_bucket_kernel<T, 512>, d.B, 512,
+                                 bucket_smem_bytes(d, 16), st, d, p);
+        if (d.H * d.m <= 256 && d.E <= 8)
+            return launch_kernel(d.pdl, gather_bucket_kernel<T, 256>, d.B, 256,
+                                 bucket_smem_bytes(d, 8), st, d, p);
+    }
     if (fits_lanes && d.E == 1)
         return launch_kernel(d.pdl, gather_reg_kernel<T, 1>, d.B, kThreads, bytes, st, d, p);
     if (fits_lanes && d.E <= 4)

@@ -481,8 +481,15 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
     const uint32_t pos = active ? pos_of(sh.win[s][qi]) : 0u;
 
     int ord = 0;
-    if (active)
-        for (int g = sub; g < k; g += G) ord += pos_of(sh.win[s][g]) < pos;
+    if (active) {
+        int g = sub;
+        for (; g + 3 * G < k; g += 4 * G) {
+            const uint32_t a = pos_of(sh.win[s][g]), b = pos_of(sh.win[s][g + G]),
+                           c = pos_of(sh.win[s][g + 2 * G]), e = pos_of(sh.win[s][g + 3 * G]);
+            ord += (a < pos) + (b < pos) + (c < pos) + (e < pos);
+        }
+        for (; g < k; g += G) ord += pos_of(sh.win[s][g]) < pos;
+    }
     for (int off = G >> 1; off > 0; off >>= 1) ord += __shfl_xor_sync(kFull, ord, off);
 
     const T *row = static_cast<const T *>(s ? p.k_col : p.k_row) + ((int64_t)h * d.K + pos) * D;
