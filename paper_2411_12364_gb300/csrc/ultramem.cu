@@ -96,11 +96,11 @@ int tc_proj_splits(const ultramem_config &c, int B) {
     return tc_splits(c.d_out, B, c.expand_e * c.d_v, 64);
 }
 
-// The tensor path needs bf16 storage, rank chunks of whole 16-wide MMA
-// steps, at most 4 chunks (TMEM columns) and 16-byte rows for TMA.
+// The tensor path needs bf16 storage and 16-byte rows for TMA (D_in, D_k and
+// E*D_v multiples of 8 elements).
 bool tc_eligible(const ultramem_config &c) {
-    return c.dtype == ULTRAMEM_BF16 && (c.d_k / c.rank) % 16 == 0 && c.rank <= 4 &&
-           c.d_in % 8 == 0 && (c.expand_e * c.d_v) % 8 == 0 && c.d_k % 8 == 0;
+    return c.dtype == ULTRAMEM_BF16 && c.d_in % 8 == 0 && (c.expand_e * c.d_v) % 8 == 0 &&
+           c.d_k % 8 == 0;
 }
 
 int proj_splits(const ultramem_config &c, int B) {
@@ -324,11 +324,11 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     const ultramem_config &c = L->cfg;
     um::TcMaps mp = L->maps;
     const int Bmax = c.max_tokens;
-    const int nt1 = um::tc_n_tile(d.B, 1), ntr = um::tc_n_tile(d.B, d.r);
+    const int nt1 = um::tc_n_tile(d.B, 1);   // N tile of every contraction (one accumulator)
     if (!um::tc_encode(&mp.x, p.x, (uint64_t)c.d_in, (uint64_t)d.B, 1, (uint32_t)nt1, 2))
         return ULTRAMEM_EINVAL;   // x must be 16-byte aligned
-    if (!um::tc_encode(&mp.qs, L->ws.qs, 3ull * c.d_k, (uint64_t)Bmax, (uint64_t)d.A * d.H,
-                       (uint32_t)ntr, 3) ||
+    if (!um::tc_encode(&mp.qs, L->ws.qs, 3ull * c.d_k, (uint64_t)Bmax, 2ull * d.H,
+                       (uint32_t)nt1, 3) ||
         !um::tc_encode(&mp.acc, L->ws.acc_bf, (uint64_t)d.E * d.d_v, (uint64_t)Bmax, 1,
                        (uint32_t)nt1, 2))
         return ULTRAMEM_ECUDA;
@@ -514,8 +514,8 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     const size_t kd = (size_t)d.E * d.d_v;
     if (e == cudaSuccess && L->tc) {
         // tensor path: split queries, bf16 acc, K-major copy of the projectors
-        e = dalloc(&ws.qs, (size_t)d.A * H * Bm * 3 * cfg->d_k);
-        if (e == cudaSuccess) e = cudaMemset(ws.qs, 0, sizeof(__nv_bfloat16) * d.A * H * Bm * 3 * cfg->d_k);
+        e = dalloc(&ws.qs, (size_t)2 * H * Bm * 3 * cfg->d_k);
+        if (e == cudaSuccess) e = cudaMemset(ws.qs, 0, sizeof(__nv_bfloat16) * 2 * H * Bm * 3 * cfg->d_k);
         if (e == cudaSuccess) e = dalloc(&ws.acc_bf, Bm * kd);
         if (e == cudaSuccess) e = cudaMemset(ws.acc_bf, 0, sizeof(__nv_bfloat16) * Bm * kd);
         if (e == cudaSuccess && cfg->has_proj) {

@@ -165,6 +165,26 @@ __device__ __forceinline__ float ord2f(uint32_t o) {
     return __uint_as_float(u);
 }
 
+// The scoring contraction's B operand for one query element: q[h][c] scaled
+// by the rank-1 coefficient of its chunk (u for the row keys, t for the
+// column keys), so that one dot product with a key row gives the folded
+// score u^T S_row (Eq. 6-7 folded into Eq. 4), written as three bf16 terms
+// q1 + q2 + q3 (each the rounding of what the previous ones leave; residual
+// <= 2^-24 of the value).  qs is [2][H][Bmax][3][D_k], axis-major; `v` is
+// the already scaled value.
+__device__ __forceinline__ void put_split_query(__nv_bfloat16 *qs, int axis, int h, int c, int n,
+                                                float v, int H, int Bmax, int d_k) {
+    const __nv_bfloat16 q1 = __float2bfloat16_rn(v);
+    const float r1 = v - __bfloat162float(q1);
+    const __nv_bfloat16 q2 = __float2bfloat16_rn(r1);
+    const float r2 = r1 - __bfloat162float(q2);
+    const __nv_bfloat16 q3 = __float2bfloat16_rn(r2);
+    __nv_bfloat16 *dst = qs + (((int64_t)(axis * H + h) * Bmax + n) * 3) * d_k + c;
+    dst[0] = q1;
+    dst[d_k] = q2;
+    dst[2 * d_k] = q3;
+}
+
 // Barrett's constant for reduction modulo M (P. Barrett, CRYPTO '86).
 inline uint64_t barrett_mu(uint64_t M) { return M ? ~0ull / M : 0; }
 

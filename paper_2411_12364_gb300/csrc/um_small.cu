@@ -11,7 +11,8 @@
 // K-slices, then a fixed 3-step shuffle sum: deterministic), and the
 // epilogue writes the result in place.  No partial sums leave the CTA.
 //
-//   Y[n][o] = sum_d x[n][d] W_q[o][d]  -> q (fp32) and its 3-term bf16 split
+//   Y[n][o] = sum_d x[n][d] W_q[o][d]  -> q (fp32), and q scaled by u (row
+//   keys) and by t (column keys) as 3-term bf16 splits for the scoring
 // (The tile re-reads each weight row once per 8 tokens, so from about 128
 // tokens on, and for the larger IVE projector, the tensor-core kernel wins.)
 #include "um_internal.cuh"
@@ -35,23 +36,33 @@ struct SmallArgs {
     int *err;
     // S1 epilogue
     float *q;                    // [A][B][HD] at a * B * HD (split 0 of q_part)
-    __nv_bfloat16 *qs;           // [A*H][Bmax][3][D_k] at a * H * Bmax * 3 * D_k
-    int d_k, Bmax;
+    __nv_bfloat16 *qs;           // [2][H][Bmax][3][D_k], the scaled split queries
+    const float *u, *t;          // [H][r] rank-1 coefficients of row / column keys
+    int a, A, H, d_k, dk, r, Bmax;
 };
 
+// Per output row o: its head, column and the rank-1 coefficients of its
+// chunk (loaded once, before the weights arrive).
+struct RowScale {
+    int h, c;
+    float cu, ct;
+};
+__device__ __forceinline__ RowScale row_scale(const SmallArgs &g, int o) {
+    RowScale rs;
+    rs.h = o / g.d_k;
+    rs.c = o - rs.h * g.d_k;
+    const int k = rs.h * g.r + rs.c / g.dk;
+    rs.cu = (g.A == 1 || g.a == 0) ? g.u[k] : 0.f;
+    rs.ct = (g.A == 1 || g.a == 1) ? g.t[k] : 0.f;
+    return rs;
+}
+
 struct QueryEp {
-    __device__ static void put(const SmallArgs &g, int o, int n, float v) {
+    __device__ static void put(const SmallArgs &g, int o, int n, float v, const RowScale &rs) {
         g.q[(int64_t)n * g.O + o] = v;
-        const __nv_bfloat16 q1 = __float2bfloat16_rn(v);
-        const float r1 = v - __bfloat162float(q1);
-        const __nv_bfloat16 q2 = __float2bfloat16_rn(r1);
-        const float r2 = r1 - __bfloat162float(q2);
-        const __nv_bfloat16 q3 = __float2bfloat16_rn(r2);
-        const int h = o / g.d_k, c = o - h * g.d_k;
-        __nv_bfloat16 *dst = g.qs + (((int64_t)h * g.Bmax + n) * 3) * g.d_k + c;
-        dst[0] = q1;
-        dst[g.d_k] = q2;
-        dst[2 * g.d_k] = q3;
+        // a shared query feeds both axes; a separate column query only axis 1
+        if (g.A == 1 || g.a == 0) put_split_query(g.qs, 0, rs.h, rs.c, n, v * rs.cu, g.H, g.Bmax, g.d_k);
+        if (g.A == 1 || g.a == 1) put_split_query(g.qs, 1, rs.h, rs.c, n, v * rs.ct, g.H, g.Bmax, g.d_k);
     }
 };
 
@@ -89,6 +100,9 @@ __global__ void __launch_bounds__(kThreads) small_gemm_kernel(SmallArgs g) {
         mbar_init(&bar, 1);
         fence_mbar_init();
     }
+    RowScale rs[2];
+#pragma unroll
+    for (int i = 0; i < 2; ++i) rs[i] = row_scale(g, min(o0 + r0 + i, g.O - 1));
     __syncthreads();
     float acc[2][2] = {};
     uint32_t phase = 0;
@@ -152,7 +166,8 @@ __global__ void __launch_bounds__(kThreads) small_gemm_kernel(SmallArgs g) {
         for (int i = 0; i < 2; ++i)
 #pragma unroll
             for (int j = 0; j < 2; ++j)
-                if (r0 + i < nrows && t0 + j < ntoks) Ep::put(g, o0 + r0 + i, n0 + t0 + j, acc[i][j]);
+                if (r0 + i < nrows && t0 + j < ntoks)
+                    Ep::put(g, o0 + r0 + i, n0 + t0 + j, acc[i][j], rs[i]);
     }
 }
 
@@ -184,8 +199,15 @@ cudaError_t launch_query_small(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, 
         g.Kd = d.d_in;
         g.err = p.err;
         g.q = p.q_part + (int64_t)a * d.B * HD;
-        g.qs = qs + (int64_t)a * d.H * Bmax * 3 * d.d_k;
+        g.qs = qs;
+        g.u = p.u;
+        g.t = p.t;
+        g.a = a;
+        g.A = d.A;
+        g.H = d.H;
         g.d_k = d.d_k;
+        g.dk = d.dk;
+        g.r = d.r;
         g.Bmax = Bmax;
         cudaError_t e = launch_small<QueryEp>(g, false, st);
         if (e != cudaSuccess) return e;

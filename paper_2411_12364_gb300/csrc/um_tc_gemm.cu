@@ -47,6 +47,7 @@ struct Tile {
     int a_sel;         // which A map (0/1)
     int a_z, b_z;      // third coordinate of 3-D maps (-1: 2-D map)
     int kb0, nkb;      // K blocks [kb0, kb0 + nkb)
+    int z;             // the tile's third grid coordinate (split or head/axis)
 };
 
 __host__ __device__ inline size_t stage_bytes_of(int nsplit, int n_tile) {
@@ -73,7 +74,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const Tile t = op.tile();
+    const Tile t = op.tile_at(blockIdx.x, blockIdx.y, blockIdx.z);
     const int n_tile = op.n_tile;
     const uint32_t b_bytes = (uint32_t)n_tile * 128;
     const uint32_t stage_bytes = kTileABytes + NSPLIT * b_bytes;
@@ -241,16 +242,215 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int q = 0; q < kMaxSplits; ++q)
                     part[e][q] = q < S ? op.load_partial(t, q, row, n + e) : 0.f;
+            float sums[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 float sum = 0.f;
 #pragma unroll
                 for (int q = 0; q < kMaxSplits; ++q)
                     if (q < S) sum += part[e][q];
-                op.store_sum(t, row, n + e, sum);
+                sums[e] = sum;
             }
+            op.store_sums(t, row, n, sums);
         }
     }
+}
+
+// ---- persistent variant (many tiles, no split-K) ----------------------------
+// One CTA per SM loops over tiles i = blockIdx.x, + gridDim.x, ... (x fastest,
+// then y, then z of the tile grid).  Warp 0 lane 0 streams A/B K-blocks of
+// successive tiles through the ring; warp 1 lane 0 issues each tile's MMAs
+// into one of two TMEM accumulator buffers; warps 2..9 drain the other
+// buffer (epilogue) meanwhile, so loads, MMAs and stores of consecutive
+// tiles overlap.  Barriers: full/empty per ring stage; tfull (MMAs of a
+// buffer done) and tempty (its epilogue done, 8 arrivals) per buffer.  Every
+// wait is bounded; a timeout raises the error word and an abort flag that
+// every role polls.
+constexpr int kPEpiWarps = 8;
+constexpr int kPThreads = 64 + 32 * kPEpiWarps;
+
+template <int NSPLIT, class Op>
+__global__ void __launch_bounds__(kPThreads, 1)
+    tc_gemm_persistent(const __grid_constant__ CUtensorMap mapA0,
+                       const __grid_constant__ CUtensorMap mapA1,
+                       const __grid_constant__ CUtensorMap mapB, Op op, int gx, int gy,
+                       int tiles, uint32_t buf_cols) {
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full[kMaxStages], empty[kMaxStages], tfull[2], tempty[2],
+        drained;
+    __shared__ uint32_t tmem_slot;
+    __shared__ volatile int abort_flag;
+    uint8_t *ring = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_tile = op.n_tile;
+    const uint32_t b_bytes = (uint32_t)n_tile * 128;
+    const uint32_t stage_bytes = kTileABytes + NSPLIT * b_bytes;
+    const int kStages = op.stages;
+    auto tile_of = [&](int i) {
+        const int bx = i % gx, r = i / gx;
+        return op.tile_at(bx, r % gy, r / gy);
+    };
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&tfull[b], 1);
+            mbar_init(&tempty[b], kPEpiWarps);
+        }
+        mbar_init(&drained, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tensormap(&mapA0);
+        prefetch_tensormap(&mapA1);
+        prefetch_tensormap(&mapB);
+    }
+    pdl_wait();
+    if (warp == 0) tmem_alloc(&tmem_slot, 2 * buf_cols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    pdl_trigger();
+    auto fail = [&]() {
+        atomicOr(op.err, kErrTimeout);
+        abort_flag = 1;
+    };
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // producer
+            int it = 0;
+            for (int i = blockIdx.x; i < tiles && !abort_flag; i += gridDim.x) {
+                const Tile t = tile_of(i);
+                const CUtensorMap *mapA = t.a_sel ? &mapA1 : &mapA0;
+                for (int kb = 0; kb < t.nkb; ++kb, ++it) {
+                    const int s = it % kStages;
+                    if (it >= kStages && !mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
+                        fail();
+                        break;
+                    }
+                    uint8_t *sa = ring + (size_t)s * stage_bytes;
+                    mbar_arrive_expect_tx(&full[s], stage_bytes);
+                    const int kx = (t.kb0 + kb) * kBlockK;
+                    if (t.a_z >= 0) tma_load_3d(sa, mapA, &full[s], kx, t.m0, t.a_z);
+                    else tma_load_2d(sa, mapA, &full[s], kx, t.m0);
+#pragma unroll
+                    for (int j = 0; j < NSPLIT; ++j) {
+                        uint8_t *sb = sa + kTileABytes + j * b_bytes;
+                        const int bx = j * op.b_split_stride + kx;
+                        if (t.b_z >= 0) tma_load_3d(sb, &mapB, &full[s], bx, t.n0, t.b_z);
+                        else tma_load_2d(sb, &mapB, &full[s], bx, t.n0);
+                    }
+                }
+            }
+            // loads still in flight (only after an abort) land before exit
+            for (int j = (it > kStages ? it - kStages : 0); j < it; ++j)
+                mbar_wait(&full[j % kStages], (j / kStages) & 1);
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // MMA issuer
+            const uint32_t idesc = idesc_bf16_f32(kTileM, n_tile);
+            int it = 0, lt = 0;
+            for (int i = blockIdx.x; i < tiles && !abort_flag; i += gridDim.x, ++lt) {
+                const Tile t = tile_of(i);
+                const int buf = lt & 1;
+                if (lt >= 2 && !mbar_wait(&tempty[buf], ((lt >> 1) - 1) & 1)) {
+                    fail();
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t dbase = tmem + (uint32_t)buf * buf_cols;
+                uint32_t started = 0;
+                int acc = (t.kb0 * kBlockK) / op.acc_chunk;
+                int next_chunk = (acc + 1) * op.acc_chunk;
+                bool ok = true;
+                for (int kb = 0; kb < t.nkb; ++kb, ++it) {
+                    const int s = it % kStages;
+                    if (!mbar_wait(&full[s], (it / kStages) & 1)) {
+                        fail();
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(ring + (size_t)s * stage_bytes);
+                    const uint64_t ad0 = desc_k_sw128(sa);
+                    uint64_t bd0[NSPLIT];
+#pragma unroll
+                    for (int j = 0; j < NSPLIT; ++j)
+                        bd0[j] = desc_k_sw128(sa + kTileABytes + j * b_bytes);
+#pragma unroll
+                    for (int k16 = 0; k16 < kBlockK / 16; ++k16) {
+                        const int kg = (t.kb0 + kb) * kBlockK + k16 * 16;
+                        while (kg >= next_chunk && acc < op.n_acc - 1) {
+                            ++acc;
+                            next_chunk += op.acc_chunk;
+                        }
+                        const uint32_t dt = dbase + (uint32_t)(acc * n_tile);
+                        const uint32_t acc_bit = 1u << acc;
+#pragma unroll
+                        for (int j = 0; j < NSPLIT; ++j) {
+                            mma_bf16(dt, ad0 + 2 * k16, bd0[j] + 2 * k16, idesc,
+                                     started & acc_bit);
+                            started |= acc_bit;
+                        }
+                    }
+                    mma_commit(&empty[s]);
+                }
+                if (!ok) break;
+                mma_commit(&tfull[buf]);
+            }
+            // every MMA issued has completed before TMEM is released
+            mma_commit(&drained);
+            mbar_wait(&drained, 0);
+        }
+        __syncwarp();
+    } else {
+        // epilogue warps: warp w reads TMEM lane quarter w % 4 and alternate
+        // 32-column chunks by warp group
+        const int quad = warp & 3, grp = (warp - 2) >> 2;
+        const int row = quad * 32 + lane;
+        int lt = 0;
+        for (int i = blockIdx.x; i < tiles && !abort_flag; i += gridDim.x, ++lt) {
+            const Tile t = tile_of(i);
+            const int buf = lt & 1;
+            if (!mbar_wait(&tfull[buf], (lt >> 1) & 1)) {
+                if (lane == 0) fail();
+                break;
+            }
+            tc_fence_after();
+            const uint32_t lane_base =
+                tmem + (uint32_t)buf * buf_cols + ((uint32_t)(quad * 32) << 16);
+            for (int c0 = grp * 32; c0 < n_tile; c0 += 64) {
+                uint32_t r[kMaxAcc][32];
+#pragma unroll
+                for (int a = 0; a < kMaxAcc; ++a)
+                    if (a < op.n_acc) tmem_ld32_nowait(lane_base + (uint32_t)(a * n_tile + c0), r[a]);
+                tmem_ld_wait();
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                    if (c0 + half * 16 >= n_tile) break;
+                    float v[kMaxAcc][16];
+#pragma unroll
+                    for (int a = 0; a < kMaxAcc; ++a)
+#pragma unroll
+                        for (int q = 0; q < 16; ++q) v[a][q] = __uint_as_float(r[a][half * 16 + q]);
+                    op.store(t, row, c0 + half * 16, v);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[buf]);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, 2 * buf_cols);
 }
 
 // ---- S1: query projection, split over D_i --------------------------------
@@ -259,54 +459,60 @@ __global__ void __launch_bounds__(kThreads, 1)
 struct QueryOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
-    int B, HD, A, a, splits, kb_total, H, d_k, Bmax;
+    int B, HD, A, a, splits, kb_total, H, d_k, dk, r, Bmax;
     float *q_part;        // [splits][A][B][HD]; the result is split 0
-    __nv_bfloat16 *qs;    // [A*H][Bmax][3][D_k]
+    __nv_bfloat16 *qs;    // [2][H][Bmax][3][D_k] scaled split queries
+    const float *u, *t;   // [H][r]
     __device__ int cluster_splits() const { return splits; }
-    __device__ Tile tile() const {
+    int cluster_splits_host() const { return splits; }
+    __device__ Tile tile_at(int bx, int by, int bz) const {
         Tile t;
-        t.m0 = blockIdx.x * kTileM;
-        t.n0 = blockIdx.y * n_tile;
+        t.m0 = bx * kTileM;
+        t.n0 = by * n_tile;
         t.a_sel = 0;
         t.a_z = -1;
         t.b_z = -1;
-        const int split = blockIdx.z;
+        t.z = bz;   // the split
         const int per = (kb_total + splits - 1) / splits;
-        t.kb0 = split * per;
+        t.kb0 = bz * per;
         t.nkb = max(0, min(kb_total, t.kb0 + per) - t.kb0);
         return t;
     }
-    __device__ void put(int m, int n, float q) const {
-        q_part[((int64_t)a * B + n) * HD + m] = q;
-        const __nv_bfloat16 q1 = __float2bfloat16_rn(q);
-        const float r1 = q - __bfloat162float(q1);
-        const __nv_bfloat16 q2 = __float2bfloat16_rn(r1);
-        const float r2 = r1 - __bfloat162float(q2);
-        const __nv_bfloat16 q3 = __float2bfloat16_rn(r2);
+    // q (fp32) and its two scaled splits for output row m over columns
+    // n0 .. n0 + cnt - 1 of the tile (the row's coefficients looked up once)
+    template <int CNT>
+    __device__ void put_row(int m, int n0, const float (&v)[CNT]) const {
         const int h = m / d_k, c = m - h * d_k;
-        __nv_bfloat16 *dst = qs + (((int64_t)(a * H + h) * Bmax + n) * 3) * d_k + c;
-        dst[0] = q1;
-        dst[d_k] = q2;
-        dst[2 * d_k] = q3;
-    }
-    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
-        const int m = t.m0 + row;
-        if (m >= HD) return;
+        const int k = h * r + c / dk;
+        const bool row_axis = A == 1 || a == 0, col_axis = A == 1 || a == 1;
+        const float cu = row_axis ? u[k] : 0.f, ct = col_axis ? t[k] : 0.f;
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            const int n = t.n0 + c + j;
-            if (n < B) put(m, n, t.nkb ? v[0][j] : 0.f);
+        for (int j = 0; j < CNT; ++j) {
+            const int n = n0 + j;
+            if (n >= B) break;
+            q_part[((int64_t)a * B + n) * HD + m] = v[j];
+            // a shared query feeds both axes; a separate column query only axis 1
+            if (row_axis) put_split_query(qs, 0, h, c, n, v[j] * cu, H, Bmax, d_k);
+            if (col_axis) put_split_query(qs, 1, h, c, n, v[j] * ct, H, Bmax, d_k);
         }
     }
-    __device__ void store_sum(const Tile &t, int row, int c, float q) const {
-        const int m = t.m0 + row, n = t.n0 + c;
-        if (m < HD && n < B) put(m, n, q);
+    __device__ void store(const Tile &tl, int row, int c, float (&v)[kMaxAcc][16]) const {
+        const int m = tl.m0 + row;
+        if (m >= HD) return;
+        float w[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) w[j] = tl.nkb ? v[0][j] : 0.f;
+        put_row<16>(m, tl.n0 + c, w);
+    }
+    __device__ void store_sums(const Tile &tl, int row, int c, const float (&s4)[4]) const {
+        const int m = tl.m0 + row;
+        if (m < HD) put_row<4>(m, tl.n0 + c, s4);
     }
     // split-K partials: q_part[split][a][n][m] (the sum later replaces split 0)
     __device__ void store_partial(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
         const int m = t.m0 + row;
         if (m >= HD) return;
-        float *dst = q_part + (((int64_t)blockIdx.z * A + a) * B + t.n0 + c) * HD + m;
+        float *dst = q_part + (((int64_t)t.z * A + a) * B + t.n0 + c) * HD + m;
 #pragma unroll
         for (int j = 0; j < 16; ++j)
             if (t.n0 + c + j < B) dst[(int64_t)j * HD] = t.nkb ? v[0][j] : 0.f;
@@ -318,29 +524,30 @@ struct QueryOp {
     }
 };
 
-// ---- S2: row/column scores, one accumulator per rank chunk ------------------
-// The epilogue folds the r chunk scores into the rank-1 score (Eq. 6-7),
-// a = sum_alpha coef[alpha] S_alpha with coef = u (row keys) or t (column
-// keys), and stores its order-preserving 32-bit key.
-template <int R>
+// ---- S2: row/column scores ---------------------------------------------------
+// The B operand is the query already scaled by the axis' rank-1 coefficients
+// (u or t per rank chunk), so one fp32 accumulator holds the folded score
+// a = sum_alpha coef[alpha] S_alpha (Eq. 4 with Eq. 6-7) and the epilogue
+// stores its order-preserving 32-bit key.
 struct ScoreOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
-    int B, H, K, A, kb_total;
-    const float *u, *t;   // [H][R]
+    int B, H, K, kb_total;
     uint32_t *akey;       // [B][H][2][K]
     __device__ int cluster_splits() const { return 1; }
-    __device__ void store_sum(const Tile &, int, int, float) const {}
+    int cluster_splits_host() const { return 1; }
+    __device__ void store_sums(const Tile &, int, int, const float (&)[4]) const {}
     __device__ void store_partial(const Tile &, int, int, float (&)[kMaxAcc][16]) const {}
     __device__ float load_partial(const Tile &, int, int, int) const { return 0.f; }
-    __device__ Tile tile() const {
+    __device__ Tile tile_at(int bx, int by, int bz) const {
         Tile tl;
-        const int h = blockIdx.z >> 1, axis = blockIdx.z & 1;
-        tl.m0 = blockIdx.x * kTileM;
-        tl.n0 = blockIdx.y * n_tile;
+        const int h = bz >> 1, axis = bz & 1;
+        tl.z = bz;   // head and axis
+        tl.m0 = bx * kTileM;
+        tl.n0 = by * n_tile;
         tl.a_sel = axis;
         tl.a_z = h;
-        tl.b_z = (A == 2 && axis == 1 ? H : 0) + h;
+        tl.b_z = axis * H + h;
         tl.kb0 = 0;
         tl.nkb = kb_total;
         return tl;
@@ -348,11 +555,7 @@ struct ScoreOp {
     __device__ void store(const Tile &tl, int row, int c, float (&v)[kMaxAcc][16]) const {
         const int i = tl.m0 + row;
         if (i >= K) return;
-        const int h = blockIdx.z >> 1, axis = blockIdx.z & 1;
-        const float *coef = (axis == 0 ? u : t) + h * R;
-        float cf[R];
-#pragma unroll
-        for (int a = 0; a < R; ++a) cf[a] = coef[a];
+        const int h = tl.z >> 1, axis = tl.z & 1;
         const int n0 = tl.n0 + c;
         const int64_t tok_stride = (int64_t)H * 2 * K;   // akey elements per token
         uint32_t *dst = akey + ((int64_t)n0 * H + h) * 2 * K + (int64_t)axis * K + i;
@@ -360,10 +563,7 @@ struct ScoreOp {
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
             if (j >= nj) break;
-            float a = cf[0] * v[0][j];
-#pragma unroll
-            for (int al = 1; al < R; ++al) a = fmaf(cf[al], v[al][j], a);
-            dst[j * tok_stride] = f2ord(a);
+            dst[j * tok_stride] = f2ord(v[0][j]);
         }
     }
 };
@@ -376,10 +576,11 @@ struct ProjOp {
     __nv_bfloat16 *out;   // [B][d_out]
     float *part;          // [splits][B][d_out] split-K partials
     __device__ int cluster_splits() const { return splits; }
+    int cluster_splits_host() const { return splits; }
     __device__ void store_partial(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
         const int o = t.m0 + row;
         if (o >= d_out) return;
-        float *dst = part + ((int64_t)blockIdx.z * B + t.n0 + c) * d_out + o;
+        float *dst = part + ((int64_t)t.z * B + t.n0 + c) * d_out + o;
 #pragma unroll
         for (int j = 0; j < 16; ++j)
             if (t.n0 + c + j < B) dst[(int64_t)j * d_out] = t.nkb ? v[0][j] : 0.f;
@@ -389,15 +590,16 @@ struct ProjOp {
         if (o >= d_out || n >= B) return 0.f;
         return __ldcg(part + ((int64_t)split * B + n) * d_out + o);
     }
-    __device__ Tile tile() const {
+    __device__ Tile tile_at(int bx, int by, int bz) const {
         Tile t;
-        t.m0 = blockIdx.x * kTileM;
-        t.n0 = blockIdx.y * n_tile;
+        t.m0 = bx * kTileM;
+        t.n0 = by * n_tile;
         t.a_sel = 0;
         t.a_z = -1;
         t.b_z = -1;
+        t.z = bz;   // the split
         const int per = (kb_total + splits - 1) / splits;
-        t.kb0 = blockIdx.z * per;
+        t.kb0 = bz * per;
         t.nkb = max(0, min(kb_total, t.kb0 + per) - t.kb0);
         return t;
     }
@@ -411,9 +613,14 @@ struct ProjOp {
             out[(int64_t)n * d_out + o] = __float2bfloat16_rn(t.nkb ? v[0][j] : 0.f);
         }
     }
-    __device__ void store_sum(const Tile &t, int row, int c, float v) const {
-        const int o = t.m0 + row, n = t.n0 + c;
-        if (o < d_out && n < B) out[(int64_t)n * d_out + o] = __float2bfloat16_rn(v);
+    __device__ void store_sums(const Tile &t, int row, int c, const float (&s4)[4]) const {
+        const int o = t.m0 + row;
+        if (o >= d_out) return;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int n = t.n0 + c + e;
+            if (n < B) out[(int64_t)n * d_out + o] = __float2bfloat16_rn(s4[e]);
+        }
     }
 };
 
@@ -485,11 +692,57 @@ int tc_n_tile(int B, int n_acc) {
     return n < cap ? n : cap;
 }
 
-// grid.z = the split count, which is also the cluster's z extent when > 1
+static int sm_count() {
+    static int n = 0;
+    if (!n) {
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+            n = 1;
+    }
+    return n;
+}
+
+// TMEM columns of one accumulator buffer: the epilogue reads 32 columns at a
+// time, so cover the last such read, rounded to 32.
+static uint32_t buf_cols_of(int n_acc, int n_tile) {
+    const uint32_t c = (uint32_t)((n_acc - 1) * n_tile + ((n_tile - 1) / 32) * 32 + 32);
+    return (c + 31) & ~31u;
+}
+
+// The persistent kernel serves grids with more tiles than SMs, no split-K and
+// two accumulator buffers within TMEM's 512 columns; returns false when it
+// does not apply.
+template <int NSPLIT, class Op>
+static bool persistent_ok(dim3 grid, const Op &op) {
+    const uint32_t bc = buf_cols_of(op.n_acc, op.n_tile);
+    return grid.z >= 1 && op.cluster_splits_host() == 1 &&
+           (int)(grid.x * grid.y * grid.z) > sm_count() && 2 * bc <= 512 &&
+           tmem_cols_for(2 * bc) == 2 * bc;
+}
+
+template <int NSPLIT, class Op>
+static cudaError_t launch_gemm_persistent(dim3 grid, const CUtensorMap &a0, const CUtensorMap &a1,
+                                          const CUtensorMap &b, Op op, int nkb, bool pdl,
+                                          cudaStream_t st) {
+    (void)nkb;   // the ring runs across tiles: as many stages as fit
+    op.stages = stages_for(NSPLIT, op.n_tile, kMaxStages);
+    const size_t smem = 1024 + (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile);
+    const int tiles = (int)(grid.x * grid.y * grid.z);
+    const int ctas = tiles < sm_count() ? tiles : sm_count();
+    return launch_kernel(pdl, tc_gemm_persistent<NSPLIT, Op>, dim3(ctas), kPThreads, smem, st, a0,
+                         a1, b, op, (int)grid.x, (int)grid.y, tiles,
+                         buf_cols_of(op.n_acc, op.n_tile));
+}
+
+// grid.z = the split count (S1, S9; also the cluster's z extent when > 1) or
+// the head/axis (S2)
 template <int NSPLIT, class Op>
 static cudaError_t launch_gemm(dim3 grid, const CUtensorMap &a0, const CUtensorMap &a1,
                                const CUtensorMap &b, Op op, int nkb, bool pdl,
                                cudaStream_t st) {
+    if (persistent_ok<NSPLIT>(grid, op))
+        return launch_gemm_persistent<NSPLIT>(grid, a0, a1, b, op, nkb, pdl, st);
     op.stages = stages_for(NSPLIT, op.n_tile, nkb);
     size_t ring = (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile);
     const size_t smem = 1024 + ring;
@@ -498,16 +751,18 @@ static cudaError_t launch_gemm(dim3 grid, const CUtensorMap &a0, const CUtensorM
 }
 
 template <int NSPLIT, class Op> static cudaError_t allow_smem() {
-    return cudaFuncSetAttribute(tc_gemm_kernel<NSPLIT, Op>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBudget);
+    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<NSPLIT, Op>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemBudget);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(tc_gemm_persistent<NSPLIT, Op>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBudget);
+    return e;
 }
 
 cudaError_t configure_tc() {
     cudaError_t e = allow_smem<1, QueryOp>();
-    if (e == cudaSuccess) e = allow_smem<3, ScoreOp<1>>();
-    if (e == cudaSuccess) e = allow_smem<3, ScoreOp<2>>();
-    if (e == cudaSuccess) e = allow_smem<3, ScoreOp<3>>();
-    if (e == cudaSuccess) e = allow_smem<3, ScoreOp<4>>();
+    if (e == cudaSuccess) e = allow_smem<3, ScoreOp>();
     if (e == cudaSuccess) e = allow_smem<1, ProjOp>();
     return e;
 }
@@ -533,9 +788,13 @@ cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int 
         op.kb_total = kb_total;
         op.H = d.H;
         op.d_k = d.d_k;
+        op.dk = d.dk;
+        op.r = d.r;
         op.Bmax = Bmax;
         op.q_part = p.q_part;
         op.qs = qs;
+        op.u = p.u;
+        op.t = p.t;
         dim3 grid((HD + kTileM - 1) / kTileM, (d.B + n_tile - 1) / n_tile, splits);
         const int per = (kb_total + splits - 1) / splits;
         cudaError_t e = launch_gemm<1>(grid, a == 0 ? mp.w_q : mp.w_q_col, mp.w_q, mp.x, op, per,
@@ -545,34 +804,20 @@ cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int 
     return cudaSuccess;
 }
 
-template <int R>
-static cudaError_t launch_score_r(const Dims &d, const Ptrs &p, const TcMaps &mp,
-                                  cudaStream_t st) {
-    ScoreOp<R> op;
-    op.n_tile = tc_n_tile(d.B, R);
-    op.n_acc = R;
-    op.acc_chunk = d.dk;
+cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
+    ScoreOp op;
+    op.n_tile = tc_n_tile(d.B, 1);
+    op.n_acc = 1;
+    op.acc_chunk = 1 << 30;
     op.b_split_stride = d.d_k;
     op.err = p.err;
     op.B = d.B;
     op.H = d.H;
     op.K = d.K;
-    op.A = d.A;
     op.kb_total = (d.d_k + kBlockK - 1) / kBlockK;
-    op.u = p.u;
-    op.t = p.t;
     op.akey = p.akey;
     dim3 grid((d.K + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 2 * d.H);
     return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs, op, op.kb_total, d.pdl, st);
-}
-
-cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
-    switch (d.r) {
-    case 1: return launch_score_r<1>(d, p, mp, st);
-    case 2: return launch_score_r<2>(d, p, mp, st);
-    case 3: return launch_score_r<3>(d, p, mp, st);
-    default: return launch_score_r<4>(d, p, mp, st);
-    }
 }
 
 cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
