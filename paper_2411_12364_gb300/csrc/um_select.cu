@@ -33,6 +33,7 @@ constexpr int kCap = 1024;                 // candidates per selection
 constexpr int kPerThread = kCap / kThreads;
 constexpr int kMaxK = 128;
 constexpr int kMaxM = 1024;
+static_assert(kMaxM <= kCap, "the final winners reuse a candidate list");
 constexpr int kMaxR = 8;
 constexpr int kRankSort = 256;             // longer lists are tightened first
 constexpr unsigned kFull = 0xffffffffu;
@@ -46,9 +47,9 @@ constexpr int kCntTopT = 5;      // tightened final top-m
 typedef unsigned long long u64;
 
 struct SelShared {
-    __align__(16) u64 cand[2][kCap];   // flat candidate lists, one per selection
+    __align__(16) u64 cand[2][kCap];   // flat candidate lists, one per selection; the
+                                       // final winners by rank reuse list 1
     __align__(16) u64 win[2][kMaxK];   // axis winners by rank
-    __align__(16) u64 fwin[kMaxM];     // final winners by rank
     float core[kMaxR * kMaxR];         // C of this head
     int cnt[8];                        // list lengths (may exceed kCap: overflow)
     uint32_t vt[2][kWarps];
@@ -502,6 +503,9 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
         // vector u of the row (EPV elements) belongs to chunk u*EPV / dk
         const uint4 *rv = reinterpret_cast<const uint4 *>(row);
         const int nvec = D / EPV;
+        // chunk of element x = floor(x / dk), as floor((x + 1/2) / dk) in fp32:
+        // exact while x, dk < 2^20 (the error stays below 1/(2 dk))
+        const float inv_dk = 1.f / (float)dk;
 #pragma unroll 1
         for (int u0 = sub; u0 < nvec; u0 += 8 * G) {
             uint4 buf[8];
@@ -527,9 +531,10 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
                         pv = fmaf(f[4 * e4 + 2], q4.z, pv);
                         pv = fmaf(f[4 * e4 + 3], q4.w, pv);
                     }
-                    const int al = iv * EPV / dk;
+                    const int al = (int)(((float)(iv * EPV) + 0.5f) * inv_dk);
 #pragma unroll
-                    for (int a = 0; a < kMaxR; ++a) S[a] += a == al ? pv : 0.f;
+                    for (int a = 0; a < kMaxR; ++a)
+                        if (a < r) S[a] += a == al ? pv : 0.f;   // r is uniform
                 }
             }
         }
@@ -571,8 +576,11 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
     }
 }
 
-template <typename T>
-__global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
+// MINB: resident CTAs per SM the registers are sized for (3: about 80
+// registers, for grids of up to about three CTAs per SM, where a CTA's
+// latency matters; 4: 64 registers, for long grids, where occupancy does).
+template <typename T, int MINB>
+__global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ SelShared sh;
     const int b = blockIdx.x / d.H, h = blockIdx.x % d.H;
@@ -628,6 +636,8 @@ __global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
     axis_survivors<T>(d, p, h, L, sh);
     __syncthreads();
 
+    u64 *const fwin = sh.cand[1];   // final winners by rank (list 1 is free now)
+
     // Eq. 10: g(i,j) = sum_b R[i][b] S_col[b,j] on I x J, R = S_row^T C
     const int k2 = k * k;
     uint32_t g1 = 0u, g2 = 0u;
@@ -635,8 +645,15 @@ __global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
         const int dii = kThreads / k, djj = kThreads % k;   // (ii, jj) step per c += kThreads
         int ii = threadIdx.x / k, jj = threadIdx.x % k;
         for (int c = threadIdx.x; c < k2; c += kThreads) {
-            float g = 0.f;
-            for (int be = 0; be < r; ++be) g = fmaf(L.R[ii * r + be], L.scol[jj * r + be], g);
+            float g;
+            if (r == 2) {   // the common rank, without the loop
+                const float2 a2 = *reinterpret_cast<const float2 *>(L.R + ii * 2);
+                const float2 b2 = *reinterpret_cast<const float2 *>(L.scol + jj * 2);
+                g = fmaf(a2.y, b2.y, a2.x * b2.x);
+            } else {
+                g = 0.f;
+                for (int be = 0; be < r; ++be) g = fmaf(L.R[ii * r + be], L.scol[jj * r + be], g);
+            }
             const uint32_t kg = f2ord(g);
             L.key0[c] = kg;
             top2(kg, g1, g2);
@@ -650,15 +667,15 @@ __global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
     compact<1>(L.key0, nullptr, k2, block_bound(0, sh), 0u, sh, kCntTop, kCntTop);
     __syncthreads();
     const int cf = settle(0, L.key0, k2, m, kCntTop, kCntTopT, sh);
-    rank_list(sh.cand[0], cf, m, sh.fwin, threadIdx.x, kThreads);
+    rank_list(sh.cand[0], cf, m, fwin, threadIdx.x, kThreads);
     __syncthreads();
 
     // PKM's softmax over the m selected scores (Eq. 3); Trick 1 skips it
-    const float gmax = ord2f(key_of(sh.fwin[0]));
+    const float gmax = ord2f(key_of(fwin[0]));
     if (d.act == ULTRAMEM_ACT_SOFTMAX) {
         if (threadIdx.x < 32) {
             float z = 0.f;
-            for (int e = threadIdx.x; e < m; e += 32) z += __expf(ord2f(key_of(sh.fwin[e])) - gmax);
+            for (int e = threadIdx.x; e < m; e += 32) z += __expf(ord2f(key_of(fwin[e])) - gmax);
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(kFull, z, off);
             if (threadIdx.x == 0) sh.scalar = z;
@@ -669,7 +686,7 @@ __global__ void __launch_bounds__(kThreads, 3) select_kernel(Dims d, Ptrs p) {
     const uint32_t N = (uint32_t)d.N;
     const uint32_t row_bytes = (uint32_t)d.d_v * (d.dtype == ULTRAMEM_BF16 ? 2u : 4u);
     for (int e = threadIdx.x; e < m; e += kThreads) {
-        const u64 wc = sh.fwin[e];
+        const u64 wc = fwin[e];
         const int c = (int)pos_of(wc);
         const int ii = c / k, jj = c - ii * k;
         const uint64_t v = (uint64_t)L.sel_i[ii] * (uint64_t)K + (uint64_t)L.sel_j[jj];
@@ -717,10 +734,16 @@ size_t select_smem_bytes(const Dims &d) { return sel_offsets(d).total; }
 
 cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st) {
     const size_t smem = select_smem_bytes(d);
+    const bool long_grid = d.B * d.H > 3 * 152;
     if (d.dtype == ULTRAMEM_BF16)
-        return launch_kernel(d.pdl, select_kernel<__nv_bfloat16>, d.B * d.H, kThreads, smem, st,
-                             d, p);
-    return launch_kernel(d.pdl, select_kernel<float>, d.B * d.H, kThreads, smem, st, d, p);
+        return long_grid ? launch_kernel(d.pdl, select_kernel<__nv_bfloat16, 4>, d.B * d.H,
+                                         kThreads, smem, st, d, p)
+                         : launch_kernel(d.pdl, select_kernel<__nv_bfloat16, 3>, d.B * d.H,
+                                         kThreads, smem, st, d, p);
+    return long_grid ? launch_kernel(d.pdl, select_kernel<float, 4>, d.B * d.H, kThreads, smem,
+                                     st, d, p)
+                     : launch_kernel(d.pdl, select_kernel<float, 3>, d.B * d.H, kThreads, smem,
+                                     st, d, p);
 }
 
 cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream_t st) {
@@ -734,11 +757,12 @@ cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream
 
 cudaError_t configure_select(const Dims &d) {
     const int bytes = (int)select_smem_bytes(d);
-    cudaError_t e = cudaFuncSetAttribute(select_kernel<float>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(select_kernel<__nv_bfloat16>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
+    cudaError_t e = cudaFuncSetAttribute(select_kernel<float, 3>, a, bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<float, 4>, a, bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<__nv_bfloat16, 3>, a, bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<__nv_bfloat16, 4>, a, bytes);
+    return e;
 }
 
 }  // namespace um

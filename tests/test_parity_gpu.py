@@ -49,6 +49,8 @@ SMALL = [
     dict(dtype=0, n=6, topk=5, topm=25),     # m = k*k
     dict(dtype=1, heads=4, topk=16, topm=40, d_v=128, d_out=40),
     dict(dtype=0, shuffle_seed=0),
+    dict(dtype=1, rank=3, d_k=48),           # tensor path, odd rank (folded query)
+    dict(dtype=1, rank=5, d_k=40, heads=3),  # tensor path, 8-wide rank chunks
 ]
 
 
