@@ -160,8 +160,10 @@ ultramem_status ultramem_lookup_reduce_noalloc(const ultramem_config *cfg, const
                                                void *out, void *stream);
 
 /* Synchronises `stream`, then reads and clears the layer's device error word:
- * ULTRAMEM_EDEVICE if a kernel recorded a bad index, ULTRAMEM_ETIMEOUT if a
- * bounded wait gave up, ULTRAMEM_ECUDA if the stream reports an error. */
+ * ULTRAMEM_EDEVICE if a kernel recorded a bad index (or, never expected, a
+ * selection position outside its grid, whose slot it then skipped),
+ * ULTRAMEM_ETIMEOUT if a bounded wait gave up, ULTRAMEM_ECUDA if the stream
+ * reports an error. */
 ultramem_status ultramem_check(ultramem_layer *layer, void *stream);
 
 /* Leading singular triplet of one r x r core (HOST, row-major fp32) with the

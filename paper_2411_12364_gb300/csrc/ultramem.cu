@@ -639,7 +639,7 @@ ultramem_status ultramem_check(ultramem_layer *L, void *stream) {
         return ULTRAMEM_ECUDA;
     if (flags && cudaMemset(L->ws.err, 0, sizeof(int)) != cudaSuccess) return ULTRAMEM_ECUDA;
     if (flags & um::kErrTimeout) return ULTRAMEM_ETIMEOUT;
-    if (flags & um::kErrBadIndex) return ULTRAMEM_EDEVICE;
+    if (flags & (um::kErrBadIndex | um::kErrInternal)) return ULTRAMEM_EDEVICE;
     return ULTRAMEM_OK;
 }
 

@@ -24,6 +24,7 @@ namespace um {
 
 constexpr int kErrBadIndex = 1;   // an address outside [0, E*N) was given
 constexpr int kErrTimeout = 2;    // a bounded wait gave up
+constexpr int kErrInternal = 4;   // a selection produced an impossible position
 
 struct Dims {
     int B;            // tokens in this call

@@ -53,6 +53,7 @@ struct SelShared {
     float core[kMaxR * kMaxR];         // C of this head
     int cnt[8];                        // list lengths (may exceed kCap: overflow)
     uint32_t vt[2][kWarps];
+    __align__(16) u64 runs[kThreads];  // sorted warp runs of rank_sorted
     int hist[256];
     int warp_tot[kWarps];
     int digit, remaining;
@@ -356,6 +357,55 @@ __device__ __forceinline__ void prefetch_l2(const void *ptr, uint32_t bytes) {
     for (uint32_t o = 0; o < bytes; o += 128) asm volatile("prefetch.global.L2 [%0];" ::"l"(c + o));
 }
 
+template <int ID>
+__device__ __forceinline__ void named_barrier(int nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"n"(ID), "r"(nthreads) : "memory");
+}
+
+// Exact ranks of the c <= nt entries of list (distinct composites) for
+// threads [0, nt) of the selection (tid the thread's index among them, nt a
+// multiple of 32): each warp sorts its run of 32 in registers (descending
+// bitonic network), the runs go to runs[nt], and an entry's rank is its place
+// in its own run plus, per other run, the number of entries above it (a
+// 5-step binary search).  Entries of rank < kk go to win[rank].  BAR: the
+// named barrier of these nt threads.
+template <int BAR, int NT>
+__device__ void rank_sorted(const u64 *list, int c, int kk, u64 *win, u64 *runs, int tid) {
+    constexpr int nt = NT, nw = NT / 32;
+    const int lane = tid & 31, w = tid >> 5;
+    u64 x = tid < c ? list[tid] : 0ull;   // padding sorts below every entry
+#pragma unroll
+    for (int blk = 2; blk <= 32; blk <<= 1)
+#pragma unroll
+        for (int st = blk >> 1; st > 0; st >>= 1) {
+            const u64 o = __shfl_xor_sync(kFull, x, st);
+            const bool keep_max = ((lane & st) == 0) == ((lane & blk) == 0);
+            x = keep_max ? (x > o ? x : o) : (x < o ? x : o);
+        }
+    runs[w * 32 + lane] = x;
+    named_barrier<BAR>(nt);
+    const int cw = min(32, max(0, c - 32 * w));   // real entries of this run
+    if (lane < cw) {
+        // the searches of the other runs are independent: interleaved steps
+        int pos[nw];
+#pragma unroll
+        for (int v = 0; v < nw; ++v) pos[v] = 0;
+#pragma unroll
+        for (int step = 16; step > 0; step >>= 1)
+#pragma unroll
+            for (int v = 0; v < nw; ++v)
+                if (runs[v * 32 + pos[v] + step - 1] > x) pos[v] += step;
+        int rank = lane;
+#pragma unroll
+        for (int v = 0; v < nw; ++v) {
+            // entries of the descending run above x: 0 .. 32 (the steps reach 31)
+            const int cnt = pos[v] + (runs[v * 32 + pos[v]] > x);
+            rank += v == w ? 0 : cnt;
+        }
+        if (rank < kk) win[rank] = x;
+    }
+}
+
 struct SelLayout {
     float *qv;          // [2][D_k] row and column query of this (token, head)
     uint32_t *key0;     // [max(K, k*k)] axis-0 keys, then the g keys
@@ -467,19 +517,25 @@ __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1
 // v = i*K + j), and its exact chunk scores S_alpha (Eq. 4) from 16-byte
 // loads of its key row split over the group.  Row survivors store
 // R[i][b] = sum_a S_row[a,i] C[a,b], column survivors S_col[j][b].
-template <typename T>
+// RM >= r bounds the rank at compile time (2 for the common ranks, else 8).
+template <typename T, int RM>
 __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLayout &L,
                                const SelShared &sh) {
     constexpr int EPV = 16 / sizeof(T);
     const int k = d.k, r = d.r, dk = d.dk, D = d.d_k;
-    int G = 1;
-    while (G < 32 && 2 * k * G * 2 <= kThreads) G <<= 1;
+    int lg = 0;   // G = 2^lg lanes per survivor
+    while (lg < 5 && 2 * k * (2 << lg) <= kThreads) ++lg;
+    const int G = 1 << lg;
     const int lane = threadIdx.x & 31, sub = lane & (G - 1);
-    const int sv = threadIdx.x / G;   // 2k * G <= kThreads: one pass
+    const int sv = threadIdx.x >> lg;   // 2k * G <= kThreads: one pass
     const bool active = sv < 2 * k;
     const int s = active && sv >= k ? 1 : 0;
     const int qi = active ? sv - s * k : 0;
-    const uint32_t pos = active ? pos_of(sh.win[s][qi]) : 0u;
+    uint32_t pos = active ? pos_of(sh.win[s][qi]) : 0u;
+    if (active && pos >= (uint32_t)d.K) {   // never expected: record and skip
+        if (sub == 0) atomicOr(p.err, kErrInternal);
+        pos = 0u;
+    }
 
     int ord = 0;
     if (active) {
@@ -495,9 +551,9 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
 
     const T *row = static_cast<const T *>(s ? p.k_col : p.k_row) + ((int64_t)h * d.K + pos) * D;
     const float *q = L.qv + s * D;
-    float S[kMaxR];
+    float S[RM];
 #pragma unroll
-    for (int a = 0; a < kMaxR; ++a) S[a] = 0.f;
+    for (int a = 0; a < RM; ++a) S[a] = 0.f;
     const bool vec = D % EPV == 0 && dk % EPV == 0 && ((uintptr_t)row & 15) == 0;
     if (vec) {
         // vector u of the row (EPV elements) belongs to chunk u*EPV / dk
@@ -533,14 +589,14 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
                     }
                     const int al = (int)(((float)(iv * EPV) + 0.5f) * inv_dk);
 #pragma unroll
-                    for (int a = 0; a < kMaxR; ++a)
+                    for (int a = 0; a < RM; ++a)
                         if (a < r) S[a] += a == al ? pv : 0.f;   // r is uniform
                 }
             }
         }
     } else {
 #pragma unroll
-        for (int a = 0; a < kMaxR; ++a) {
+        for (int a = 0; a < RM; ++a) {
             if (a < r && active) {
                 float acc = 0.f;
                 for (int c = a * dk + sub; c < (a + 1) * dk; c += G)
@@ -550,7 +606,7 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
         }
     }
 #pragma unroll
-    for (int a = 0; a < kMaxR; ++a) {
+    for (int a = 0; a < RM; ++a) {
         if (a < r)
             for (int off = G >> 1; off > 0; off >>= 1) S[a] += __shfl_xor_sync(kFull, S[a], off);
     }
@@ -558,11 +614,11 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
         if (s == 0) {
             L.sel_i[ord] = (int)pos;
 #pragma unroll
-            for (int b = 0; b < kMaxR; ++b) {
+            for (int b = 0; b < RM; ++b) {
                 if (b < r) {
                     float acc = 0.f;
 #pragma unroll
-                    for (int a = 0; a < kMaxR; ++a)
+                    for (int a = 0; a < RM; ++a)
                         if (a < r) acc = fmaf(S[a], sh.core[a * r + b], acc);
                     L.R[ord * r + b] = acc;
                 }
@@ -570,7 +626,7 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
         } else {
             L.sel_j[ord] = (int)pos;
 #pragma unroll
-            for (int b = 0; b < kMaxR; ++b)
+            for (int b = 0; b < RM; ++b)
                 if (b < r) L.scol[ord * r + b] = S[b];
         }
     }
@@ -627,13 +683,24 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     const int c0 = settle(0, L.key0, K, k, kCntAxis, kCntAxisT, sh);
     const int c1 = settle(1, L.key1, K, k, kCntAxis + 1, kCntAxisT + 1, sh);
     {
-        const int s = threadIdx.x >= kThreads / 2;
-        rank_list(sh.cand[s], s ? c1 : c0, k, sh.win[s], threadIdx.x & (kThreads / 2 - 1),
-                  kThreads / 2);
+        const int s = threadIdx.x >= kThreads / 2, cs = s ? c1 : c0;
+        const int tid = threadIdx.x & (kThreads / 2 - 1);
+        // long grids (issue-bound) rank by sorted runs, which execute fewer
+        // instructions; decode grids (latency-bound) by counting, which
+        // has the shorter dependency chain
+        if (MINB >= 4 && c0 <= kThreads / 2 && c1 <= kThreads / 2) {   // uniform
+            if (s)   // warp-uniform: each half of the block has its own barrier
+                rank_sorted<2, kThreads / 2>(sh.cand[1], cs, k, sh.win[1], sh.runs + kThreads / 2,
+                                             tid);
+            else
+                rank_sorted<1, kThreads / 2>(sh.cand[0], cs, k, sh.win[0], sh.runs, tid);
+        } else
+            rank_list(sh.cand[s], cs, k, sh.win[s], tid, kThreads / 2);
     }
     __syncthreads();
     // survivors in increasing index with their exact chunk scores (Eq. 4)
-    axis_survivors<T>(d, p, h, L, sh);
+    if (r <= 2) axis_survivors<T, 2>(d, p, h, L, sh);
+    else axis_survivors<T, kMaxR>(d, p, h, L, sh);
     __syncthreads();
 
     u64 *const fwin = sh.cand[1];   // final winners by rank (list 1 is free now)
@@ -667,7 +734,9 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     compact<1>(L.key0, nullptr, k2, block_bound(0, sh), 0u, sh, kCntTop, kCntTop);
     __syncthreads();
     const int cf = settle(0, L.key0, k2, m, kCntTop, kCntTopT, sh);
-    rank_list(sh.cand[0], cf, m, fwin, threadIdx.x, kThreads);
+    if (MINB >= 4 && cf <= kThreads)
+        rank_sorted<3, kThreads>(sh.cand[0], cf, m, fwin, sh.runs, threadIdx.x);
+    else rank_list(sh.cand[0], cf, m, fwin, threadIdx.x, kThreads);
     __syncthreads();
 
     // PKM's softmax over the m selected scores (Eq. 3); Trick 1 skips it
@@ -687,7 +756,11 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     const uint32_t row_bytes = (uint32_t)d.d_v * (d.dtype == ULTRAMEM_BF16 ? 2u : 4u);
     for (int e = threadIdx.x; e < m; e += kThreads) {
         const u64 wc = fwin[e];
-        const int c = (int)pos_of(wc);
+        int c = (int)pos_of(wc);
+        if ((uint32_t)c >= (uint32_t)k2) {   // never expected: record and skip
+            atomicOr(p.err, kErrInternal);
+            c = 0;
+        }
         const int ii = c / k, jj = c - ii * k;
         const uint64_t v = (uint64_t)L.sel_i[ii] * (uint64_t)K + (uint64_t)L.sel_j[jj];
         const float g = ord2f(key_of(wc));

@@ -243,3 +243,27 @@ def test_last_launches_counts_each_call(gpu_lib):
     cfg32 = workloads.small_config(dtype=0)
     layer32, *_ = _run(cfg32, 16, gpu_lib)
     assert layer32.last_launches() == 6
+
+
+LONG_GRID = [
+    dict(dtype=1, topk=48, topm=1),                          # k = K: every key a candidate
+    dict(dtype=0, n=6, topk=5, topm=25),                     # m = k*k
+    dict(dtype=1, heads=4, topk=16, topm=40, d_v=128, d_out=40),
+    dict(dtype=1, topk=24, topm=64),
+]
+
+
+@pytest.mark.parametrize("over", LONG_GRID, ids=[str(i) for i in range(len(LONG_GRID))])
+def test_long_grid_selection(over, gpu_lib):
+    """Batches whose selection grid exceeds three CTAs per SM (here 300 tokens
+    x H heads) take the long-grid selection, which ranks candidates by
+    sorted warp runs instead of counting; its lists here fill several runs."""
+    cfg = workloads.small_config(**over)
+    _run(cfg, 300, gpu_lib)
+
+
+@pytest.mark.parametrize("rows_tied", [1200, 500])
+def test_tied_keys_long_grid(rows_tied, gpu_lib):
+    """The tie cases above on the long-grid selection (240 tokens x 2 heads)."""
+    cfg = workloads.small_config(dtype=1, n=600, topk=40, topm=64)
+    _run_weights(cfg, _tied_weights(cfg, rows_tied), 240, gpu_lib)
