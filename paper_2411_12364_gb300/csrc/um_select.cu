@@ -635,7 +635,9 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
 // MINB: resident CTAs per SM the registers are sized for (3: about 80
 // registers, for grids of up to about three CTAs per SM, where a CTA's
 // latency matters; 4: 64 registers, for long grids, where occupancy does).
-template <typename T, int MINB>
+// RM >= r: the rank bound of the survivor phase (2, or 8 for larger ranks),
+// one per kernel so that each carries a single copy of it.
+template <typename T, int MINB, int RM>
 __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ SelShared sh;
@@ -699,8 +701,7 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     }
     __syncthreads();
     // survivors in increasing index with their exact chunk scores (Eq. 4)
-    if (r <= 2) axis_survivors<T, 2>(d, p, h, L, sh);
-    else axis_survivors<T, kMaxR>(d, p, h, L, sh);
+    axis_survivors<T, RM>(d, p, h, L, sh);
     __syncthreads();
 
     u64 *const fwin = sh.cand[1];   // final winners by rank (list 1 is free now)
@@ -805,18 +806,20 @@ __global__ void slots_kernel(Dims d, Ptrs p) {
 
 size_t select_smem_bytes(const Dims &d) { return sel_offsets(d).total; }
 
+template <typename T, int RM>
+static cudaError_t launch_select_t(const Dims &d, const Ptrs &p, size_t smem, cudaStream_t st) {
+    if (d.B * d.H > 3 * 152)
+        return launch_kernel(d.pdl, select_kernel<T, 4, RM>, d.B * d.H, kThreads, smem, st, d, p);
+    return launch_kernel(d.pdl, select_kernel<T, 3, RM>, d.B * d.H, kThreads, smem, st, d, p);
+}
+
 cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st) {
     const size_t smem = select_smem_bytes(d);
-    const bool long_grid = d.B * d.H > 3 * 152;
     if (d.dtype == ULTRAMEM_BF16)
-        return long_grid ? launch_kernel(d.pdl, select_kernel<__nv_bfloat16, 4>, d.B * d.H,
-                                         kThreads, smem, st, d, p)
-                         : launch_kernel(d.pdl, select_kernel<__nv_bfloat16, 3>, d.B * d.H,
-                                         kThreads, smem, st, d, p);
-    return long_grid ? launch_kernel(d.pdl, select_kernel<float, 4>, d.B * d.H, kThreads, smem,
-                                     st, d, p)
-                     : launch_kernel(d.pdl, select_kernel<float, 3>, d.B * d.H, kThreads, smem,
-                                     st, d, p);
+        return d.r <= 2 ? launch_select_t<__nv_bfloat16, 2>(d, p, smem, st)
+                        : launch_select_t<__nv_bfloat16, kMaxR>(d, p, smem, st);
+    return d.r <= 2 ? launch_select_t<float, 2>(d, p, smem, st)
+                    : launch_select_t<float, kMaxR>(d, p, smem, st);
 }
 
 cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream_t st) {
@@ -828,13 +831,19 @@ cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream
     return cudaGetLastError();
 }
 
+template <typename T, int RM> static cudaError_t allow_select(int bytes) {
+    const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
+    cudaError_t e = cudaFuncSetAttribute(select_kernel<T, 3, RM>, a, bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<T, 4, RM>, a, bytes);
+    return e;
+}
+
 cudaError_t configure_select(const Dims &d) {
     const int bytes = (int)select_smem_bytes(d);
-    const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
-    cudaError_t e = cudaFuncSetAttribute(select_kernel<float, 3>, a, bytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<float, 4>, a, bytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<__nv_bfloat16, 3>, a, bytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<__nv_bfloat16, 4>, a, bytes);
+    cudaError_t e = allow_select<float, 2>(bytes);
+    if (e == cudaSuccess) e = allow_select<float, kMaxR>(bytes);
+    if (e == cudaSuccess) e = allow_select<__nv_bfloat16, 2>(bytes);
+    if (e == cudaSuccess) e = allow_select<__nv_bfloat16, kMaxR>(bytes);
     return e;
 }
 
