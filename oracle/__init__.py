@@ -31,7 +31,7 @@ ACT_NONE, ACT_SOFTMAX = 0, 1
 class Config(C.Structure):
     _fields_ = [(name, C.c_int32) for name in (
         "d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out",
-        "topk", "topm", "has_proj", "share_query", "act", "dtype")] + [
+        "topk", "topm", "has_proj", "share_query", "act", "dtype", "cores")] + [
         ("shuffle_seed", C.c_uint64)]
 
 
@@ -80,7 +80,13 @@ def make_config(cfg: dict) -> Config:
     c = Config()
     for k in _CFG_KEYS:
         setattr(c, k, int(cfg[k]))
+    c.cores = int(cfg.get("cores", 0))
     return c
+
+
+def cores_of(cfg: dict) -> int:
+    """h, the component cores per head (Multi-Core Scoring, Sec. 3.2)."""
+    return max(1, int(cfg.get("cores", 0)))
 
 
 def keys_per_axis(cfg: dict) -> int:
@@ -120,7 +126,9 @@ def _tensors(cfg: dict, t: dict):
 def forward(cfg: dict, tensors: dict, B: int, tokens=None, threads: int = 0):
     """Eq. 4-10 then Eq. 13-15 for the listed tokens (all B if None).
 
-    Returns ``(out [n, d_out] f64, idx [n, H, m] i64, w [n, H, m] f64)``."""
+    Returns ``(out [n, d_out] f64, idx [n, H, m] i64, w [n, H, m] f64)``;
+    with h > 1 component cores (MCS) ``w`` is ``[n, H, m, h]``, the score of
+    each core at the slot."""
     lib = _load()
     c = make_config(cfg)
     s, keep = _tensors(cfg, tensors)
@@ -129,7 +137,8 @@ def forward(cfg: dict, tensors: dict, B: int, tokens=None, threads: int = 0):
     H, m = int(cfg["heads"]), int(cfg["topm"])
     out = np.zeros((n, int(cfg["d_out"])), np.float64)
     idx = np.zeros((n, H, m), np.int64)
-    w = np.zeros((n, H, m), np.float64)
+    h = cores_of(cfg)
+    w = np.zeros((n, H, m) if h == 1 else (n, H, m, h), np.float64)
     st = lib.uo_forward(C.byref(c), C.byref(s), int(B), _ptr(tok), int(n),
                         out.ctypes.data, idx.ctypes.data, w.ctypes.data, int(threads))
     del keep
@@ -139,13 +148,16 @@ def forward(cfg: dict, tensors: dict, B: int, tokens=None, threads: int = 0):
 
 
 def lookup_reduce(cfg: dict, tensors: dict, idx, w, threads: int = 0):
-    """Eq. 14-15 alone on given (virtual address, weight) pairs [n, H, m]."""
+    """Eq. 14-15 alone on given virtual addresses [n, H, m] and weights
+    [n, H, m] (or [n, H, m, h], one per value slice, with h > 1 cores)."""
     lib = _load()
     c = make_config(cfg)
     s, keep = _tensors(cfg, tensors)
     idx = np.ascontiguousarray(idx, dtype=np.int64)
     w = np.ascontiguousarray(w, dtype=np.float64)
     n = idx.shape[0]
+    if w.size != idx.size * cores_of(cfg):
+        raise ValueError(f"weights {w.shape} do not match addresses {idx.shape}")
     out = np.zeros((n, int(cfg["d_out"])), np.float64)
     st = lib.uo_lookup_reduce(C.byref(c), C.byref(s), int(n), idx.ctypes.data,
                               w.ctypes.data, out.ctypes.data, int(threads))

@@ -66,8 +66,14 @@ static int check_config(const uo_config *cfg)
     if (cfg->has_proj && cfg->d_out <= 0) return UO_EINVAL;
     if (cfg->dtype != UO_F32 && cfg->dtype != UO_BF16) return UO_EINVAL;
     if (cfg->act != UO_ACT_NONE && cfg->act != UO_ACT_SOFTMAX) return UO_EINVAL;
+    if (cfg->cores < 0 || cfg->cores > 8) return UO_EINVAL;
+    if (cfg->cores > 1 && (cfg->d_v % cfg->cores != 0 || cfg->act != UO_ACT_NONE))
+        return UO_EINVAL;
     return UO_OK;
 }
+
+/* h, the number of component cores of each head (Sec. 3.2, MCS) */
+static int32_t cores_of(const uo_config *cfg) { return cfg->cores > 1 ? cfg->cores : 1; }
 
 /* ---- Eq. 7 / Eq. 11: leading singular triplet of the Tucker core -------- */
 
@@ -287,12 +293,15 @@ static void pool_and_project(const uo_config *cfg, const uo_tensors *x,
     const int64_t N = (int64_t)cfg->n * cfg->n;
     const int32_t E = cfg->expand_e, Dv = cfg->d_v, Do = cfg->d_out;
     const int64_t hm = (int64_t)cfg->heads * cfg->topm;
+    const int32_t nc = cores_of(cfg), slice = Dv / nc;
     memset(acc, 0, sizeof(double) * E * Dv);
     for (int64_t e = 0; e < hm; ++e) {
         int64_t vs = uo_shuffle(cfg, x->perm, idx[e]);
         int64_t p = vs / N, row = vs % N;
+        /* MCS: element c of the row lies in slice c / (D_v/h), weighted by
+         * that core's score (one slice, the plain weight, without MCS) */
         for (int32_t c = 0; c < Dv; ++c)
-            acc[p * Dv + c] += w[e] * load(x->values, cfg->dtype, row * Dv + c);
+            acc[p * Dv + c] += w[e * nc + c / slice] * load(x->values, cfg->dtype, row * Dv + c);
     }
     if (!cfg->has_proj) {
         for (int32_t c = 0; c < Dv; ++c) out[c] = acc[c];
@@ -333,7 +342,7 @@ int uo_lookup_reduce(const uo_config *cfg, const uo_tensors *x, int64_t n_tokens
         } else {
 #pragma omp for schedule(dynamic, 1)
             for (int64_t b = 0; b < n_tokens; ++b)
-                pool_and_project(cfg, x, idx + b * hm, w + b * hm, acc,
+                pool_and_project(cfg, x, idx + b * hm, w + b * hm * cores_of(cfg), acc,
                                  out + b * cfg->d_out);
         }
         free(acc);
@@ -344,7 +353,7 @@ int uo_lookup_reduce(const uo_config *cfg, const uo_tensors *x, int64_t n_tokens
 /* ---- the whole layer for one token ------------------------------------- */
 
 typedef struct {
-    double *q, *s_row, *s_col, *a, *bcol, *acc, *sel_w, *pool_w;
+    double *q, *s_row, *s_col, *a, *bcol, *acc, *sel_w, *pool_w, *core;
     scored *axis, *cand;
     int64_t *sel_i, *sel_j, *sel_v;
 } scratch;
@@ -362,9 +371,16 @@ static void token_forward(const uo_config *cfg, const uo_tensors *x, int64_t b,
     if (cfg->share_query) memcpy(sc->q + HD, sc->q, sizeof(double) * HD);
     else query(cfg, x->w_q_col, x->x, b, sc->q + HD);
 
+    const int32_t nc = cores_of(cfg);
     for (int32_t h = 0; h < H; ++h) {
         const double *u = u_all + (int64_t)h * r, *t = t_all + (int64_t)h * r;
-        const float *C = x->core + (int64_t)h * r * r;
+        /* the Tucker core is the sum of the head's component cores (MCS) */
+        const float *Ci = x->core + (int64_t)h * nc * r * r;
+        double *C = sc->core;
+        for (int32_t e = 0; e < r * r; ++e) {
+            C[e] = 0.0;
+            for (int32_t i = 0; i < nc; ++i) C[e] += (double)Ci[(int64_t)i * r * r + e];
+        }
 
         /* Eq. 4: S_row, S_col in R^{r x K} */
         row_col_scores(cfg, x, h, sc->q + (int64_t)h * cfg->d_k,
@@ -398,21 +414,21 @@ static void token_forward(const uo_config *cfg, const uo_tensors *x, int64_t b,
         for (int32_t e = 0; e < k; ++e) sc->sel_j[e] = sc->axis[e].index;
 
         /* Eq. 10: exact Tucker score S_row^T C S_col on the k*k survivors */
-        int64_t nc = 0;
+        int64_t ncand = 0;
         for (int32_t ei = 0; ei < k; ++ei)
             for (int32_t ej = 0; ej < k; ++ej) {
                 int64_t i = sc->sel_i[ei], j = sc->sel_j[ej];
                 double g = 0.0;
                 for (int32_t al = 0; al < r; ++al)
                     for (int32_t be = 0; be < r; ++be)
-                        g += sc->s_row[(int64_t)al * K + i] * (double)C[al * r + be] *
+                        g += sc->s_row[(int64_t)al * K + i] * C[al * r + be] *
                              sc->s_col[(int64_t)be * K + j];
-                sc->cand[nc].key = (float)g;
-                sc->cand[nc].index = i * K + j; /* virtual address v */
-                sc->cand[nc].value = g;
-                ++nc;
+                sc->cand[ncand].key = (float)g;
+                sc->cand[ncand].index = i * K + j; /* virtual address v */
+                sc->cand[ncand].value = g;
+                ++ncand;
             }
-        qsort(sc->cand, (size_t)nc, sizeof(scored), by_score_desc_index_asc);
+        qsort(sc->cand, (size_t)ncand, sizeof(scored), by_score_desc_index_asc);
 
         /* Trick 1 uses the selected scores as weights; PKM softmaxes them
          * over the m selected slots (Eq. 3). */
@@ -423,16 +439,31 @@ static void token_forward(const uo_config *cfg, const uo_tensors *x, int64_t b,
             for (int32_t e = 0; e < m; ++e) z += exp(sc->cand[e].value - mx);
             for (int32_t e = 0; e < m; ++e)
                 sc->sel_w[e] = exp(sc->cand[e].value - mx) / z;
-        } else {
+        } else if (nc == 1) {
             for (int32_t e = 0; e < m; ++e) sc->sel_w[e] = sc->cand[e].value;
+        } else {
+            /* MCS: each selected slot's individual scores S_row^T C^(i) S_col */
+            for (int32_t e = 0; e < m; ++e) {
+                const int64_t i = sc->cand[e].index / K, j = sc->cand[e].index % K;
+                for (int32_t ci = 0; ci < nc; ++ci) {
+                    const float *Cc = Ci + (int64_t)ci * r * r;
+                    double g = 0.0;
+                    for (int32_t al = 0; al < r; ++al)
+                        for (int32_t be = 0; be < r; ++be)
+                            g += sc->s_row[(int64_t)al * K + i] * (double)Cc[al * r + be] *
+                                 sc->s_col[(int64_t)be * K + j];
+                    sc->sel_w[(int64_t)e * nc + ci] = g;
+                }
+            }
         }
         for (int32_t e = 0; e < m; ++e) {
             sc->sel_v[(int64_t)h * m + e] = sc->cand[e].index;
             if (idx_out) idx_out[(int64_t)h * m + e] = sc->cand[e].index;
-            if (w_out) w_out[(int64_t)h * m + e] = sc->sel_w[e];
+            for (int32_t ci = 0; ci < nc; ++ci)
+                if (w_out) w_out[((int64_t)h * m + e) * nc + ci] = sc->sel_w[(int64_t)e * nc + ci];
         }
         /* keep this head's weights next to its addresses for pooling */
-        memcpy(sc->pool_w + (int64_t)h * m, sc->sel_w, sizeof(double) * m);
+        memcpy(sc->pool_w + (int64_t)h * m * nc, sc->sel_w, sizeof(double) * m * nc);
     }
     /* Eq. 14-15 over all heads' slots together (heads are summed) */
     pool_and_project(cfg, x, sc->sel_v, sc->pool_w, sc->acc, out);
@@ -471,7 +502,12 @@ int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
             }
         } else {
             double sigma;
-            for (int32_t e = 0; e < r * r; ++e) cd[e] = x->core[(int64_t)h * r * r + e];
+            const int32_t nc = cores_of(cfg);
+            for (int32_t e = 0; e < r * r; ++e) {   /* the aggregate core (MCS) */
+                cd[e] = 0.0;
+                for (int32_t i = 0; i < nc; ++i)
+                    cd[e] += x->core[((int64_t)h * nc + i) * r * r + e];
+            }
             if (uo_rank1(cd, r, u_all + h * r, t_all + h * r, &sigma) != UO_OK) {
                 free(u_all); free(t_all); free(cd);
                 return UO_EINVAL;
@@ -494,18 +530,19 @@ int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
         sc.s_row = malloc(sizeof(double) * r * K);
         sc.s_col = malloc(sizeof(double) * r * K);
         sc.a = malloc(sizeof(double) * K);
-        sc.pool_w = malloc(sizeof(double) * hm);
+        sc.pool_w = malloc(sizeof(double) * hm * cores_of(cfg));
+        sc.core = malloc(sizeof(double) * r * r);
         sc.bcol = malloc(sizeof(double) * K);
         sc.acc = malloc(sizeof(double) * cfg->expand_e * cfg->d_v);
-        sc.sel_w = malloc(sizeof(double) * cfg->topm);
+        sc.sel_w = malloc(sizeof(double) * cfg->topm * cores_of(cfg));
         sc.axis = malloc(sizeof(scored) * K);
         sc.cand = malloc(sizeof(scored) * kk);
         sc.sel_i = malloc(sizeof(int64_t) * cfg->topk);
         sc.sel_j = malloc(sizeof(int64_t) * cfg->topk);
         sc.sel_v = malloc(sizeof(int64_t) * hm);
         int ok = sc.q && sc.s_row && sc.s_col && sc.a && sc.bcol && sc.acc &&
-                 sc.sel_w && sc.pool_w && sc.axis && sc.cand && sc.sel_i && sc.sel_j &&
-                 sc.sel_v;
+                 sc.sel_w && sc.pool_w && sc.core && sc.axis && sc.cand && sc.sel_i &&
+                 sc.sel_j && sc.sel_v;
         if (!ok) {
 #pragma omp atomic write
             status = UO_ENOMEM;
@@ -514,11 +551,12 @@ int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
             for (int64_t e = 0; e < n_tokens; ++e) {
                 int64_t b = tokens ? tokens[e] : e;
                 token_forward(cfg, x, b, u_all, t_all, &sc, out + e * cfg->d_out,
-                              idx ? idx + e * hm : NULL, w ? w + e * hm : NULL);
+                              idx ? idx + e * hm : NULL, w ? w + e * hm * cores_of(cfg) : NULL);
             }
         }
         free(sc.q); free(sc.s_row); free(sc.s_col); free(sc.a); free(sc.bcol);
-        free(sc.acc); free(sc.sel_w); free(sc.pool_w); free(sc.axis); free(sc.cand);
+        free(sc.acc); free(sc.sel_w); free(sc.pool_w); free(sc.core); free(sc.axis);
+        free(sc.cand);
         free(sc.sel_i); free(sc.sel_j); free(sc.sel_v);
     }
     free(u_all);

@@ -24,6 +24,9 @@
  *   Eq. 13  virtual blocks                V~_p = V W_p
  *   Eq. 14  shuffle of virtual addresses  s^ = Shuffle(vec(S_grid))
  *   Eq. 15  implicit value expansion      o = sum_p W_p^T (V^T s^_p)
+ *   Eq. 16-17 Multi-Core Scoring (MCS)    C = sum_i C^(i); top-m on the
+ *           aggregate S_row^T C S_col; physical value slice i (D_v/h wide)
+ *           weighted by the individual score S_row^T C^(i) S_col
  */
 #ifndef ULTRAMEM_ORACLE_H
 #define ULTRAMEM_ORACLE_H
@@ -52,6 +55,8 @@ typedef struct {
     int32_t share_query; /* 1: one query for both key sets (Trick 5)            */
     int32_t act;         /* UO_ACT_NONE (Trick 1) or UO_ACT_SOFTMAX (PKM)       */
     int32_t dtype;       /* UO_F32 or UO_BF16 for x, W_q, keys, V, W_p          */
+    int32_t cores;       /* h: component cores per head (MCS); 0 or 1 = one core.
+                            h > 1 needs D_v % h == 0 and UO_ACT_NONE            */
     uint64_t shuffle_seed; /* 0: identity shuffle; else the seeded bijection   */
 } uo_config;
 
@@ -61,7 +66,8 @@ typedef struct {
     const void *w_q_col;  /* [H*d_k][d_in] column query when share_query == 0   */
     const void *k_row;    /* [H][K][d_k], K = sqrt(E)*n keys per axis            */
     const void *k_col;    /* [H][K][d_k]                                         */
-    const float *core;    /* [H][r][r] Tucker cores C_h, always fp32             */
+    const float *core;    /* [H][h][r][r] component cores C_h^(i), always fp32;
+                             the Tucker core of head h is their sum            */
     const float *u;       /* [H][r] or NULL: leading left singular vectors       */
     const float *t;       /* [H][r] or NULL: leading right singular vectors      */
     const void *values;   /* [N][d_v] physical table V                           */
@@ -78,14 +84,16 @@ enum { UO_OK = 0, UO_EINVAL = -1, UO_ENOMEM = -2 };
  *   out [n_tokens][d_out]   layer output o
  *   idx [n_tokens][H][m]    virtual address v = i*K + j of each selected slot,
  *                           ordered by (score desc, v asc); may be NULL
- *   w   [n_tokens][H][m]    the weight applied to that slot; may be NULL
+ *   w   [n_tokens][H][m][h] the weights applied to that slot, one per core
+ *                           (slice of the value row); may be NULL
  * n_threads <= 0 uses the OpenMP default. */
 int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
                const int64_t *tokens, int64_t n_tokens,
                double *out, int64_t *idx, double *w, int32_t n_threads);
 
-/* Eq. 14-15 alone: pool the given (virtual address, weight) pairs and project.
- * idx/w are [n_tokens][H][m]; only values, w_proj and perm of `x` are read. */
+/* Eq. 14-15 alone: pool the given (virtual address, weights) and project.
+ * idx is [n_tokens][H][m], w [n_tokens][H][m][h]; only values, w_proj and
+ * perm of `x` are read. */
 int uo_lookup_reduce(const uo_config *cfg, const uo_tensors *x, int64_t n_tokens,
                      const int64_t *idx, const double *w, double *out,
                      int32_t n_threads);

@@ -9,7 +9,8 @@ tensor here is drawn from a seeded Gaussian with the scale the layer sees:
   x      ~ N(0, 1)                [B, D_i]
   W_q    ~ N(0, 1/D_i)  variance  [H*D_k, D_i]   (query variance ~1)
   K_row, K_col ~ N(0, 1/D_k) variance [H, K, D_k]  K = sqrt(E) * n
-  C      ~ N(0, 1)                [H, r, r]      Tucker cores
+  C      ~ N(0, 1)                [H, r, r]      Tucker cores; with h > 1
+                                  component cores (MCS) [H, h, r, r] ~ N(0, 1/h)
   V      ~ N(0, 0.02^2)  (std 0.02) [N, D_v]     N = n * n physical rows
   W_p    ~ N(0, 1/(E*D_v)) variance [E, D_v, D'_v]
 
@@ -122,7 +123,9 @@ def make_weights(cfg: dict, device="cpu", with_table=True) -> dict:
         _randn(gen, (H * dk, din), 1.0 / math.sqrt(din), dt)
     w["k_row"] = _randn(gen, (H, K, dk), 1.0 / math.sqrt(dk), dt)
     w["k_col"] = _randn(gen, (H, K, dk), 1.0 / math.sqrt(dk), dt)
-    w["core"] = _randn(gen, (H, r, r), 1.0, torch.float32)
+    h = int(cfg.get("cores", 0))
+    w["core"] = _randn(gen, (H, h, r, r), 1.0 / math.sqrt(h), torch.float32) if h > 1 \
+        else _randn(gen, (H, r, r), 1.0, torch.float32)
     w["w_proj"] = _randn(gen, (E, dv, do), 1.0 / math.sqrt(E * dv), dt) \
         if int(cfg["has_proj"]) else None
     w = {k: (None if v is None else v.to(device)) for k, v in w.items()}

@@ -2,7 +2,9 @@
 examples, the brute-force definition of Eq. 5, the exactness of the
 two-phase search for a rank-1 core (Eq. 6), the PKM reduction at r = 1
 (Eq. 2-3), the explicit virtual table (Eq. 13-15), numpy's SVD (Eq. 7),
-the published SplitMix64 outputs and plain invariants of top-m and softmax."""
+the published SplitMix64 outputs, plain invariants of top-m and softmax,
+and Eq. 16-17 of Multi-Core Scoring (per-core grids by brute force, the
+explicit sliced table, the h = 1 and equal-core reductions)."""
 import json
 import os
 
@@ -26,7 +28,8 @@ def _golden(name):
     return cfg, t, d["expected"]
 
 
-@pytest.mark.parametrize("name", ["hand_tucker_ive.json", "hand_pruning_rows.json"])
+@pytest.mark.parametrize("name", ["hand_tucker_ive.json", "hand_pruning_rows.json",
+                                  "hand_mcs.json"])
 def test_hand_worked_examples(name):
     cfg, t, exp = _golden(name)
     out, idx, w = oracle.forward(cfg, t, B=1)
@@ -396,7 +399,107 @@ def test_invalid_configs_are_rejected():
     base = _f32_cfg()
     t = util.numpy_layer(base, B=1)
     bad = [dict(rank=3), dict(expand_e=3), dict(topk=10 ** 6), dict(topm=26),
-           dict(has_proj=0), dict(act=5)]
+           dict(has_proj=0), dict(act=5), dict(cores=3), dict(cores=2, act=1),
+           dict(cores=9), dict(cores=-1)]
     for kw in bad:
         with pytest.raises(ValueError):
             oracle.forward(dict(base, **kw), t, B=1)
+
+
+# ---- Multi-Core Scoring (Sec. 3.2, Eq. 16-17) -------------------------------
+
+def _mcs_layer(cfg, B, seed=21):
+    """A layer whose h component cores are multiples of 1/8, so that their
+    fp32 sum is exact and a one-core layer can be given the same aggregate."""
+    t = util.numpy_layer(cfg, B=B)
+    H, h, r = cfg["heads"], cfg["cores"], cfg["rank"]
+    rng = np.random.default_rng(seed)
+    t["core"] = (rng.integers(-16, 17, (H, h, r, r)) / 8.0).astype(np.float32)
+    return t
+
+
+def test_mcs_selection_uses_the_aggregate_core():
+    """Eq. 16: top-m runs on S_row^T (sum_i C^(i)) S_col, so the addresses
+    equal those of one core C = sum_i C^(i) (with u, t from its SVD), and the
+    h per-core weights of a slot sum to that slot's aggregate score."""
+    cfg = _f32_cfg(cores=3, rank=3, d_k=12, d_v=9, d_out=10, topk=6, topm=7)
+    t = _mcs_layer(cfg, B=4)
+    out, idx, w = oracle.forward(cfg, t, B=4)
+    assert w.shape == (4, cfg["heads"], cfg["topm"], 3)
+    one = dict(t)
+    one["core"] = t["core"].sum(1)
+    cfg1 = dict(cfg, cores=0)
+    _, idx1, w1 = oracle.forward(cfg1, one, B=4)
+    np.testing.assert_array_equal(idx, idx1)
+    np.testing.assert_allclose(w.sum(-1), w1, rtol=1e-12, atol=1e-13)
+
+
+def test_mcs_weights_are_the_per_core_grids():
+    """Eq. 16-17 by brute force: with k = K (no pruning) the addresses are
+    the top-m of the whole aggregate grid, and weight i of each is the
+    individual map S_row^T C^(i) S_col (numpy reshapes, numpy SVD) there."""
+    cfg = _f32_cfg(cores=2, d_v=8)
+    K = workloads.keys_per_axis(cfg)
+    cfg["topk"] = K
+    t = _mcs_layer(cfg, B=3)
+    out, idx, w = oracle.forward(cfg, t, B=3)
+    for b in range(3):
+        for h in range(cfg["heads"]):
+            agg = t["core"][h].astype(np.float64).sum(0)
+            v, g = util.brute_force_grid(cfg, t, b, h, agg)
+            np.testing.assert_array_equal(idx[b, h], v)
+            s_row, s_col = util.numpy_scores(cfg, t, b, h)
+            for i in range(2):
+                Gi = s_row.T @ t["core"][h, i].astype(np.float64) @ s_col
+                np.testing.assert_allclose(w[b, h, :, i], Gi.ravel()[v], rtol=1e-11,
+                                           atol=1e-12)
+
+
+def test_mcs_explicit_sliced_table():
+    """Eq. 17 with IVE (Eq. 15 on the split physical table): o is the sum
+    over slices i of the explicit virtual-table output of a table whose
+    columns outside slice i are zero, weighted by the i-th scores."""
+    cfg = _f32_cfg(cores=4, d_v=8, d_out=11, heads=3, topm=7, expand_e=4)
+    t = _mcs_layer(cfg, B=5)
+    M = cfg["expand_e"] * cfg["n"] ** 2
+    t["perm"] = np.random.default_rng(9).permutation(M).astype(np.int64)
+    out, idx, w = oracle.forward(cfg, t, B=5)
+    ref = np.zeros_like(out)
+    sl = cfg["d_v"] // 4
+    for i in range(4):
+        ti = dict(t)
+        V = util.widen(t["values"]).copy()
+        V[:, :i * sl] = 0
+        V[:, (i + 1) * sl:] = 0
+        ti["values"] = V.astype(np.float32)
+        ref += util.explicit_ive(cfg, ti, idx, w[..., i], t["perm"])
+    np.testing.assert_allclose(out, ref, rtol=1e-11, atol=1e-13)
+    # lookup_reduce pools the same (address, weights) pairs the same way
+    np.testing.assert_allclose(oracle.lookup_reduce(cfg, t, idx, w), out,
+                               rtol=1e-12, atol=1e-14)
+
+
+def test_mcs_equal_cores_scale_the_output():
+    """h equal component cores C/h: every individual score is g/h, so each
+    slice gets weight g/h and the output is 1/h of the one-core layer's."""
+    cfg = _f32_cfg(cores=2, d_v=8, heads=2)
+    t = util.numpy_layer(cfg, B=3)
+    t1 = util.numpy_layer(dict(cfg, cores=0), B=3)
+    core = t1["core"] * 2
+    t["core"] = np.stack([core / 2, core / 2], axis=1).astype(np.float32)
+    t1["core"] = core.astype(np.float32)
+    out, idx, w = oracle.forward(cfg, t, B=3)
+    out1, idx1, w1 = oracle.forward(dict(cfg, cores=0), t1, B=3)
+    np.testing.assert_array_equal(idx, idx1)
+    np.testing.assert_allclose(w, np.repeat(w1[..., None] / 2, 2, axis=-1), rtol=1e-12)
+    np.testing.assert_allclose(out, out1 / 2, rtol=1e-11, atol=1e-14)
+
+
+def test_mcs_one_core_is_plain():
+    """h = 1 is the layer without MCS: same addresses, weights and output."""
+    cfg = _f32_cfg()
+    t = util.numpy_layer(cfg, B=3)
+    a = oracle.forward(cfg, t, B=3)
+    b = oracle.forward(dict(cfg, cores=1), dict(t, core=t["core"][:, None]), B=3)
+    for x, y in zip(a, b):
+        np.testing.assert_array_equal(x, y)
