@@ -41,6 +41,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=None)
     ap.add_argument("--batch", type=int, default=None)
+    ap.add_argument("--cores", type=int, default=0,
+                    help="component cores per head (Multi-Core Scoring); 0 = one core")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -67,7 +69,8 @@ def algorithmic_bytes(cfg, B):
     with heads: the gather reads min(B*H*m, N) rows of D_v).  The selection
     reads, per (token, head), the rank-1 score keys of both axes (2 K x 4 B),
     the query (A D_k x 4 B) and the key rows of the 2k survivors
-    (2 k D_k x es), and writes m slots (row, block, weight: 12 B)."""
+    (2 k D_k x es), and writes m slots (row, block and h weights: 8 + 4h B,
+    h = 1 without Multi-Core Scoring)."""
     es = 4 if int(cfg["dtype"]) == 0 else 2
     H, dk, din = cfg["heads"], cfg["d_k"], cfg["d_in"]
     K = int(round(cfg["expand_e"] ** 0.5)) * cfg["n"]
@@ -78,7 +81,8 @@ def algorithmic_bytes(cfg, B):
     return {
         "query": A * H * dk * din * es + B * din * es,
         "score": 2 * H * K * dk * es,
-        "select": B * H * (2 * K * 4 + A * dk * 4 + 2 * k * dk * es + m * 12),
+        "select": B * H * (2 * K * 4 + A * dk * 4 + 2 * k * dk * es
+                           + m * (8 + 4 * max(1, int(cfg.get("cores", 0))))),
         "gather": rows * cfg["d_v"] * es,
         "project": (cfg["expand_e"] * cfg["d_v"] * cfg["d_out"] * es if cfg["has_proj"] else 0)
         + B * cfg["d_out"] * es,
@@ -239,6 +243,8 @@ def _cfg_brief(cfg):
     keys = ("d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out", "topk", "topm")
     d = {k: int(cfg[k]) for k in keys}
     d["storage"] = "f32" if int(cfg["dtype"]) == 0 else "bf16"
+    if int(cfg.get("cores", 0)) > 1:
+        d["mcs_cores"] = int(cfg["cores"])
     return d
 
 
@@ -248,7 +254,7 @@ def main():
     wl = args.workload or workloads.HEADLINE[0]
     B = args.batch or (workloads.HEADLINE[1] if wl == workloads.HEADLINE[0]
                        else workloads.CONFIGS[wl]["batches"][-1])
-    cfg = workloads.layer_config(wl)
+    cfg = workloads.layer_config(wl, **({"cores": args.cores} if args.cores > 1 else {}))
     if args.impl == "reference":
         return run_reference(args, cfg, B, wl)
 
@@ -352,7 +358,8 @@ def main():
     dom_bytes = alg[dominant]
     roof = {"kernel": dominant, "bound": "hbm", "achieved": dom_bytes / (stage_avg[dominant] * 1e6),
             "peak": peak, "unit": "GB/s", "peak_kind": peak_kind,
-            "traffic": ncu_traffic(dominant, wl, B), "algorithmic_bytes": dom_bytes,
+            "traffic": None if int(cfg.get("cores", 0)) > 1 else ncu_traffic(dominant, wl, B),
+            "algorithmic_bytes": dom_bytes,
             "avg_ms": stage_avg[dominant]}
     roof["frac"] = roof["achieved"] / peak
     gms = stage_avg.get("gather")

@@ -16,6 +16,13 @@
  *   S8  acc[p] += w * V[row]                       Eq. 15, pooled per virtual block
  *   S9  o = sum_p W_p^T acc[p]                     Eq. 13/15 (IVE) + Trick 6 output
  *
+ * Multi-Core Scoring (Sec. 3.2, Eq. 16-17), when cfg.cores = h > 1: each head's
+ * Tucker core is the sum of h component cores, C = sum_i C^(i).  S3-S6 run on
+ * that sum; each selected slot then carries h weights, the individual scores
+ * g_i(i,j) = S_row[:,i]^T C^(i) S_col[:,j], and weight i scales slice i (columns
+ * i*D_v/h .. (i+1)*D_v/h - 1) of the physical value row in S8 (with IVE the
+ * physical table is split, so Eq. 15 still holds per block).
+ *
  * Shapes (all row-major and contiguous):
  *   K = sqrt(E) * n keys per axis ("the key size is expanded by sqrt(E) times",
  *   Sec. 3.2 IVE); N = n*n physical value rows; the virtual grid has K*K = E*N
@@ -71,7 +78,9 @@ typedef struct ultramem_config {
     int32_t act;         /* ULTRAMEM_ACT_NONE or ULTRAMEM_ACT_SOFTMAX                 */
     int32_t dtype;       /* ULTRAMEM_F32 or ULTRAMEM_BF16                              */
     int32_t max_tokens;  /* largest B any later call may pass; sizes the workspace    */
-    int32_t reserved;    /* must be 0                                                 */
+    int32_t cores;       /* h, component cores per head (MCS, Eq. 16-17): 0 or 1 = one
+                            core; 2..8 needs act == ULTRAMEM_ACT_NONE and
+                            (d_v / h) % 8 == 0                                        */
     uint64_t shuffle_seed; /* Eq. 14 shuffle: 0 = identity, otherwise the seeded
                               bijection pi(v) = (a v + c) mod E*N whose a and c come
                               from the first two SplitMix64 outputs of the seed
@@ -86,10 +95,12 @@ typedef struct ultramem_weights {
     const void *w_q_col;   /* [H*D_k][D_i] column query when share_query == 0, else NULL */
     const void *k_row;     /* [H][K][D_k]; rank chunk alpha = columns alpha*D_k/r..    */
     const void *k_col;     /* [H][K][D_k]                                              */
-    const float *core;     /* HOST fp32 [H][r][r], Tucker cores C_h, copied at create  */
+    const float *core;     /* HOST fp32 [H][h][r][r] (h = max(1, cores)): component
+                              cores C_h^(i), copied at create; C_h is their sum         */
     const float *u;        /* HOST fp32 [H][r] or NULL: leading left singular vectors  */
     const float *t;        /* HOST fp32 [H][r] or NULL (both or neither); when NULL
-                              they are computed at create from the SVD of C_h with the
+                              they are computed at create from the SVD of C_h (the sum
+                              of the head's component cores) with the
                               sign rule sum(u) > 0 (first non-zero entry if the sum is 0) */
     const void *values;    /* [N][D_v], physical table V; 16-byte aligned              */
     const void *w_proj;    /* [E][D_v][D'_v] projectors W_p, or NULL when has_proj == 0 */
@@ -113,8 +124,9 @@ void ultramem_destroy(ultramem_layer *layer);
 
 /* S1-S9 for B tokens: x [B][D_i] -> out [B][D'_v] (both cfg.dtype).  Optional
  * outputs (NULL to skip): idx_out [B][H][m] int64 virtual addresses v = i*K + j,
- * w_out [B][H][m] fp32 weights, each head's m slots ordered by (score desc,
- * v asc).  0 <= B <= max_tokens (B == 0 launches nothing). */
+ * w_out [B][H][m][h] fp32 weights (h = max(1, cores): the slot's score, or its h
+ * individual scores under MCS), each head's m slots ordered by (aggregate score
+ * desc, v asc).  0 <= B <= max_tokens (B == 0 launches nothing). */
 ultramem_status ultramem_forward(ultramem_layer *layer, const void *x, int32_t B,
                                  void *out, int64_t *idx_out, float *w_out, void *stream);
 
@@ -125,12 +137,13 @@ ultramem_status ultramem_forward_host(ultramem_layer *layer, const void *x_host,
                                       void *out_host, void *stream);
 
 /* S1-S6 only (retrieval, Eq. 4-10): idx_out [B][H][m] int64 and w_out
- * [B][H][m] fp32 as in ultramem_forward; both required. */
+ * [B][H][m][h] fp32 as in ultramem_forward; both required. */
 ultramem_status ultramem_retrieve(ultramem_layer *layer, const void *x, int32_t B,
                                   int64_t *idx_out, float *w_out, void *stream);
 
 /* S7-S9 only (the lookup-reduce of Eq. 14-15) on given slots: idx [B][H][m]
- * int64 virtual addresses in [0, E*N), w [B][H][m] fp32 -> out [B][D'_v].  An
+ * int64 virtual addresses in [0, E*N), w [B][H][m][h] fp32 (weight i scales value
+ * slice i, as in ultramem_forward) -> out [B][D'_v].  An
  * address out of range is not read: the kernel records it and the next
  * ultramem_check returns ULTRAMEM_EDEVICE. */
 ultramem_status ultramem_lookup_reduce(ultramem_layer *layer, const int64_t *idx,
@@ -144,10 +157,10 @@ ultramem_status ultramem_lookup_reduce(ultramem_layer *layer, const int64_t *idx
  * is one 8 MiB array of static device memory that every GPU loading the
  * library holds until the process exits; a batch whose scratch would exceed
  * it is rejected with ULTRAMEM_EINVAL.  cfg: d_k, rank, topk, max_tokens are
- * ignored; heads, topm, n, expand_e, d_v, d_out, has_proj, dtype and
+ * ignored; heads, topm, n, expand_e, d_v, d_out, has_proj, dtype, cores and
  * shuffle_seed are used as in ultramem_create.  values [N][D_v] and w_proj
  * [E][D_v][D'_v] as in ultramem_weights (w_proj may be NULL when has_proj is
- * 0), perm optional; idx [B][H][m] int64 and w [B][H][m] fp32 as in
+ * 0), perm optional; idx [B][H][m] int64 and w [B][H][m][h] fp32 as in
  * ultramem_lookup_reduce; out [B][D'_v].  Out-of-range addresses are skipped
  * (weight 0).  Asynchronous on `stream`.  The first call on a device looks up
  * the array's device address and sets a kernel attribute; make that first

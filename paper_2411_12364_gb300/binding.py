@@ -31,7 +31,7 @@ EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
 class Config(C.Structure):
     _fields_ = [(name, C.c_int32) for name in (
         "d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out", "topk", "topm",
-        "has_proj", "share_query", "act", "dtype", "max_tokens", "reserved")] + [
+        "has_proj", "share_query", "act", "dtype", "max_tokens", "cores")] + [
         ("shuffle_seed", C.c_uint64)]
 
 
@@ -141,9 +141,11 @@ class UltraMemLayer:
 
     ``weights`` holds device tensors in the layer's storage type (``w_q``,
     ``w_q_col``, ``k_row``, ``k_col``, ``values``, ``w_proj``), the cores
-    ``core`` [H, r, r] (any device, fp32) and optionally ``u``, ``t`` [H, r]
-    and an explicit shuffle ``perm`` (int32/uint32 device tensor).  The layer
-    keeps references to them for its lifetime."""
+    ``core`` [H, r, r] (with ``cfg["cores"]`` = h > 1 component cores,
+    [H, h, r, r]; any device, fp32) and optionally ``u``, ``t`` [H, r] and an
+    explicit shuffle ``perm`` (int32/uint32 device tensor).  The layer keeps
+    references to them for its lifetime.  Slot weights ``w`` are [B, H, m],
+    or [B, H, m, h] with h > 1 cores (one per value slice, Eq. 17)."""
 
     def __init__(self, cfg: dict, weights: dict, max_tokens: int):
         if not torch.cuda.is_available():
@@ -154,7 +156,7 @@ class UltraMemLayer:
         for k in _CFG_KEYS:
             setattr(c, k, int(cfg[k]))
         c.max_tokens = int(max_tokens)
-        c.reserved = 0
+        c.cores = int(cfg.get("cores", 0))
         c.shuffle_seed = int(cfg.get("shuffle_seed", 0))
         self._c = c
         dev_keys = ("w_q", "w_q_col", "k_row", "k_col", "values", "w_proj", "perm")
@@ -177,6 +179,11 @@ class UltraMemLayer:
         self._h = h
         self.max_tokens = int(max_tokens)
         self.dtype = torch.float32 if int(cfg["dtype"]) == F32 else torch.bfloat16
+        self.cores = max(1, int(cfg.get("cores", 0)))
+
+    def _w_shape(self, B: int):
+        H, m = int(self.cfg["heads"]), int(self.cfg["topm"])
+        return (B, H, m) if self.cores == 1 else (B, H, m, self.cores)
 
     # -- calls ------------------------------------------------------------
     def forward(self, x: torch.Tensor, out: torch.Tensor | None = None, with_slots=False):
@@ -190,7 +197,7 @@ class UltraMemLayer:
         if with_slots:
             H, m = int(self.cfg["heads"]), int(self.cfg["topm"])
             idx = torch.empty((B, H, m), dtype=torch.int64, device=x.device)
-            w = torch.empty((B, H, m), dtype=torch.float32, device=x.device)
+            w = torch.empty(self._w_shape(B), dtype=torch.float32, device=x.device)
         _check(self.lib.ultramem_forward(self._h, x.data_ptr(), B, out.data_ptr(), _ptr(idx),
                                          _ptr(w), _stream()), "ultramem_forward")
         return (out, idx, w) if with_slots else out
@@ -208,7 +215,7 @@ class UltraMemLayer:
         B = x.shape[0]
         H, m = int(self.cfg["heads"]), int(self.cfg["topm"])
         idx = torch.empty((B, H, m), dtype=torch.int64, device=x.device)
-        w = torch.empty((B, H, m), dtype=torch.float32, device=x.device)
+        w = torch.empty(self._w_shape(B), dtype=torch.float32, device=x.device)
         _check(self.lib.ultramem_retrieve(self._h, x.data_ptr(), B, idx.data_ptr(),
                                           w.data_ptr(), _stream()), "ultramem_retrieve")
         return idx, w
@@ -218,6 +225,8 @@ class UltraMemLayer:
         idx = idx.contiguous().to(torch.int64)
         w = w.contiguous().to(torch.float32)
         B = idx.shape[0]
+        if w.numel() != idx.numel() * self.cores:
+            raise ValueError(f"weights {tuple(w.shape)} do not match addresses {tuple(idx.shape)}")
         out = torch.empty((B, int(self.cfg["d_out"])), dtype=self.dtype, device=idx.device)
         _check(self.lib.ultramem_lookup_reduce(self._h, idx.data_ptr(), w.data_ptr(), B,
                                                out.data_ptr(), _stream()),

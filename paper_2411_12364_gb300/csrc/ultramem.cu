@@ -23,6 +23,7 @@ struct Workspace {
     uint32_t *akey = nullptr;
     int32_t *sel_row = nullptr, *sel_p = nullptr;
     float *core = nullptr, *u = nullptr, *t = nullptr;
+    float *cores = nullptr;   // MCS component cores [H][h][r][r] (h > 1 only)
     int *err = nullptr;
     void *x_stage = nullptr, *out_stage = nullptr;
     __nv_bfloat16 *qs = nullptr, *acc_bf = nullptr, *w_pt = nullptr;   // tensor path
@@ -116,7 +117,9 @@ int proj_splits(const ultramem_config &c, int B) {
 
 ultramem_status validate(const ultramem_config *c, const ultramem_weights *w) {
     if (!c || !w) return ULTRAMEM_EINVAL;
-    if (c->reserved != 0) return ULTRAMEM_EINVAL;
+    if (c->cores < 0 || c->cores > 8) return ULTRAMEM_EINVAL;
+    if (c->cores > 1 && (c->act != ULTRAMEM_ACT_NONE || c->d_v % (8 * c->cores)))
+        return ULTRAMEM_EINVAL;   // MCS: raw scores, value slices of whole 16-byte words
     if (c->d_in <= 0 || c->d_k <= 0 || c->heads <= 0 || c->rank < 1 || c->rank > 8)
         return ULTRAMEM_EINVAL;
     if (c->d_k % c->rank) return ULTRAMEM_EINVAL;
@@ -236,7 +239,7 @@ void free_workspace(Workspace &ws) {
     void *ptrs[] = {ws.q_part, ws.akey, ws.sel_w,   ws.acc,       ws.proj_part,
                     ws.sel_row, ws.sel_p, ws.core,   ws.u,         ws.t,
                     ws.err,    ws.x_stage, ws.out_stage, ws.qs,     ws.acc_bf,
-                    ws.w_pt};
+                    ws.w_pt,   ws.cores};
     for (void *p : ptrs)
         if (p) cudaFree(p);
     ws = Workspace();
@@ -253,6 +256,7 @@ Ptrs make_ptrs(ultramem_layer *L) {
     p.w_proj = L->w.w_proj;
     p.perm = L->w.perm;
     p.core = L->ws.core;
+    p.cores = L->ws.cores;
     p.u = L->ws.u;
     p.t = L->ws.t;
     p.q_part = L->ws.q_part;
@@ -426,27 +430,39 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
     if (major != 10 || minor != 3) return ULTRAMEM_ENODEV;
 
-    const int H = cfg->heads, r = cfg->rank;
-    // (u, t) per head: given, or the SVD of each core (Eq. 7)
+    const int H = cfg->heads, r = cfg->rank, nc = cfg->cores > 1 ? cfg->cores : 1;
+    // each head's Tucker core: the sum of its component cores (MCS, Eq. 16),
+    // summed in fp64 and kept in fp32 for the Tucker combine
     float *hu = (float *)malloc(sizeof(float) * H * r);
     float *ht = (float *)malloc(sizeof(float) * H * r);
-    if (!hu || !ht) { free(hu); free(ht); return ULTRAMEM_ENOMEM; }
+    float *hc = (float *)malloc(sizeof(float) * H * r * r);
+    if (!hu || !ht || !hc) { free(hu); free(ht); free(hc); return ULTRAMEM_ENOMEM; }
     for (int h = 0; h < H; ++h) {
+        double cd[64];
+        for (int e = 0; e < r * r; ++e) {
+            cd[e] = 0.0;
+            for (int i = 0; i < nc; ++i) cd[e] += w->core[((size_t)h * nc + i) * r * r + e];
+            hc[h * r * r + e] = (float)cd[e];
+        }
+        // (u, t): given, or the SVD of the summed core (Eq. 7)
         if (w->u) {
             memcpy(hu + h * r, w->u + h * r, sizeof(float) * r);
             memcpy(ht + h * r, w->t + h * r, sizeof(float) * r);
         } else {
-            float sg;
-            if (ultramem_rank1(w->core + (size_t)h * r * r, r, hu + h * r, ht + h * r, &sg) !=
-                ULTRAMEM_OK) {
-                free(hu); free(ht);
+            double uu[8], tt[8], sg;
+            if (rank1_host(cd, r, uu, tt, &sg) != ULTRAMEM_OK) {
+                free(hu); free(ht); free(hc);
                 return ULTRAMEM_EINVAL;
+            }
+            for (int i = 0; i < r; ++i) {
+                hu[h * r + i] = (float)uu[i];
+                ht[h * r + i] = (float)tt[i];
             }
         }
     }
 
     ultramem_layer *L = new (std::nothrow) ultramem_layer();
-    if (!L) { free(hu); free(ht); return ULTRAMEM_ENOMEM; }
+    if (!L) { free(hu); free(ht); free(hc); return ULTRAMEM_ENOMEM; }
     L->cfg = *cfg;
     L->w = *w;
     L->device = dev;
@@ -465,6 +481,7 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     d.d_out = cfg->d_out;
     d.k = cfg->topk;
     d.m = cfg->topm;
+    d.nc = nc;
     d.A = cfg->share_query ? 1 : 2;
     d.act = cfg->act;
     d.dtype = cfg->dtype;
@@ -491,12 +508,13 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     const size_t hm = Bm * H * cfg->topm;
     if (e == cudaSuccess) e = dalloc(&ws.q_part, qmax * d.A * HD);
     if (e == cudaSuccess) e = dalloc(&ws.akey, Bm * H * 2 * (size_t)d.K);
-    if (e == cudaSuccess) e = dalloc(&ws.sel_w, hm);
+    if (e == cudaSuccess) e = dalloc(&ws.sel_w, hm * nc);
     if (e == cudaSuccess) e = dalloc(&ws.sel_row, hm);
     if (e == cudaSuccess) e = dalloc(&ws.sel_p, hm);
     if (e == cudaSuccess) e = dalloc(&ws.acc, cfg->has_proj ? Bm * d.E * d.d_v : 1);
     if (e == cudaSuccess) e = dalloc(&ws.proj_part, cfg->has_proj ? pmax * d.d_out : 1);
     if (e == cudaSuccess) e = dalloc(&ws.core, (size_t)H * r * r);
+    if (e == cudaSuccess && nc > 1) e = dalloc(&ws.cores, (size_t)H * nc * r * r);
     if (e == cudaSuccess) e = dalloc(&ws.u, (size_t)H * r);
     if (e == cudaSuccess) e = dalloc(&ws.t, (size_t)H * r);
     if (e == cudaSuccess) e = dalloc(&ws.err, 1);
@@ -505,12 +523,16 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     if (e == cudaSuccess)
         e = cudaMalloc(&ws.out_stage, Bm * cfg->d_out * elt_size(*cfg));
     if (e == cudaSuccess)
-        e = cudaMemcpy(ws.core, w->core, sizeof(float) * H * r * r, cudaMemcpyHostToDevice);
+        e = cudaMemcpy(ws.core, hc, sizeof(float) * H * r * r, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess && nc > 1)
+        e = cudaMemcpy(ws.cores, w->core, sizeof(float) * H * nc * r * r,
+                       cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(ws.u, hu, sizeof(float) * H * r, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(ws.t, ht, sizeof(float) * H * r, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemset(ws.err, 0, sizeof(int));
     free(hu);
     free(ht);
+    free(hc);
     const size_t kd = (size_t)d.E * d.d_v;
     if (e == cudaSuccess && L->tc) {
         // tensor path: split queries, bf16 acc, K-major copy of the projectors

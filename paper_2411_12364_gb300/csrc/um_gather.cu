@@ -14,6 +14,11 @@
 //     fixed order at the end (deterministic).
 // Wider rows or more slots take the per-lane multi-block kernels below.  Row
 // loads bypass L1 (read-only path).
+//
+// Multi-Core Scoring (Eq. 17): a slot has nc weights and weight i scales
+// columns [i*D_v/nc, (i+1)*D_v/nc) of the row.  Slices are whole 16-byte
+// vectors (D_v/nc is a multiple of 8), so a lane's vector lies in one slice
+// and the lane picks that slice's weight.
 #include "um_internal.cuh"
 
 namespace um {
@@ -151,10 +156,12 @@ __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
 }
 
 constexpr int kBMaxE = 16;
+constexpr int kMaxCores = 8;   // MCS component cores per head
 
 size_t bucket_smem_bytes(const Dims &d, int warps) {
     const int hm = d.H * d.m;
-    return sizeof(int) * 2 * (size_t)hm + sizeof(float) * (size_t)warps * d.d_v;
+    return sizeof(int) * (size_t)hm + sizeof(float) * (size_t)hm * d.nc +
+           sizeof(float) * (size_t)warps * d.d_v;
 }
 
 // THREADS = 512 (2 CTAs per SM) for batches up to about two CTAs per SM,
@@ -174,17 +181,22 @@ __global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(
     const int64_t base = (int64_t)b * hm;
     float *red = reinterpret_cast<float *>(gsm);                 // [kBWarps][D_v]
     int *row_s = reinterpret_cast<int *>(red + kBWarps * Dv);    // [hm] bucketed rows
-    float *w_s = reinterpret_cast<float *>(row_s + hm);          // [hm] their weights
+    float *w_s = reinterpret_cast<float *>(row_s + hm);          // [hm][nc] their weights
+    const int nc = d.nc;
     pdl_wait();
     pdl_trigger();
 
     // stable counting sort of the slots by block (slot order kept within a block)
     int row = 0, blk = -1;
-    float w = 0.f;
+    float w[kMaxCores];   // the slot's weight, or its nc slice weights (MCS)
+#pragma unroll
+    for (int ci = 0; ci < kMaxCores; ++ci) w[ci] = 0.f;
     if (t < hm) {
         row = p.sel_row[base + t];
         blk = p.sel_p[base + t];
-        w = p.sel_w[base + t];
+#pragma unroll
+        for (int ci = 0; ci < kMaxCores; ++ci)
+            if (ci < nc) w[ci] = p.sel_w[(base + t) * nc + ci];
         if (blk < 0 || blk >= E) blk = -1;   // not a slot of this layer: skipped
     }
     int rank = 0;
@@ -215,7 +227,9 @@ __global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(
     if (blk >= 0) {
         const int pos = start[blk] + wcnt[warp][blk] + rank;
         row_s[pos] = row;
-        w_s[pos] = w;
+#pragma unroll
+        for (int ci = 0; ci < kMaxCores; ++ci)
+            if (ci < nc) w_s[pos * nc + ci] = w[ci];
     }
     __syncthreads();
 
@@ -223,6 +237,7 @@ __global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(
     const int wpb = kBWarps / E;
     const int q = warp / wpb, sub = warp - q * wpb;
     const bool active = lane * EPV < Dv;
+    const int wsel = nc == 1 || !active ? 0 : (lane * EPV) / (Dv / nc);   // this lane's slice
     const T *V = static_cast<const T *>(p.values) + lane * EPV;
     float acc[EPV];
 #pragma unroll
@@ -237,7 +252,7 @@ __global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(
             for (int u = 0; u < kUnroll; ++u) {
                 const int j = j0 + u;
                 const bool ok = j < hi;
-                wu[u] = ok ? w_s[j] : 0.f;
+                wu[u] = ok ? w_s[j * nc + wsel] : 0.f;
                 val[u] = (ok && active) ? ld_stream(V + (int64_t)row_s[j] * Dv)
                                         : make_uint4(0, 0, 0, 0);
             }
@@ -295,7 +310,7 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Dims d, Ptrs p) {
             bool ok = e < hm;
             row[u] = ok ? p.sel_row[base + e] : 0;
             blk[u] = ok ? p.sel_p[base + e] : 0;
-            w[u] = ok ? p.sel_w[base + e] : 0.f;
+            w[u] = ok && d.nc == 1 ? p.sel_w[base + e] : 0.f;
         }
         for (int vv = lane; vv < VPR; vv += 32) {
             uint4 val[kUnroll];
@@ -303,6 +318,12 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Dims d, Ptrs p) {
             for (int u = 0; u < kUnroll; ++u)
                 val[u] = (e0 + u < hm) ? ld_stream(V + (int64_t)row[u] * d.d_v + vv * EPV)
                                        : make_uint4(0, 0, 0, 0);
+            if (d.nc > 1) {   // MCS: the weight of this vector's value slice
+                const int ws = (vv * EPV) / (d.d_v / d.nc);
+#pragma unroll
+                for (int u = 0; u < kUnroll; ++u)
+                    if (e0 + u < hm) w[u] = p.sel_w[(base + e0 + u) * d.nc + ws];
+            }
 #pragma unroll
             for (int u = 0; u < kUnroll; ++u)
                 if (e0 + u < hm) fma_vec(mine + blk[u] * d.d_v + vv * EPV, val[u], w[u], T());
@@ -416,6 +437,8 @@ static cudaError_t launch_gather_t(const Dims &d, const Ptrs &p, cudaStream_t st
             return launch_kernel(d.pdl, gather_bucket_kernel<T, 256>, d.B, 256,
                                  bucket_smem_bytes(d, 8), st, d, p);
     }
+    if (d.nc > 1)   // MCS beyond the bucketed kernel's range
+        return launch_kernel(d.pdl, gather_kernel<T>, d.B, kThreads, bytes, st, d, p);
     if (fits_lanes && d.E == 1)
         return launch_kernel(d.pdl, gather_reg_kernel<T, 1>, d.B, kThreads, bytes, st, d, p);
     if (fits_lanes && d.E <= 4)

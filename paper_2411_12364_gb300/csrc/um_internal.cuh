@@ -8,7 +8,8 @@
 //                                      u^T S_row (axis 0) / t^T S_col (axis 1), Eq. 6
 //   sel_row  [B][H][m] int32           physical row of each selected slot
 //   sel_p    [B][H][m] int32           virtual block p of each selected slot
-//   sel_w    [B][H][m]                 weight of each selected slot
+//   sel_w    [B][H][m][nc]             weights of each selected slot (nc > 1:
+//                                      one per value slice, Multi-Core Scoring)
 //   acc      [B][E*D_v]                per-block pooled rows, Eq. 15 inner sum
 //   proj_part[p_splits][B][D'_v]       split-K partial sums of the projection
 #pragma once
@@ -33,6 +34,7 @@ struct Dims {
     int64_t N;        // physical rows
     uint64_t M;       // virtual slots E*N
     int E, d_v, d_out, k, m;
+    int nc;           // component cores per head (MCS, Eq. 16-17); 1 = one core
     int A;            // 1 = shared query, 2 = separate column query
     int act, dtype, has_proj;
     uint64_t shuf_a, shuf_c;
@@ -45,7 +47,8 @@ struct Dims {
 struct Ptrs {
     const void *x, *w_q, *w_q_col, *k_row, *k_col, *values, *w_proj;
     const uint32_t *perm;
-    const float *core, *u, *t;   // library copies: [H][r][r], [H][r], [H][r]
+    const float *core, *u, *t;   // library copies: [H][r][r] (the summed core), [H][r], [H][r]
+    const float *cores;          // [H][nc][r][r] component cores when nc > 1
     float *q_part, *sel_w, *acc, *proj_part;
     uint32_t *akey;
     int32_t *sel_row, *sel_p;
@@ -54,7 +57,7 @@ struct Ptrs {
     float *w_out;
     __nv_bfloat16 *acc_bf;       // tensor path: acc rounded to bf16 [B][E*D_v]
     const int64_t *idx_in;       // lookup_reduce input addresses
-    const float *w_in;           // lookup_reduce input weights
+    const float *w_in;           // lookup_reduce input weights [B][H][m][nc]
     int *err;                    // device error word (bit flags above)
 };
 

@@ -64,7 +64,8 @@ extern "C" ultramem_status ultramem_lookup_reduce_noalloc(const ultramem_config 
         c.expand_e < 1 || c.expand_e > 16 || s * s != c.expand_e ||
         (c.dtype != ULTRAMEM_F32 && c.dtype != ULTRAMEM_BF16) ||
         (c.has_proj != 0 && c.has_proj != 1) ||
-        (!c.has_proj && (c.expand_e != 1 || c.d_out != c.d_v)) || (c.has_proj && c.d_out <= 0))
+        (!c.has_proj && (c.expand_e != 1 || c.d_out != c.d_v)) || (c.has_proj && c.d_out <= 0) ||
+        c.cores < 0 || c.cores > 8 || (c.cores > 1 && c.d_v % (8 * c.cores)))
         return ULTRAMEM_EINVAL;
     const uint64_t N = (uint64_t)c.n * c.n, M = (uint64_t)c.expand_e * N;
     if (M >= (1ull << 32)) return ULTRAMEM_EINVAL;
@@ -76,6 +77,7 @@ extern "C" ultramem_status ultramem_lookup_reduce_noalloc(const ultramem_config 
     d.B = B;
     d.H = c.heads;
     d.m = c.topm;
+    d.nc = c.cores > 1 ? c.cores : 1;
     d.N = (int64_t)N;
     d.M = M;
     d.E = c.expand_e;
@@ -99,7 +101,7 @@ extern "C" ultramem_status ultramem_lookup_reduce_noalloc(const ultramem_config 
     const size_t o_blk = off;
     off = align256(off + slots * sizeof(int32_t));
     const size_t o_w = off;
-    off = align256(off + slots * sizeof(float));
+    off = align256(off + slots * d.nc * sizeof(float));
     const size_t o_acc = off;
     if (c.has_proj) off = align256(off + (size_t)B * kd * sizeof(float));
     const size_t o_part = off;

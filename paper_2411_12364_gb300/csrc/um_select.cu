@@ -4,6 +4,8 @@
 //   exact Tucker score g on the k*k survivor pairs      (Eq. 10)
 //   top-m of g, ordered by (score desc, v asc)          (Eq. 10)
 //   weights (raw scores, or PKM's softmax), shuffle     (Trick 1, Eq. 3, Eq. 14)
+//   with h component cores (MCS), the h individual scores of each winner
+//                                                        (Eq. 16-17)
 // No K*K grid is ever formed.  The scoring kernel leaves, per key, the
 // order-preserving 32-bit key of its fp32 rank-1 score; the exact chunk
 // scores of the k survivors of each axis are recomputed here from q and the
@@ -409,14 +411,16 @@ __device__ void rank_sorted(const u64 *list, int c, int kk, u64 *win, u64 *runs,
 struct SelLayout {
     float *qv;          // [2][D_k] row and column query of this (token, head)
     uint32_t *key0;     // [max(K, k*k)] axis-0 keys, then the g keys
-    uint32_t *key1;     // [K] axis-1 keys
+    uint32_t *key1;     // [K] axis-1 keys (free once the axis winners are ranked)
     int *sel_i, *sel_j; // [k] surviving rows / columns in increasing index
     float *R, *scol;    // [k][r] R = S_row^T C and S_col of the survivors
+    float *srow;        // MCS: [k][r] S_row of the row survivors      } in key1's
+    float *cparts;      // MCS: [nc][r][r] component cores of this head } space
 };
 
 // Dynamic shared memory layout; every section starts on 16 bytes.
 struct SelOffsets {
-    size_t qv, key0, key1, sel_i, sel_j, R, scol, total;
+    size_t qv, key0, key1, sel_i, sel_j, R, scol, srow, cparts, total;
 };
 __host__ __device__ inline SelOffsets sel_offsets(const Dims &d) {
     auto up = [](size_t x) { return (x + 15) & ~size_t(15); };
@@ -424,7 +428,13 @@ __host__ __device__ inline SelOffsets sel_offsets(const Dims &d) {
     size_t off = 0;
     o.qv = off;    off = up(off + sizeof(float) * 2 * d.d_k);
     o.key0 = off;  off = up(off + sizeof(uint32_t) * (d.K > d.k * d.k ? d.K : d.k * d.k));
-    o.key1 = off;  off = up(off + sizeof(uint32_t) * d.K);
+    // with MCS, key1's space later holds S_row of the row survivors and the
+    // component cores (so that the block's shared memory does not grow)
+    const bool mcs = d.nc > 1;
+    const int mcs_floats = mcs ? d.k * d.r + d.nc * d.r * d.r : 0;
+    o.key1 = off;  off = up(off + sizeof(uint32_t) * (d.K > mcs_floats ? d.K : mcs_floats));
+    o.srow = o.key1;
+    o.cparts = o.key1 + sizeof(float) * d.k * d.r;
     o.sel_i = off; off = up(off + sizeof(int) * d.k);
     o.sel_j = off; off = up(off + sizeof(int) * d.k);
     o.R = off;     off = up(off + sizeof(float) * d.k * d.r);
@@ -443,6 +453,8 @@ __device__ SelLayout carve(const Dims &d, unsigned char *base) {
     L.sel_j = reinterpret_cast<int *>(base + o.sel_j);
     L.R = reinterpret_cast<float *>(base + o.R);
     L.scol = reinterpret_cast<float *>(base + o.scol);
+    L.srow = reinterpret_cast<float *>(base + o.srow);
+    L.cparts = reinterpret_cast<float *>(base + o.cparts);
     return L;
 }
 
@@ -613,6 +625,10 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
     if (active && sub == 0) {
         if (s == 0) {
             L.sel_i[ord] = (int)pos;
+            if (d.nc > 1)   // MCS: the individual scores need S_row itself
+#pragma unroll
+                for (int a = 0; a < RM; ++a)
+                    if (a < r) L.srow[ord * r + a] = S[a];
 #pragma unroll
             for (int b = 0; b < RM; ++b) {
                 if (b < r) {
@@ -652,6 +668,11 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     // row/column query of this (token, head), summed over its D_i splits:
     // loaded before the keys, stored after them
     const float core_e = threadIdx.x < r * r ? p.core[(int64_t)h * r * r + threadIdx.x] : 0.f;
+    // MCS component cores (nc r^2 <= 2 kThreads), stored once key1 is free
+    const int ncrr = d.nc > 1 ? d.nc * r * r : 0;
+    const float *cp = p.cores + (int64_t)h * ncrr;
+    const float cp0 = threadIdx.x < ncrr ? cp[threadIdx.x] : 0.f;
+    const float cp1 = threadIdx.x + kThreads < ncrr ? cp[threadIdx.x + kThreads] : 0.f;
     pdl_wait();
     pdl_trigger();
     const int HD = d.H * d.d_k;
@@ -700,6 +721,8 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
             rank_list(sh.cand[s], cs, k, sh.win[s], tid, kThreads / 2);
     }
     __syncthreads();
+    if (threadIdx.x < ncrr) L.cparts[threadIdx.x] = cp0;   // key1 is free now
+    if (threadIdx.x + kThreads < ncrr) L.cparts[threadIdx.x + kThreads] = cp1;
     // survivors in increasing index with their exact chunk scores (Eq. 4)
     axis_survivors<T, RM>(d, p, h, L, sh);
     __syncthreads();
@@ -774,31 +797,58 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
                     row_bytes);
         p.sel_row[base + e] = (int32_t)prow;
         p.sel_p[base + e] = (int32_t)pb;
-        p.sel_w[base + e] = w;
         if (p.idx_out) p.idx_out[base + e] = (int64_t)v;
-        if (p.w_out) p.w_out[base + e] = w;
+        if (d.nc == 1) {
+            p.sel_w[base + e] = w;
+            if (p.w_out) p.w_out[base + e] = w;
+        } else {
+            // MCS (Eq. 16-17): the individual scores S_row^T C^(i) S_col of
+            // this slot, one per value slice (the softmax is not allowed here)
+            float sr[RM], sc[RM];
+#pragma unroll
+            for (int a = 0; a < RM; ++a) {
+                sr[a] = a < r ? L.srow[ii * r + a] : 0.f;
+                sc[a] = a < r ? L.scol[jj * r + a] : 0.f;
+            }
+            for (int ci = 0; ci < d.nc; ++ci) {
+                const float *Cc = L.cparts + ci * r * r;
+                float gi = 0.f;
+#pragma unroll
+                for (int a = 0; a < RM; ++a) {
+                    if (a < r) {
+                        float cs = 0.f;
+#pragma unroll
+                        for (int be = 0; be < RM; ++be)
+                            if (be < r) cs = fmaf(Cc[a * r + be], sc[be], cs);
+                        gi = fmaf(sr[a], cs, gi);
+                    }
+                }
+                p.sel_w[(base + e) * d.nc + ci] = gi;
+                if (p.w_out) p.w_out[(base + e) * d.nc + ci] = gi;
+            }
+        }
     }
 }
 
 // lookup_reduce input: given virtual addresses and weights -> (row, p, w).
 // An address outside [0, E*N) is recorded in the error word and skipped
-// (weight 0, row 0).
+// (weights 0, row 0).  With MCS each slot has nc weights.
 __global__ void slots_kernel(Dims d, Ptrs p) {
     const int64_t total = (int64_t)d.B * d.H * d.m;
     for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
          e += (int64_t)gridDim.x * blockDim.x) {
         int64_t v = p.idx_in[e];
-        float w = p.w_in[e];
-        if (v < 0 || (uint64_t)v >= d.M) {
+        const bool bad = v < 0 || (uint64_t)v >= d.M;
+        if (bad) {
             atomicOr(p.err, kErrBadIndex);
             v = 0;
-            w = 0.f;
         }
+        for (int ci = 0; ci < d.nc; ++ci)
+            p.sel_w[e * d.nc + ci] = bad ? 0.f : p.w_in[e * d.nc + ci];
         uint64_t vs = shuffle_address(d, p.perm, (uint64_t)v);
         uint64_t pb = vs / (uint64_t)d.N;
         p.sel_row[e] = (int32_t)(vs - pb * (uint64_t)d.N);
         p.sel_p[e] = (int32_t)pb;
-        p.sel_w[e] = w;
     }
 }
 

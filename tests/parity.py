@@ -11,7 +11,8 @@ lookup-reduce of the GPU's own slots.
 
 Output tolerance: per token, max_e |y - y_ref| / max_e |y_ref| <= 1e-4 in
 fp32 mode and 2e-2 in bf16 mode.  Weights: |w - w_ref| <= 1e-4 * max |w_ref|
-per head.
+per head (over all h weights of a slot with Multi-Core Scoring).  With MCS
+the selection and the near-tie rule use each head's summed core (Eq. 16).
 """
 from __future__ import annotations
 
@@ -37,6 +38,13 @@ def _gap_is_tie(vals, kk):
     return (srt[kk - 1] - srt[kk]) <= TIE_REL * scale
 
 
+def tucker_core(cfg, t):
+    """[H, r, r] fp64: each head's Tucker core, the sum of its component
+    cores when there are h > 1 of them (Eq. 16)."""
+    c = np.asarray(t["core"], np.float64)
+    return c.sum(axis=1) if int(cfg.get("cores", 0)) > 1 else c
+
+
 def head_scores(cfg, t, b, h):
     """Oracle's Eq. 4 scores, rank-1 scores and the survivors' exact scores."""
     s_row, s_col = oracle.row_col_scores(cfg, t, b, h)
@@ -52,7 +60,7 @@ def near_tie(cfg, t, b, h):
         return True
     I = np.argsort(-a, kind="stable")[:k]
     J = np.argsort(-bb, kind="stable")[:k]
-    G = s_row[:, I].T @ np.asarray(t["core"], np.float64)[h] @ s_col[:, J]
+    G = s_row[:, I].T @ tucker_core(cfg, t)[h] @ s_col[:, J]
     return _gap_is_tie(G.ravel(), m)
 
 
@@ -60,7 +68,7 @@ def slot_scores(cfg, t, b, h, v):
     """Exact Eq. 5 score of given virtual addresses v = i*K + j."""
     K = workloads.keys_per_axis(cfg)
     s_row, s_col, _, _ = head_scores(cfg, t, b, h)
-    C = np.asarray(t["core"], np.float64)[h]
+    C = tucker_core(cfg, t)[h]
     i, j = np.asarray(v) // K, np.asarray(v) % K
     return np.einsum("an,ab,bn->n", s_row[:, i], C, s_col[:, j])
 
@@ -112,6 +120,6 @@ def numpy_inputs(cfg, weights, x):
     numpy's SVD so that both sides prune with the same singular pair."""
     t = {k: workloads.stored_numpy(v) for k, v in weights.items() if k not in ("u", "t")}
     t["x"] = workloads.stored_numpy(x)
-    u, tt = util.numpy_rank1(t["core"])
+    u, tt = util.numpy_rank1(tucker_core(cfg, t))
     t["u"], t["t"] = u.astype(np.float32), tt.astype(np.float32)
     return t

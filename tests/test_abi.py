@@ -65,7 +65,7 @@ def _create(cfg_over=None, **w_over):
     lib = binding.load()
     c = binding.Config(d_in=64, d_k=32, heads=2, rank=2, n=16, expand_e=4, d_v=64, d_out=96,
                        topk=8, topm=8, has_proj=1, share_query=1, act=0, dtype=1,
-                       max_tokens=16, reserved=0, shuffle_seed=3)
+                       max_tokens=16, cores=0, shuffle_seed=3)
     for k, v in (cfg_over or {}).items():
         setattr(c, k, v)
     core = np.ones((2, 2, 2), np.float32)
@@ -81,8 +81,9 @@ def _create(cfg_over=None, **w_over):
 @pytest.mark.parametrize("bad", [dict(rank=3), dict(expand_e=3), dict(expand_e=25),
                                  dict(topk=200), dict(topm=65), dict(d_v=60),
                                  dict(has_proj=0), dict(act=7), dict(dtype=9),
-                                 dict(max_tokens=0), dict(reserved=1), dict(n=30000),
-                                 dict(rank=9, d_k=36)])
+                                 dict(max_tokens=0), dict(n=30000),
+                                 dict(rank=9, d_k=36), dict(cores=-1), dict(cores=9),
+                                 dict(cores=2, act=1), dict(cores=3), dict(cores=16)])
 def test_create_rejects_invalid_configs(bad):
     st, h = _create(bad)
     assert st == binding.EINVAL

@@ -51,6 +51,12 @@ SMALL = [
     dict(dtype=0, shuffle_seed=0),
     dict(dtype=1, rank=3, d_k=48),           # tensor path, odd rank (folded query)
     dict(dtype=1, rank=5, d_k=40, heads=3),  # tensor path, 8-wide rank chunks
+    dict(dtype=0, cores=2),                  # Multi-Core Scoring (Eq. 16-17)
+    dict(dtype=1, cores=2),
+    dict(dtype=1, cores=4, rank=3, d_k=48),  # four 16-wide value slices
+    dict(dtype=0, cores=2, expand_e=1, has_proj=0, d_out=64, n=40),
+    dict(dtype=1, cores=8, d_v=128, d_out=40, heads=4, topk=16, topm=40),
+    dict(dtype=1, cores=2, heads=4, topk=24, topm=160),   # H*m > 512: per-lane gather
 ]
 
 
@@ -69,6 +75,15 @@ def test_tiny_fp32_workload(gpu_lib):
 def test_decode_1m_workload(gpu_lib):
     cfg = workloads.layer_config("decode_1m")
     _run(cfg, 64, gpu_lib)
+
+
+@pytest.mark.parametrize("name,B", [("decode_1m", 64), ("mid_4m", 128)])
+def test_multi_core_scoring_workloads(name, B, gpu_lib):
+    """The paper's default h = 2 component cores (Sec. 3.2, Eq. 16-17) on the
+    decode-shaped layers: top-m on the summed core, two weights per slot,
+    each scaling one 128-wide half of the physical value row."""
+    cfg = workloads.layer_config(name, cores=2)
+    _run(cfg, B, gpu_lib)
 
 
 @pytest.mark.parametrize("B", [1, 8, 32, 128])
@@ -93,10 +108,12 @@ def test_prefill_16k_sampled(gpu_lib):
     _run(cfg, 16384, gpu_lib, tokens=sample)
 
 
-def test_lookup_reduce_on_oracle_slots(gpu_lib):
-    """S7-S9 alone: the GPU pools the oracle's own (v, w) like the oracle."""
+@pytest.mark.parametrize("cores", [0, 2])
+def test_lookup_reduce_on_oracle_slots(cores, gpu_lib):
+    """S7-S9 alone: the GPU pools the oracle's own (v, w) like the oracle
+    (with MCS, h weights per slot, one per value slice)."""
     from paper_2411_12364_gb300.binding import UltraMemLayer
-    cfg = workloads.layer_config("decode_1m")
+    cfg = workloads.layer_config("decode_1m", cores=cores)
     w = workloads.make_weights(cfg, device="cuda")
     x = workloads.make_tokens(cfg, 16, device="cuda")
     t = parity.numpy_inputs(cfg, w, x)
@@ -250,6 +267,8 @@ LONG_GRID = [
     dict(dtype=0, n=6, topk=5, topm=25),                     # m = k*k
     dict(dtype=1, heads=4, topk=16, topm=40, d_v=128, d_out=40),
     dict(dtype=1, topk=24, topm=64),
+    dict(dtype=1, topk=24, topm=64, cores=2),                # MCS
+    dict(dtype=1, heads=4, topk=24, topm=160, cores=2),      # MCS, per-lane gather
 ]
 
 

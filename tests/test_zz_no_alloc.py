@@ -21,7 +21,7 @@ def _config_struct(cfg, max_tokens):
               "has_proj", "share_query", "act", "dtype"):
         setattr(c, k, int(cfg[k]))
     c.max_tokens = max_tokens
-    c.reserved = 0
+    c.cores = int(cfg.get("cores", 0))
     c.shuffle_seed = int(cfg["shuffle_seed"])
     return c
 
@@ -35,9 +35,10 @@ def _noalloc(lib, c, w, idx, wt, out):
     return st
 
 
-@pytest.mark.parametrize("name,B", [("decode_1m", 64), ("tiny_fp32", 16)])
-def test_noalloc_matches_lookup_reduce_twice(name, B, gpu_lib):
-    cfg = workloads.layer_config(name)
+@pytest.mark.parametrize("name,B,cores", [("decode_1m", 64, 0), ("tiny_fp32", 16, 0),
+                                          ("decode_1m", 64, 2)])
+def test_noalloc_matches_lookup_reduce_twice(name, B, cores, gpu_lib):
+    cfg = workloads.layer_config(name, cores=cores)
     w = workloads.make_weights(cfg, device="cuda")
     layer = binding.UltraMemLayer(cfg, w, B)
     c = _config_struct(cfg, B)
