@@ -31,15 +31,17 @@ ACT_NONE, ACT_SOFTMAX = 0, 1
 class Config(C.Structure):
     _fields_ = [(name, C.c_int32) for name in (
         "d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out",
-        "topk", "topm", "has_proj", "share_query", "act", "dtype", "cores")] + [
-        ("shuffle_seed", C.c_uint64)]
+        "topk", "topm", "has_proj", "share_query", "act", "dtype", "cores", "conv_k",
+        "query_ln")] + [("shuffle_seed", C.c_uint64), ("ln_eps", C.c_double)]
 
 
 class Tensors(C.Structure):
     _fields_ = [("x", C.c_void_p), ("w_q", C.c_void_p), ("w_q_col", C.c_void_p),
                 ("k_row", C.c_void_p), ("k_col", C.c_void_p),
                 ("core", C.c_void_p), ("u", C.c_void_p), ("t", C.c_void_p),
-                ("values", C.c_void_p), ("w_proj", C.c_void_p), ("perm", C.c_void_p)]
+                ("values", C.c_void_p), ("w_proj", C.c_void_p), ("perm", C.c_void_p),
+                ("conv_w", C.c_void_p), ("conv_b", C.c_void_p), ("conv_state", C.c_void_p),
+                ("seq_len", C.c_int64), ("ln_g", C.c_void_p), ("ln_b", C.c_void_p)]
 
 
 def build(force: bool = False) -> str:
@@ -61,7 +63,9 @@ def _load():
             P = C.c_void_p
             lib.uo_forward.argtypes = [P, P, C.c_int64, P, C.c_int64, P, P, P, C.c_int32]
             lib.uo_lookup_reduce.argtypes = [P, P, C.c_int64, P, P, P, C.c_int32]
-            lib.uo_row_col_scores.argtypes = [P, P, C.c_int64, C.c_int32, P, P]
+            lib.uo_row_col_scores.argtypes = [P, P, C.c_int64, C.c_int64, C.c_int32, P, P]
+            lib.uo_conv_state.argtypes = [P, P, C.c_int64, P]
+            lib.uo_key_ln.argtypes = [P, C.c_int32, C.c_int64, C.c_int32, P, P, C.c_double, P]
             lib.uo_rank1.argtypes = [P, C.c_int32, P, P, P]
             lib.uo_shuffle.argtypes = [P, P, C.c_int64]
             lib.uo_shuffle.restype = C.c_int64
@@ -81,6 +85,9 @@ def make_config(cfg: dict) -> Config:
     for k in _CFG_KEYS:
         setattr(c, k, int(cfg[k]))
     c.cores = int(cfg.get("cores", 0))
+    c.conv_k = int(cfg.get("conv_k", 0))
+    c.query_ln = int(cfg.get("query_ln", 0))
+    c.ln_eps = float(cfg.get("ln_eps", 1e-5))
     return c
 
 
@@ -113,13 +120,18 @@ def _tensors(cfg: dict, t: dict):
     keep = {}
     for k in ("x", "w_q", "w_q_col", "k_row", "k_col", "values", "w_proj"):
         keep[k] = _stored(t.get(k), dt)
-    for k in ("core", "u", "t"):
+    for k in ("core", "u", "t", "conv_w", "conv_b", "ln_g", "ln_b"):
         a = t.get(k)
         keep[k] = None if a is None else np.ascontiguousarray(a, dtype=np.float32)
+    keep["conv_state"] = _stored(t.get("conv_state"), dt)
     p = t.get("perm")
     keep["perm"] = None if p is None else np.ascontiguousarray(p, dtype=np.int64)
     s = Tensors(*[_ptr(keep[k]) for k in ("x", "w_q", "w_q_col", "k_row", "k_col",
-                                          "core", "u", "t", "values", "w_proj", "perm")])
+                                          "core", "u", "t", "values", "w_proj", "perm",
+                                          "conv_w", "conv_b", "conv_state")])
+    s.seq_len = int(t.get("seq_len", 0))
+    s.ln_g = _ptr(keep["ln_g"])
+    s.ln_b = _ptr(keep["ln_b"])
     return s, keep
 
 
@@ -167,20 +179,54 @@ def lookup_reduce(cfg: dict, tensors: dict, idx, w, threads: int = 0):
     return out
 
 
-def row_col_scores(cfg: dict, tensors: dict, b: int, h: int):
-    """Eq. 4 for token b, head h: ``(S_row [r, K], S_col [r, K])`` in fp64."""
+def row_col_scores(cfg: dict, tensors: dict, b: int, h: int, B: int | None = None):
+    """Eq. 4 for token b of the batch (B tokens, default all rows of x),
+    head h: ``(S_row [r, K], S_col [r, K])`` in fp64."""
     lib = _load()
     c = make_config(cfg)
     s, keep = _tensors(cfg, tensors)
     r, K = int(cfg["rank"]), keys_per_axis(cfg)
+    if B is None:
+        B = np.asarray(tensors["x"]).shape[0]
     sr = np.zeros((r, K), np.float64)
     sc = np.zeros((r, K), np.float64)
-    st = lib.uo_row_col_scores(C.byref(c), C.byref(s), int(b), int(h),
+    st = lib.uo_row_col_scores(C.byref(c), C.byref(s), int(B), int(b), int(h),
                                sr.ctypes.data, sc.ctypes.data)
     del keep
     if st != 0:
         raise ValueError(f"uo_row_col_scores failed with status {st}")
     return sr, sc
+
+
+def conv_state(cfg: dict, tensors: dict, B: int):
+    """Trick 4's state after a batch of B tokens: [B/seq_len, conv_k-1, d_in]
+    f64, the last conv_k - 1 inputs of each sequence, oldest first."""
+    lib = _load()
+    c = make_config(cfg)
+    s, keep = _tensors(cfg, tensors)
+    L = int(tensors.get("seq_len", 0)) or B
+    out = np.zeros((B // L, int(cfg["conv_k"]) - 1, int(cfg["d_in"])), np.float64)
+    st = lib.uo_conv_state(C.byref(c), C.byref(s), int(B), out.ctypes.data)
+    del keep
+    if st != 0:
+        raise ValueError(f"uo_conv_state failed with status {st}")
+    return out
+
+
+def key_ln(keys, dtype: int, g, b=None, eps: float = 1e-5):
+    """Trick 2 for keys: LayerNorm of each row of ``keys`` [..., d] (stored
+    as ``dtype``) with gain g [d] and bias b [d]; f64 of the same shape."""
+    lib = _load()
+    k = _stored(np.asarray(keys), dtype)
+    g = np.ascontiguousarray(g, dtype=np.float32)
+    bb = None if b is None else np.ascontiguousarray(b, dtype=np.float32)
+    d = k.shape[-1]
+    out = np.zeros(k.shape, np.float64)
+    st = lib.uo_key_ln(k.ctypes.data, int(dtype), int(k.size // d), int(d), g.ctypes.data,
+                       _ptr(bb), float(eps), out.ctypes.data)
+    if st != 0:
+        raise ValueError(f"uo_key_ln failed with status {st}")
+    return out
 
 
 def rank1(core):

@@ -16,7 +16,14 @@
  *  - heads are summed: all H*m weighted rows are pooled into one output;
  *  - virtual block p = v' div N, physical row = v' mod N where v' is the
  *    shuffled address (blocks concatenated in order, Eq. 13-14);
- *  - the shuffle is the seeded affine bijection documented at uo_shuffle.
+ *  - the shuffle is the seeded affine bijection documented at uo_shuffle;
+ *  - Trick 4's convolution feeds the query linear directly (no activation);
+ *    tap j multiplies the input j tokens back, within the token's sequence
+ *    or from the state before it;
+ *  - Trick 2's query LayerNorm runs over each head's D_k query entries
+ *    (population variance, epsilon inside the square root), after the
+ *    projection and before the key scores; a separate column query has its
+ *    own gain and bias.
  */
 #include "ultramem_oracle.h"
 
@@ -69,8 +76,14 @@ static int check_config(const uo_config *cfg)
     if (cfg->cores < 0 || cfg->cores > 8) return UO_EINVAL;
     if (cfg->cores > 1 && (cfg->d_v % cfg->cores != 0 || cfg->act != UO_ACT_NONE))
         return UO_EINVAL;
+    if (cfg->conv_k < 0 || cfg->conv_k > 64) return UO_EINVAL;
+    if (cfg->query_ln != 0 && cfg->query_ln != 1) return UO_EINVAL;
+    if (cfg->query_ln && !(cfg->ln_eps >= 0.0)) return UO_EINVAL;
     return UO_OK;
 }
+
+/* tokens per sequence of a batch of B (Trick 4) */
+static int64_t seq_len_of(const uo_tensors *x, int64_t B) { return x->seq_len > 0 ? x->seq_len : B; }
 
 /* h, the number of component cores of each head (Sec. 3.2, MCS) */
 static int32_t cores_of(const uo_config *cfg) { return cfg->cores > 1 ? cfg->cores : 1; }
@@ -252,33 +265,136 @@ static void row_col_scores(const uo_config *cfg, const uo_tensors *x, int32_t h,
         }
 }
 
-/* q = W_q x for all heads; q has H*D_k entries. */
-static void query(const uo_config *cfg, const void *w, const void *xv, int64_t b,
-                  double *q)
+/* Input d of the token j positions before token b (j >= 0) of a batch of B:
+ * from the same sequence, else from the state before it (zero without one). */
+static double input_back(const uo_config *cfg, const uo_tensors *x, int64_t B, int64_t b,
+                         int64_t j, int32_t d)
+{
+    const int64_t L = seq_len_of(x, B), s = b / L, pos = b - s * L - j;
+    if (pos >= 0) return load(x->x, cfg->dtype, (b - j) * cfg->d_in + d);
+    if (!x->conv_state) return 0.0;
+    /* the state holds the conv_k - 1 inputs before position 0, oldest first */
+    const int64_t row = (cfg->conv_k - 1) + pos;
+    return load(x->conv_state, cfg->dtype, (s * (cfg->conv_k - 1) + row) * cfg->d_in + d);
+}
+
+/* The query's input row: x itself, or (Trick 4) its causal depthwise
+ * convolution  x~[d] = b[d] + sum_j w[j][d] x[t - j][d]. */
+static void query_input(const uo_config *cfg, const uo_tensors *x, int64_t B, int64_t b,
+                        double *xin)
+{
+    for (int32_t d = 0; d < cfg->d_in; ++d) {
+        if (cfg->conv_k == 0) {
+            xin[d] = load(x->x, cfg->dtype, b * cfg->d_in + d);
+            continue;
+        }
+        double acc = x->conv_b ? (double)x->conv_b[d] : 0.0;
+        for (int32_t j = 0; j < cfg->conv_k; ++j)
+            acc += (double)x->conv_w[(int64_t)j * cfg->d_in + d] * input_back(cfg, x, B, b, j, d);
+        xin[d] = acc;
+    }
+}
+
+/* q = W_q x for all heads; q has H*D_k entries.  With Trick 2, each head's
+ * D_k entries are then layer-normalised with gain g and bias bb. */
+static void query(const uo_config *cfg, const void *w, const double *xin, const float *g,
+                  const float *bb, double *q)
 {
     const int64_t rows = (int64_t)cfg->heads * cfg->d_k;
     for (int64_t o = 0; o < rows; ++o) {
         double acc = 0.0;
         for (int32_t d = 0; d < cfg->d_in; ++d)
-            acc += load(w, cfg->dtype, o * cfg->d_in + d) *
-                   load(xv, cfg->dtype, b * cfg->d_in + d);
+            acc += load(w, cfg->dtype, o * cfg->d_in + d) * xin[d];
         q[o] = acc;
+    }
+    if (!cfg->query_ln) return;
+    for (int32_t h = 0; h < cfg->heads; ++h) {
+        double *qh = q + (int64_t)h * cfg->d_k;
+        double mean = 0.0, var = 0.0;
+        for (int32_t c = 0; c < cfg->d_k; ++c) mean += qh[c];
+        mean /= cfg->d_k;
+        for (int32_t c = 0; c < cfg->d_k; ++c) var += (qh[c] - mean) * (qh[c] - mean);
+        var /= cfg->d_k;
+        const double inv = 1.0 / sqrt(var + cfg->ln_eps);
+        for (int32_t c = 0; c < cfg->d_k; ++c) {
+            const int64_t o = (int64_t)h * cfg->d_k + c;
+            qh[c] = (qh[c] - mean) * inv * (double)g[o] + (bb ? (double)bb[o] : 0.0);
+        }
     }
 }
 
-int uo_row_col_scores(const uo_config *cfg, const uo_tensors *x, int64_t b,
+/* Both queries of token b (Trick 5: the column keys share the row query). */
+static void queries(const uo_config *cfg, const uo_tensors *x, int64_t B, int64_t b,
+                    double *xin, double *q)
+{
+    const int64_t HD = (int64_t)cfg->heads * cfg->d_k;
+    query_input(cfg, x, B, b, xin);
+    query(cfg, x->w_q, xin, x->ln_g, x->ln_b, q);
+    if (cfg->share_query) memcpy(q + HD, q, sizeof(double) * HD);
+    else query(cfg, x->w_q_col, xin, x->ln_g ? x->ln_g + HD : NULL,
+               x->ln_b ? x->ln_b + HD : NULL, q + HD);
+}
+
+/* Checks the query-side tensors a forward of B tokens reads. */
+static int check_query_extras(const uo_config *cfg, const uo_tensors *x, int64_t B)
+{
+    if (cfg->conv_k > 0) {
+        if (!x->conv_w || x->seq_len < 0) return UO_EINVAL;
+        if (x->seq_len > 0 && B % x->seq_len != 0) return UO_EINVAL;
+    }
+    if (cfg->query_ln && !x->ln_g) return UO_EINVAL;
+    return UO_OK;
+}
+
+int uo_conv_state(const uo_config *cfg, const uo_tensors *x, int64_t B, double *state_out)
+{
+    if (check_config(cfg) != UO_OK || !x || !x->x || !state_out || B <= 0) return UO_EINVAL;
+    if (cfg->conv_k <= 0 || check_query_extras(cfg, x, B) != UO_OK) return UO_EINVAL;
+    const int64_t L = seq_len_of(x, B), S = B / L, kk = cfg->conv_k - 1;
+    for (int64_t s = 0; s < S; ++s)
+        for (int64_t i = 0; i < kk; ++i)   /* row i holds input L - kk + i of sequence s */
+            for (int32_t d = 0; d < cfg->d_in; ++d)
+                state_out[(s * kk + i) * cfg->d_in + d] =
+                    input_back(cfg, x, B, s * L + L - 1, kk - 1 - i, d);
+    return UO_OK;
+}
+
+int uo_key_ln(const void *keys, int32_t dtype, int64_t n_rows, int32_t d, const float *g,
+              const float *b, double eps, double *out)
+{
+    if (!keys || !g || !out || n_rows < 0 || d <= 0 || !(eps >= 0.0)) return UO_EINVAL;
+    if (dtype != UO_F32 && dtype != UO_BF16) return UO_EINVAL;
+    for (int64_t i = 0; i < n_rows; ++i) {
+        double mean = 0.0, var = 0.0;
+        for (int32_t c = 0; c < d; ++c) mean += load(keys, dtype, i * d + c);
+        mean /= d;
+        for (int32_t c = 0; c < d; ++c) {
+            const double e = load(keys, dtype, i * d + c) - mean;
+            var += e * e;
+        }
+        var /= d;
+        const double inv = 1.0 / sqrt(var + eps);
+        for (int32_t c = 0; c < d; ++c)
+            out[i * d + c] = (load(keys, dtype, i * d + c) - mean) * inv * (double)g[c] +
+                             (b ? (double)b[c] : 0.0);
+    }
+    return UO_OK;
+}
+
+int uo_row_col_scores(const uo_config *cfg, const uo_tensors *x, int64_t B, int64_t b,
                       int32_t h, double *s_row, double *s_col)
 {
-    if (check_config(cfg) != UO_OK) return UO_EINVAL;
+    if (check_config(cfg) != UO_OK || check_query_extras(cfg, x, B) != UO_OK) return UO_EINVAL;
+    if (b < 0 || b >= B) return UO_EINVAL;
     const int64_t HD = (int64_t)cfg->heads * cfg->d_k;
     double *q = malloc(sizeof(double) * HD * 2);
-    if (!q) return UO_ENOMEM;
-    query(cfg, x->w_q, x->x, b, q);
-    if (cfg->share_query) memcpy(q + HD, q, sizeof(double) * HD);
-    else query(cfg, x->w_q_col, x->x, b, q + HD);
+    double *xin = malloc(sizeof(double) * cfg->d_in);
+    if (!q || !xin) { free(q); free(xin); return UO_ENOMEM; }
+    queries(cfg, x, B, b, xin, q);
     row_col_scores(cfg, x, h, q + (int64_t)h * cfg->d_k,
                    q + HD + (int64_t)h * cfg->d_k, s_row, s_col);
     free(q);
+    free(xin);
     return UO_OK;
 }
 
@@ -353,12 +469,12 @@ int uo_lookup_reduce(const uo_config *cfg, const uo_tensors *x, int64_t n_tokens
 /* ---- the whole layer for one token ------------------------------------- */
 
 typedef struct {
-    double *q, *s_row, *s_col, *a, *bcol, *acc, *sel_w, *pool_w, *core;
+    double *q, *xin, *s_row, *s_col, *a, *bcol, *acc, *sel_w, *pool_w, *core;
     scored *axis, *cand;
     int64_t *sel_i, *sel_j, *sel_v;
 } scratch;
 
-static void token_forward(const uo_config *cfg, const uo_tensors *x, int64_t b,
+static void token_forward(const uo_config *cfg, const uo_tensors *x, int64_t B, int64_t b,
                           const double *u_all, const double *t_all, scratch *sc,
                           double *out, int64_t *idx_out, double *w_out)
 {
@@ -366,10 +482,9 @@ static void token_forward(const uo_config *cfg, const uo_tensors *x, int64_t b,
     const int32_t H = cfg->heads, r = cfg->rank, k = cfg->topk, m = cfg->topm;
     const int64_t HD = (int64_t)H * cfg->d_k;
 
-    /* query projection (Sec. 3.1; Trick 5 shares it between the key sets) */
-    query(cfg, x->w_q, x->x, b, sc->q);
-    if (cfg->share_query) memcpy(sc->q + HD, sc->q, sizeof(double) * HD);
-    else query(cfg, x->w_q_col, x->x, b, sc->q + HD);
+    /* query projection (Sec. 3.1; Trick 5 shares it between the key sets,
+     * Trick 4 convolves its input, Trick 2 normalises it) */
+    queries(cfg, x, B, b, sc->xin, sc->q);
 
     const int32_t nc = cores_of(cfg);
     for (int32_t h = 0; h < H; ++h) {
@@ -479,6 +594,7 @@ int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
     if (!cfg->share_query && !x->w_q_col) return UO_EINVAL;
     if (cfg->has_proj && !x->w_proj) return UO_EINVAL;
     if ((x->u == NULL) != (x->t == NULL)) return UO_EINVAL;
+    if (check_query_extras(cfg, x, B) != UO_OK) return UO_EINVAL;
     uint64_t M = (uint64_t)cfg->expand_e * (uint64_t)cfg->n * (uint64_t)cfg->n;
     if (M >= (1ull << 32)) return UO_EINVAL;
     if (!tokens) n_tokens = B;
@@ -527,6 +643,7 @@ int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
         scratch sc;
         int64_t kk = (int64_t)cfg->topk * cfg->topk;
         sc.q = malloc(sizeof(double) * 2 * H * cfg->d_k);
+        sc.xin = malloc(sizeof(double) * cfg->d_in);
         sc.s_row = malloc(sizeof(double) * r * K);
         sc.s_col = malloc(sizeof(double) * r * K);
         sc.a = malloc(sizeof(double) * K);
@@ -540,7 +657,7 @@ int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
         sc.sel_i = malloc(sizeof(int64_t) * cfg->topk);
         sc.sel_j = malloc(sizeof(int64_t) * cfg->topk);
         sc.sel_v = malloc(sizeof(int64_t) * hm);
-        int ok = sc.q && sc.s_row && sc.s_col && sc.a && sc.bcol && sc.acc &&
+        int ok = sc.q && sc.xin && sc.s_row && sc.s_col && sc.a && sc.bcol && sc.acc &&
                  sc.sel_w && sc.pool_w && sc.core && sc.axis && sc.cand && sc.sel_i &&
                  sc.sel_j && sc.sel_v;
         if (!ok) {
@@ -550,11 +667,11 @@ int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
 #pragma omp for schedule(dynamic, 1)
             for (int64_t e = 0; e < n_tokens; ++e) {
                 int64_t b = tokens ? tokens[e] : e;
-                token_forward(cfg, x, b, u_all, t_all, &sc, out + e * cfg->d_out,
+                token_forward(cfg, x, B, b, u_all, t_all, &sc, out + e * cfg->d_out,
                               idx ? idx + e * hm : NULL, w ? w + e * hm * cores_of(cfg) : NULL);
             }
         }
-        free(sc.q); free(sc.s_row); free(sc.s_col); free(sc.a); free(sc.bcol);
+        free(sc.q); free(sc.xin); free(sc.s_row); free(sc.s_col); free(sc.a); free(sc.bcol);
         free(sc.acc); free(sc.sel_w); free(sc.pool_w); free(sc.core); free(sc.axis);
         free(sc.cand);
         free(sc.sel_i); free(sc.sel_j); free(sc.sel_v);

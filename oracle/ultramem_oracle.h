@@ -27,6 +27,10 @@
  *   Eq. 16-17 Multi-Core Scoring (MCS)    C = sum_i C^(i); top-m on the
  *           aggregate S_row^T C S_col; physical value slice i (D_v/h wide)
  *           weighted by the individual score S_row^T C^(i) S_col
+ *   Sec. 3.1 Trick 4  causal depthwise convolution of the input before the
+ *           query linear: x~[t] = b + sum_j w_j (.) x[t - j], per channel
+ *   Sec. 3.1 Trick 2  LayerNorm of each head's query (and of the keys, which
+ *           at inference is a fixed transform of the key table: uo_key_ln)
  */
 #ifndef ULTRAMEM_ORACLE_H
 #define ULTRAMEM_ORACLE_H
@@ -57,7 +61,11 @@ typedef struct {
     int32_t dtype;       /* UO_F32 or UO_BF16 for x, W_q, keys, V, W_p          */
     int32_t cores;       /* h: component cores per head (MCS); 0 or 1 = one core.
                             h > 1 needs D_v % h == 0 and UO_ACT_NONE            */
+    int32_t conv_k;      /* taps of the causal depthwise conv on x (Trick 4);
+                            0 = no convolution                                  */
+    int32_t query_ln;    /* 1: LayerNorm over each head's D_k query (Trick 2)   */
     uint64_t shuffle_seed; /* 0: identity shuffle; else the seeded bijection   */
+    double ln_eps;       /* LayerNorm epsilon (inside the square root)          */
 } uo_config;
 
 typedef struct {
@@ -73,6 +81,17 @@ typedef struct {
     const void *values;   /* [N][d_v] physical table V                           */
     const void *w_proj;   /* [E][d_v][d_out] projectors W_p, or NULL             */
     const int64_t *perm;  /* [E*N] explicit shuffle, or NULL for the seeded one  */
+    /* query-side extras (read only when conv_k > 0 / query_ln == 1) */
+    const float *conv_w;  /* [conv_k][d_in]: tap j multiplies x[t - j]            */
+    const float *conv_b;  /* [d_in] or NULL                                       */
+    const void *conv_state; /* [B/seq_len][conv_k-1][d_in], storage type: the
+                             inputs before each sequence, oldest first; NULL =
+                             zeros (every sequence starts fresh)                */
+    int64_t seq_len;      /* tokens per sequence, the batch being B/seq_len
+                             sequences back to back; 0 = one sequence of B      */
+    const float *ln_g;    /* [A][H*d_k] query LayerNorm gain (A = 1 shared
+                             query, 2 with a column query)                      */
+    const float *ln_b;    /* [A][H*d_k] or NULL                                 */
 } uo_tensors;
 
 /* Status codes. */
@@ -98,14 +117,24 @@ int uo_lookup_reduce(const uo_config *cfg, const uo_tensors *x, int64_t n_tokens
                      const int64_t *idx, const double *w, double *out,
                      int32_t n_threads);
 
-/* Eq. 4 for one (token b, head h): s_row[r][K], s_col[r][K]. */
-int uo_row_col_scores(const uo_config *cfg, const uo_tensors *x, int64_t b,
+/* Eq. 4 for one (token b of a batch of B, head h): s_row[r][K], s_col[r][K]. */
+int uo_row_col_scores(const uo_config *cfg, const uo_tensors *x, int64_t B, int64_t b,
                       int32_t h, double *s_row, double *s_col);
 
 /* Leading singular triplet of an r x r matrix (row-major), Eq. 7 / Eq. 11.
  * Sign rule: sum(u) > 0, or if that sum is exactly 0 the first non-zero
  * entry of u is positive; t = C^T u / sigma.  Returns UO_OK. */
 int uo_rank1(const double *c, int32_t r, double *u, double *t, double *sigma);
+
+/* Trick 4: the conv state after the batch, [B/seq_len][conv_k-1][d_in] in
+ * double: the last conv_k - 1 inputs of each sequence, oldest first (from the
+ * previous state when a sequence is shorter than conv_k - 1). */
+int uo_conv_state(const uo_config *cfg, const uo_tensors *x, int64_t B, double *state_out);
+
+/* Trick 2 for keys: LayerNorm of each of n_rows rows of width d (stored in
+ * `dtype`), gain g [d], bias b [d] or NULL, epsilon eps; out [n_rows][d]. */
+int uo_key_ln(const void *keys, int32_t dtype, int64_t n_rows, int32_t d, const float *g,
+              const float *b, double eps, double *out);
 
 /* Eq. 14: the shuffled virtual address pi(v) for v in [0, E*N). */
 int64_t uo_shuffle(const uo_config *cfg, const int64_t *perm, int64_t v);

@@ -13,9 +13,14 @@ tensor here is drawn from a seeded Gaussian with the scale the layer sees:
                                   component cores (MCS) [H, h, r, r] ~ N(0, 1/h)
   V      ~ N(0, 0.02^2)  (std 0.02) [N, D_v]     N = n * n physical rows
   W_p    ~ N(0, 1/(E*D_v)) variance [E, D_v, D'_v]
+  query-side extras, when enabled (Tricks 2 and 4):
+  conv taps ~ N(0, 1/conv_k) variance [conv_k, D_i], conv bias ~ N(0, 0.1^2)
+  query LayerNorm gain ~ 1 + N(0, 0.1^2), bias ~ N(0, 0.1^2)  [A, H*D_k]
+  conv state (the inputs before each sequence) ~ N(0, 1) like the tokens
 
 Draw order from one generator seeded with the workload seed: W_q, (W_q_col),
-K_row, K_col, C, V, W_p.  Token batches come from a second generator seeded
+K_row, K_col, C, W_p, then the conv taps and bias and the LayerNorm gain and
+bias (when enabled).  V has a generator of its own.  Token batches come from a second generator seeded
 with ``seed + 10_000 + 7919 * batch_index``.  Tables above 256 Mi elements
 are drawn on the GPU (when one is used) in chunks, seeded the same way.
 """
@@ -128,6 +133,14 @@ def make_weights(cfg: dict, device="cpu", with_table=True) -> dict:
         else _randn(gen, (H, r, r), 1.0, torch.float32)
     w["w_proj"] = _randn(gen, (E, dv, do), 1.0 / math.sqrt(E * dv), dt) \
         if int(cfg["has_proj"]) else None
+    kc = int(cfg.get("conv_k", 0))
+    if kc > 0:   # Trick 4: causal depthwise convolution of x
+        w["conv_w"] = _randn(gen, (kc, din), 1.0 / math.sqrt(kc), torch.float32)
+        w["conv_b"] = _randn(gen, (din,), 0.1, torch.float32)
+    if int(cfg.get("query_ln", 0)):   # Trick 2: query LayerNorm per head
+        A = 1 if int(cfg["share_query"]) else 2
+        w["ln_g"] = 1.0 + _randn(gen, (A, H * dk), 0.1, torch.float32)
+        w["ln_b"] = _randn(gen, (A, H * dk), 0.1, torch.float32)
     w = {k: (None if v is None else v.to(device)) for k, v in w.items()}
     w["values"] = _table(cfg, seed, dt, device) if with_table else None
     return w
@@ -137,6 +150,14 @@ def make_tokens(cfg: dict, B: int, batch_index: int = 0, device="cpu") -> torch.
     """One batch x [B, D_i] ~ N(0, 1) in the layer's storage type."""
     gen = torch.Generator().manual_seed(int(cfg["seed"]) + 10_000 + 7919 * batch_index)
     return _randn(gen, (B, int(cfg["d_in"])), 1.0, torch_dtype(cfg)).to(device)
+
+
+def make_conv_state(cfg: dict, n_seq: int, batch_index: int = 0, device="cpu"):
+    """The conv_k - 1 inputs before each of n_seq sequences, [n_seq, conv_k-1,
+    D_i] ~ N(0, 1) in the storage type (Trick 4's decode state)."""
+    kc = int(cfg["conv_k"])
+    gen = torch.Generator().manual_seed(int(cfg["seed"]) + 30_000 + 7919 * batch_index)
+    return _randn(gen, (n_seq, kc - 1, int(cfg["d_in"])), 1.0, torch_dtype(cfg)).to(device)
 
 
 def stored_numpy(t):

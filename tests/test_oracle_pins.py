@@ -29,10 +29,10 @@ def _golden(name):
 
 
 @pytest.mark.parametrize("name", ["hand_tucker_ive.json", "hand_pruning_rows.json",
-                                  "hand_mcs.json"])
+                                  "hand_mcs.json", "hand_conv_ln.json"])
 def test_hand_worked_examples(name):
     cfg, t, exp = _golden(name)
-    out, idx, w = oracle.forward(cfg, t, B=1)
+    out, idx, w = oracle.forward(cfg, t, B=len(t["x"]))
     np.testing.assert_array_equal(idx, np.array(exp["idx"]))
     np.testing.assert_array_equal(w, np.array(exp["w"], dtype=np.float64))
     np.testing.assert_array_equal(out, np.array(exp["out"], dtype=np.float64))
@@ -400,7 +400,8 @@ def test_invalid_configs_are_rejected():
     t = util.numpy_layer(base, B=1)
     bad = [dict(rank=3), dict(expand_e=3), dict(topk=10 ** 6), dict(topm=26),
            dict(has_proj=0), dict(act=5), dict(cores=3), dict(cores=2, act=1),
-           dict(cores=9), dict(cores=-1)]
+           dict(cores=9), dict(cores=-1), dict(conv_k=-1), dict(conv_k=65),
+           dict(conv_k=2), dict(query_ln=2), dict(query_ln=1)]
     for kw in bad:
         with pytest.raises(ValueError):
             oracle.forward(dict(base, **kw), t, B=1)
@@ -503,3 +504,160 @@ def test_mcs_one_core_is_plain():
     b = oracle.forward(dict(cfg, cores=1), dict(t, core=t["core"][:, None]), B=3)
     for x, y in zip(a, b):
         np.testing.assert_array_equal(x, y)
+
+
+# ---- query-side extras (Sec. 3.1, Trick 4 convolution, Trick 2 LayerNorm) ----
+
+def _conv_layer(cfg, B, taps=None, bias=None, state_seqs=None):
+    t = util.numpy_layer(cfg, B=B)
+    if taps is not None:
+        t["conv_w"] = np.asarray(taps, np.float32)
+        t["conv_b"] = None if bias is None else np.asarray(bias, np.float32)
+    if state_seqs:
+        t["conv_state"] = workloads.stored_numpy(workloads.make_conv_state(cfg, state_seqs))
+    return t
+
+
+def test_identity_conv_is_no_conv():
+    """Taps [1, 0, ..] without bias leave the query input unchanged."""
+    cfg = _f32_cfg(conv_k=3)
+    taps = np.zeros((3, cfg["d_in"]))
+    taps[0] = 1
+    t = _conv_layer(cfg, 6, taps)
+    plain = oracle.forward(dict(cfg, conv_k=0), t, B=6)
+    for a, b in zip(oracle.forward(cfg, t, B=6), plain):
+        np.testing.assert_array_equal(a, b)
+
+
+@pytest.mark.parametrize("lag", [1, 2])
+def test_shift_conv_reads_previous_tokens(lag):
+    """One tap at lag j makes the query input the token j positions back in
+    its own sequence, or the state row before the sequence: the layer then
+    equals the plain layer on those shifted rows."""
+    cfg = _f32_cfg(conv_k=3)
+    S, L = 3, 4
+    taps = np.zeros((3, cfg["d_in"]))
+    taps[lag] = 1
+    t = _conv_layer(cfg, S * L, taps, state_seqs=S)
+    t["seq_len"] = L
+    x, st = t["x"].reshape(S, L, -1), t["conv_state"]
+    shifted = np.concatenate([st, x], axis=1)[:, 2 - lag:2 - lag + L].reshape(S * L, -1)
+    t0 = dict(t, x=np.ascontiguousarray(shifted))
+    plain = oracle.forward(dict(cfg, conv_k=0), t0, B=S * L)
+    for a, b in zip(oracle.forward(cfg, t, B=S * L), plain):
+        np.testing.assert_array_equal(a, b)
+
+
+def test_conv_equals_numpy_convolution():
+    """The causal depthwise convolution against numpy's np.convolve per
+    channel, on small integers and quarter taps so that every input, product
+    and sum is exact in fp32: the layer equals the plain layer on x~."""
+    cfg = _f32_cfg(conv_k=4)
+    B, rng = 9, np.random.default_rng(3)
+    t = util.numpy_layer(cfg, B=B)
+    t["x"] = rng.integers(-3, 4, (B, cfg["d_in"])).astype(np.float32)
+    t["conv_w"] = (rng.integers(-4, 5, (4, cfg["d_in"])) / 4).astype(np.float32)
+    t["conv_b"] = (rng.integers(-2, 3, cfg["d_in"]) / 2).astype(np.float32)
+    xt = np.stack([np.convolve(t["x"][:, c], t["conv_w"][:, c])[:B]
+                   for c in range(cfg["d_in"])], axis=1) + t["conv_b"]
+    plain = oracle.forward(dict(cfg, conv_k=0), dict(t, x=xt.astype(np.float32)), B=B)
+    for a, b in zip(oracle.forward(cfg, t, B=B), plain):
+        np.testing.assert_array_equal(a, b)
+
+
+@pytest.mark.parametrize("first", [1, 2, 5])
+def test_conv_state_carries_sequences_across_calls(first):
+    """Two sequences of 7 tokens in one call equal the same sequences cut
+    after `first` tokens, the second call starting from the state the first
+    left (decode is the case of one token per call)."""
+    cfg = _f32_cfg(conv_k=4, query_ln=1, ln_eps=1e-5)
+    S, L = 2, 7
+    t = _conv_layer(cfg, S * L, state_seqs=S)
+    t["seq_len"] = L
+    whole = oracle.forward(cfg, t, B=S * L)
+    x = t["x"].reshape(S, L, -1)
+    t1 = dict(t, x=np.ascontiguousarray(x[:, :first].reshape(S * first, -1)), seq_len=first)
+    part1 = oracle.forward(cfg, t1, B=S * first)
+    st = oracle.conv_state(cfg, t1, B=S * first).astype(np.float32)
+    rest = L - first
+    t2 = dict(t, x=np.ascontiguousarray(x[:, first:].reshape(S * rest, -1)), seq_len=rest,
+              conv_state=st)
+    part2 = oracle.forward(cfg, t2, B=S * rest)
+    for a, p1, p2 in zip(whole, part1, part2):
+        a = a.reshape(S, L, *a.shape[1:])
+        np.testing.assert_array_equal(a[:, :first], p1.reshape(S, first, *p1.shape[1:]))
+        np.testing.assert_array_equal(a[:, first:], p2.reshape(S, rest, *p2.shape[1:]))
+
+
+def test_conv_state_is_the_last_inputs():
+    """The state after a call: the last conv_k - 1 inputs of each sequence,
+    reaching into the previous state when a sequence is shorter."""
+    cfg = _f32_cfg(conv_k=4)
+    t = _conv_layer(cfg, 6, state_seqs=3)
+    x = t["x"]
+    for L in (3, 2, 1):
+        S = 6 // L if L != 1 else 3
+        tt = dict(t, x=np.ascontiguousarray(x[:S * L]), seq_len=L)
+        got = oracle.conv_state(cfg, tt, B=S * L)
+        hist = np.concatenate([t["conv_state"][:S], x[:S * L].reshape(S, L, -1)], axis=1)
+        np.testing.assert_array_equal(got, hist[:, -3:])
+
+
+@pytest.mark.parametrize("share", [1, 0])
+def test_query_layernorm_against_torch(share):
+    """Trick 2 on each head's query against torch.nn.functional.layer_norm,
+    then Eq. 4 by numpy reshapes; a separate column query has its own gain
+    and bias."""
+    torch = pytest.importorskip("torch")
+    cfg = _f32_cfg(query_ln=1, ln_eps=1e-3, share_query=share)
+    t = util.numpy_layer(cfg, B=3)
+    r, dk, H = cfg["rank"], cfg["d_k"], cfg["heads"]
+    K = workloads.keys_per_axis(cfg)
+    g = t["ln_g"].astype(np.float64)
+    bb = t["ln_b"].astype(np.float64)
+    for b in range(3):
+        for h in range(H):
+            x = util.widen(t["x"])[b]
+            qs = []
+            for a, w in enumerate([t["w_q"], t["w_q"] if share else t["w_q_col"]]):
+                q = util.widen(w)[h * dk:(h + 1) * dk] @ x
+                a = 0 if share else a
+                q = torch.nn.functional.layer_norm(
+                    torch.from_numpy(q), (dk,), torch.from_numpy(g[a, h * dk:(h + 1) * dk]),
+                    torch.from_numpy(bb[a, h * dk:(h + 1) * dk]), eps=1e-3).numpy()
+                qs.append(q)
+            kr = util.widen(t["k_row"])[h].reshape(K, r, dk // r)
+            kc = util.widen(t["k_col"])[h].reshape(K, r, dk // r)
+            s_row = np.einsum("iac,ac->ai", kr, qs[0].reshape(r, dk // r))
+            s_col = np.einsum("jbc,bc->bj", kc, qs[1].reshape(r, dk // r))
+            o_row, o_col = oracle.row_col_scores(cfg, t, b, h)
+            np.testing.assert_allclose(o_row, s_row, rtol=1e-10, atol=1e-12)
+            np.testing.assert_allclose(o_col, s_col, rtol=1e-10, atol=1e-12)
+
+
+def test_query_layernorm_is_scale_invariant():
+    """With eps = 0, LayerNorm removes any positive scale of the query:
+    W_q scaled by 4 (exact in fp32) leaves the layer unchanged."""
+    cfg = _f32_cfg(query_ln=1, ln_eps=0.0, conv_k=2)
+    t = util.numpy_layer(cfg, B=4)
+    base = oracle.forward(cfg, t, B=4)
+    scaled = oracle.forward(cfg, dict(t, w_q=t["w_q"] * np.float32(4)), B=4)
+    for a, b in zip(base, scaled):
+        np.testing.assert_array_equal(a, b)
+
+
+def test_key_layernorm_against_torch():
+    """Trick 2 for keys: each stored key row layer-normalised like
+    torch.nn.functional.layer_norm."""
+    torch = pytest.importorskip("torch")
+    cfg = _f32_cfg(dtype=1)
+    t = util.numpy_layer(cfg, B=1)
+    dk = cfg["d_k"]
+    rng = np.random.default_rng(8)
+    g = (1 + 0.1 * rng.standard_normal(dk)).astype(np.float32)
+    bb = (0.1 * rng.standard_normal(dk)).astype(np.float32)
+    got = oracle.key_ln(t["k_row"], 1, g, bb, eps=1e-5)
+    ref = torch.nn.functional.layer_norm(
+        torch.from_numpy(util.widen(t["k_row"])), (dk,), torch.from_numpy(g.astype(np.float64)),
+        torch.from_numpy(bb.astype(np.float64)), eps=1e-5).numpy()
+    np.testing.assert_allclose(got, ref, rtol=1e-10, atol=1e-12)
