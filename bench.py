@@ -43,6 +43,12 @@ def parse():
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--cores", type=int, default=0,
                     help="component cores per head (Multi-Core Scoring); 0 = one core")
+    ap.add_argument("--conv-k", type=int, default=0,
+                    help="taps of the causal query convolution; each step continues B/L "
+                         "sequences by L tokens, the conv state carried from step to step")
+    ap.add_argument("--seq-len", type=int, default=1,
+                    help="L, tokens per sequence per step with a query convolution")
+    ap.add_argument("--query-ln", action="store_true", help="LayerNorm of each head's query")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -245,6 +251,11 @@ def _cfg_brief(cfg):
     d["storage"] = "f32" if int(cfg["dtype"]) == 0 else "bf16"
     if int(cfg.get("cores", 0)) > 1:
         d["mcs_cores"] = int(cfg["cores"])
+    if int(cfg.get("conv_k", 0)) > 0:
+        d["conv_k"] = int(cfg["conv_k"])
+        d["seq_len_per_step"] = int(cfg.get("seq_len_per_step", 1))
+    if int(cfg.get("query_ln", 0)):
+        d["query_ln"] = 1
     return d
 
 
@@ -254,7 +265,14 @@ def main():
     wl = args.workload or workloads.HEADLINE[0]
     B = args.batch or (workloads.HEADLINE[1] if wl == workloads.HEADLINE[0]
                        else workloads.CONFIGS[wl]["batches"][-1])
-    cfg = workloads.layer_config(wl, **({"cores": args.cores} if args.cores > 1 else {}))
+    over = {"cores": args.cores} if args.cores > 1 else {}
+    if args.conv_k > 0:
+        over["conv_k"] = args.conv_k
+    if args.query_ln:
+        over.update(query_ln=1, ln_eps=1e-5)
+    if args.conv_k > 0:
+        over["seq_len_per_step"] = args.seq_len
+    cfg = workloads.layer_config(wl, **over)
     if args.impl == "reference":
         return run_reference(args, cfg, B, wl)
 
@@ -273,20 +291,33 @@ def main():
     xs = [workloads.make_tokens(cfg, B, 100 * rank + i, device="cuda") for i in range(NB)]
     out = torch.empty((B, cfg["d_out"]), dtype=layer.dtype, device="cuda")
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
+    kc = int(cfg.get("conv_k", 0))
+    # with a query convolution every step continues B/L sequences by L tokens
+    # (L = 1: a decode step); batch i reads state i % 2 and writes the other
+    n_seq = B // max(1, args.seq_len)
+    states = [workloads.make_conv_state(cfg, n_seq, 0, device="cuda") for _ in range(2)] \
+        if kc > 1 else None
+
+    def fwd(i):
+        if states is None:
+            layer.forward(xs[i % NB], out=out)
+        else:
+            layer.forward_seq(xs[i % NB], n_seq, states[i % 2], states[(i + 1) % 2], out=out)
+
     stream = torch.cuda.Stream()
 
     use_graph = not args.no_graph
     graphs = []
     with torch.cuda.stream(stream):
         for i in range(3):
-            layer.forward(xs[0], out=out)
+            fwd(0)
         torch.cuda.synchronize()
         launches = layer.last_launches()   # kernels per forward (and per graph replay)
         if use_graph:
             for i in range(NB):
                 g = torch.cuda.CUDAGraph()
                 with torch.cuda.graph(g, stream=stream):
-                    layer.forward(xs[i], out=out)
+                    fwd(i)
                 graphs.append(g)
     torch.cuda.synchronize()
 
@@ -294,7 +325,7 @@ def main():
         if use_graph:
             graphs[i % NB].replay()
         else:
-            layer.forward(xs[i % NB], out=out)
+            fwd(i)
 
     with torch.cuda.stream(stream):
         for i in range(args.warmup):
@@ -329,12 +360,12 @@ def main():
     layer.profile(True)
     pgraphs = []
     with torch.cuda.stream(stream):
-        layer.forward(xs[0], out=out)
+        fwd(0)
         torch.cuda.synchronize()
         for i in range(NB if use_graph else 0):
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g, stream=stream):
-                layer.forward(xs[i], out=out)
+                fwd(i)
             pgraphs.append(g)
     torch.cuda.synchronize()
     stage_ms = {}
@@ -343,7 +374,7 @@ def main():
             if use_graph:
                 pgraphs[i % NB].replay()
             else:
-                layer.forward(xs[i % NB], out=out)
+                fwd(i)
             torch.cuda.synchronize()
             for k, v in layer.profile_read().items():
                 stage_ms.setdefault(k, []).append(v)

@@ -16,6 +16,14 @@
  *   S8  acc[p] += w * V[row]                       Eq. 15, pooled per virtual block
  *   S9  o = sum_p W_p^T acc[p]                     Eq. 13/15 (IVE) + Trick 6 output
  *
+ * Query-side extras (Sec. 3.1): with cfg.conv_k > 0 (Trick 4) the query input
+ * is the causal depthwise convolution x~[t] = conv_b + sum_j conv_w[j] (.) x[t-j]
+ * over the tokens of each sequence (the conv state supplies the inputs before
+ * a sequence); with cfg.query_ln = 1 (Trick 2) each head's D_k-wide query is
+ * layer-normalised (gain ln_g, bias ln_b, epsilon ln_eps) before S2.  The key
+ * LayerNorm of Trick 2 is a fixed transform of the key table at inference:
+ * ultramem_key_ln applies it once to stored keys.
+ *
  * Multi-Core Scoring (Sec. 3.2, Eq. 16-17), when cfg.cores = h > 1: each head's
  * Tucker core is the sum of h component cores, C = sum_i C^(i).  S3-S6 run on
  * that sum; each selected slot then carries h weights, the individual scores
@@ -81,11 +89,15 @@ typedef struct ultramem_config {
     int32_t cores;       /* h, component cores per head (MCS, Eq. 16-17): 0 or 1 = one
                             core; 2..8 needs act == ULTRAMEM_ACT_NONE and
                             (d_v / h) % 8 == 0                                        */
+    int32_t conv_k;      /* taps of the causal depthwise query convolution (Trick 4),
+                            0..64; 0 = none                                           */
+    int32_t query_ln;    /* 1: LayerNorm of each head's query (Trick 2); d_k <= 256  */
     uint64_t shuffle_seed; /* Eq. 14 shuffle: 0 = identity, otherwise the seeded
                               bijection pi(v) = (a v + c) mod E*N whose a and c come
                               from the first two SplitMix64 outputs of the seed
                               (a = 1 + o1 mod (E*N - 1) stepped up to gcd(a, E*N) = 1,
                               c = o2 mod E*N); E*N must be < 2^32                     */
+    float ln_eps;        /* query LayerNorm epsilon, >= 0 (inside the square root)   */
 } ultramem_config;
 
 /* The layer's parameters.  Device tensors are in the storage type cfg.dtype
@@ -105,6 +117,12 @@ typedef struct ultramem_weights {
     const void *values;    /* [N][D_v], physical table V; 16-byte aligned              */
     const void *w_proj;    /* [E][D_v][D'_v] projectors W_p, or NULL when has_proj == 0 */
     const uint32_t *perm;  /* [E*N] explicit shuffle v -> v', or NULL for the seeded one */
+    const float *conv_w;   /* fp32 [conv_k][D_i] when conv_k > 0: tap j multiplies the
+                              input j tokens back (j = 0: the token itself), else NULL */
+    const float *conv_b;   /* fp32 [D_i] convolution bias, or NULL                     */
+    const float *ln_g;     /* fp32 [A][H*D_k] query LayerNorm gain when query_ln == 1
+                              (A = 1 with share_query, 2 with a column query), else NULL */
+    const float *ln_b;     /* fp32 [A][H*D_k] LayerNorm bias, or NULL                   */
 } ultramem_weights;
 
 typedef struct ultramem_layer ultramem_layer;
@@ -122,13 +140,30 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
  * a no-op.  Waits for work still queued on the layer's workspace. */
 void ultramem_destroy(ultramem_layer *layer);
 
-/* S1-S9 for B tokens: x [B][D_i] -> out [B][D'_v] (both cfg.dtype).  Optional
+/* S1-S9 for B tokens: x [B][D_i] -> out [B][D'_v] (both cfg.dtype).  With a
+ * query convolution the B tokens are one sequence with nothing before it
+ * (ultramem_forward_seq gives the general case).  Optional
  * outputs (NULL to skip): idx_out [B][H][m] int64 virtual addresses v = i*K + j,
  * w_out [B][H][m][h] fp32 weights (h = max(1, cores): the slot's score, or its h
  * individual scores under MCS), each head's m slots ordered by (aggregate score
  * desc, v asc).  0 <= B <= max_tokens (B == 0 launches nothing). */
 ultramem_status ultramem_forward(ultramem_layer *layer, const void *x, int32_t B,
                                  void *out, int64_t *idx_out, float *w_out, void *stream);
+
+/* The forward on n_seq sequences of seq_len tokens each, back to back in x
+ * [n_seq*seq_len][D_i] (B = n_seq*seq_len <= max_tokens); out, idx_out and w_out
+ * as in ultramem_forward.  The query convolution (Trick 4) reaches back only
+ * within a sequence and, before its first token, into conv_state_in
+ * [n_seq][conv_k-1][D_i] (cfg.dtype, the inputs before each sequence, oldest
+ * first; NULL = zeros).  conv_state_out (same shape, may be NULL) receives the
+ * last conv_k-1 inputs of each sequence, reaching into conv_state_in when
+ * seq_len < conv_k-1; it must not overlap conv_state_in.  Decode is seq_len = 1
+ * with the states of the previous step.  Without a convolution the sequence
+ * layout changes nothing and the states are ignored. */
+ultramem_status ultramem_forward_seq(ultramem_layer *layer, const void *x, int32_t n_seq,
+                                     int32_t seq_len, const void *conv_state_in,
+                                     void *conv_state_out, void *out, int64_t *idx_out,
+                                     float *w_out, void *stream);
 
 /* The same forward on HOST buffers: copies x to the device, runs the forward
  * and copies out back, all on `stream`, and returns after the stream has
@@ -179,6 +214,16 @@ ultramem_status ultramem_lookup_reduce_noalloc(const ultramem_config *cfg, const
  * reports an error. */
 ultramem_status ultramem_check(ultramem_layer *layer, void *stream);
 
+/* Trick 2 for keys: LayerNorm of each of n_rows rows of width d (DEVICE, dtype
+ * ULTRAMEM_F32 or ULTRAMEM_BF16) with gain g [d] and bias b [d] (DEVICE fp32, b
+ * may be NULL) and epsilon eps, computed in fp32 and written to out (same type
+ * and shape; out == keys works in place).  At inference the key LayerNorm is a
+ * fixed transform of the key table: apply it once and create the layer with
+ * the result.  Asynchronous on `stream`. */
+ultramem_status ultramem_key_ln(const void *keys, int32_t dtype, int64_t n_rows, int32_t d,
+                                const float *g, const float *b, float eps, void *out,
+                                void *stream);
+
 /* Leading singular triplet of one r x r core (HOST, row-major fp32) with the
  * sign rule above (Eq. 7; the SVD of Eq. 11).  ULTRAMEM_EINVAL if sigma == 0. */
 ultramem_status ultramem_rank1(const float *core, int32_t r, float *u, float *t,
@@ -206,7 +251,7 @@ const char *ultramem_last_error(void);
 /* Human-readable name of a status code. */
 const char *ultramem_status_string(ultramem_status s);
 
-/* ABI version, currently 1. */
+/* ABI version, currently 2. */
 int32_t ultramem_version(void);
 
 #ifdef __cplusplus

@@ -25,21 +25,22 @@ EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
            "ultramem_check", "ultramem_rank1", "ultramem_profile_enable",
            "ultramem_profile_read", "ultramem_stage_name", "ultramem_status_string",
            "ultramem_last_error", "ultramem_version", "ultramem_lookup_reduce_noalloc",
-           "ultramem_last_launches")
+           "ultramem_last_launches", "ultramem_forward_seq", "ultramem_key_ln")
 
 
 class Config(C.Structure):
     _fields_ = [(name, C.c_int32) for name in (
         "d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out", "topk", "topm",
-        "has_proj", "share_query", "act", "dtype", "max_tokens", "cores")] + [
-        ("shuffle_seed", C.c_uint64)]
+        "has_proj", "share_query", "act", "dtype", "max_tokens", "cores", "conv_k",
+        "query_ln")] + [("shuffle_seed", C.c_uint64), ("ln_eps", C.c_float)]
 
 
 class Weights(C.Structure):
     _fields_ = [("w_q", C.c_void_p), ("w_q_col", C.c_void_p), ("k_row", C.c_void_p),
                 ("k_col", C.c_void_p), ("core", C.c_void_p), ("u", C.c_void_p),
                 ("t", C.c_void_p), ("values", C.c_void_p), ("w_proj", C.c_void_p),
-                ("perm", C.c_void_p)]
+                ("perm", C.c_void_p), ("conv_w", C.c_void_p), ("conv_b", C.c_void_p),
+                ("ln_g", C.c_void_p), ("ln_b", C.c_void_p)]
 
 
 class UltraMemError(RuntimeError):
@@ -72,6 +73,10 @@ def load(path: str | None = None) -> C.CDLL:
         lib.ultramem_destroy.restype = None
         lib.ultramem_forward.argtypes = [P, P, I32, P, P, P, P]
         lib.ultramem_forward.restype = I32
+        lib.ultramem_forward_seq.argtypes = [P, P, I32, I32, P, P, P, P, P, P]
+        lib.ultramem_forward_seq.restype = I32
+        lib.ultramem_key_ln.argtypes = [P, I32, I64, I32, P, P, C.c_float, P, P]
+        lib.ultramem_key_ln.restype = I32
         lib.ultramem_forward_host.argtypes = [P, P, I32, P, P]
         lib.ultramem_forward_host.restype = I32
         lib.ultramem_retrieve.argtypes = [P, P, I32, P, P, P]
@@ -128,6 +133,23 @@ def _ptr(t):
     return None if t is None else t.data_ptr()
 
 
+def key_ln(keys: torch.Tensor, g: torch.Tensor, b: torch.Tensor | None = None,
+           eps: float = 1e-5, out: torch.Tensor | None = None) -> torch.Tensor:
+    """Trick 2 for keys: LayerNorm of each row of ``keys`` (fp32 or bf16 on
+    the device) with gain g and bias b (fp32), in the keys' type."""
+    lib = load()
+    keys = keys.contiguous()
+    dt = {torch.float32: F32, torch.bfloat16: BF16}[keys.dtype]
+    d = keys.shape[-1]
+    out = torch.empty_like(keys) if out is None else out
+    g = g.to(torch.float32).contiguous()
+    bb = None if b is None else b.to(torch.float32).contiguous()
+    _check(lib.ultramem_key_ln(keys.data_ptr(), dt, keys.numel() // d, d, g.data_ptr(),
+                               _ptr(bb), float(eps), out.data_ptr(), _stream()),
+           "ultramem_key_ln")
+    return out
+
+
 def _stream():
     return torch.cuda.current_stream().cuda_stream
 
@@ -157,9 +179,13 @@ class UltraMemLayer:
             setattr(c, k, int(cfg[k]))
         c.max_tokens = int(max_tokens)
         c.cores = int(cfg.get("cores", 0))
+        c.conv_k = int(cfg.get("conv_k", 0))
+        c.query_ln = int(cfg.get("query_ln", 0))
+        c.ln_eps = float(cfg.get("ln_eps", 1e-5))
         c.shuffle_seed = int(cfg.get("shuffle_seed", 0))
         self._c = c
-        dev_keys = ("w_q", "w_q_col", "k_row", "k_col", "values", "w_proj", "perm")
+        dev_keys = ("w_q", "w_q_col", "k_row", "k_col", "values", "w_proj", "perm", "conv_w",
+                    "conv_b", "ln_g", "ln_b")
         self._keep = {k: (None if weights.get(k) is None else weights[k].contiguous())
                       for k in dev_keys}
         for k, v in self._keep.items():
@@ -173,7 +199,9 @@ class UltraMemLayer:
                     _ptr(self._keep["k_row"]), _ptr(self._keep["k_col"]),
                     self._core.data_ptr(), _ptr(self._u), _ptr(self._t),
                     _ptr(self._keep["values"]), _ptr(self._keep["w_proj"]),
-                    _ptr(self._keep["perm"]))
+                    _ptr(self._keep["perm"]), _ptr(self._keep["conv_w"]),
+                    _ptr(self._keep["conv_b"]), _ptr(self._keep["ln_g"]),
+                    _ptr(self._keep["ln_b"]))
         h = C.c_void_p()
         _check(self.lib.ultramem_create(C.byref(c), C.byref(w), C.byref(h)), "ultramem_create")
         self._h = h
@@ -200,6 +228,28 @@ class UltraMemLayer:
             w = torch.empty(self._w_shape(B), dtype=torch.float32, device=x.device)
         _check(self.lib.ultramem_forward(self._h, x.data_ptr(), B, out.data_ptr(), _ptr(idx),
                                          _ptr(w), _stream()), "ultramem_forward")
+        return (out, idx, w) if with_slots else out
+
+    def forward_seq(self, x: torch.Tensor, n_seq: int, state_in=None, state_out=None,
+                    out: torch.Tensor | None = None, with_slots=False):
+        """S1-S9 on n_seq sequences back to back in x [n_seq*L, D_i]; the
+        query convolution (Trick 4) reads state_in [n_seq, conv_k-1, D_i]
+        before each sequence and writes state_out (both optional)."""
+        x = x.contiguous()
+        B = x.shape[0]
+        if n_seq < 1 or B % n_seq:
+            raise ValueError(f"{B} tokens do not split into {n_seq} sequences")
+        if out is None:
+            out = torch.empty((B, int(self.cfg["d_out"])), dtype=self.dtype, device=x.device)
+        idx = w = None
+        if with_slots:
+            H, m = int(self.cfg["heads"]), int(self.cfg["topm"])
+            idx = torch.empty((B, H, m), dtype=torch.int64, device=x.device)
+            w = torch.empty(self._w_shape(B), dtype=torch.float32, device=x.device)
+        si = None if state_in is None else state_in.contiguous()
+        _check(self.lib.ultramem_forward_seq(self._h, x.data_ptr(), n_seq, B // n_seq, _ptr(si),
+                                             _ptr(state_out), out.data_ptr(), _ptr(idx),
+                                             _ptr(w), _stream()), "ultramem_forward_seq")
         return (out, idx, w) if with_slots else out
 
     def forward_host(self, x_host: torch.Tensor, out_host: torch.Tensor):

@@ -26,6 +26,7 @@ struct Workspace {
     float *cores = nullptr;   // MCS component cores [H][h][r][r] (h > 1 only)
     int *err = nullptr;
     void *x_stage = nullptr, *out_stage = nullptr;
+    void *xs = nullptr;   // the convolved query input (Trick 4)
     __nv_bfloat16 *qs = nullptr, *acc_bf = nullptr, *w_pt = nullptr;   // tensor path
 };
 
@@ -120,6 +121,11 @@ ultramem_status validate(const ultramem_config *c, const ultramem_weights *w) {
     if (c->cores < 0 || c->cores > 8) return ULTRAMEM_EINVAL;
     if (c->cores > 1 && (c->act != ULTRAMEM_ACT_NONE || c->d_v % (8 * c->cores)))
         return ULTRAMEM_EINVAL;   // MCS: raw scores, value slices of whole 16-byte words
+    if (c->conv_k < 0 || c->conv_k > 64 || (c->conv_k > 0 && !w->conv_w)) return ULTRAMEM_EINVAL;
+    if (c->query_ln != 0 && c->query_ln != 1) return ULTRAMEM_EINVAL;
+    if (c->query_ln && (!w->ln_g || c->d_k > 256 || !(c->ln_eps >= 0.f) ||
+                        !(c->ln_eps < INFINITY)))
+        return ULTRAMEM_EINVAL;
     if (c->d_in <= 0 || c->d_k <= 0 || c->heads <= 0 || c->rank < 1 || c->rank > 8)
         return ULTRAMEM_EINVAL;
     if (c->d_k % c->rank) return ULTRAMEM_EINVAL;
@@ -239,7 +245,7 @@ void free_workspace(Workspace &ws) {
     void *ptrs[] = {ws.q_part, ws.akey, ws.sel_w,   ws.acc,       ws.proj_part,
                     ws.sel_row, ws.sel_p, ws.core,   ws.u,         ws.t,
                     ws.err,    ws.x_stage, ws.out_stage, ws.qs,     ws.acc_bf,
-                    ws.w_pt,   ws.cores};
+                    ws.w_pt,   ws.cores,   ws.xs};
     for (void *p : ptrs)
         if (p) cudaFree(p);
     ws = Workspace();
@@ -255,6 +261,11 @@ Ptrs make_ptrs(ultramem_layer *L) {
     p.values = L->w.values;
     p.w_proj = L->w.w_proj;
     p.perm = L->w.perm;
+    p.conv_w = L->w.conv_w;
+    p.conv_b = L->w.conv_b;
+    p.ln_g = L->w.ln_g;
+    p.ln_b = L->w.ln_b;
+    p.xs = L->ws.xs;
     p.core = L->ws.core;
     p.cores = L->ws.cores;
     p.u = L->ws.u;
@@ -273,6 +284,7 @@ Ptrs make_ptrs(ultramem_layer *L) {
 Dims dims_for(const ultramem_layer *L, int B) {
     Dims d = L->base;
     d.B = B;
+    d.seq_len = B;   // one sequence unless the caller says otherwise
     d.q_splits = L->tc ? tc_query_splits(L->cfg, B) : query_splits(L->cfg, B);
     d.p_splits = L->tc ? tc_proj_splits(L->cfg, B) : proj_splits(L->cfg, B);
     return d;
@@ -301,23 +313,35 @@ void mark(ultramem_layer *L, int i, cudaStream_t st) {
 }
 
 // S1..S6 (retrieval) then S7..S9; `retrieve_only` stops after S6.
-ultramem_status run_cuda_core(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
+ultramem_status run_cuda_core(ultramem_layer *L, const Dims &d0, Ptrs p, cudaStream_t st,
                               bool retrieve_only, int *launches) {
     cudaError_t e;
+    Dims d = d0;
+    const int extras = (d.conv_k > 0) + d.query_ln;   // convolution, LayerNorm
     mark(L, 0, st);
-    if ((e = um::launch_query(d, p, st)) != cudaSuccess) return from_cuda(e);
+    if (d.conv_k > 0 && (e = um::launch_query_conv(d, p, false, st)) != cudaSuccess)
+        return from_cuda(e);
+    {
+        Ptrs pq = p;
+        if (d.conv_k > 0) pq.x = p.xs;   // the fp32 convolved rows
+        if ((e = um::launch_query(d, pq, d.conv_k > 0, st)) != cudaSuccess) return from_cuda(e);
+    }
+    if (d.query_ln) {
+        if ((e = um::launch_query_ln(d, p, nullptr, 0, st)) != cudaSuccess) return from_cuda(e);
+        d.q_splits = 1;   // the normalised query is split 0
+    }
     mark(L, 1, st);
     if ((e = um::launch_score(d, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 2, st);
     if ((e = um::launch_select(d, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 3, st);
-    *launches = 3;
+    *launches = 3 + extras;
     if (retrieve_only) return ULTRAMEM_OK;
     if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 4, st);
     if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 5, st);
-    *launches = 4 + (d.has_proj ? 2 : 0);   // the projection and its split-K reduce
+    *launches = 4 + (d.has_proj ? 2 : 0) + extras;   // the projection and its split-K reduce
     if (L->profiling) L->profiled_once = true;
     return ULTRAMEM_OK;
 }
@@ -329,8 +353,12 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     um::TcMaps mp = L->maps;
     const int Bmax = c.max_tokens;
     const int nt1 = um::tc_n_tile(d.B, 1);   // N tile of every contraction (one accumulator)
-    if (!um::tc_encode(&mp.x, p.x, (uint64_t)c.d_in, (uint64_t)d.B, 1, (uint32_t)nt1, 2))
+    const bool conv = d.conv_k > 0;
+    if (!conv && !um::tc_encode(&mp.x, p.x, (uint64_t)c.d_in, (uint64_t)d.B, 1, (uint32_t)nt1, 2))
         return ULTRAMEM_EINVAL;   // x must be 16-byte aligned
+    if (conv && !um::tc_encode(&mp.xs, L->ws.xs, 3ull * c.d_in, (uint64_t)d.B, 1,
+                               (uint32_t)nt1, 2))
+        return ULTRAMEM_ECUDA;
     if (!um::tc_encode(&mp.qs, L->ws.qs, 3ull * c.d_k, (uint64_t)Bmax, 2ull * d.H,
                        (uint32_t)nt1, 3) ||
         !um::tc_encode(&mp.acc, L->ws.acc_bf, (uint64_t)d.E * d.d_v, (uint64_t)Bmax, 1,
@@ -339,16 +367,30 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     p.acc_bf = c.has_proj ? L->ws.acc_bf : nullptr;
     cudaError_t e;
     mark(L, 0, st);
-    // Every kernel after the query projection is a programmatic dependent
-    // launch of its predecessor (not while profiling: the stage events sit
-    // between the kernels).  The query projection itself waits for all
-    // earlier work on the stream.
+    // Every kernel after the first is a programmatic dependent launch of its
+    // predecessor (not while profiling: the stage events sit between the
+    // kernels).  The first (the convolution, else the query projection)
+    // waits for all earlier work on the stream.
     Dims dd = d;
     dd.pdl = L->profiling ? 0 : 1;
+    // Trick 4: the convolution runs first and the query projection reads its
+    // output (fp32 for the CUDA-core query, three bf16 terms for the tensor
+    // cores); with Trick 2 the LayerNorm writes the scaled splits
     const bool small = d.B <= kSmallQueryBatch;
-    if ((e = small ? um::launch_query_small(d, p, L->ws.qs, Bmax, st)
-                   : um::launch_query_tc(d, p, mp, d.q_splits, L->ws.qs, Bmax, st)) != cudaSuccess)
+    if (conv && (e = um::launch_query_conv(d, p, !small, st)) != cudaSuccess) return from_cuda(e);
+    const bool write_qs = !d.query_ln;
+    const bool qpdl = conv && dd.pdl;   // a dependent of the convolution only
+    if ((e = small ? um::launch_query_small(d, p, L->ws.qs, Bmax, conv, write_qs, qpdl, st)
+                   : um::launch_query_tc(d, p, mp, d.q_splits, L->ws.qs, Bmax, conv, write_qs,
+                                         qpdl, st)) != cudaSuccess)
         return from_cuda(e);
+    if (d.query_ln) {
+        Dims dl = dd;
+        dl.q_splits = 1;   // the projection left the summed query in split 0
+        if ((e = um::launch_query_ln(dl, p, L->ws.qs, Bmax, st)) != cudaSuccess)
+            return from_cuda(e);
+    }
+    const int extras = conv + d.query_ln;
     mark(L, 1, st);
     if ((e = um::launch_score_tc(dd, p, mp, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 2, st);
@@ -356,13 +398,13 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     ds.q_splits = 1;   // the query projection wrote the summed query
     if ((e = um::launch_select(ds, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 3, st);
-    *launches = d.A + 2;   // one query projection per query
+    *launches = d.A + 2 + extras;   // one query projection per query
     if (retrieve_only) return ULTRAMEM_OK;
     if ((e = um::launch_gather(dd, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 4, st);
     if (d.has_proj && (e = um::launch_proj_tc(dd, p, mp, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 5, st);
-    *launches = d.A + 3 + (d.has_proj ? 1 : 0);
+    *launches = d.A + 3 + (d.has_proj ? 1 : 0) + extras;
     if (L->profiling) L->profiled_once = true;
     return ULTRAMEM_OK;
 }
@@ -381,7 +423,7 @@ ultramem_status run(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
 
 extern "C" {
 
-int32_t ultramem_version(void) { return 1; }
+int32_t ultramem_version(void) { return 2; }
 
 const char *ultramem_last_error(void) { return g_last_error; }
 
@@ -482,6 +524,9 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     d.k = cfg->topk;
     d.m = cfg->topm;
     d.nc = nc;
+    d.conv_k = cfg->conv_k;
+    d.query_ln = cfg->query_ln;
+    d.ln_eps = cfg->ln_eps;
     d.A = cfg->share_query ? 1 : 2;
     d.act = cfg->act;
     d.dtype = cfg->dtype;
@@ -522,6 +567,8 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
         e = cudaMalloc(&ws.x_stage, Bm * cfg->d_in * elt_size(*cfg));
     if (e == cudaSuccess)
         e = cudaMalloc(&ws.out_stage, Bm * cfg->d_out * elt_size(*cfg));
+    // the convolved input: three bf16 terms (tensor path) or fp32, 6 B a value covers both
+    if (e == cudaSuccess && cfg->conv_k > 0) e = cudaMalloc(&ws.xs, Bm * cfg->d_in * 6);
     if (e == cudaSuccess)
         e = cudaMemcpy(ws.core, hc, sizeof(float) * H * r * r, cudaMemcpyHostToDevice);
     if (e == cudaSuccess && nc > 1)
@@ -597,6 +644,44 @@ ultramem_status ultramem_forward(ultramem_layer *L, const void *x, int32_t B, vo
     p.idx_out = idx_out;
     p.w_out = w_out;
     return run(L, d, p, (cudaStream_t)stream, false);
+}
+
+ultramem_status ultramem_forward_seq(ultramem_layer *L, const void *x, int32_t n_seq,
+                                     int32_t seq_len, const void *conv_state_in,
+                                     void *conv_state_out, void *out, int64_t *idx_out,
+                                     float *w_out, void *stream) {
+    if (!L || n_seq < 0 || seq_len < 1) return ULTRAMEM_EINVAL;
+    if ((int64_t)n_seq * seq_len > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    const int B = n_seq * seq_len;
+    if (B == 0) return ULTRAMEM_OK;
+    if (!x || !out) return ULTRAMEM_EINVAL;
+    Dims d = dims_for(L, B);
+    d.seq_len = seq_len;
+    Ptrs p = make_ptrs(L);
+    p.x = x;
+    p.out = out;
+    p.idx_out = idx_out;
+    p.w_out = w_out;
+    if (L->cfg.conv_k > 1) {
+        const size_t bytes = (size_t)n_seq * (L->cfg.conv_k - 1) * L->cfg.d_in * elt_size(L->cfg);
+        const char *a = static_cast<const char *>(conv_state_in);
+        const char *b = static_cast<const char *>(conv_state_out);
+        if (a && b && a < b + bytes && b < a + bytes) return ULTRAMEM_EINVAL;   // overlap
+        p.state_in = conv_state_in;
+        p.state_out = conv_state_out;
+    }
+    return run(L, d, p, (cudaStream_t)stream, false);
+}
+
+ultramem_status ultramem_key_ln(const void *keys, int32_t dtype, int64_t n_rows, int32_t dd,
+                                const float *g, const float *b, float eps, void *out,
+                                void *stream) {
+    if (!keys || !g || !out || n_rows < 0 || dd < 1 || !(eps >= 0.f) || !(eps < INFINITY))
+        return ULTRAMEM_EINVAL;
+    if (dtype != ULTRAMEM_F32 && dtype != ULTRAMEM_BF16) return ULTRAMEM_EINVAL;
+    cudaGetLastError();
+    return from_cuda(um::launch_key_ln(keys, dtype, n_rows, dd, g, b, eps, out,
+                                       (cudaStream_t)stream));
 }
 
 ultramem_status ultramem_retrieve(ultramem_layer *L, const void *x, int32_t B,
@@ -694,6 +779,20 @@ int32_t ultramem_profile_read(ultramem_layer *L, float *ms, int32_t n) {
 }  // extern "C"
 
 namespace um {
+int device_sm_count() {
+    static int n = 0;
+    if (!n) {
+        int dev = 0, v = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v < 1) {
+            cudaGetLastError();
+            v = 1;
+        }
+        n = v;
+    }
+    return n;
+}
+
 // The seeded shuffle's multiplier and offset, for entry points defined in
 // other translation units.
 void host_shuffle_params(uint64_t seed, uint64_t M, uint64_t *a, uint64_t *c) {

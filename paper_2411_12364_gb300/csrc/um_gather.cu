@@ -407,6 +407,9 @@ size_t gather_smem_bytes(const Dims &d) { return sizeof(float) * kWarps * d.E * 
 template <typename K> static cudaError_t allow(K kern, size_t bytes) {
     return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
+template <auto K> static cudaError_t allow_padded() {
+    return allow(K, kSmemPerCta - static_smem_of<K>());
+}
 
 cudaError_t configure_gather(const Dims &d) {
     const size_t bytes = gather_smem_bytes(d);
@@ -416,12 +419,11 @@ cudaError_t configure_gather(const Dims &d) {
     if (e == cudaSuccess) e = allow(gather_reg_kernel<float, 4>, bytes);
     if (e == cudaSuccess) e = allow(gather_reg_kernel<__nv_bfloat16, 1>, bytes);
     if (e == cudaSuccess) e = allow(gather_reg_kernel<__nv_bfloat16, 4>, bytes);
-    if (e == cudaSuccess) e = allow(gather_bucket_kernel<float, 512>, bucket_smem_bytes(d, 16));
-    if (e == cudaSuccess)
-        e = allow(gather_bucket_kernel<__nv_bfloat16, 512>, bucket_smem_bytes(d, 16));
-    if (e == cudaSuccess) e = allow(gather_bucket_kernel<float, 256>, bucket_smem_bytes(d, 8));
-    if (e == cudaSuccess)
-        e = allow(gather_bucket_kernel<__nv_bfloat16, 256>, bucket_smem_bytes(d, 8));
+    // the bucketed kernels may be padded up to a whole SM's share (spread_smem)
+    if (e == cudaSuccess) e = allow_padded<gather_bucket_kernel<float, 512>>();
+    if (e == cudaSuccess) e = allow_padded<gather_bucket_kernel<__nv_bfloat16, 512>>();
+    if (e == cudaSuccess) e = allow_padded<gather_bucket_kernel<float, 256>>();
+    if (e == cudaSuccess) e = allow_padded<gather_bucket_kernel<__nv_bfloat16, 256>>();
     return e;
 }
 
@@ -430,12 +432,19 @@ static cudaError_t launch_gather_t(const Dims &d, const Ptrs &p, cudaStream_t st
     const size_t bytes = gather_smem_bytes(d);
     const bool fits_lanes = d.d_v / (16 / (int)sizeof(T)) <= 32;
     if (fits_lanes && d.d_v % (16 / (int)sizeof(T)) == 0 && d.E <= kBMaxE) {
-        if (d.B <= 2 * 152 && d.H * d.m <= 512)
-            return launch_kernel(d.pdl, gather_bucket_kernel<T, 512>, d.B, 512,
-                                 bucket_smem_bytes(d, 16), st, d, p);
-        if (d.H * d.m <= 256 && d.E <= 8)
-            return launch_kernel(d.pdl, gather_bucket_kernel<T, 256>, d.B, 256,
-                                 bucket_smem_bytes(d, 8), st, d, p);
+        // spread over the SMs (see spread_smem)
+        if (d.B <= 2 * 152 && d.H * d.m <= 512) {
+            constexpr auto k = gather_bucket_kernel<T, 512>;
+            return launch_kernel(d.pdl, k, d.B, 512,
+                                 spread_smem(bucket_smem_bytes(d, 16), static_smem_of<k>(), d.B),
+                                 st, d, p);
+        }
+        if (d.H * d.m <= 256 && d.E <= 8) {
+            constexpr auto k = gather_bucket_kernel<T, 256>;
+            return launch_kernel(d.pdl, k, d.B, 256,
+                                 spread_smem(bucket_smem_bytes(d, 8), static_smem_of<k>(), d.B),
+                                 st, d, p);
+        }
     }
     if (d.nc > 1)   // MCS beyond the bucketed kernel's range
         return launch_kernel(d.pdl, gather_kernel<T>, d.B, kThreads, bytes, st, d, p);

@@ -12,6 +12,9 @@
 //                                      one per value slice, Multi-Core Scoring)
 //   acc      [B][E*D_v]                per-block pooled rows, Eq. 15 inner sum
 //   proj_part[p_splits][B][D'_v]       split-K partial sums of the projection
+//   xs       the convolved query input x~ (Trick 4): bf16 [B][3][D_i], three
+//            terms per value, for the tensor-core query; fp32 [B][D_i] for
+//            the CUDA-core ones
 #pragma once
 
 #include <cuda.h>
@@ -35,6 +38,10 @@ struct Dims {
     uint64_t M;       // virtual slots E*N
     int E, d_v, d_out, k, m;
     int nc;           // component cores per head (MCS, Eq. 16-17); 1 = one core
+    int conv_k;       // taps of the causal depthwise query convolution; 0 = none
+    int seq_len;      // tokens per sequence of this call (the convolution's scope)
+    int query_ln;     // 1: LayerNorm of each head's query
+    float ln_eps;
     int A;            // 1 = shared query, 2 = separate column query
     int act, dtype, has_proj;
     uint64_t shuf_a, shuf_c;
@@ -58,6 +65,11 @@ struct Ptrs {
     __nv_bfloat16 *acc_bf;       // tensor path: acc rounded to bf16 [B][E*D_v]
     const int64_t *idx_in;       // lookup_reduce input addresses
     const float *w_in;           // lookup_reduce input weights [B][H][m][nc]
+    const float *conv_w, *conv_b;   // [conv_k][D_i], [D_i] or null
+    const float *ln_g, *ln_b;       // [A][H*D_k] each (ln_b may be null)
+    const void *state_in;        // [B/seq_len][conv_k-1][D_i] storage type, or null
+    void *state_out;             // same shape, or null
+    void *xs;                    // the convolved input (layout above)
     int *err;                    // device error word (bit flags above)
 };
 
@@ -66,6 +78,7 @@ struct Ptrs {
 struct TcMaps {
     CUtensorMap w_q, w_q_col, k_row, k_col, w_pt;
     CUtensorMap x, qs, acc;
+    CUtensorMap xs;      // the convolved input's three bf16 terms [B][3 D_i]
 };
 
 bool tc_init();
@@ -74,17 +87,31 @@ bool tc_encode(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid,
 int tc_n_tile(int B, int n_acc);
 cudaError_t configure_tc();
 cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int splits,
-                            __nv_bfloat16 *qs, int Bmax, cudaStream_t st);
+                            __nv_bfloat16 *qs, int Bmax, bool x_splits, bool write_qs,
+                            bool pdl, cudaStream_t st);
 cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st);
 // small batches: S1 on CUDA cores, 16 weight rows x 8 tokens per CTA
 cudaError_t configure_small();
+// x_f32: the token rows are the fp32 convolved input (p.xs, [B][D_i])
+// instead of x itself
 cudaError_t launch_query_small(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, int Bmax,
-                               cudaStream_t st);
+                               bool x_f32, bool write_qs, bool pdl, cudaStream_t st);
 cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st);
 cudaError_t launch_transpose_bf16(const void *src, void *dst, int rows, int cols,
                                   cudaStream_t st);
 
-cudaError_t launch_query(const Dims &d, const Ptrs &p, cudaStream_t st);
+// x_f32: the token rows p.x are fp32 (the convolved input) whatever the storage type
+cudaError_t launch_query(const Dims &d, const Ptrs &p, bool x_f32, cudaStream_t st);
+// Trick 4: the causal depthwise convolution of the call's tokens into p.xs
+// (three bf16 terms when `splits`, else fp32) and the conv state after them
+cudaError_t launch_query_conv(const Dims &d, const Ptrs &p, bool splits, cudaStream_t st);
+// Trick 2: LayerNorm of each head's query in place (split 0 of q_part, the
+// sum of d.q_splits partials), and its scaled splits when qs is not null
+cudaError_t launch_query_ln(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, int Bmax,
+                            cudaStream_t st);
+// LayerNorm of n_rows stored rows of width dd (keys), result in the same type
+cudaError_t launch_key_ln(const void *keys, int dtype, int64_t n_rows, int dd, const float *g,
+                          const float *b, float eps, void *out, cudaStream_t st);
 cudaError_t launch_score(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream_t st);
@@ -146,6 +173,46 @@ template <typename... KArgs, typename... Args>
 cudaError_t launch_kernel(bool pdl, void (*kernel)(KArgs...), dim3 grid, dim3 block,
                           size_t smem, cudaStream_t st, Args &&...args) {
     return launch_kernel(pdl, 1u, kernel, grid, block, smem, st, static_cast<Args &&>(args)...);
+}
+
+// ---- CTA placement of dependent launches ----------------------------------
+// The CTAs of a programmatic dependent launch are placed while the previous
+// kernel still holds SMs, and the scheduler packs them onto whichever SMs have
+// room at that moment.  Measured on GB300: the selection's 128 CTAs at decode
+// ran 1.15x (decode_1m) to 1.5x (mid_4m) slower packed 2-3 per SM than spread
+// one per SM.  A launch of `ctas` CTAs therefore asks for enough dynamic
+// shared memory that at most ceil(ctas / SMs) of them fit on one SM.
+constexpr size_t kSmemPerSM = 233472;     // 228 KB per SM
+constexpr size_t kSmemPerCta = 232448;    // 227 KB at most per CTA
+constexpr size_t kSmemReserved = 1024;    // the driver's reservation per CTA
+
+int device_sm_count();
+
+// Dynamic shared memory for a launch of `ctas` CTAs that need `need` bytes
+// each and have `static_bytes` of static shared memory.
+inline size_t spread_smem(size_t need, size_t static_bytes, int64_t ctas) {
+    const int sms = device_sm_count();
+    const int64_t per_sm = (ctas + sms - 1) / sms;
+    if (per_sm < 1 || per_sm >= 8) return need;
+    // (per_sm + 1) CTAs must not fit: each takes more than this
+    const size_t share = kSmemPerSM / (size_t)(per_sm + 1);
+    if (share <= kSmemReserved + static_bytes) return need;
+    const size_t pad = ((share - kSmemReserved - static_bytes + 1 + 127) / 128) * 128;
+    if (pad + static_bytes > kSmemPerCta) return need;
+    return pad > need ? pad : need;
+}
+
+// The static shared memory of kernel K (looked up once per kernel).
+template <auto K> size_t static_smem_of() {
+    static size_t bytes = [] {
+        cudaFuncAttributes a;
+        if (cudaFuncGetAttributes(&a, K) != cudaSuccess) {
+            cudaGetLastError();
+            return (size_t)0;
+        }
+        return (size_t)a.sharedSizeBytes;
+    }();
+    return bytes;
 }
 
 // ---- small device helpers ------------------------------------------------

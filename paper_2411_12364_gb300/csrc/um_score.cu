@@ -10,11 +10,15 @@ namespace {
 constexpr int kThreads = 256;
 
 // q_part[split][a][b][o] = sum over this split's slice of D_i of x[b][d] W[o][d]
-// Tile: 32 tokens x 64 outputs; each thread owns 2 tokens x 4 outputs.
-template <typename T>
+// Tile: 32 tokens x 64 outputs; each thread owns 2 tokens x 4 outputs.  TX:
+// the token rows' type (T, or fp32 for the convolved input x~ of Trick 4,
+// which the caller then passes as p.x).
+template <typename T, typename TX>
 __global__ void __launch_bounds__(kThreads) query_kernel(Dims d, Ptrs p) {
+    pdl_wait();
+    pdl_trigger();
     const int a = blockIdx.z / d.q_splits, split = blockIdx.z % d.q_splits;
-    const T *X = static_cast<const T *>(p.x);
+    const TX *X = static_cast<const TX *>(p.x);
     const T *W = static_cast<const T *>(a == 0 ? p.w_q : p.w_q_col);
     const int HD = d.H * d.d_k;
     const int o0 = blockIdx.x * 64, b0 = blockIdx.y * 32;
@@ -121,14 +125,15 @@ __global__ void __launch_bounds__(kThreads) score_kernel(Dims d, Ptrs p) {
 
 }  // namespace
 
-cudaError_t launch_query(const Dims &d, const Ptrs &p, cudaStream_t st) {
+cudaError_t launch_query(const Dims &d, const Ptrs &p, bool x_f32, cudaStream_t st) {
     const int HD = d.H * d.d_k;
     dim3 grid((HD + 63) / 64, (d.B + 31) / 32, d.A * d.q_splits);
     if (d.dtype == ULTRAMEM_BF16)
-        query_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(d, p);
-    else
-        query_kernel<float><<<grid, kThreads, 0, st>>>(d, p);
-    return cudaGetLastError();
+        return x_f32 ? launch_kernel(d.pdl, query_kernel<__nv_bfloat16, float>, grid, kThreads,
+                                     0, st, d, p)
+                     : launch_kernel(d.pdl, query_kernel<__nv_bfloat16, __nv_bfloat16>, grid,
+                                     kThreads, 0, st, d, p);
+    return launch_kernel(d.pdl, query_kernel<float, float>, grid, kThreads, 0, st, d, p);
 }
 
 cudaError_t launch_score(const Dims &d, const Ptrs &p, cudaStream_t st) {

@@ -860,7 +860,9 @@ template <typename T, int RM>
 static cudaError_t launch_select_t(const Dims &d, const Ptrs &p, size_t smem, cudaStream_t st) {
     if (d.B * d.H > 3 * 152)
         return launch_kernel(d.pdl, select_kernel<T, 4, RM>, d.B * d.H, kThreads, smem, st, d, p);
-    return launch_kernel(d.pdl, select_kernel<T, 3, RM>, d.B * d.H, kThreads, smem, st, d, p);
+    // decode grids: spread over the SMs (see spread_smem)
+    const size_t sm = spread_smem(smem, static_smem_of<select_kernel<T, 3, RM>>(), d.B * d.H);
+    return launch_kernel(d.pdl, select_kernel<T, 3, RM>, d.B * d.H, kThreads, sm, st, d, p);
 }
 
 cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st) {
@@ -883,7 +885,9 @@ cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream
 
 template <typename T, int RM> static cudaError_t allow_select(int bytes) {
     const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
-    cudaError_t e = cudaFuncSetAttribute(select_kernel<T, 3, RM>, a, bytes);
+    // the decode-grid kernel may be padded up to a whole SM's share
+    const int pad = (int)(kSmemPerCta - static_smem_of<select_kernel<T, 3, RM>>());
+    cudaError_t e = cudaFuncSetAttribute(select_kernel<T, 3, RM>, a, bytes > pad ? bytes : pad);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<T, 4, RM>, a, bytes);
     return e;
 }

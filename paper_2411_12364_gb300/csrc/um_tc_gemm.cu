@@ -460,6 +460,7 @@ struct QueryOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
     int B, HD, A, a, splits, kb_total, H, d_k, dk, r, Bmax;
+    int write_qs;         // 0: the query LayerNorm writes the splits later
     float *q_part;        // [splits][A][B][HD]; the result is split 0
     __nv_bfloat16 *qs;    // [2][H][Bmax][3][D_k] scaled split queries
     const float *u, *t;   // [H][r]
@@ -491,6 +492,7 @@ struct QueryOp {
             const int n = n0 + j;
             if (n >= B) break;
             q_part[((int64_t)a * B + n) * HD + m] = v[j];
+            if (!write_qs) continue;
             // a shared query feeds both axes; a separate column query only axis 1
             if (row_axis) put_split_query(qs, 0, h, c, n, v[j] * cu, H, Bmax, d_k);
             if (col_axis) put_split_query(qs, 1, h, c, n, v[j] * ct, H, Bmax, d_k);
@@ -692,16 +694,7 @@ int tc_n_tile(int B, int n_acc) {
     return n < cap ? n : cap;
 }
 
-static int sm_count() {
-    static int n = 0;
-    if (!n) {
-        int dev = 0;
-        if (cudaGetDevice(&dev) != cudaSuccess ||
-            cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
-            n = 1;
-    }
-    return n;
-}
+static int sm_count() { return device_sm_count(); }
 
 // TMEM columns of one accumulator buffer: the epilogue reads 32 columns at a
 // time, so cover the last such read, rounded to 32.
@@ -762,13 +755,17 @@ template <int NSPLIT, class Op> static cudaError_t allow_smem() {
 
 cudaError_t configure_tc() {
     cudaError_t e = allow_smem<1, QueryOp>();
+    if (e == cudaSuccess) e = allow_smem<3, QueryOp>();
     if (e == cudaSuccess) e = allow_smem<3, ScoreOp>();
     if (e == cudaSuccess) e = allow_smem<1, ProjOp>();
     return e;
 }
 
+// x_splits: the B operand is the convolved input as three bf16 terms (map
+// xs over [B][3 D_i]), contracted as three MMAs into one accumulator
 cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int splits,
-                            __nv_bfloat16 *qs, int Bmax, cudaStream_t st) {
+                            __nv_bfloat16 *qs, int Bmax, bool x_splits, bool write_qs,
+                            bool pdl, cudaStream_t st) {
     const int HD = d.H * d.d_k;
     const int n_tile = tc_n_tile(d.B, 1);
     const int kb_total = (d.d_in + kBlockK - 1) / kBlockK;
@@ -778,7 +775,8 @@ cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int 
         op.n_tile = n_tile;
         op.n_acc = 1;
         op.acc_chunk = 1 << 30;
-        op.b_split_stride = 0;
+        op.b_split_stride = x_splits ? d.d_in : 0;
+        op.write_qs = write_qs ? 1 : 0;
         op.err = p.err;
         op.B = d.B;
         op.HD = HD;
@@ -797,8 +795,11 @@ cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int 
         op.t = p.t;
         dim3 grid((HD + kTileM - 1) / kTileM, (d.B + n_tile - 1) / n_tile, splits);
         const int per = (kb_total + splits - 1) / splits;
-        cudaError_t e = launch_gemm<1>(grid, a == 0 ? mp.w_q : mp.w_q_col, mp.w_q, mp.x, op, per,
-                                       false, st);
+        const CUtensorMap &wa = a == 0 ? mp.w_q : mp.w_q_col;
+        // the first query waits for all earlier work on the stream, unless it
+        // follows this call's convolution
+        cudaError_t e = x_splits ? launch_gemm<3>(grid, wa, mp.w_q, mp.xs, op, per, pdl && a == 0, st)
+                                 : launch_gemm<1>(grid, wa, mp.w_q, mp.x, op, per, pdl && a == 0, st);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;

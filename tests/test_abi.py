@@ -30,7 +30,7 @@ def test_library_exports_every_declared_function():
 
 def test_version_and_status_strings():
     lib = binding.load()
-    assert lib.ultramem_version() == 1
+    assert lib.ultramem_version() == 2
     for s in (0, -1, -2, -3, -4, -5, -6):
         assert binding.status_string(s) not in ("", "unknown status")
     assert binding.status_string(-99) == "unknown status"
@@ -83,7 +83,9 @@ def _create(cfg_over=None, **w_over):
                                  dict(has_proj=0), dict(act=7), dict(dtype=9),
                                  dict(max_tokens=0), dict(n=30000),
                                  dict(rank=9, d_k=36), dict(cores=-1), dict(cores=9),
-                                 dict(cores=2, act=1), dict(cores=3), dict(cores=16)])
+                                 dict(cores=2, act=1), dict(cores=3), dict(cores=16),
+                                 dict(conv_k=2), dict(conv_k=-1), dict(query_ln=1),
+                                 dict(query_ln=2)])
 def test_create_rejects_invalid_configs(bad):
     st, h = _create(bad)
     assert st == binding.EINVAL
