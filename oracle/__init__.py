@@ -26,13 +26,14 @@ _lib = None
 
 F32, BF16 = 0, 1
 ACT_NONE, ACT_SOFTMAX = 0, 1
+SCORE_TUCKER, SCORE_PKM = 0, 1
 
 
 class Config(C.Structure):
     _fields_ = [(name, C.c_int32) for name in (
         "d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out",
         "topk", "topm", "has_proj", "share_query", "act", "dtype", "cores", "conv_k",
-        "query_ln")] + [("shuffle_seed", C.c_uint64), ("ln_eps", C.c_double)]
+        "query_ln", "score_mode")] + [("shuffle_seed", C.c_uint64), ("ln_eps", C.c_double)]
 
 
 class Tensors(C.Structure):
@@ -65,6 +66,7 @@ def _load():
             lib.uo_lookup_reduce.argtypes = [P, P, C.c_int64, P, P, P, C.c_int32]
             lib.uo_row_col_scores.argtypes = [P, P, C.c_int64, C.c_int64, C.c_int32, P, P]
             lib.uo_conv_state.argtypes = [P, P, C.c_int64, P]
+            lib.uo_exact_topm.argtypes = [P, P, C.c_int64, P, C.c_int64, P, P, C.c_int32]
             lib.uo_key_ln.argtypes = [P, C.c_int32, C.c_int64, C.c_int32, P, P, C.c_double, P]
             lib.uo_rank1.argtypes = [P, C.c_int32, P, P, P]
             lib.uo_shuffle.argtypes = [P, P, C.c_int64]
@@ -88,6 +90,7 @@ def make_config(cfg: dict) -> Config:
     c.conv_k = int(cfg.get("conv_k", 0))
     c.query_ln = int(cfg.get("query_ln", 0))
     c.ln_eps = float(cfg.get("ln_eps", 1e-5))
+    c.score_mode = int(cfg.get("score_mode", 0))
     return c
 
 
@@ -157,6 +160,25 @@ def forward(cfg: dict, tensors: dict, B: int, tokens=None, threads: int = 0):
     if st != 0:
         raise ValueError(f"uo_forward failed with status {st}")
     return out, idx, w
+
+
+def exact_topm(cfg: dict, tensors: dict, B: int, tokens=None, threads: int = 0):
+    """Eq. 5 (or Eq. 2 with PKM scoring) by brute force over the whole K x K
+    grid: ``(idx [n, H, m] i64, w [n, H, m] f64)`` in uo_forward's order."""
+    lib = _load()
+    c = make_config(cfg)
+    s, keep = _tensors(cfg, tensors)
+    tok = None if tokens is None else np.ascontiguousarray(tokens, dtype=np.int64)
+    n = B if tok is None else len(tok)
+    H, m = int(cfg["heads"]), int(cfg["topm"])
+    idx = np.zeros((n, H, m), np.int64)
+    w = np.zeros((n, H, m), np.float64)
+    st = lib.uo_exact_topm(C.byref(c), C.byref(s), int(B), _ptr(tok), int(n), idx.ctypes.data,
+                           w.ctypes.data, int(threads))
+    del keep
+    if st != 0:
+        raise ValueError(f"uo_exact_topm failed with status {st}")
+    return idx, w
 
 
 def lookup_reduce(cfg: dict, tensors: dict, idx, w, threads: int = 0):

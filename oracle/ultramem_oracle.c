@@ -79,6 +79,8 @@ static int check_config(const uo_config *cfg)
     if (cfg->conv_k < 0 || cfg->conv_k > 64) return UO_EINVAL;
     if (cfg->query_ln != 0 && cfg->query_ln != 1) return UO_EINVAL;
     if (cfg->query_ln && !(cfg->ln_eps >= 0.0)) return UO_EINVAL;
+    if (cfg->score_mode != UO_SCORE_TUCKER && cfg->score_mode != UO_SCORE_PKM) return UO_EINVAL;
+    if (cfg->score_mode == UO_SCORE_PKM && (cfg->rank != 1 || cfg->cores > 1)) return UO_EINVAL;
     return UO_OK;
 }
 
@@ -466,6 +468,33 @@ int uo_lookup_reduce(const uo_config *cfg, const uo_tensors *x, int64_t n_tokens
     return status;
 }
 
+/* ---- grid scores --------------------------------------------------------- */
+
+/* The score of slot (i, j): Eq. 5's S_row[:,i]^T C S_col[:,j] (TDQKR), or
+ * Eq. 2's s_row[i] + s_col[j] (product keys, rank 1). */
+static double grid_score(const uo_config *cfg, const double *s_row, const double *s_col,
+                         const double *C, int64_t K, int64_t i, int64_t j)
+{
+    if (cfg->score_mode == UO_SCORE_PKM) return s_row[i] + s_col[j];
+    const int32_t r = cfg->rank;
+    double g = 0.0;
+    for (int32_t al = 0; al < r; ++al)
+        for (int32_t be = 0; be < r; ++be)
+            g += s_row[(int64_t)al * K + i] * C[al * r + be] * s_col[(int64_t)be * K + j];
+    return g;
+}
+
+/* Each head's Tucker core, the sum of its component cores (MCS), in C. */
+static void head_core(const uo_config *cfg, const uo_tensors *x, int32_t h, double *C)
+{
+    const int32_t r = cfg->rank, nc = cores_of(cfg);
+    for (int32_t e = 0; e < r * r; ++e) {
+        C[e] = 0.0;
+        if (cfg->score_mode == UO_SCORE_PKM) continue;
+        for (int32_t i = 0; i < nc; ++i) C[e] += (double)x->core[((int64_t)h * nc + i) * r * r + e];
+    }
+}
+
 /* ---- the whole layer for one token ------------------------------------- */
 
 typedef struct {
@@ -490,12 +519,9 @@ static void token_forward(const uo_config *cfg, const uo_tensors *x, int64_t B, 
     for (int32_t h = 0; h < H; ++h) {
         const double *u = u_all + (int64_t)h * r, *t = t_all + (int64_t)h * r;
         /* the Tucker core is the sum of the head's component cores (MCS) */
-        const float *Ci = x->core + (int64_t)h * nc * r * r;
+        const float *Ci = x->core ? x->core + (int64_t)h * nc * r * r : NULL;
         double *C = sc->core;
-        for (int32_t e = 0; e < r * r; ++e) {
-            C[e] = 0.0;
-            for (int32_t i = 0; i < nc; ++i) C[e] += (double)Ci[(int64_t)i * r * r + e];
-        }
+        head_core(cfg, x, h, C);
 
         /* Eq. 4: S_row, S_col in R^{r x K} */
         row_col_scores(cfg, x, h, sc->q + (int64_t)h * cfg->d_k,
@@ -528,16 +554,13 @@ static void token_forward(const uo_config *cfg, const uo_tensors *x, int64_t B, 
         qsort(sc->axis, (size_t)K, sizeof(scored), by_score_desc_index_asc);
         for (int32_t e = 0; e < k; ++e) sc->sel_j[e] = sc->axis[e].index;
 
-        /* Eq. 10: exact Tucker score S_row^T C S_col on the k*k survivors */
+        /* Eq. 10: exact Tucker score S_row^T C S_col on the k*k survivors
+         * (with product keys, Eq. 2's sum s_row + s_col) */
         int64_t ncand = 0;
         for (int32_t ei = 0; ei < k; ++ei)
             for (int32_t ej = 0; ej < k; ++ej) {
                 int64_t i = sc->sel_i[ei], j = sc->sel_j[ej];
-                double g = 0.0;
-                for (int32_t al = 0; al < r; ++al)
-                    for (int32_t be = 0; be < r; ++be)
-                        g += sc->s_row[(int64_t)al * K + i] * C[al * r + be] *
-                             sc->s_col[(int64_t)be * K + j];
+                const double g = grid_score(cfg, sc->s_row, sc->s_col, C, K, i, j);
                 sc->cand[ncand].key = (float)g;
                 sc->cand[ncand].index = i * K + j; /* virtual address v */
                 sc->cand[ncand].value = g;
@@ -589,8 +612,8 @@ int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
                int64_t *idx, double *w, int32_t n_threads)
 {
     if (check_config(cfg) != UO_OK || !x || !out || B < 0) return UO_EINVAL;
-    if (!x->x || !x->w_q || !x->k_row || !x->k_col || !x->core || !x->values)
-        return UO_EINVAL;
+    if (!x->x || !x->w_q || !x->k_row || !x->k_col || !x->values) return UO_EINVAL;
+    if (!x->core && cfg->score_mode != UO_SCORE_PKM) return UO_EINVAL;
     if (!cfg->share_query && !x->w_q_col) return UO_EINVAL;
     if (cfg->has_proj && !x->w_proj) return UO_EINVAL;
     if ((x->u == NULL) != (x->t == NULL)) return UO_EINVAL;
@@ -611,19 +634,17 @@ int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
     double *cd = malloc(sizeof(double) * r * r);
     if (!u_all || !t_all || !cd) { free(u_all); free(t_all); free(cd); return UO_ENOMEM; }
     for (int32_t h = 0; h < H; ++h) {
-        if (x->u) {
+        if (cfg->score_mode == UO_SCORE_PKM) {   /* r = 1: the axis scores themselves */
+            u_all[h] = 1.0;
+            t_all[h] = 1.0;
+        } else if (x->u) {
             for (int32_t al = 0; al < r; ++al) {
                 u_all[h * r + al] = x->u[h * r + al];
                 t_all[h * r + al] = x->t[h * r + al];
             }
         } else {
             double sigma;
-            const int32_t nc = cores_of(cfg);
-            for (int32_t e = 0; e < r * r; ++e) {   /* the aggregate core (MCS) */
-                cd[e] = 0.0;
-                for (int32_t i = 0; i < nc; ++i)
-                    cd[e] += x->core[((int64_t)h * nc + i) * r * r + e];
-            }
+            head_core(cfg, x, h, cd);   /* the aggregate core (MCS) */
             if (uo_rank1(cd, r, u_all + h * r, t_all + h * r, &sigma) != UO_OK) {
                 free(u_all); free(t_all); free(cd);
                 return UO_EINVAL;
@@ -678,5 +699,103 @@ int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
     }
     free(u_all);
     free(t_all);
+    return status;
+}
+
+/* ---- Eq. 5 by brute force: the exact top-m of the whole grid ------------ */
+
+/* a ranks before b: score (fp32 key) descending, then index ascending */
+static int better(const scored *a, const scored *b)
+{
+    return a->key > b->key || (a->key == b->key && a->index < b->index);
+}
+
+/* Min-heap of the m best so far (the root is the worst kept). */
+static void heap_sift_down(scored *hp, int32_t n, int32_t i)
+{
+    for (;;) {
+        int32_t l = 2 * i + 1, r = l + 1, w = i;
+        if (l < n && better(&hp[w], &hp[l])) w = l;
+        if (r < n && better(&hp[w], &hp[r])) w = r;
+        if (w == i) return;
+        scored t = hp[i]; hp[i] = hp[w]; hp[w] = t;
+        i = w;
+    }
+}
+
+static void heap_push(scored *hp, int32_t *n, int32_t cap, scored c)
+{
+    if (*n < cap) {   /* sift up */
+        int32_t i = (*n)++;
+        hp[i] = c;
+        while (i > 0) {
+            int32_t p = (i - 1) / 2;
+            if (!better(&hp[p], &hp[i])) break;
+            scored t = hp[i]; hp[i] = hp[p]; hp[p] = t;
+            i = p;
+        }
+    } else if (better(&c, &hp[0])) {
+        hp[0] = c;
+        heap_sift_down(hp, *n, 0);
+    }
+}
+
+int uo_exact_topm(const uo_config *cfg, const uo_tensors *x, int64_t B, const int64_t *tokens,
+                  int64_t n_tokens, int64_t *idx, double *w, int32_t n_threads)
+{
+    if (check_config(cfg) != UO_OK || !x || B < 0) return UO_EINVAL;
+    if (!x->x || !x->w_q || !x->k_row || !x->k_col) return UO_EINVAL;
+    if (!x->core && cfg->score_mode != UO_SCORE_PKM) return UO_EINVAL;
+    if (!cfg->share_query && !x->w_q_col) return UO_EINVAL;
+    if (check_query_extras(cfg, x, B) != UO_OK) return UO_EINVAL;
+    if (!tokens) n_tokens = B;
+    for (int64_t e = 0; tokens && e < n_tokens; ++e)
+        if (tokens[e] < 0 || tokens[e] >= B) return UO_EINVAL;
+    const int32_t H = cfg->heads, r = cfg->rank, m = cfg->topm;
+    const int64_t K = keys_per_axis(cfg), HD = (int64_t)H * cfg->d_k;
+    int status = UO_OK;
+#ifdef _OPENMP
+    if (n_threads > 0) omp_set_num_threads(n_threads);
+#else
+    (void)n_threads;
+#endif
+#pragma omp parallel
+    {
+        double *q = malloc(sizeof(double) * 2 * HD), *xin = malloc(sizeof(double) * cfg->d_in);
+        double *s_row = malloc(sizeof(double) * r * K), *s_col = malloc(sizeof(double) * r * K);
+        double *C = malloc(sizeof(double) * r * r);
+        scored *hp = malloc(sizeof(scored) * m);
+        if (!q || !xin || !s_row || !s_col || !C || !hp) {
+#pragma omp atomic write
+            status = UO_ENOMEM;
+        } else {
+#pragma omp for schedule(dynamic, 1)
+            for (int64_t e = 0; e < n_tokens; ++e) {
+                const int64_t b = tokens ? tokens[e] : e;
+                queries(cfg, x, B, b, xin, q);
+                for (int32_t h = 0; h < H; ++h) {
+                    head_core(cfg, x, h, C);
+                    row_col_scores(cfg, x, h, q + (int64_t)h * cfg->d_k,
+                                   q + HD + (int64_t)h * cfg->d_k, s_row, s_col);
+                    int32_t n = 0;
+                    for (int64_t i = 0; i < K; ++i)
+                        for (int64_t j = 0; j < K; ++j) {
+                            scored c;
+                            c.value = grid_score(cfg, s_row, s_col, C, K, i, j);
+                            c.key = (float)c.value;
+                            c.index = i * K + j;
+                            heap_push(hp, &n, m, c);
+                        }
+                    qsort(hp, (size_t)n, sizeof(scored), by_score_desc_index_asc);
+                    for (int32_t t = 0; t < m; ++t) {
+                        const int64_t o = (e * H + h) * m + t;
+                        if (idx) idx[o] = hp[t].index;
+                        if (w) w[o] = hp[t].value;
+                    }
+                }
+            }
+        }
+        free(q); free(xin); free(s_row); free(s_col); free(C); free(hp);
+    }
     return status;
 }

@@ -16,6 +16,7 @@
  * Paper sections and equations cited below use the paper's own numbering:
  *   Eq. 1   generic memory layer          s = sigma(K q),  o = V^T s
  *   Eq. 2-3 product keys (PKM)            two-phase top-m, softmax pooling
+ *           (score_mode UO_SCORE_PKM: additive grid score, exact two-phase)
  *   Eq. 4   row/column scores             S_row = K_row q_row, S_col = K_col q_col
  *   Eq. 5   Tucker grid score             S_grid = TopM(S_row^T C S_col)
  *   Eq. 6-7 rank-1 approximation          C ~ u t^T (leading singular pair)
@@ -43,6 +44,7 @@ extern "C" {
 
 enum { UO_F32 = 0, UO_BF16 = 1 };          /* storage type of the big tensors */
 enum { UO_ACT_NONE = 0, UO_ACT_SOFTMAX = 1 }; /* Trick 1 removes the softmax   */
+enum { UO_SCORE_TUCKER = 0, UO_SCORE_PKM = 1 }; /* grid score: Eq. 5 or Eq. 2   */
 
 typedef struct {
     int32_t d_in;        /* D_i: width of the input hidden x                    */
@@ -64,6 +66,9 @@ typedef struct {
     int32_t conv_k;      /* taps of the causal depthwise conv on x (Trick 4);
                             0 = no convolution                                  */
     int32_t query_ln;    /* 1: LayerNorm over each head's D_k query (Trick 2)   */
+    int32_t score_mode;  /* UO_SCORE_TUCKER: S_row^T C S_col (TDQKR, Eq. 5, 10);
+                            UO_SCORE_PKM: s_row[i] + s_col[j] (product keys,
+                            Eq. 2-3), needs rank 1 and one core; no core read  */
     uint64_t shuffle_seed; /* 0: identity shuffle; else the seeded bijection   */
     double ln_eps;       /* LayerNorm epsilon (inside the square root)          */
 } uo_config;
@@ -109,6 +114,14 @@ enum { UO_OK = 0, UO_EINVAL = -1, UO_ENOMEM = -2 };
 int uo_forward(const uo_config *cfg, const uo_tensors *x, int64_t B,
                const int64_t *tokens, int64_t n_tokens,
                double *out, int64_t *idx, double *w, int32_t n_threads);
+
+/* Eq. 5 (or Eq. 2 with PKM scoring) without the two-phase search: the top-m
+ * of the whole K x K grid of each head, by brute force, in the order and tie
+ * rule of uo_forward.  idx [n_tokens][H][m], w [n_tokens][H][m] (the grid
+ * scores of the summed core, raw), either may be NULL.  Used to measure the
+ * recall of the approximate search of Eq. 6-10. */
+int uo_exact_topm(const uo_config *cfg, const uo_tensors *x, int64_t B, const int64_t *tokens,
+                  int64_t n_tokens, int64_t *idx, double *w, int32_t n_threads);
 
 /* Eq. 14-15 alone: pool the given (virtual address, weights) and project.
  * idx is [n_tokens][H][m], w [n_tokens][H][m][h]; only values, w_proj and

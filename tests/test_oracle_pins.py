@@ -661,3 +661,82 @@ def test_key_layernorm_against_torch():
         torch.from_numpy(util.widen(t["k_row"])), (dk,), torch.from_numpy(g.astype(np.float64)),
         torch.from_numpy(bb.astype(np.float64)), eps=1e-5).numpy()
     np.testing.assert_allclose(got, ref, rtol=1e-10, atol=1e-12)
+
+
+# ---- product-key scoring (Eq. 2-3) and the exact grid top-m (Eq. 5) ----------
+
+def _pkm_cfg(**kw):
+    return _f32_cfg(rank=1, score_mode=1, **kw)
+
+
+def test_exact_topm_is_the_brute_force_grid():
+    """uo_exact_topm against numpy's grid S_row^T C S_col (Eq. 5) over every
+    slot, with the summed core under Multi-Core Scoring."""
+    for cfg in (_f32_cfg(), _f32_cfg(cores=2, d_v=8), _f32_cfg(rank=3, d_k=12)):
+        t = _mcs_layer(cfg, B=3) if cfg.get("cores") else util.numpy_layer(cfg, B=3)
+        idx, w = oracle.exact_topm(cfg, t, 3)
+        core = parity_core(cfg, t)
+        for b in range(3):
+            for h in range(cfg["heads"]):
+                v, g = util.brute_force_grid(cfg, t, b, h, core[h])
+                np.testing.assert_array_equal(idx[b, h], v)
+                np.testing.assert_allclose(w[b, h], g, rtol=1e-12, atol=1e-13)
+
+
+def parity_core(cfg, t):
+    c = np.asarray(t["core"], np.float64)
+    return c.sum(axis=1) if int(cfg.get("cores", 0)) > 1 else c
+
+
+def test_exact_topm_equals_search_without_pruning():
+    """With k = K the two-phase search keeps every key and is exact."""
+    cfg = _f32_cfg()
+    cfg["topk"] = workloads.keys_per_axis(cfg)
+    t = util.numpy_layer(cfg, B=4)
+    _, idx, w = oracle.forward(cfg, t, 4)
+    ei, ew = oracle.exact_topm(cfg, t, 4)
+    np.testing.assert_array_equal(idx, ei)
+    np.testing.assert_array_equal(w, ew)
+
+
+def test_pkm_scores_are_additive():
+    """Eq. 2: with product keys the grid score is s_row[i] + s_col[j]
+    (numpy reshapes, rank 1), searched over every slot when k = K."""
+    cfg = _pkm_cfg()
+    K = workloads.keys_per_axis(cfg)
+    cfg["topk"] = K
+    t = util.numpy_layer(cfg, B=3)
+    t.pop("core")
+    _, idx, w = oracle.forward(cfg, t, 3)
+    for b in range(3):
+        for h in range(cfg["heads"]):
+            s_row, s_col = util.numpy_scores(cfg, t, b, h)
+            G = (s_row[0][:, None] + s_col[0][None, :]).ravel()
+            v = np.arange(K * K)
+            pos = util.topm_desc(G, v, cfg["topm"])
+            np.testing.assert_array_equal(idx[b, h], v[pos])
+            np.testing.assert_allclose(w[b, h], G[pos], rtol=1e-12, atol=1e-13)
+
+
+@pytest.mark.parametrize("act", [0, 1])
+def test_pkm_two_phase_is_exact(act):
+    """Product keys' two-phase top-m is exact once k >= m: a slot of the
+    grid's top m has its row among the top m rows (else m rows would beat
+    it in its own column), and its column likewise (Sec. 3.1)."""
+    cfg = _pkm_cfg(topk=6, topm=6, act=act)
+    t = util.numpy_layer(cfg, B=5)
+    t.pop("core")
+    _, idx, w = oracle.forward(cfg, t, 5)
+    ei, ew = oracle.exact_topm(cfg, t, 5)
+    np.testing.assert_array_equal(idx, ei)
+    if act == 0:
+        np.testing.assert_array_equal(w, ew)
+    else:
+        np.testing.assert_allclose(w.sum(-1), 1.0, rtol=1e-12)
+
+
+def test_pkm_needs_rank_one():
+    cfg = dict(_pkm_cfg(), rank=2)
+    t = util.numpy_layer(_f32_cfg(), B=1)
+    with pytest.raises(ValueError):
+        oracle.forward(cfg, t, 1)
