@@ -49,6 +49,12 @@ def parse():
     ap.add_argument("--seq-len", type=int, default=1,
                     help="L, tokens per sequence per step with a query convolution")
     ap.add_argument("--query-ln", action="store_true", help="LayerNorm of each head's query")
+    ap.add_argument("--pkm", action="store_true",
+                    help="the layer as a product-key memory: rank 1, additive grid scores, "
+                         "softmax weights")
+    ap.add_argument("--recall", action="store_true",
+                    help="also measure the two-phase search's recall@m against the "
+                         "brute-force grid top-m, and the brute force's time")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -245,6 +251,27 @@ def run_reference(args, cfg, B, wl):
     print(json.dumps(line), flush=True)
 
 
+def measure_recall(layer, x, cfg, stream):
+    """recall@m of the forward's two-phase search (Eq. 6-10) against the
+    brute-force top-m of each head's whole grid (Eq. 5), over one batch,
+    and the device time of the brute force."""
+    import torch
+    with torch.cuda.stream(stream):
+        _, a_idx, _ = layer.forward(x, with_slots=True)
+        layer.retrieve_exact(x)   # warm-up
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        ev[0].record(stream)
+        e_idx, _ = layer.retrieve_exact(x)
+        ev[1].record(stream)
+    torch.cuda.synchronize()
+    a, e = a_idx.cpu().numpy(), e_idx.cpu().numpy()
+    B, H, m = a.shape
+    hits = sum(len(set(a[b, h].tolist()) & set(e[b, h].tolist()))
+               for b in range(B) for h in range(H))
+    return {"recall_at_m": hits / (B * H * m), "heads": B * H, "m": m,
+            "exact_ms": ev[0].elapsed_time(ev[1])}
+
+
 def _cfg_brief(cfg):
     keys = ("d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out", "topk", "topm")
     d = {k: int(cfg[k]) for k in keys}
@@ -256,6 +283,8 @@ def _cfg_brief(cfg):
         d["seq_len_per_step"] = int(cfg.get("seq_len_per_step", 1))
     if int(cfg.get("query_ln", 0)):
         d["query_ln"] = 1
+    if int(cfg.get("score_mode", 0)) == 1:
+        d["score"] = "product keys (Eq. 2-3)"
     return d
 
 
@@ -272,6 +301,8 @@ def main():
         over.update(query_ln=1, ln_eps=1e-5)
     if args.conv_k > 0:
         over["seq_len_per_step"] = args.seq_len
+    if args.pkm:
+        over.update(rank=1, score_mode=1, act=1)
     cfg = workloads.layer_config(wl, **over)
     if args.impl == "reference":
         return run_reference(args, cfg, B, wl)
@@ -418,6 +449,10 @@ def main():
            "h2d_bytes_per_step": B * cfg["d_in"] * es, "d2h_bytes_per_step": B * cfg["d_out"] * es,
            "ms_per_step": e2e_ms}
 
+    recall = None
+    if args.recall and rank == 0:
+        recall = measure_recall(layer, xs[0], cfg, stream)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(cfg, numpy_weights(w), B)
@@ -433,6 +468,8 @@ def main():
                 "roofline": roof, "gather": gather, "stages_ms": stage_avg,
                 "gpu_launches": K * launches, "e2e": e2e,
                 "cpu_baseline": cpu, "clocks": clk}
+        if recall is not None:
+            line["recall"] = recall
         print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()

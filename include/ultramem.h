@@ -68,6 +68,7 @@ typedef enum ultramem_status {
 
 enum { ULTRAMEM_F32 = 0, ULTRAMEM_BF16 = 1 };          /* storage of x, W_q, keys, V, W_p, out */
 enum { ULTRAMEM_ACT_NONE = 0, ULTRAMEM_ACT_SOFTMAX = 1 }; /* Trick 1 vs PKM's softmax (Eq. 3)  */
+enum { ULTRAMEM_SCORE_TUCKER = 0, ULTRAMEM_SCORE_PKM = 1 };   /* grid score: Eq. 5 or Eq. 2 */
 
 /* Hyper-parameters of one layer, in the paper's notation. */
 typedef struct ultramem_config {
@@ -92,6 +93,10 @@ typedef struct ultramem_config {
     int32_t conv_k;      /* taps of the causal depthwise query convolution (Trick 4),
                             0..64; 0 = none                                           */
     int32_t query_ln;    /* 1: LayerNorm of each head's query (Trick 2); d_k <= 256  */
+    int32_t score_mode;  /* ULTRAMEM_SCORE_TUCKER: g(i,j) = S_row[:,i]^T C S_col[:,j]
+                            (TDQKR, Eq. 5, 10); ULTRAMEM_SCORE_PKM: the product-key
+                            memory's g(i,j) = s_row[i] + s_col[j] (Eq. 2-3), exact
+                            two-phase search; needs rank 1 and one core, no core read */
     uint64_t shuffle_seed; /* Eq. 14 shuffle: 0 = identity, otherwise the seeded
                               bijection pi(v) = (a v + c) mod E*N whose a and c come
                               from the first two SplitMix64 outputs of the seed
@@ -108,7 +113,8 @@ typedef struct ultramem_weights {
     const void *k_row;     /* [H][K][D_k]; rank chunk alpha = columns alpha*D_k/r..    */
     const void *k_col;     /* [H][K][D_k]                                              */
     const float *core;     /* HOST fp32 [H][h][r][r] (h = max(1, cores)): component
-                              cores C_h^(i), copied at create; C_h is their sum         */
+                              cores C_h^(i), copied at create; C_h is their sum.  NULL
+                              with ULTRAMEM_SCORE_PKM                                   */
     const float *u;        /* HOST fp32 [H][r] or NULL: leading left singular vectors  */
     const float *t;        /* HOST fp32 [H][r] or NULL (both or neither); when NULL
                               they are computed at create from the SVD of C_h (the sum
@@ -175,6 +181,17 @@ ultramem_status ultramem_forward_host(ultramem_layer *layer, const void *x_host,
  * [B][H][m][h] fp32 as in ultramem_forward; both required. */
 ultramem_status ultramem_retrieve(ultramem_layer *layer, const void *x, int32_t B,
                                   int64_t *idx_out, float *w_out, void *stream);
+
+/* Eq. 5 (Eq. 2 with ULTRAMEM_SCORE_PKM) without the approximate search: S1
+ * (with the query extras), then the top-m of each head's whole K x K grid by
+ * brute force, for measuring the recall of the two-phase search of Eq. 6-10.
+ * idx_out [B][H][m] int64 and w_out [B][H][m] fp32 (raw grid scores of the
+ * summed core, no activation), ordered as in ultramem_forward; both required.
+ * Much slower than ultramem_retrieve (every grid score is computed several
+ * times).  ULTRAMEM_EINVAL when the layer's chunk scores do not fit one CTA's
+ * shared memory (K r > about 25000). */
+ultramem_status ultramem_retrieve_exact(ultramem_layer *layer, const void *x, int32_t B,
+                                        int64_t *idx_out, float *w_out, void *stream);
 
 /* S7-S9 only (the lookup-reduce of Eq. 14-15) on given slots: idx [B][H][m]
  * int64 virtual addresses in [0, E*N), w [B][H][m][h] fp32 (weight i scales value

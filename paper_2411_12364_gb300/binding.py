@@ -18,6 +18,7 @@ from . import build as _build
 OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EDEVICE, ENODEV = 0, -1, -2, -3, -4, -5, -6
 F32, BF16 = 0, 1
 ACT_NONE, ACT_SOFTMAX = 0, 1
+SCORE_TUCKER, SCORE_PKM = 0, 1
 
 # every function include/ultramem.h declares
 EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
@@ -25,14 +26,15 @@ EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
            "ultramem_check", "ultramem_rank1", "ultramem_profile_enable",
            "ultramem_profile_read", "ultramem_stage_name", "ultramem_status_string",
            "ultramem_last_error", "ultramem_version", "ultramem_lookup_reduce_noalloc",
-           "ultramem_last_launches", "ultramem_forward_seq", "ultramem_key_ln")
+           "ultramem_last_launches", "ultramem_forward_seq", "ultramem_key_ln",
+           "ultramem_retrieve_exact")
 
 
 class Config(C.Structure):
     _fields_ = [(name, C.c_int32) for name in (
         "d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out", "topk", "topm",
         "has_proj", "share_query", "act", "dtype", "max_tokens", "cores", "conv_k",
-        "query_ln")] + [("shuffle_seed", C.c_uint64), ("ln_eps", C.c_float)]
+        "query_ln", "score_mode")] + [("shuffle_seed", C.c_uint64), ("ln_eps", C.c_float)]
 
 
 class Weights(C.Structure):
@@ -80,6 +82,8 @@ def load(path: str | None = None) -> C.CDLL:
         lib.ultramem_forward_host.argtypes = [P, P, I32, P, P]
         lib.ultramem_forward_host.restype = I32
         lib.ultramem_retrieve.argtypes = [P, P, I32, P, P, P]
+        lib.ultramem_retrieve_exact.argtypes = [P, P, I32, P, P, P]
+        lib.ultramem_retrieve_exact.restype = I32
         lib.ultramem_retrieve.restype = I32
         lib.ultramem_lookup_reduce.argtypes = [P, P, P, I32, P, P]
         lib.ultramem_lookup_reduce.restype = I32
@@ -182,6 +186,7 @@ class UltraMemLayer:
         c.conv_k = int(cfg.get("conv_k", 0))
         c.query_ln = int(cfg.get("query_ln", 0))
         c.ln_eps = float(cfg.get("ln_eps", 1e-5))
+        c.score_mode = int(cfg.get("score_mode", 0))
         c.shuffle_seed = int(cfg.get("shuffle_seed", 0))
         self._c = c
         dev_keys = ("w_q", "w_q_col", "k_row", "k_col", "values", "w_proj", "perm", "conv_w",
@@ -191,13 +196,15 @@ class UltraMemLayer:
         for k, v in self._keep.items():
             if v is not None and not v.is_cuda:
                 raise ValueError(f"{k} must be a CUDA tensor")
-        self._core = weights["core"].detach().to("cpu", torch.float32).contiguous()
+        core = weights.get("core")
+        self._core = None if core is None else \
+            core.detach().to("cpu", torch.float32).contiguous()
         u, t = weights.get("u"), weights.get("t")
         self._u = None if u is None else torch.as_tensor(u).to("cpu", torch.float32).contiguous()
         self._t = None if t is None else torch.as_tensor(t).to("cpu", torch.float32).contiguous()
         w = Weights(_ptr(self._keep["w_q"]), _ptr(self._keep["w_q_col"]),
                     _ptr(self._keep["k_row"]), _ptr(self._keep["k_col"]),
-                    self._core.data_ptr(), _ptr(self._u), _ptr(self._t),
+                    _ptr(self._core), _ptr(self._u), _ptr(self._t),
                     _ptr(self._keep["values"]), _ptr(self._keep["w_proj"]),
                     _ptr(self._keep["perm"]), _ptr(self._keep["conv_w"]),
                     _ptr(self._keep["conv_b"]), _ptr(self._keep["ln_g"]),
@@ -268,6 +275,19 @@ class UltraMemLayer:
         w = torch.empty(self._w_shape(B), dtype=torch.float32, device=x.device)
         _check(self.lib.ultramem_retrieve(self._h, x.data_ptr(), B, idx.data_ptr(),
                                           w.data_ptr(), _stream()), "ultramem_retrieve")
+        return idx, w
+
+    def retrieve_exact(self, x: torch.Tensor):
+        """Eq. 5 (Eq. 2 for product keys) by brute force over each head's
+        whole grid: (idx [B,H,m] int64, w [B,H,m] fp32 raw scores)."""
+        x = x.contiguous()
+        B = x.shape[0]
+        H, m = int(self.cfg["heads"]), int(self.cfg["topm"])
+        idx = torch.empty((B, H, m), dtype=torch.int64, device=x.device)
+        w = torch.empty((B, H, m), dtype=torch.float32, device=x.device)
+        _check(self.lib.ultramem_retrieve_exact(self._h, x.data_ptr(), B, idx.data_ptr(),
+                                                w.data_ptr(), _stream()),
+               "ultramem_retrieve_exact")
         return idx, w
 
     def lookup_reduce(self, idx: torch.Tensor, w: torch.Tensor):

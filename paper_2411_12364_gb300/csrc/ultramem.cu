@@ -44,6 +44,7 @@ struct ultramem_layer {
     bool profiled_once = false;
     cudaEvent_t ev[kStages + 1] = {};
     int launches = 0;    // kernels launched by the most recent successful call
+    bool exact_ok = false;   // the brute-force top-m fits this layer's grid
 };
 
 namespace {
@@ -122,6 +123,10 @@ ultramem_status validate(const ultramem_config *c, const ultramem_weights *w) {
     if (c->cores > 1 && (c->act != ULTRAMEM_ACT_NONE || c->d_v % (8 * c->cores)))
         return ULTRAMEM_EINVAL;   // MCS: raw scores, value slices of whole 16-byte words
     if (c->conv_k < 0 || c->conv_k > 64 || (c->conv_k > 0 && !w->conv_w)) return ULTRAMEM_EINVAL;
+    if (c->score_mode != ULTRAMEM_SCORE_TUCKER && c->score_mode != ULTRAMEM_SCORE_PKM)
+        return ULTRAMEM_EINVAL;
+    const bool pkm = c->score_mode == ULTRAMEM_SCORE_PKM;
+    if (pkm && (c->rank != 1 || c->cores > 1)) return ULTRAMEM_EINVAL;
     if (c->query_ln != 0 && c->query_ln != 1) return ULTRAMEM_EINVAL;
     if (c->query_ln && (!w->ln_g || c->d_k > 256 || !(c->ln_eps >= 0.f) ||
                         !(c->ln_eps < INFINITY)))
@@ -145,7 +150,8 @@ ultramem_status validate(const ultramem_config *c, const ultramem_weights *w) {
     if (c->act != ULTRAMEM_ACT_NONE && c->act != ULTRAMEM_ACT_SOFTMAX) return ULTRAMEM_EINVAL;
     if (c->dtype != ULTRAMEM_F32 && c->dtype != ULTRAMEM_BF16) return ULTRAMEM_EINVAL;
     if (c->max_tokens < 1 || c->max_tokens > (1 << 20)) return ULTRAMEM_EINVAL;
-    if (!w->w_q || !w->k_row || !w->k_col || !w->core || !w->values) return ULTRAMEM_EINVAL;
+    if (!w->w_q || !w->k_row || !w->k_col || !w->values || (!w->core && !pkm))
+        return ULTRAMEM_EINVAL;
     if (!c->share_query && !w->w_q_col) return ULTRAMEM_EINVAL;
     if (c->has_proj && !w->w_proj) return ULTRAMEM_EINVAL;
     if ((w->u == nullptr) != (w->t == nullptr)) return ULTRAMEM_EINVAL;
@@ -312,9 +318,13 @@ void mark(ultramem_layer *L, int i, cudaStream_t st) {
         cudaEventRecord(L->ev[i], st);
 }
 
-// S1..S6 (retrieval) then S7..S9; `retrieve_only` stops after S6.
+// What a call runs: the whole forward, S1..S6 (retrieval), or S1 and the
+// brute-force exact top-m of the whole grid (recall measurement).
+enum RunMode { kForward, kRetrieve, kExact };
+
+// S1..S6 (retrieval) then S7..S9.
 ultramem_status run_cuda_core(ultramem_layer *L, const Dims &d0, Ptrs p, cudaStream_t st,
-                              bool retrieve_only, int *launches) {
+                              RunMode mode, int *launches) {
     cudaError_t e;
     Dims d = d0;
     const int extras = (d.conv_k > 0) + d.query_ln;   // convolution, LayerNorm
@@ -331,12 +341,18 @@ ultramem_status run_cuda_core(ultramem_layer *L, const Dims &d0, Ptrs p, cudaStr
         d.q_splits = 1;   // the normalised query is split 0
     }
     mark(L, 1, st);
+    if (mode == kExact) {
+        if ((e = um::launch_exact(d, p, p.idx_out, p.w_out, st)) != cudaSuccess)
+            return from_cuda(e);
+        *launches = 2 + extras;
+        return ULTRAMEM_OK;
+    }
     if ((e = um::launch_score(d, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 2, st);
     if ((e = um::launch_select(d, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 3, st);
     *launches = 3 + extras;
-    if (retrieve_only) return ULTRAMEM_OK;
+    if (mode == kRetrieve) return ULTRAMEM_OK;
     if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 4, st);
     if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
@@ -348,7 +364,7 @@ ultramem_status run_cuda_core(ultramem_layer *L, const Dims &d0, Ptrs p, cudaStr
 
 // The bf16 path: S1, S2 and S9 on tcgen05 tensor cores, S3-S8 as above.
 ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
-                           bool retrieve_only, int *launches) {
+                           RunMode mode, int *launches) {
     const ultramem_config &c = L->cfg;
     um::TcMaps mp = L->maps;
     const int Bmax = c.max_tokens;
@@ -392,6 +408,14 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     }
     const int extras = conv + d.query_ln;
     mark(L, 1, st);
+    if (mode == kExact) {
+        Dims dx = dd;
+        dx.q_splits = 1;   // the summed query is split 0
+        if ((e = um::launch_exact(dx, p, p.idx_out, p.w_out, st)) != cudaSuccess)
+            return from_cuda(e);
+        *launches = d.A + 1 + extras;
+        return ULTRAMEM_OK;
+    }
     if ((e = um::launch_score_tc(dd, p, mp, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 2, st);
     Dims ds = dd;
@@ -399,7 +423,7 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     if ((e = um::launch_select(ds, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 3, st);
     *launches = d.A + 2 + extras;   // one query projection per query
-    if (retrieve_only) return ULTRAMEM_OK;
+    if (mode == kRetrieve) return ULTRAMEM_OK;
     if ((e = um::launch_gather(dd, p, st)) != cudaSuccess) return from_cuda(e);
     mark(L, 4, st);
     if (d.has_proj && (e = um::launch_proj_tc(dd, p, mp, st)) != cudaSuccess) return from_cuda(e);
@@ -409,12 +433,11 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     return ULTRAMEM_OK;
 }
 
-ultramem_status run(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st,
-                    bool retrieve_only) {
+ultramem_status run(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_t st, RunMode mode) {
     cudaGetLastError();   // a stale error from unrelated work is not ours to report
     int n = 0;
-    const ultramem_status s = L->tc ? run_tensor(L, d, p, st, retrieve_only, &n)
-                                    : run_cuda_core(L, d, p, st, retrieve_only, &n);
+    const ultramem_status s = L->tc ? run_tensor(L, d, p, st, mode, &n)
+                                    : run_cuda_core(L, d, p, st, mode, &n);
     if (s == ULTRAMEM_OK) L->launches = n;
     return s;
 }
@@ -479,8 +502,15 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     float *ht = (float *)malloc(sizeof(float) * H * r);
     float *hc = (float *)malloc(sizeof(float) * H * r * r);
     if (!hu || !ht || !hc) { free(hu); free(ht); free(hc); return ULTRAMEM_ENOMEM; }
+    const bool pkm = cfg->score_mode == ULTRAMEM_SCORE_PKM;
     for (int h = 0; h < H; ++h) {
         double cd[64];
+        if (pkm) {   // product keys (rank 1): the axis scores themselves, summed
+            hc[h] = 1.f;
+            hu[h] = 1.f;
+            ht[h] = 1.f;
+            continue;
+        }
         for (int e = 0; e < r * r; ++e) {
             cd[e] = 0.0;
             for (int i = 0; i < nc; ++i) cd[e] += w->core[((size_t)h * nc + i) * r * r + e];
@@ -526,6 +556,7 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     d.nc = nc;
     d.conv_k = cfg->conv_k;
     d.query_ln = cfg->query_ln;
+    d.pkm = pkm ? 1 : 0;
     d.ln_eps = cfg->ln_eps;
     d.A = cfg->share_query ? 1 : 2;
     d.act = cfg->act;
@@ -611,6 +642,8 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
             return ULTRAMEM_EINVAL;   // a weight is not 16-byte aligned
         }
     }
+    L->exact_ok = um::exact_fits(d);
+    if (e == cudaSuccess && L->exact_ok) e = um::configure_exact(d);
     if (e == cudaSuccess) e = um::configure_select(d);
     if (e == cudaSuccess) e = um::configure_gather(d);
     if (e != cudaSuccess) {
@@ -643,7 +676,7 @@ ultramem_status ultramem_forward(ultramem_layer *L, const void *x, int32_t B, vo
     p.out = out;
     p.idx_out = idx_out;
     p.w_out = w_out;
-    return run(L, d, p, (cudaStream_t)stream, false);
+    return run(L, d, p, (cudaStream_t)stream, kForward);
 }
 
 ultramem_status ultramem_forward_seq(ultramem_layer *L, const void *x, int32_t n_seq,
@@ -670,7 +703,7 @@ ultramem_status ultramem_forward_seq(ultramem_layer *L, const void *x, int32_t n
         p.state_in = conv_state_in;
         p.state_out = conv_state_out;
     }
-    return run(L, d, p, (cudaStream_t)stream, false);
+    return run(L, d, p, (cudaStream_t)stream, kForward);
 }
 
 ultramem_status ultramem_key_ln(const void *keys, int32_t dtype, int64_t n_rows, int32_t dd,
@@ -694,7 +727,20 @@ ultramem_status ultramem_retrieve(ultramem_layer *L, const void *x, int32_t B,
     p.x = x;
     p.idx_out = idx_out;
     p.w_out = w_out;
-    return run(L, d, p, (cudaStream_t)stream, true);
+    return run(L, d, p, (cudaStream_t)stream, kRetrieve);
+}
+
+ultramem_status ultramem_retrieve_exact(ultramem_layer *L, const void *x, int32_t B,
+                                        int64_t *idx_out, float *w_out, void *stream) {
+    if (!L || B < 0 || B > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (B == 0) return ULTRAMEM_OK;
+    if (!x || !idx_out || !w_out || !L->exact_ok) return ULTRAMEM_EINVAL;
+    Dims d = dims_for(L, B);
+    Ptrs p = make_ptrs(L);
+    p.x = x;
+    p.idx_out = idx_out;
+    p.w_out = w_out;
+    return run(L, d, p, (cudaStream_t)stream, kExact);
 }
 
 ultramem_status ultramem_lookup_reduce(ultramem_layer *L, const int64_t *idx, const float *w,

@@ -41,6 +41,7 @@ struct Dims {
     int conv_k;       // taps of the causal depthwise query convolution; 0 = none
     int seq_len;      // tokens per sequence of this call (the convolution's scope)
     int query_ln;     // 1: LayerNorm of each head's query
+    int pkm;          // 1: product-key grid score s_row[i] + s_col[j] (rank 1)
     float ln_eps;
     int A;            // 1 = shared query, 2 = separate column query
     int act, dtype, has_proj;
@@ -117,6 +118,13 @@ cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_gather(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_proj(const Dims &d, const Ptrs &p, cudaStream_t st);
+
+// Eq. 5 by brute force (recall measurement): the exact top-m of every
+// (token, head)'s whole grid into idx_out / w_out [B][H][m]
+bool exact_fits(const Dims &d);
+cudaError_t configure_exact(const Dims &d);
+cudaError_t launch_exact(const Dims &d, const Ptrs &p, int64_t *idx_out, float *w_out,
+                         cudaStream_t st);
 
 // kernel attributes for large dynamic shared memory, set at layer creation
 cudaError_t configure_select(const Dims &d);

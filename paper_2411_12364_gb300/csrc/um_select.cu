@@ -1,7 +1,8 @@
 // um_select.cu -- S4..S7 for one (token, head) per CTA:
 //   top-k of each axis on the rank-1 score keys         (Eq. 8-9)
 //   exact chunk scores S_alpha of the 2k survivors      (Eq. 4)
-//   exact Tucker score g on the k*k survivor pairs      (Eq. 10)
+//   exact Tucker score g on the k*k survivor pairs      (Eq. 10; with product
+//                                                         keys s_row + s_col, Eq. 2)
 //   top-m of g, ordered by (score desc, v asc)          (Eq. 10)
 //   weights (raw scores, or PKM's softmax), shuffle     (Trick 1, Eq. 3, Eq. 14)
 //   with h component cores (MCS), the h individual scores of each winner
@@ -737,7 +738,9 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
         int ii = threadIdx.x / k, jj = threadIdx.x % k;
         for (int c = threadIdx.x; c < k2; c += kThreads) {
             float g;
-            if (r == 2) {   // the common rank, without the loop
+            if (d.pkm) {    // product keys (Eq. 2): s_row[i] + s_col[j]
+                g = L.R[ii] + L.scol[jj];
+            } else if (r == 2) {   // the common rank, without the loop
                 const float2 a2 = *reinterpret_cast<const float2 *>(L.R + ii * 2);
                 const float2 b2 = *reinterpret_cast<const float2 *>(L.scol + jj * 2);
                 g = fmaf(a2.y, b2.y, a2.x * b2.x);

@@ -60,16 +60,26 @@ def near_tie(cfg, t, b, h):
         return True
     I = np.argsort(-a, kind="stable")[:k]
     J = np.argsort(-bb, kind="stable")[:k]
-    G = s_row[:, I].T @ tucker_core(cfg, t)[h] @ s_col[:, J]
+    G = grid(cfg, t, h, s_row[:, I], s_col[:, J])
     return _gap_is_tie(G.ravel(), m)
+
+
+def grid(cfg, t, h, s_row, s_col):
+    """Grid scores of the given row and column score columns: Eq. 5's
+    S_row^T C S_col, or Eq. 2's s_row + s_col with product keys."""
+    if int(cfg.get("score_mode", 0)) == 1:
+        return s_row[0][:, None] + s_col[0][None, :]
+    return s_row.T @ tucker_core(cfg, t)[h] @ s_col
 
 
 def slot_scores(cfg, t, b, h, v):
     """Exact Eq. 5 score of given virtual addresses v = i*K + j."""
     K = workloads.keys_per_axis(cfg)
     s_row, s_col, _, _ = head_scores(cfg, t, b, h)
-    C = tucker_core(cfg, t)[h]
     i, j = np.asarray(v) // K, np.asarray(v) % K
+    if int(cfg.get("score_mode", 0)) == 1:
+        return s_row[0][i] + s_col[0][j]
+    C = tucker_core(cfg, t)[h]
     return np.einsum("an,ab,bn->n", s_row[:, i], C, s_col[:, j])
 
 
@@ -120,6 +130,10 @@ def numpy_inputs(cfg, weights, x):
     numpy's SVD so that both sides prune with the same singular pair."""
     t = {k: workloads.stored_numpy(v) for k, v in weights.items() if k not in ("u", "t")}
     t["x"] = workloads.stored_numpy(x)
+    if int(cfg.get("score_mode", 0)) == 1:   # product keys: the axis scores themselves
+        H = int(cfg["heads"])
+        t["u"] = t["t"] = np.ones((H, 1), np.float32)
+        return t
     u, tt = util.numpy_rank1(tucker_core(cfg, t))
     t["u"], t["t"] = u.astype(np.float32), tt.astype(np.float32)
     return t

@@ -85,7 +85,8 @@ def _create(cfg_over=None, **w_over):
                                  dict(rank=9, d_k=36), dict(cores=-1), dict(cores=9),
                                  dict(cores=2, act=1), dict(cores=3), dict(cores=16),
                                  dict(conv_k=2), dict(conv_k=-1), dict(query_ln=1),
-                                 dict(query_ln=2)])
+                                 dict(query_ln=2), dict(score_mode=2), dict(score_mode=1),
+                                 dict(score_mode=1, rank=1, d_k=32, cores=2)])
 def test_create_rejects_invalid_configs(bad):
     st, h = _create(bad)
     assert st == binding.EINVAL

@@ -57,6 +57,9 @@ SMALL = [
     dict(dtype=0, cores=2, expand_e=1, has_proj=0, d_out=64, n=40),
     dict(dtype=1, cores=8, d_v=128, d_out=40, heads=4, topk=16, topm=40),
     dict(dtype=1, cores=2, heads=4, topk=24, topm=160),   # H*m > 512: per-lane gather
+    dict(dtype=1, rank=1, score_mode=1),                  # product keys (Eq. 2), raw
+    dict(dtype=0, rank=1, score_mode=1, act=1),           # PKM with its softmax (Eq. 3)
+    dict(dtype=1, rank=1, score_mode=1, share_query=0, topk=16, topm=16),
 ]
 
 
@@ -75,6 +78,14 @@ def test_tiny_fp32_workload(gpu_lib):
 def test_decode_1m_workload(gpu_lib):
     cfg = workloads.layer_config("decode_1m")
     _run(cfg, 64, gpu_lib)
+
+
+@pytest.mark.parametrize("B", [64, 300])
+def test_product_key_workload(B, gpu_lib):
+    """The decode-shaped layer as a product-key memory (Eq. 2-3): rank 1,
+    additive grid scores, PKM's softmax over the m slots."""
+    cfg = workloads.layer_config("decode_1m", rank=1, score_mode=1, act=1)
+    _run(cfg, B, gpu_lib)
 
 
 @pytest.mark.parametrize("name,B", [("decode_1m", 64), ("mid_4m", 128)])
