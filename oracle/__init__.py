@@ -67,6 +67,7 @@ def _load():
             lib.uo_row_col_scores.argtypes = [P, P, C.c_int64, C.c_int64, C.c_int32, P, P]
             lib.uo_conv_state.argtypes = [P, P, C.c_int64, P]
             lib.uo_exact_topm.argtypes = [P, P, C.c_int64, P, C.c_int64, P, P, C.c_int32]
+            lib.uo_lookup_reduce_backward.argtypes = [P, P, C.c_int64, P, P, P, P, P, P]
             lib.uo_key_ln.argtypes = [P, C.c_int32, C.c_int64, C.c_int32, P, P, C.c_double, P]
             lib.uo_rank1.argtypes = [P, C.c_int32, P, P, P]
             lib.uo_shuffle.argtypes = [P, P, C.c_int64]
@@ -199,6 +200,31 @@ def lookup_reduce(cfg: dict, tensors: dict, idx, w, threads: int = 0):
     if st != 0:
         raise ValueError(f"uo_lookup_reduce failed with status {st}")
     return out
+
+
+def lookup_reduce_backward(cfg: dict, tensors: dict, idx, w, g):
+    """Backward of Eq. 14-15 for slots idx [n, H, m], weights w [n, H, m]
+    (or [n, H, m, h]) and dL/do g [n, d_out] (stored type): ``(dv [N, d_v],
+    dw (w's shape), dwp [E, d_v, d_out])`` in f64, dv accumulated from 0."""
+    lib = _load()
+    c = make_config(cfg)
+    s, keep = _tensors(cfg, tensors)
+    idx = np.ascontiguousarray(idx, dtype=np.int64)
+    w = np.ascontiguousarray(w, dtype=np.float64)
+    g = _stored(np.asarray(g), int(cfg["dtype"]))
+    n = idx.shape[0]
+    N = int(cfg["n"]) ** 2
+    E, dv_, do = int(cfg["expand_e"]), int(cfg["d_v"]), int(cfg["d_out"])
+    dv = np.zeros((N, dv_), np.float64)
+    dw = np.zeros(w.shape, np.float64)
+    dwp = np.zeros((E, dv_, do), np.float64)
+    st = lib.uo_lookup_reduce_backward(C.byref(c), C.byref(s), int(n), idx.ctypes.data,
+                                       w.ctypes.data, g.ctypes.data, dv.ctypes.data,
+                                       dw.ctypes.data, dwp.ctypes.data)
+    del keep
+    if st != 0:
+        raise ValueError(f"uo_lookup_reduce_backward failed with status {st}")
+    return dv, dw, dwp
 
 
 def row_col_scores(cfg: dict, tensors: dict, b: int, h: int, B: int | None = None):

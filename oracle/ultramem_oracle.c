@@ -495,6 +495,64 @@ static void head_core(const uo_config *cfg, const uo_tensors *x, int32_t h, doub
     }
 }
 
+/* ---- backward of Eq. 14-15 (App. D's fused lookup-reduce) -------------- */
+
+int uo_lookup_reduce_backward(const uo_config *cfg, const uo_tensors *x, int64_t n_tokens,
+                              const int64_t *idx, const double *w, const void *g, double *dv,
+                              double *dw, double *dwp)
+{
+    if (check_config(cfg) != UO_OK || !x || !x->values || !idx || !w || !g || n_tokens < 0)
+        return UO_EINVAL;
+    if (cfg->has_proj && !x->w_proj) return UO_EINVAL;
+    const int32_t E = cfg->expand_e, Dv = cfg->d_v, Do = cfg->d_out, nc = cores_of(cfg);
+    const int32_t slice = Dv / nc;
+    const int64_t N = (int64_t)cfg->n * cfg->n, M = (int64_t)E * N;
+    const int64_t hm = (int64_t)cfg->heads * cfg->topm;
+    for (int64_t e = 0; e < n_tokens * hm; ++e)
+        if (idx[e] < 0 || idx[e] >= M) return UO_EINVAL;
+    double *acc = malloc(sizeof(double) * E * Dv), *dacc = malloc(sizeof(double) * E * Dv);
+    if (!acc || !dacc) { free(acc); free(dacc); return UO_ENOMEM; }
+    if (dwp) memset(dwp, 0, sizeof(double) * E * Dv * Do);
+    for (int64_t b = 0; b < n_tokens; ++b) {
+        /* dL/dacc_p = W_p dL/do (the output is acc_0 itself without a projector) */
+        for (int32_t p = 0; p < E; ++p)
+            for (int32_t c = 0; c < Dv; ++c) {
+                double s = 0.0;
+                if (!cfg->has_proj) s = load(g, cfg->dtype, b * Do + c);
+                else
+                    for (int32_t o = 0; o < Do; ++o)
+                        s += load(x->w_proj, cfg->dtype, ((int64_t)p * Dv + c) * Do + o) *
+                             load(g, cfg->dtype, b * Do + o);
+                dacc[p * Dv + c] = s;
+                acc[p * Dv + c] = 0.0;
+            }
+        for (int64_t e = 0; e < hm; ++e) {
+            const int64_t slot = b * hm + e;
+            const int64_t vs = uo_shuffle(cfg, x->perm, idx[slot]);
+            const int64_t p = vs / N, row = vs % N;
+            if (dw)
+                for (int32_t i = 0; i < nc; ++i) dw[slot * nc + i] = 0.0;
+            for (int32_t c = 0; c < Dv; ++c) {
+                const int32_t sl = c / slice;
+                const double we = w[slot * nc + sl], V = load(x->values, cfg->dtype, row * Dv + c);
+                if (dv) dv[row * Dv + c] += we * dacc[p * Dv + c];
+                if (dw) dw[slot * nc + sl] += dacc[p * Dv + c] * V;
+                acc[p * Dv + c] += we * V;
+            }
+        }
+        /* dL/dW_p[c][o] = sum over tokens of acc_p[c] dL/do[o] */
+        if (dwp && cfg->has_proj)
+            for (int32_t p = 0; p < E; ++p)
+                for (int32_t c = 0; c < Dv; ++c)
+                    for (int32_t o = 0; o < Do; ++o)
+                        dwp[((int64_t)p * Dv + c) * Do + o] +=
+                            acc[p * Dv + c] * load(g, cfg->dtype, b * Do + o);
+    }
+    free(acc);
+    free(dacc);
+    return UO_OK;
+}
+
 /* ---- the whole layer for one token ------------------------------------- */
 
 typedef struct {

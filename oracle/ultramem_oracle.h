@@ -130,6 +130,20 @@ int uo_lookup_reduce(const uo_config *cfg, const uo_tensors *x, int64_t n_tokens
                      const int64_t *idx, const double *w, double *out,
                      int32_t n_threads);
 
+/* The backward of Eq. 14-15 (the fused lookup-reduce of App. D), by the chain
+ * rule on its definition.  For slots idx [n_tokens][H][m] with weights w
+ * [n_tokens][H][m][h] and the gradient g = dL/do [n_tokens][d_out] (stored in
+ * the config's type), with acc_p = sum_e w_e V[row_e] (block p) and
+ * o = sum_p W_p^T acc_p:
+ *   dacc_p = W_p g                       (g itself without a projector)
+ *   dv[row][c]   += w_e^(slice c) dacc_{p_e}[c]        accumulated, [N][d_v]
+ *   dw[e][i]      = sum_{c in slice i} dacc_{p_e}[c] V[row_e][c]   [n][H][m][h]
+ *   dwp[p][c][o]  = sum_tokens acc_p[c] g[o]                       [E][d_v][d_out]
+ * Any output may be NULL.  An address outside [0, E*N) is an error. */
+int uo_lookup_reduce_backward(const uo_config *cfg, const uo_tensors *x, int64_t n_tokens,
+                              const int64_t *idx, const double *w, const void *g, double *dv,
+                              double *dw, double *dwp);
+
 /* Eq. 4 for one (token b of a batch of B, head h): s_row[r][K], s_col[r][K]. */
 int uo_row_col_scores(const uo_config *cfg, const uo_tensors *x, int64_t B, int64_t b,
                       int32_t h, double *s_row, double *s_col);

@@ -740,3 +740,82 @@ def test_pkm_needs_rank_one():
     t = util.numpy_layer(_f32_cfg(), B=1)
     with pytest.raises(ValueError):
         oracle.forward(cfg, t, 1)
+
+
+# ---- backward of the lookup-reduce (Eq. 14-15, App. D) ----------------------
+
+def _torch_lookup_reduce(cfg, t, idx, w, perm):
+    """Eq. 14-15 restated in torch (float64, autograd on V, w and W_p)."""
+    torch = pytest.importorskip("torch")
+    N = cfg["n"] ** 2
+    E, dv, do = cfg["expand_e"], cfg["d_v"], cfg["d_out"]
+    h = max(1, int(cfg.get("cores", 0)))
+    V = torch.tensor(util.widen(t["values"]), requires_grad=True)
+    W = torch.tensor(util.widen(t["w_proj"]).reshape(E, dv, do), requires_grad=True) \
+        if cfg["has_proj"] else None
+    wt = torch.tensor(np.asarray(w, np.float64).reshape(idx.shape + (h,)), requires_grad=True)
+    vs = torch.from_numpy(perm[idx.ravel()]).reshape(idx.shape)
+    p, row = vs // N, vs % N
+    rows = V[row]                                                  # [n, H, m, dv]
+    wexp = wt.repeat_interleave(dv // h, dim=-1)                   # slice weights per column
+    contrib = wexp * rows
+    acc = torch.zeros(idx.shape[0], E, dv, dtype=torch.float64)
+    for b in range(idx.shape[0]):
+        acc[b] = acc[b].index_add(0, p[b].ravel(), contrib[b].reshape(-1, dv))
+    out = torch.einsum("bpc,pco->bo", acc, W) if W is not None else acc[:, 0]
+    return out, V, wt, W
+
+
+@pytest.mark.parametrize("over", [dict(), dict(cores=2, d_v=8), dict(expand_e=1, has_proj=0,
+                                                                     d_out=8, d_v=8, n=12)])
+def test_lookup_reduce_backward_against_autograd(over):
+    """The backward against torch's autograd of the lookup-reduce restated
+    in torch (the forward itself checked against the oracle's)."""
+    torch = pytest.importorskip("torch")
+    cfg = _f32_cfg(**over)
+    t = _mcs_layer(cfg, B=4) if cfg.get("cores") else util.numpy_layer(cfg, B=4)
+    _, idx, w = oracle.forward(cfg, t, 4)
+    # one slot of token 1 repeats one of token 0's: its row gradient accumulates twice
+    idx[1, 0, 0] = idx[0, 1, 2]
+    M = cfg["expand_e"] * cfg["n"] ** 2
+    perm = oracle.shuffle(cfg, np.arange(M))
+    out, V, wt, W = _torch_lookup_reduce(cfg, t, idx, w, perm)
+    np.testing.assert_allclose(out.detach().numpy(), oracle.lookup_reduce(cfg, t, idx, w),
+                               rtol=1e-12, atol=1e-14)
+    g = np.random.default_rng(4).standard_normal(out.shape).astype(np.float32)
+    (out * torch.from_numpy(g.astype(np.float64))).sum().backward()
+    dv, dw, dwp = oracle.lookup_reduce_backward(cfg, t, idx, w, g)
+    np.testing.assert_allclose(dv, V.grad.numpy(), rtol=1e-12, atol=1e-14)
+    np.testing.assert_allclose(dw.reshape(wt.grad.shape), wt.grad.numpy(), rtol=1e-12,
+                               atol=1e-14)
+    if W is not None:
+        np.testing.assert_allclose(dwp, W.grad.numpy(), rtol=1e-12, atol=1e-14)
+
+
+def test_lookup_reduce_backward_finite_differences():
+    """The loss sum(g * o) is linear in each of V, w and W_p, so a change of
+    one stored entry by d changes it by exactly d times that entry's
+    gradient (up to fp64 rounding): checked through the oracle's forward."""
+    cfg = _f32_cfg()
+    t = util.numpy_layer(cfg, B=3)
+    _, idx, w = oracle.forward(cfg, t, 3)
+    g = np.random.default_rng(6).standard_normal((3, cfg["d_out"])).astype(np.float32)
+    dv, dw, dwp = oracle.lookup_reduce_backward(cfg, t, idx, w, g)
+    base = (oracle.lookup_reduce(cfg, t, idx, w) * g).sum()
+    perm = oracle.shuffle(cfg, np.arange(cfg["expand_e"] * cfg["n"] ** 2))
+    row = int(perm[idx[2, 1, 3]] % cfg["n"] ** 2)
+    for c in (0, 5):
+        V = t["values"].copy()
+        V[row, c] = np.float32(V[row, c] + 2.0 ** -10)
+        d = float(V[row, c]) - float(t["values"][row, c])
+        got = (oracle.lookup_reduce(cfg, dict(t, values=V), idx, w) * g).sum() - base
+        np.testing.assert_allclose(got, d * dv[row, c], rtol=1e-9, atol=1e-15)
+    w2 = w.copy()
+    w2[2, 1, 3] += 0.125
+    got = (oracle.lookup_reduce(cfg, t, idx, w2) * g).sum() - base
+    np.testing.assert_allclose(got, 0.125 * dw[2, 1, 3], rtol=1e-9, atol=1e-15)
+    Wp = t["w_proj"].copy()
+    Wp[1, 3, 4] = np.float32(Wp[1, 3, 4] + 2.0 ** -8)
+    d = float(Wp[1, 3, 4]) - float(t["w_proj"][1, 3, 4])
+    got = (oracle.lookup_reduce(cfg, dict(t, w_proj=Wp), idx, w) * g).sum() - base
+    np.testing.assert_allclose(got, d * dwp[1, 3, 4], rtol=1e-9, atol=1e-15)
