@@ -52,6 +52,9 @@ def parse():
     ap.add_argument("--pkm", action="store_true",
                     help="the layer as a product-key memory: rank 1, additive grid scores, "
                          "softmax weights")
+    ap.add_argument("--backward", action="store_true",
+                    help="also time the lookup-reduce backward (dV, dw, dW_p) on the "
+                         "batch's slots")
     ap.add_argument("--recall", action="store_true",
                     help="also measure the two-phase search's recall@m against the "
                          "brute-force grid top-m, and the brute force's time")
@@ -249,6 +252,39 @@ def run_reference(args, cfg, B, wl):
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def measure_backward(layer, x, cfg, stream, K, flush):
+    """Device time of the lookup-reduce backward (dV accumulated, dw, dW_p)
+    on one batch's slots, K timed calls with the L2 flushed between them,
+    and the same without dW_p (whose forward re-gather and token-reduction
+    contraction are the training-only extra)."""
+    import torch
+    B = x.shape[0]
+    with torch.cuda.stream(stream):
+        _, idx, w = layer.forward(x, with_slots=True)
+        g = torch.randn((B, cfg["d_out"]), device="cuda").to(layer.dtype)
+        dv, _, _ = layer.lookup_reduce_backward(idx, w, g)
+
+        def timed(want_dwp):
+            ts = []
+            for i in range(K):
+                flush.fill_(float(i))
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                layer.lookup_reduce_backward(idx, w, g, dvalues=dv, want_dw_proj=want_dwp)
+                b.record(stream)
+                ts.append((a, b))
+            torch.cuda.synchronize()
+            return sum(a.elapsed_time(b) for a, b in ts) / K
+        full = timed(True)
+        rows_only = timed(False)
+    es = 4 if int(cfg["dtype"]) == 0 else 2
+    slots = B * cfg["heads"] * cfg["topm"]
+    # the rows kernel: value rows read (D_v es), dV rows read and written (fp32)
+    rows_bytes = slots * cfg["d_v"] * (es + 8)
+    return {"ms": full, "ms_without_dw_proj": rows_only, "slots": slots,
+            "rows_bytes": rows_bytes, "launches": layer.last_launches()}
 
 
 def measure_recall(layer, x, cfg, stream):
@@ -452,6 +488,9 @@ def main():
     recall = None
     if args.recall and rank == 0:
         recall = measure_recall(layer, xs[0], cfg, stream)
+    backward = None
+    if args.backward and rank == 0:
+        backward = measure_backward(layer, xs[0], cfg, stream, K, flush)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -470,6 +509,8 @@ def main():
                 "cpu_baseline": cpu, "clocks": clk}
         if recall is not None:
             line["recall"] = recall
+        if backward is not None:
+            line["backward"] = backward
         print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()

@@ -201,6 +201,24 @@ ultramem_status ultramem_retrieve_exact(ultramem_layer *layer, const void *x, in
 ultramem_status ultramem_lookup_reduce(ultramem_layer *layer, const int64_t *idx,
                                        const float *w, int32_t B, void *out, void *stream);
 
+/* The backward of the lookup-reduce (S7-S9; App. D's fused lookup-reduce
+ * operator) for the slots idx [B][H][m] int64 and weights w [B][H][m][h] fp32
+ * of a forward, given g = dL/dout [B][D'_v] (cfg.dtype), all DEVICE:
+ *   dvalues [N][D_v] fp32: += sum over slots of w_e (.) dacc_{p_e} at row_e,
+ *           dacc_p = W_p g (g itself without projectors); accumulated, so zero
+ *           it first for a fresh gradient; repeated rows add (fp32 atomics:
+ *           the summation order is not fixed)
+ *   dw      [B][H][m][h] fp32: dacc_{p_e} . V[row_e] over each value slice
+ *   dw_proj [E][D_v][D'_v] fp32: sum over tokens of acc_p g^T (written; ignored
+ *           without projectors)
+ * Any output may be NULL.  Out-of-range addresses are skipped (their dw is 0)
+ * and reported by ultramem_check.  ULTRAMEM_EINVAL when a value row is wider
+ * than 32 16-byte vectors.  Asynchronous on `stream`. */
+ultramem_status ultramem_lookup_reduce_backward(ultramem_layer *layer, const int64_t *idx,
+                                                const float *w, const void *g, int32_t B,
+                                                float *dvalues, float *dw, float *dw_proj,
+                                                void *stream);
+
 /* The lookup-reduce of ultramem_lookup_reduce (S7-S9) without a layer handle
  * and without allocating anything.  The paper has no counterpart: this entry
  * point exists for callers that cannot call cudaMalloc or create a layer -- a

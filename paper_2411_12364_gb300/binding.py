@@ -27,7 +27,7 @@ EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
            "ultramem_profile_read", "ultramem_stage_name", "ultramem_status_string",
            "ultramem_last_error", "ultramem_version", "ultramem_lookup_reduce_noalloc",
            "ultramem_last_launches", "ultramem_forward_seq", "ultramem_key_ln",
-           "ultramem_retrieve_exact")
+           "ultramem_retrieve_exact", "ultramem_lookup_reduce_backward")
 
 
 class Config(C.Structure):
@@ -84,6 +84,8 @@ def load(path: str | None = None) -> C.CDLL:
         lib.ultramem_retrieve.argtypes = [P, P, I32, P, P, P]
         lib.ultramem_retrieve_exact.argtypes = [P, P, I32, P, P, P]
         lib.ultramem_retrieve_exact.restype = I32
+        lib.ultramem_lookup_reduce_backward.argtypes = [P, P, P, P, I32, P, P, P, P]
+        lib.ultramem_lookup_reduce_backward.restype = I32
         lib.ultramem_retrieve.restype = I32
         lib.ultramem_lookup_reduce.argtypes = [P, P, P, I32, P, P]
         lib.ultramem_lookup_reduce.restype = I32
@@ -302,6 +304,28 @@ class UltraMemLayer:
                                                out.data_ptr(), _stream()),
                "ultramem_lookup_reduce")
         return out
+
+    def lookup_reduce_backward(self, idx: torch.Tensor, w: torch.Tensor, g: torch.Tensor,
+                               dvalues: torch.Tensor | None = None, want_dw=True,
+                               want_dw_proj=True):
+        """Backward of S7-S9: (dvalues [N, D_v] fp32, accumulated into the given
+        tensor or a new zero one; dw like w; dw_proj [E, D_v, D'_v] or None)."""
+        idx = idx.contiguous().to(torch.int64)
+        w = w.contiguous().to(torch.float32)
+        g = g.contiguous().to(self.dtype)
+        B = idx.shape[0]
+        c = self.cfg
+        N = int(c["n"]) ** 2
+        if dvalues is None:
+            dvalues = torch.zeros((N, int(c["d_v"])), dtype=torch.float32, device=idx.device)
+        dw = torch.empty_like(w) if want_dw else None
+        dwp = torch.empty((int(c["expand_e"]), int(c["d_v"]), int(c["d_out"])),
+                          dtype=torch.float32, device=idx.device) \
+            if want_dw_proj and int(c["has_proj"]) else None
+        _check(self.lib.ultramem_lookup_reduce_backward(
+            self._h, idx.data_ptr(), w.data_ptr(), g.data_ptr(), B, _ptr(dvalues), _ptr(dw),
+            _ptr(dwp), _stream()), "ultramem_lookup_reduce_backward")
+        return dvalues, dw, dwp
 
     def check(self) -> int:
         """Syncs the current stream and returns the device error status."""

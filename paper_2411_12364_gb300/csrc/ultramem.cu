@@ -27,6 +27,7 @@ struct Workspace {
     int *err = nullptr;
     void *x_stage = nullptr, *out_stage = nullptr;
     void *xs = nullptr;   // the convolved query input (Trick 4)
+    float *dacc = nullptr;   // backward: dL/dacc [B][E*D_v]
     __nv_bfloat16 *qs = nullptr, *acc_bf = nullptr, *w_pt = nullptr;   // tensor path
 };
 
@@ -45,6 +46,7 @@ struct ultramem_layer {
     cudaEvent_t ev[kStages + 1] = {};
     int launches = 0;    // kernels launched by the most recent successful call
     bool exact_ok = false;   // the brute-force top-m fits this layer's grid
+    bool backward_ok = false;   // the lookup-reduce backward fits this layer
 };
 
 namespace {
@@ -251,7 +253,7 @@ void free_workspace(Workspace &ws) {
     void *ptrs[] = {ws.q_part, ws.akey, ws.sel_w,   ws.acc,       ws.proj_part,
                     ws.sel_row, ws.sel_p, ws.core,   ws.u,         ws.t,
                     ws.err,    ws.x_stage, ws.out_stage, ws.qs,     ws.acc_bf,
-                    ws.w_pt,   ws.cores,   ws.xs};
+                    ws.w_pt,   ws.cores,   ws.xs,      ws.dacc};
     for (void *p : ptrs)
         if (p) cudaFree(p);
     ws = Workspace();
@@ -643,6 +645,9 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
         }
     }
     L->exact_ok = um::exact_fits(d);
+    L->backward_ok = um::backward_fits(d);
+    if (e == cudaSuccess && L->backward_ok) e = um::configure_backward(d);
+    if (e == cudaSuccess && L->backward_ok && cfg->has_proj) e = dalloc(&ws.dacc, Bm * d.E * d.d_v);
     if (e == cudaSuccess && L->exact_ok) e = um::configure_exact(d);
     if (e == cudaSuccess) e = um::configure_select(d);
     if (e == cudaSuccess) e = um::configure_gather(d);
@@ -760,6 +765,38 @@ ultramem_status ultramem_lookup_reduce(ultramem_layer *L, const int64_t *idx, co
     if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
     if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
     L->launches = 2 + (d.has_proj ? 2 : 0);
+    return ULTRAMEM_OK;
+}
+
+ultramem_status ultramem_lookup_reduce_backward(ultramem_layer *L, const int64_t *idx,
+                                                const float *w, const void *g, int32_t B,
+                                                float *dvalues, float *dw, float *dw_proj,
+                                                void *stream) {
+    if (!L || B < 0 || B > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (B == 0) return ULTRAMEM_OK;
+    if (!idx || !w || !g || !L->backward_ok) return ULTRAMEM_EINVAL;
+    Dims d = dims_for(L, B);
+    Ptrs p = make_ptrs(L);
+    p.idx_in = idx;
+    p.w_in = w;
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e;
+    cudaGetLastError();
+    int n = 0;
+    if (dw_proj && d.has_proj) {
+        // dW_p needs the forward's pooled rows: the forward's slots and gather
+        if ((e = um::launch_slots_from_addresses(d, p, st)) != cudaSuccess) return from_cuda(e);
+        if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
+        if ((e = um::launch_backward_proj(d, L->ws.acc, g, dw_proj, st)) != cudaSuccess)
+            return from_cuda(e);
+        n += 3;
+    }
+    if (dvalues || dw) {
+        if ((e = um::launch_backward_rows(d, p, g, L->ws.dacc, dvalues, dw, st)) != cudaSuccess)
+            return from_cuda(e);
+        n += d.has_proj ? 2 : 1;
+    }
+    L->launches = n;
     return ULTRAMEM_OK;
 }
 

@@ -126,6 +126,15 @@ cudaError_t configure_exact(const Dims &d);
 cudaError_t launch_exact(const Dims &d, const Ptrs &p, int64_t *idx_out, float *w_out,
                          cudaStream_t st);
 
+// The backward of the lookup-reduce (App. D): dacc = W_p g, then dV (+=) and
+// dw from the slots (p.idx_in, p.w_in); dW_p from the forward's pooled rows
+bool backward_fits(const Dims &d);
+cudaError_t configure_backward(const Dims &d);
+cudaError_t launch_backward_rows(const Dims &d, const Ptrs &p, const void *g, float *dacc,
+                                 float *dV, float *dw, cudaStream_t st);
+cudaError_t launch_backward_proj(const Dims &d, const float *acc, const void *g, float *dW,
+                                 cudaStream_t st);
+
 // kernel attributes for large dynamic shared memory, set at layer creation
 cudaError_t configure_select(const Dims &d);
 cudaError_t configure_gather(const Dims &d);
