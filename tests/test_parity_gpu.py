@@ -168,13 +168,18 @@ def test_library_svd_and_explicit_perm(gpu_lib):
 
 
 def test_workspace_reuse_across_batch_sizes(gpu_lib):
-    """One handle sized for 70 tokens serves smaller batches too."""
+    """One handle sized for 70 tokens serves smaller batches too: the same
+    slots, and the same outputs up to the query's summation order (70 tokens
+    take the tensor-core query, 64 and fewer the CUDA-core one)."""
     cfg = workloads.small_config(dtype=1)
     layer, (w, x, t), (out, idx, wt), _ = _run(cfg, 70, gpu_lib)
     for B in (1, 5, 32, 64):
         o2, i2, w2 = layer.forward(x[:B].contiguous(), with_slots=True)
         assert torch.equal(i2, idx[:B])
-        assert torch.equal(o2, out[:B])
+        torch.testing.assert_close(w2, wt[:B], rtol=1e-5, atol=1e-6)
+        ref = out[:B].float()
+        err = (o2.float() - ref).abs().amax(1) / ref.abs().amax(1)
+        assert err.max().item() <= 2 ** -7   # one bf16 rounding of the output
 
 
 def test_bad_address_is_reported_not_read(gpu_lib):
