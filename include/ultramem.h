@@ -171,9 +171,11 @@ ultramem_status ultramem_forward_seq(ultramem_layer *layer, const void *x, int32
                                      void *conv_state_out, void *out, int64_t *idx_out,
                                      float *w_out, void *stream);
 
-/* The same forward on HOST buffers: copies x to the device, runs the forward
- * and copies out back, all on `stream`, and returns after the stream has
- * finished.  Pinned host memory gives asynchronous copies; pageable works. */
+/* The same forward on HOST buffers: moves x to the device, runs the forward
+ * and moves out back, all on `stream`, and returns after the stream has
+ * finished.  Page-locked (pinned, mapped) buffers that are 16-byte aligned are
+ * moved by a copy kernel that reads and writes them over the host link;
+ * other host memory (pageable works) by the copy engines. */
 ultramem_status ultramem_forward_host(ultramem_layer *layer, const void *x_host, int32_t B,
                                       void *out_host, void *stream);
 

@@ -205,6 +205,12 @@ constexpr size_t kSmemReserved = 1024;    // the driver's reservation per CTA
 
 int device_sm_count();
 
+// Host buffers: the device address of mapped pinned memory (null otherwise),
+// and a 16-byte copy kernel (host link or device memory).
+const void *mapped_host(const void *p, size_t bytes);
+void *mapped_host(void *p, size_t bytes);
+cudaError_t launch_copy16(const void *src, void *dst, size_t bytes, cudaStream_t st);
+
 // Dynamic shared memory for a launch of `ctas` CTAs that need `need` bytes
 // each and have `static_bytes` of static shared memory.
 inline size_t spread_smem(size_t need, size_t static_bytes, int64_t ctas) {

@@ -146,8 +146,12 @@ def test_retrieve_and_host_forward_agree_with_forward(gpu_lib):
     assert torch.equal(i2, idx) and torch.equal(w2, wt)
     xh = x.cpu().pin_memory()
     oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
-    layer.forward_host(xh, oh)
+    layer.forward_host(xh, oh)              # pinned: copy kernels over the host link
     assert torch.equal(oh, out.cpu())
+    xp = x.cpu().clone()
+    op = torch.empty(out.shape, dtype=out.dtype)
+    layer.forward_host(xp, op)              # pageable: the copy engines
+    assert torch.equal(op, out.cpu())
 
 
 def test_forward_is_deterministic(gpu_lib):
