@@ -107,4 +107,22 @@ def test_null_handle_calls_are_rejected():
     assert lib.ultramem_forward(None, None, 1, None, None, None, None) == binding.EINVAL
     assert lib.ultramem_lookup_reduce(None, None, None, 1, None, None) == binding.EINVAL
     assert lib.ultramem_check(None, None) == binding.EINVAL
+    assert lib.ultramem_forward_seq(None, None, 1, 1, None, None, None, None, None,
+                                    None) == binding.EINVAL
+    assert lib.ultramem_retrieve_exact(None, None, 1, None, None, None) == binding.EINVAL
+    assert lib.ultramem_lookup_reduce_backward(None, None, None, None, 1, None, None, None,
+                                               None) == binding.EINVAL
+    assert lib.ultramem_last_launches(None) == 0
     lib.ultramem_destroy(None)
+
+
+def test_key_ln_rejects_invalid_arguments():
+    """Checked before anything is launched (no device needed)."""
+    lib = binding.load()
+    fake = 4096   # never dereferenced
+    assert lib.ultramem_key_ln(None, 1, 4, 8, fake, None, 1e-5, fake, None) == binding.EINVAL
+    assert lib.ultramem_key_ln(fake, 7, 4, 8, fake, None, 1e-5, fake, None) == binding.EINVAL
+    assert lib.ultramem_key_ln(fake, 1, 4, 0, fake, None, 1e-5, fake, None) == binding.EINVAL
+    assert lib.ultramem_key_ln(fake, 1, -1, 8, fake, None, 1e-5, fake, None) == binding.EINVAL
+    assert lib.ultramem_key_ln(fake, 1, 4, 8, fake, None, -1.0, fake, None) == binding.EINVAL
+    assert lib.ultramem_key_ln(fake, 1, 4, 8, None, None, 1e-5, fake, None) == binding.EINVAL
