@@ -28,6 +28,7 @@ struct Workspace {
     void *x_stage = nullptr, *out_stage = nullptr;
     void *xs = nullptr;   // the convolved query input (Trick 4)
     float *dacc = nullptr;   // backward: dL/dacc [B][E*D_v]
+    __nv_bfloat16 *bwd_t = nullptr;   // backward (tensor cores): acc^T [E*D_v][B], g^T [D'_v][B]
     __nv_bfloat16 *qs = nullptr, *acc_bf = nullptr, *w_pt = nullptr;   // tensor path
 };
 
@@ -62,6 +63,7 @@ struct ultramem_layer {
     int host_graph_next = 0;
     cudaStream_t capture = nullptr;
     bool x_after_copy = false;   // x is written by the copy kernel just before the forward
+    bool dacc_tc = false;        // the backward's dacc may run on the tensor cores
 };
 
 namespace {
@@ -268,7 +270,7 @@ void free_workspace(Workspace &ws) {
     void *ptrs[] = {ws.q_part, ws.akey, ws.sel_w,   ws.acc,       ws.proj_part,
                     ws.sel_row, ws.sel_p, ws.core,   ws.u,         ws.t,
                     ws.err,    ws.x_stage, ws.out_stage, ws.qs,     ws.acc_bf,
-                    ws.w_pt,   ws.cores,   ws.xs,      ws.dacc};
+                    ws.w_pt,   ws.cores,   ws.xs,      ws.dacc,    ws.bwd_t};
     for (void *p : ptrs)
         if (p) cudaFree(p);
     ws = Workspace();
@@ -586,7 +588,11 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     const size_t Bm = (size_t)cfg->max_tokens, HD = (size_t)H * cfg->d_k;
     size_t qmax = 0, pmax = 0;
     L->tc = tc_eligible(*cfg) && um::tc_init();
-    for (size_t B = 1; B <= Bm; B = (B < 256 ? B + 1 : B + 16)) {
+    // The split-K partial buffers hold splits(B) * B rows for every batch up
+    // to Bm.  splits(B) only falls as B grows and changes only at multiples
+    // of 16 tokens, so within a run of equal splits the product peaks at its
+    // last batch: every batch up to 256, then every 16th, then Bm itself.
+    auto visit = [&](size_t B) {
         size_t q = (size_t)query_splits(*cfg, (int)B) * B;
         size_t qt = (size_t)tc_query_splits(*cfg, (int)B) * B;
         size_t pp = (size_t)proj_splits(*cfg, (int)B) * B;
@@ -595,8 +601,10 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
         if (qt > qmax) qmax = qt;
         if (pp > pmax) pmax = pp;
         if (pt > pmax) pmax = pt;
-        if (B + 16 > Bm && B < Bm && B >= 256) B = Bm - 16;   // visit Bm itself
-    }
+    };
+    for (size_t B = 1; B <= Bm && B <= 256; ++B) visit(B);
+    for (size_t B = 272; B < Bm; B += 16) visit(B);
+    if (Bm > 256) visit(Bm);
     Workspace &ws = L->ws;
     cudaError_t e = cudaSuccess;
     const size_t hm = Bm * H * cfg->topm;
@@ -650,10 +658,14 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
                                  cfg->d_in, HD, 1, 128, 2);
         ok = ok && um::tc_encode(&L->maps.k_row, w->k_row, cfg->d_k, d.K, H, 128, 3);
         ok = ok && um::tc_encode(&L->maps.k_col, w->k_col, cfg->d_k, d.K, H, 128, 3);
-        if (cfg->has_proj)
+        if (cfg->has_proj) {
             ok = ok && um::tc_encode(&L->maps.w_pt, ws.w_pt, kd, cfg->d_out, 1, 128, 2);
-        else
+            // the projectors as stored, for the backward's dacc = W_p g (when
+            // D'_v rows are whole 16-byte vectors; else the CUDA-core path)
+            L->dacc_tc = um::tc_encode(&L->maps.w_p, w->w_proj, cfg->d_out, kd, 1, 128, 2);
+        } else {
             L->maps.w_pt = L->maps.w_q;
+        }
         if (e == cudaSuccess && !ok) {
             free_workspace(ws);
             delete L;
@@ -664,6 +676,8 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     L->backward_ok = um::backward_fits(d);
     if (e == cudaSuccess && L->backward_ok) e = um::configure_backward(d);
     if (e == cudaSuccess && L->backward_ok && cfg->has_proj) e = dalloc(&ws.dacc, Bm * d.E * d.d_v);
+    if (e == cudaSuccess && L->backward_ok && cfg->has_proj && L->tc)
+        e = dalloc(&ws.bwd_t, Bm * ((size_t)d.E * d.d_v + cfg->d_out));
     if (e == cudaSuccess && L->exact_ok) e = um::configure_exact(d);
     if (e == cudaSuccess) e = um::configure_select(d);
     if (e == cudaSuccess) e = um::configure_gather(d);
@@ -805,15 +819,53 @@ ultramem_status ultramem_lookup_reduce_backward(ultramem_layer *L, const int64_t
     if (dw_proj && d.has_proj) {
         // dW_p needs the forward's pooled rows: the forward's slots and gather
         if ((e = um::launch_slots_from_addresses(d, p, st)) != cudaSuccess) return from_cuda(e);
-        if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
-        if ((e = um::launch_backward_proj(d, L->ws.acc, g, dw_proj, st)) != cudaSuccess)
-            return from_cuda(e);
-        n += 3;
+        const int kd = d.E * d.d_v;
+        // tensor cores from 256 tokens on (below, the transposes and extra
+        // launches cost more than the CUDA-core contraction over few tokens,
+        // measured: 65 against 51 us at 64 tokens, 112 against 143 us at 256):
+        // the pooled rows in bf16 (as the forward's projection reads them) and
+        // both operands transposed to put the tokens on K
+        bool tc_dw = L->tc && L->ws.bwd_t && B >= 256 && B % 8 == 0 && L->cfg.d_out % 8 == 0;
+        CUtensorMap am, gm;
+        __nv_bfloat16 *acc_t = L->ws.bwd_t, *g_t = L->ws.bwd_t + (size_t)B * kd;
+        tc_dw = tc_dw && um::tc_encode(&am, acc_t, (uint64_t)B, (uint64_t)kd, 1, 128, 2) &&
+                um::tc_encode(&gm, g_t, (uint64_t)B, (uint64_t)L->cfg.d_out, 1,
+                              (uint32_t)um::tc_n_tile(L->cfg.d_out, 1), 2);
+        Ptrs pg = p;
+        if (tc_dw) pg.acc_bf = L->ws.acc_bf;
+        if ((e = um::launch_gather(d, pg, st)) != cudaSuccess) return from_cuda(e);
+        if (tc_dw) {
+            if ((e = um::launch_transpose_bf16(L->ws.acc_bf, acc_t, B, kd, st)) != cudaSuccess ||
+                (e = um::launch_transpose_bf16(g, g_t, B, L->cfg.d_out, st)) != cudaSuccess ||
+                (e = um::launch_dw_tc(d, am, gm, dw_proj, L->ws.err, st)) != cudaSuccess)
+                return from_cuda(e);
+            n += 5;
+        } else {
+            if ((e = um::launch_backward_proj(d, L->ws.acc, g, dw_proj, st)) != cudaSuccess)
+                return from_cuda(e);
+            n += 3;
+        }
     }
     if (dvalues || dw) {
-        if ((e = um::launch_backward_rows(d, p, g, L->ws.dacc, dvalues, dw, st)) != cudaSuccess)
+        // dacc = W_p g: on the tensor cores when the layer has its maps and g
+        // is 16-byte aligned, else the CUDA-core contraction
+        bool ready = false;
+        if (d.has_proj && L->tc && L->dacc_tc) {
+            um::TcMaps mp = L->maps;
+            CUtensorMap gm;
+            if (um::tc_encode(&gm, g, (uint64_t)d.d_out, (uint64_t)B, 1,
+                              (uint32_t)um::tc_n_tile(B, 1), 2)) {
+                if ((e = um::launch_dacc_tc(d, mp.w_p, gm, L->ws.dacc, L->ws.err, st)) !=
+                    cudaSuccess)
+                    return from_cuda(e);
+                ready = true;
+                ++n;
+            }
+        }
+        if ((e = um::launch_backward_rows(d, p, g, L->ws.dacc, ready, dvalues, dw, st)) !=
+            cudaSuccess)
             return from_cuda(e);
-        n += d.has_proj ? 2 : 1;
+        n += (d.has_proj && !ready) ? 2 : 1;
     }
     L->launches = n;
     return ULTRAMEM_OK;

@@ -192,9 +192,9 @@ cudaError_t configure_backward(const Dims &) { return cudaSuccess; }
 
 // dacc (with a projector) then dV and dw; g [B][D'_v] in the storage type.
 cudaError_t launch_backward_rows(const Dims &d, const Ptrs &p, const void *g, float *dacc,
-                                 float *dV, float *dw, cudaStream_t st) {
+                                 bool dacc_ready, float *dV, float *dw, cudaStream_t st) {
     const bool bf = d.dtype == ULTRAMEM_BF16;
-    if (d.has_proj) {
+    if (d.has_proj && !dacc_ready) {
         // slices of D'_v so that about two waves of CTAs run
         const int tiles = ((d.E * d.d_v + 63) / 64) * ((d.B + 31) / 32);
         int ks = (2 * device_sm_count() + tiles - 1) / tiles;

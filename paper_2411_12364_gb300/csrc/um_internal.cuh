@@ -80,6 +80,7 @@ struct TcMaps {
     CUtensorMap w_q, w_q_col, k_row, k_col, w_pt;
     CUtensorMap x, qs, acc;
     CUtensorMap xs;      // the convolved input's three bf16 terms [B][3 D_i]
+    CUtensorMap w_p;     // the projectors as stored, [E D_v][D'_v] (backward's A)
 };
 
 bool tc_init();
@@ -98,6 +99,13 @@ cudaError_t configure_small();
 cudaError_t launch_query_small(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, int Bmax,
                                bool x_f32, bool write_qs, bool pdl, cudaStream_t st);
 cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st);
+// the backward's dacc = W_p g on the tensor cores (g: map over [B][D'_v] bf16)
+cudaError_t launch_dacc_tc(const Dims &d, const CUtensorMap &w_p, const CUtensorMap &g,
+                           float *dacc, int *err, cudaStream_t st);
+// the backward's dW_p = sum_tokens acc g^T on the tensor cores, from the
+// transposed pooled rows [E D_v][B] and gradient rows [D'_v][B] (bf16)
+cudaError_t launch_dw_tc(const Dims &d, const CUtensorMap &acc_t, const CUtensorMap &g_t,
+                         float *dW, int *err, cudaStream_t st);
 cudaError_t launch_transpose_bf16(const void *src, void *dst, int rows, int cols,
                                   cudaStream_t st);
 
@@ -130,8 +138,9 @@ cudaError_t launch_exact(const Dims &d, const Ptrs &p, int64_t *idx_out, float *
 // dw from the slots (p.idx_in, p.w_in); dW_p from the forward's pooled rows
 bool backward_fits(const Dims &d);
 cudaError_t configure_backward(const Dims &d);
+// dacc_ready: dacc already holds W_p g (the tensor-core contraction ran)
 cudaError_t launch_backward_rows(const Dims &d, const Ptrs &p, const void *g, float *dacc,
-                                 float *dV, float *dw, cudaStream_t st);
+                                 bool dacc_ready, float *dV, float *dw, cudaStream_t st);
 cudaError_t launch_backward_proj(const Dims &d, const float *acc, const void *g, float *dW,
                                  cudaStream_t st);
 

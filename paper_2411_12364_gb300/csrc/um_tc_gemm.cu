@@ -626,6 +626,80 @@ struct ProjOp {
     }
 };
 
+// The backward's dacc = W_p g (the projectors as stored, [E D_v][D'_v], are
+// the K-major A operand; the gradient rows g [B][D'_v] the B operand): fp32
+// rows dacc[B][E D_v], unsplit.
+struct DaccOp {
+    int n_tile, stages, n_acc, acc_chunk, b_split_stride;
+    int *err;
+    int B, M, kb_total;
+    float *out;   // [B][M]
+    __device__ int cluster_splits() const { return 1; }
+    int cluster_splits_host() const { return 1; }
+    __device__ void store_partial(const Tile &, int, int, float (&)[kMaxAcc][16]) const {}
+    __device__ float load_partial(const Tile &, int, int, int) const { return 0.f; }
+    __device__ void store_sums(const Tile &, int, int, const float (&)[4]) const {}
+    __device__ Tile tile_at(int bx, int by, int) const {
+        Tile t;
+        t.m0 = bx * kTileM;
+        t.n0 = by * n_tile;
+        t.a_sel = 0;
+        t.a_z = -1;
+        t.b_z = -1;
+        t.z = 0;
+        t.kb0 = 0;
+        t.nkb = kb_total;
+        return t;
+    }
+    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
+        const int o = t.m0 + row;
+        if (o >= M) return;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int n = t.n0 + c + j;
+            if (n >= B) break;
+            out[(int64_t)n * M + o] = t.nkb ? v[0][j] : 0.f;
+        }
+    }
+};
+
+// The backward's dW_p = sum_tokens acc_p g^T: A = the pooled rows transposed
+// ([E D_v][B] bf16, K = tokens), B = the gradient rows transposed ([D'_v][B]);
+// fp32 dW [E D_v][D'_v] row-major, unsplit.
+struct DwOp {
+    int n_tile, stages, n_acc, acc_chunk, b_split_stride;
+    int *err;
+    int M, N, kb_total;
+    float *out;   // [M][N]
+    __device__ int cluster_splits() const { return 1; }
+    int cluster_splits_host() const { return 1; }
+    __device__ void store_partial(const Tile &, int, int, float (&)[kMaxAcc][16]) const {}
+    __device__ float load_partial(const Tile &, int, int, int) const { return 0.f; }
+    __device__ void store_sums(const Tile &, int, int, const float (&)[4]) const {}
+    __device__ Tile tile_at(int bx, int by, int) const {
+        Tile t;
+        t.m0 = bx * kTileM;
+        t.n0 = by * n_tile;
+        t.a_sel = 0;
+        t.a_z = -1;
+        t.b_z = -1;
+        t.z = 0;
+        t.kb0 = 0;
+        t.nkb = kb_total;
+        return t;
+    }
+    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
+        const int m = t.m0 + row;
+        if (m >= M) return;
+        float *dst = out + (int64_t)m * N;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int n = t.n0 + c + j;
+            if (n < N) dst[n] = t.nkb ? v[0][j] : 0.f;
+        }
+    }
+};
+
 // dst[c][r] = src[r][c] for a rows x cols bf16 matrix (32 x 32 tiles)
 __global__ void transpose_kernel(const __nv_bfloat16 *__restrict__ src,
                                  __nv_bfloat16 *__restrict__ dst, int rows, int cols) {
@@ -758,7 +832,41 @@ cudaError_t configure_tc() {
     if (e == cudaSuccess) e = allow_smem<3, QueryOp>();
     if (e == cudaSuccess) e = allow_smem<3, ScoreOp>();
     if (e == cudaSuccess) e = allow_smem<1, ProjOp>();
+    if (e == cudaSuccess) e = allow_smem<1, DaccOp>();
+    if (e == cudaSuccess) e = allow_smem<1, DwOp>();
     return e;
+}
+
+cudaError_t launch_dw_tc(const Dims &d, const CUtensorMap &acc_t, const CUtensorMap &g_t,
+                         float *dW, int *err, cudaStream_t st) {
+    DwOp op;
+    op.n_tile = tc_n_tile(d.d_out, 1);
+    op.n_acc = 1;
+    op.acc_chunk = 1 << 30;
+    op.b_split_stride = 0;
+    op.err = err;
+    op.M = d.E * d.d_v;
+    op.N = d.d_out;
+    op.kb_total = (d.B + kBlockK - 1) / kBlockK;
+    op.out = dW;
+    dim3 grid((op.M + kTileM - 1) / kTileM, (op.N + op.n_tile - 1) / op.n_tile, 1);
+    return launch_gemm<1>(grid, acc_t, acc_t, g_t, op, op.kb_total, false, st);
+}
+
+cudaError_t launch_dacc_tc(const Dims &d, const CUtensorMap &w_p, const CUtensorMap &g,
+                           float *dacc, int *err, cudaStream_t st) {
+    DaccOp op;
+    op.n_tile = tc_n_tile(d.B, 1);
+    op.n_acc = 1;
+    op.acc_chunk = 1 << 30;
+    op.b_split_stride = 0;
+    op.err = err;
+    op.B = d.B;
+    op.M = d.E * d.d_v;
+    op.kb_total = (d.d_out + kBlockK - 1) / kBlockK;
+    op.out = dacc;
+    dim3 grid((op.M + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 1);
+    return launch_gemm<1>(grid, w_p, w_p, g, op, op.kb_total, false, st);
 }
 
 // x_splits: the B operand is the convolved input as three bf16 terms (map
