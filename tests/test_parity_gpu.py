@@ -212,6 +212,26 @@ def test_batch_limits(gpu_lib):
         layer.forward(big)
 
 
+MAXIMA = [
+    # K = sqrt(16) * 5120 = 20480 keys per axis, k = 128, m = 1024 = the
+    # selection's limits (the final list overflows into the radix select),
+    # r = 8, E = 16 virtual blocks, 26 M physical rows
+    dict(dtype=1, d_in=64, d_k=64, heads=2, rank=8, n=5120, expand_e=16, d_v=16, d_out=32,
+         topk=128, topm=1024),
+    # the same limits with fp32 storage (CUDA-core path) and eight cores
+    dict(dtype=0, d_in=64, d_k=64, heads=1, rank=8, n=5120, expand_e=16, d_v=64, d_out=32,
+         topk=128, topm=1024, cores=8),
+]
+
+
+@pytest.mark.parametrize("case", range(len(MAXIMA)))
+def test_maximum_sizes(case, gpu_lib):
+    """The ABI's upper limits at once, on 6 tokens against the oracle."""
+    cfg = workloads.small_config(**MAXIMA[case])
+    assert workloads.keys_per_axis(cfg) == 20480
+    _run(cfg, 6, gpu_lib)
+
+
 def _tied_weights(cfg, rows_tied):
     """Weights whose first `rows_tied` keys of each axis are one and the same
     row, so that their rank-1 and exact scores tie exactly."""
