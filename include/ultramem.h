@@ -72,9 +72,9 @@ enum { ULTRAMEM_SCORE_TUCKER = 0, ULTRAMEM_SCORE_PKM = 1 };   /* grid score: Eq.
 
 /* Hyper-parameters of one layer, in the paper's notation. */
 typedef struct ultramem_config {
-    int32_t d_in;        /* D_i, width of x                                          */
-    int32_t d_k;         /* D_k, query/key width of one head; d_k % rank == 0        */
-    int32_t heads;       /* H, key sets that read the shared table (Sec. 3.1)        */
+    int32_t d_in;        /* D_i, width of x, <= 2^20                                 */
+    int32_t d_k;         /* D_k, query/key width of one head; d_k % rank == 0, <= 4096 */
+    int32_t heads;       /* H, key sets that read the shared table (Sec. 3.1), 1..64  */
     int32_t rank;        /* r, Tucker rank (Eq. 5), 1..8                              */
     int32_t n;           /* physical grid side, N = n*n rows; K = sqrt(E)*n <= 20480  */
     int32_t expand_e;    /* E, virtual expansion, a perfect square 1..16 (Eq. 13)    */

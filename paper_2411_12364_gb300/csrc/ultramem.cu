@@ -150,8 +150,10 @@ ultramem_status validate(const ultramem_config *c, const ultramem_weights *w) {
     if (c->query_ln && (!w->ln_g || c->d_k > 256 || !(c->ln_eps >= 0.f) ||
                         !(c->ln_eps < INFINITY)))
         return ULTRAMEM_EINVAL;
-    if (c->d_in <= 0 || c->d_k <= 0 || c->heads <= 0 || c->rank < 1 || c->rank > 8)
+    if (c->d_in <= 0 || c->d_k <= 0 || c->heads <= 0 || c->heads > 64 || c->rank < 1 ||
+        c->rank > 8)
         return ULTRAMEM_EINVAL;
+    if (c->d_k > 4096 || c->d_in > (1 << 20)) return ULTRAMEM_EINVAL;
     if (c->d_k % c->rank) return ULTRAMEM_EINVAL;
     if (c->n <= 0 || c->d_v <= 0 || c->d_v % 8) return ULTRAMEM_EINVAL;
     int s = (int)lround(sqrt((double)c->expand_e));

@@ -86,6 +86,7 @@ def _create(cfg_over=None, **w_over):
                                  dict(cores=2, act=1), dict(cores=3), dict(cores=16),
                                  dict(conv_k=2), dict(conv_k=-1), dict(query_ln=1),
                                  dict(query_ln=2), dict(score_mode=2), dict(score_mode=1),
+                                 dict(heads=65), dict(d_k=8192),
                                  dict(score_mode=1, rank=1, d_k=32, cores=2)])
 def test_create_rejects_invalid_configs(bad):
     st, h = _create(bad)
