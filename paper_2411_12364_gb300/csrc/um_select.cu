@@ -39,6 +39,9 @@ constexpr int kMaxM = 1024;
 static_assert(kMaxM <= kCap, "the final winners reuse a candidate list");
 constexpr int kMaxR = 8;
 constexpr int kRankSort = 256;             // longer lists are tightened first
+// value rows of a batch beyond this are not prefetched into L2 by the
+// selection: they would be evicted before the gather reads them
+constexpr uint64_t kPrefetchMaxBytes = 64ull << 20;
 constexpr unsigned kFull = 0xffffffffu;
 
 // counter slots of SelShared::cnt
@@ -243,41 +246,58 @@ __device__ __forceinline__ void warp_append(bool pr, u64 comp, u64 *list, int *c
     if (pr && slot < kCap) list[slot] = comp;
 }
 
-// Appends key[i] >= tau_s (i < n) of NS selections to their lists.  Each
-// warp handles 32-key batches in a strided share, 8 batches per round with
-// one atomic per selection and round.
+// Appends key[i] >= tau_s (i < n) of NS selections to their lists.  A round
+// covers 4 kThreads 16-byte groups of keys; lane l of warp w reads groups
+// (q kWarps + w) 32 + l, q < 4, so that a warp's loads are contiguous, and
+// marks its hits in a 16-bit mask.  A warp scan of the lanes' hit counts
+// places them, one shared atomic per warp and selection reserves the room,
+// and each lane writes its hits by walking its mask (re-reading a hit's key).
+// The last group may extend past n (up to the 16-byte end of the array's
+// section); its extra entries are masked.
 template <int NS>
 __device__ void compact(const uint32_t *key0, const uint32_t *key1, int n, uint32_t tau0,
                         uint32_t tau1, SelShared &sh, int slot0, int slot1) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    constexpr int kB = 8;
+    const int n4 = (n + 3) >> 2;
 #pragma unroll 1
-    for (int c0 = warp * 32 + lane; c0 - lane < n; c0 += kB * kThreads) {
+    for (int r0 = 0; r0 < n4; r0 += 4 * kThreads) {
 #pragma unroll
         for (int s = 0; s < NS; ++s) {
             const uint32_t *key = s ? key1 : key0;
+            const uint4 *k4 = reinterpret_cast<const uint4 *>(key);
             const uint32_t tau = s ? tau1 : tau0;
-            uint32_t v[kB];
-            unsigned bal[kB];
-            int tot = 0;
+            uint32_t mask = 0u;
 #pragma unroll
-            for (int u = 0; u < kB; ++u) {
-                const int i = c0 + u * kThreads;
-                v[u] = i < n ? key[i] : 0u;
-                bal[u] = __ballot_sync(kFull, i < n && v[u] >= tau);
-                tot += __popc(bal[u]);
+            for (int q = 0; q < 4; ++q) {
+                const int g = r0 + (q * kWarps + warp) * 32 + lane;
+                if (g < n4) {
+                    const uint4 v = k4[g];
+                    uint32_t m4 = (uint32_t)(v.x >= tau) | (uint32_t)(v.y >= tau) << 1 |
+                                  (uint32_t)(v.z >= tau) << 2 | (uint32_t)(v.w >= tau) << 3;
+                    const int valid = n - 4 * g;   // >= 1
+                    if (valid < 4) m4 &= (1u << valid) - 1u;
+                    mask |= m4 << (4 * q);
+                }
             }
-            if (tot == 0) continue;
-            int base = 0;
-            if (lane == 0) base = atomicAdd(&sh.cnt[s ? slot1 : slot0], tot);
-            base = __shfl_sync(kFull, base, 0);
-            u64 *list = sh.cand[s];
+            const int cnt = __popc(mask);
+            int incl = cnt;
 #pragma unroll
-            for (int u = 0; u < kB; ++u) {
-                const int slot = base + __popc(bal[u] & ((1u << lane) - 1u));
-                if (((bal[u] >> lane) & 1u) && slot < kCap)
-                    list[slot] = comp_of(v[u], (uint32_t)(c0 + u * kThreads));
-                base += __popc(bal[u]);
+            for (int off = 1; off < 32; off <<= 1) {
+                const int y = __shfl_up_sync(kFull, incl, off);
+                if (lane >= off) incl += y;
+            }
+            const int tot = __shfl_sync(kFull, incl, 31);
+            if (tot == 0) continue;   // warp-uniform
+            int base = 0;
+            if (lane == 31) base = atomicAdd(&sh.cnt[s ? slot1 : slot0], tot);
+            int slot = __shfl_sync(kFull, base, 31) + incl - cnt;
+            u64 *list = sh.cand[s];
+            while (mask) {
+                const int b = __ffs(mask) - 1;
+                mask &= mask - 1u;
+                const int i = 4 * (r0 + ((b >> 2) * kWarps + warp) * 32 + lane) + (b & 3);
+                if (slot < kCap) list[slot] = comp_of(key[i], (uint32_t)i);
+                ++slot;
             }
         }
     }
@@ -462,7 +482,9 @@ __device__ SelLayout carve(const Dims &d, unsigned char *base) {
 // Loads the rank-1 score keys of both axes (Eq. 6-7, written by the scoring
 // kernel) into shared memory and returns this thread's two largest of each
 // axis (padding reads as 0, below every key); all loads of a round are
-// issued before any store.
+// issued before any store.  Each key is read once: the loads are streaming
+// (L2 evict-first), so that a long batch's keys do not push the key rows,
+// which every (token, head) reads again, out of L2.
 __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1, int K,
                                           const SelLayout &L, uint32_t (&top)[2][2]) {
     uint32_t a1 = 0u, a2 = 0u, b1 = 0u, b2 = 0u;
@@ -477,8 +499,8 @@ __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int i = v0 + q * kThreads;
-                a[q] = i < nv ? V0[i] : make_uint4(0, 0, 0, 0);
-                c[q] = i < nv ? V1[i] : make_uint4(0, 0, 0, 0);
+                a[q] = i < nv ? __ldcs(V0 + i) : make_uint4(0, 0, 0, 0);
+                c[q] = i < nv ? __ldcs(V1 + i) : make_uint4(0, 0, 0, 0);
             }
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -504,8 +526,8 @@ __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int i = i0 + q * kThreads;
-                a[q] = i < K ? A0[i] : 0u;
-                c[q] = i < K ? A1[i] : 0u;
+                a[q] = i < K ? __ldcs(A0 + i) : 0u;
+                c[q] = i < K ? __ldcs(A1 + i) : 0u;
             }
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -523,6 +545,18 @@ __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1
     top[0][1] = a2;
     top[1][0] = b1;
     top[1][1] = b2;
+}
+
+// A 16-byte load of a key row with the L2 evict-last policy: the rows are
+// read again by the other (token, head) pairs of the batch.
+__device__ __forceinline__ uint4 ld_key_row(const uint4 *ptr) {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+    uint4 v;
+    asm volatile("ld.global.nc.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(ptr), "l"(pol));
+    return v;
 }
 
 // The 2k axis survivors, one group of G lanes each: the survivor's place in
@@ -550,6 +584,20 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
         pos = 0u;
     }
 
+    const T *row = static_cast<const T *>(s ? p.k_col : p.k_row) + ((int64_t)h * d.K + pos) * D;
+    const float *q = L.qv + s * D;
+    const bool vec = D % EPV == 0 && dk % EPV == 0 && ((uintptr_t)row & 15) == 0;
+    const uint4 *rv = reinterpret_cast<const uint4 *>(row);
+    const int nvec = vec ? D / EPV : 0;
+    // the first batch of the row's 16-byte loads is issued before the order
+    // scan below, which reads shared memory only
+    uint4 buf[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+        const int iv = sub + u * G;
+        buf[u] = active && iv < nvec ? ld_key_row(rv + iv) : make_uint4(0, 0, 0, 0);
+    }
+
     int ord = 0;
     if (active) {
         int g = sub;
@@ -562,26 +610,23 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
     }
     for (int off = G >> 1; off > 0; off >>= 1) ord += __shfl_xor_sync(kFull, ord, off);
 
-    const T *row = static_cast<const T *>(s ? p.k_col : p.k_row) + ((int64_t)h * d.K + pos) * D;
-    const float *q = L.qv + s * D;
     float S[RM];
 #pragma unroll
     for (int a = 0; a < RM; ++a) S[a] = 0.f;
-    const bool vec = D % EPV == 0 && dk % EPV == 0 && ((uintptr_t)row & 15) == 0;
     if (vec) {
-        // vector u of the row (EPV elements) belongs to chunk u*EPV / dk
-        const uint4 *rv = reinterpret_cast<const uint4 *>(row);
-        const int nvec = D / EPV;
-        // chunk of element x = floor(x / dk), as floor((x + 1/2) / dk) in fp32:
-        // exact while x, dk < 2^20 (the error stays below 1/(2 dk))
+        // 16-byte group iv of the row belongs to chunk iv / cpv
+        const int cpv = dk / EPV;
+        // (rank > 2) chunk of element x = floor(x / dk), as floor((x + 1/2) /
+        // dk) in fp32: exact while x, dk < 2^20 (the error stays below 1/(2 dk))
         const float inv_dk = 1.f / (float)dk;
 #pragma unroll 1
         for (int u0 = sub; u0 < nvec; u0 += 8 * G) {
-            uint4 buf[8];
+            if (u0 != sub) {
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                const int iv = u0 + u * G;
-                buf[u] = active && iv < nvec ? rv[iv] : make_uint4(0, 0, 0, 0);
+                for (int u = 0; u < 8; ++u) {
+                    const int iv = u0 + u * G;
+                    buf[u] = active && iv < nvec ? ld_key_row(rv + iv) : make_uint4(0, 0, 0, 0);
+                }
             }
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
@@ -600,10 +645,16 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
                         pv = fmaf(f[4 * e4 + 2], q4.z, pv);
                         pv = fmaf(f[4 * e4 + 3], q4.w, pv);
                     }
-                    const int al = (int)(((float)(iv * EPV) + 0.5f) * inv_dk);
+                    if (RM == 2) {   // rank 1 or 2: the second chunk starts at cpv
+                        const bool hi = iv >= cpv;
+                        S[0] += hi ? 0.f : pv;
+                        S[RM - 1] += hi ? pv : 0.f;
+                    } else {
+                        const int al = (int)(((float)(iv * EPV) + 0.5f) * inv_dk);
 #pragma unroll
-                    for (int a = 0; a < RM; ++a)
-                        if (a < r) S[a] += a == al ? pv : 0.f;   // r is uniform
+                        for (int a = 0; a < RM; ++a)
+                            if (a < r) S[a] += a == al ? pv : 0.f;   // r is uniform
+                    }
                 }
             }
         }
@@ -733,7 +784,17 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     // Eq. 10: g(i,j) = sum_b R[i][b] S_col[b,j] on I x J, R = S_row^T C
     const int k2 = k * k;
     uint32_t g1 = 0u, g2 = 0u;
-    {
+    if (!d.pkm && r == 2 && kThreads % k == 0) {   // uniform: a thread keeps one column jj
+        const int jj = threadIdx.x % k, dii = kThreads / k;
+        const float2 b2 = *reinterpret_cast<const float2 *>(L.scol + jj * 2);
+        int ii = threadIdx.x / k;
+        for (int c = threadIdx.x; c < k2; c += kThreads, ii += dii) {
+            const float2 a2 = *reinterpret_cast<const float2 *>(L.R + ii * 2);
+            const uint32_t kg = f2ord(fmaf(a2.y, b2.y, a2.x * b2.x));
+            L.key0[c] = kg;
+            top2(kg, g1, g2);
+        }
+    } else {
         const int dii = kThreads / k, djj = kThreads % k;   // (ii, jj) step per c += kThreads
         int ii = threadIdx.x / k, jj = threadIdx.x % k;
         for (int c = threadIdx.x; c < k2; c += kThreads) {
@@ -781,6 +842,7 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     const int64_t base = ((int64_t)b * d.H + h) * m;
     const uint32_t N = (uint32_t)d.N;
     const uint32_t row_bytes = (uint32_t)d.d_v * (d.dtype == ULTRAMEM_BF16 ? 2u : 4u);
+    const bool prefetch = (uint64_t)d.B * d.H * m * row_bytes <= kPrefetchMaxBytes;
     for (int e = threadIdx.x; e < m; e += kThreads) {
         const u64 wc = fwin[e];
         int c = (int)pos_of(wc);
@@ -795,9 +857,11 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
         const uint32_t vs = (uint32_t)shuffle_address(d, p.perm, v);   // Eq. 14, < M < 2^32
         const uint32_t pb = vs / N;
         const uint32_t prow = vs - pb * N;
-        // the gather will read this value row: start moving it into L2
-        prefetch_l2(static_cast<const unsigned char *>(p.values) + (size_t)prow * row_bytes,
-                    row_bytes);
+        // the gather will read this value row: start moving it into L2,
+        // unless the batch's rows would not stay there until then
+        if (prefetch)
+            prefetch_l2(static_cast<const unsigned char *>(p.values) + (size_t)prow * row_bytes,
+                        row_bytes);
         p.sel_row[base + e] = (int32_t)prow;
         p.sel_p[base + e] = (int32_t)pb;
         if (p.idx_out) p.idx_out[base + e] = (int64_t)v;

@@ -309,6 +309,8 @@ LONG_GRID = [
     dict(dtype=1, topk=24, topm=64),
     dict(dtype=1, topk=24, topm=64, cores=2),                # MCS
     dict(dtype=1, heads=4, topk=24, topm=160, cores=2),      # MCS, per-lane gather
+    dict(dtype=1, topk=32, topm=100),
+    dict(dtype=0, n=600, topk=100, topm=128),                # axis lists over 128: counted
 ]
 
 
@@ -316,7 +318,8 @@ LONG_GRID = [
 def test_long_grid_selection(over, gpu_lib):
     """Batches whose selection grid exceeds three CTAs per SM (here 300 tokens
     x H heads) take the long-grid selection, which ranks candidates by
-    sorted warp runs instead of counting; its lists here fill several runs."""
+    sorted warp runs instead of counting (longer lists are counted); its
+    lists here fill several runs."""
     cfg = workloads.small_config(**over)
     _run(cfg, 300, gpu_lib)
 
