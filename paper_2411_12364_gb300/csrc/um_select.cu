@@ -39,6 +39,9 @@ constexpr int kMaxM = 1024;
 static_assert(kMaxM <= kCap, "the final winners reuse a candidate list");
 constexpr int kMaxR = 8;
 constexpr int kRankSort = 256;             // longer lists are tightened first
+constexpr uint32_t kPairMix = 421;         // prime > kMaxK: the order of the Tucker pairs
+static_assert(kWarps == 8, "the Tucker pairs' assignment spreads rows over 8 warps");
+static_assert(kPairMix > kMaxK, "kPairMix must be coprime with every k^2");
 // value rows of a batch beyond this are not prefetched into L2 by the
 // selection: they would be evicted before the gather reads them
 constexpr uint64_t kPrefetchMaxBytes = 64ull << 20;
@@ -781,23 +784,43 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
 
     u64 *const fwin = sh.cand[1];   // final winners by rank (list 1 is free now)
 
-    // Eq. 10: g(i,j) = sum_b R[i][b] S_col[b,j] on I x J, R = S_row^T C
+    // Eq. 10: g(i,j) = sum_b R[i][b] S_col[b,j] on I x J, R = S_row^T C.
+    // Which thread computes which pair decides how tight the bound below is:
+    // it is the smallest of the 8 warps' values, so every warp should hold a
+    // spread sample of rows and columns.  In index order (pair c to thread
+    // c mod 256) a warp holds a few rows and half of the columns, and about
+    // twice as many candidates pass (final list at decode_1m, median over
+    // CTAs: 126 of 1024 for m = 32; 49 with a spread assignment).
     const int k2 = k * k;
     uint32_t g1 = 0u, g2 = 0u;
-    if (!d.pkm && r == 2 && kThreads % k == 0) {   // uniform: a thread keeps one column jj
-        const int jj = threadIdx.x % k, dii = kThreads / k;
-        const float2 b2 = *reinterpret_cast<const float2 *>(L.scol + jj * 2);
-        int ii = threadIdx.x / k;
-        for (int c = threadIdx.x; c < k2; c += kThreads, ii += dii) {
-            const float2 a2 = *reinterpret_cast<const float2 *>(L.R + ii * 2);
-            const uint32_t kg = f2ord(fmaf(a2.y, b2.y, a2.x * b2.x));
-            L.key0[c] = kg;
-            top2(kg, g1, g2);
+    if (!d.pkm && r == 2 && (k & 31) == 0) {   // uniform
+        // lane l of warp w owns columns l + 32 h (h < k/32; S_col in
+        // registers) and, of each, the rows ((w + l) mod 8) + 8 i (i < k/8):
+        // a warp holds every row and every column (8 warps, kThreads = 256)
+        const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+        const int i0 = (w + lane) & 7;
+        for (int jj = lane; jj < k; jj += 32) {
+            const float2 b2 = *reinterpret_cast<const float2 *>(L.scol + jj * 2);
+            for (int ii = i0; ii < k; ii += 8) {
+                const float2 a2 = *reinterpret_cast<const float2 *>(L.R + ii * 2);
+                const uint32_t kg = f2ord(fmaf(a2.y, b2.y, a2.x * b2.x));
+                L.key0[ii * k + jj] = kg;
+                top2(kg, g1, g2);
+            }
         }
     } else {
-        const int dii = kThreads / k, djj = kThreads % k;   // (ii, jj) step per c += kThreads
-        int ii = threadIdx.x / k, jj = threadIdx.x % k;
+        // any shape: thread t visits the pairs p = t, t + kThreads, ... as
+        // pair index pp = p kPairMix mod k^2 (a bijection: kPairMix is a
+        // prime above kMaxK)
+        const uint32_t uk2 = (uint32_t)k2;
+        const uint32_t step = (uint32_t)(((uint64_t)kThreads * kPairMix) % uk2);
+        uint32_t pp = (uint32_t)(((uint64_t)threadIdx.x * kPairMix) % uk2);
+        // ii = pp / k as floor((pp + 1/2) / k) in fp32: pp < 2^14 and k <= 128,
+        // so the rounding error (< 2^-16) stays below the 1/(2k) margin
+        const float inv_k = 1.f / (float)k;
         for (int c = threadIdx.x; c < k2; c += kThreads) {
+            const int ii = (int)(((float)pp + 0.5f) * inv_k);
+            const int jj = (int)pp - ii * k;
             float g;
             if (d.pkm) {    // product keys (Eq. 2): s_row[i] + s_col[j]
                 g = L.R[ii] + L.scol[jj];
@@ -810,11 +833,10 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
                 for (int be = 0; be < r; ++be) g = fmaf(L.R[ii * r + be], L.scol[jj * r + be], g);
             }
             const uint32_t kg = f2ord(g);
-            L.key0[c] = kg;
+            L.key0[pp] = kg;
             top2(kg, g1, g2);
-            ii += dii;
-            jj += djj;
-            if (jj >= k) { jj -= k; ++ii; }
+            pp += step;
+            if (pp >= uk2) pp -= uk2;
         }
     }
     warp_bounds(g1, g2, 0u, 0u, 1, m, sh);

@@ -60,6 +60,7 @@ SMALL = [
     dict(dtype=1, rank=1, score_mode=1),                  # product keys (Eq. 2), raw
     dict(dtype=0, rank=1, score_mode=1, act=1),           # PKM with its softmax (Eq. 3)
     dict(dtype=1, rank=1, score_mode=1, share_query=0, topk=16, topm=16),
+    dict(dtype=1, n=600, topk=128, topm=128),             # k = 128: four S_col columns a lane
 ]
 
 
@@ -311,6 +312,7 @@ LONG_GRID = [
     dict(dtype=1, heads=4, topk=24, topm=160, cores=2),      # MCS, per-lane gather
     dict(dtype=1, topk=32, topm=100),
     dict(dtype=0, n=600, topk=100, topm=128),                # axis lists over 128: counted
+    dict(dtype=1, n=600, topk=96, topm=64),                  # k = 96: three S_col columns a lane
 ]
 
 
