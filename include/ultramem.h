@@ -32,9 +32,9 @@
  * physical table is split, so Eq. 15 still holds per block).
  *
  * Shapes (all row-major and contiguous):
- *   K = sqrt(E) * n keys per axis ("the key size is expanded by sqrt(E) times",
- *   Sec. 3.2 IVE); N = n*n physical value rows; the virtual grid has K*K = E*N
- *   slots.  Heads share the value table and their pooled rows are summed.
+ *   K = sqrt(E) * n keys per axis (IVE grows each axis' key count by a factor
+ *   sqrt(E), Sec. 3.2); N = n*n physical value rows; the virtual grid has
+ *   K*K = E*N slots.  Heads share the value table and their pooled rows are summed.
  *
  * Conventions for every entry point:
  *   - Tensor pointers are DEVICE pointers unless a comment says HOST.  The

@@ -203,8 +203,8 @@ static uint64_t gcd_u64(uint64_t a, uint64_t b)
     return a;
 }
 
-/* The paper asks for "a random shuffle" of the E*N virtual addresses and
- * fixes nothing more.  Reading: pi(v) = (a*v + c) mod M with M = E*N, where
+/* The paper shuffles the E*N virtual addresses at random (Eq. 14) and fixes
+ * nothing more about the permutation.  Reading: pi(v) = (a*v + c) mod M with M = E*N, where
  * o1, o2 are the first two outputs of SplitMix64 seeded with `seed`:
  *   a = 1 + o1 mod (M-1), stepped up by one until gcd(a, M) = 1 (wrapping
  *       from M back to 1), which makes pi a bijection,
