@@ -17,14 +17,15 @@
 // lanes' 64 values (j = ceil(k / 8): j rounds of a warp max that removes one
 // instance) and tau is the smallest of the 8 warp values.  Every warp owns at
 // least j keys >= tau, so at least k keys are >= tau whatever the input:
-// every key of the top k is >= tau.  The keys >= tau are appended to one flat list per selection
-// (ballot, one shared atomic per warp).  When the list is long the same
-// bound is taken again over it; when it overflows (heavy ties) an exact radix
-// select replaces it.  Order: the candidates are 64-bit composites (key,
-// ~position) whose descending order is key descending then position
-// ascending; the rank of each is the number of candidates above it, counted
-// in parallel (a group of lanes per candidate), and the ones ranked below k
-// are the winners, in rank order.
+// every key of the top k is >= tau.  The keys >= tau are appended to one
+// flat list per selection (a hit mask per lane, a warp scan, one shared
+// atomic per warp).  When the list is long the same bound is taken again over
+// it; when it overflows (heavy ties) an exact radix select replaces it.
+// Order: the candidates are 64-bit composites (key, ~position) whose
+// descending order is key descending then position ascending; the rank of
+// each is the number of candidates above it (counted by a group of lanes per
+// candidate, or by binary searches in sorted warp runs on long grids), and the
+// ones ranked below k are the winners, in rank order.
 #include "um_internal.cuh"
 
 namespace um {
