@@ -23,7 +23,16 @@
  *  - Trick 2's query LayerNorm runs over each head's D_k query entries
  *    (population variance, epsilon inside the square root), after the
  *    projection and before the key scores; a separate column query has its
- *    own gain and bias.
+ *    own gain and bias;
+ *  - precision of the discrete decisions: every score is computed in fp64,
+ *    but each top-k / top-m orders the scores rounded to fp32 (the `key` of
+ *    `scored` below), with the value itself kept in fp64 for the weights.
+ *    The paper fixes no precision for these decisions; fp32 is the
+ *    precision the GPU kernels decide in, so a pair of scores that are
+ *    equal in fp32 is ordered by the tie rule on both sides instead of by a
+ *    difference below fp32 resolution that only the oracle sees.  Scores
+ *    closer than 1e-5 relative are treated as near-ties by the parity
+ *    tests, so this choice moves no test outcome outside that band.
  */
 #include "ultramem_oracle.h"
 

@@ -28,7 +28,8 @@ struct Workspace {
     void *x_stage = nullptr, *out_stage = nullptr;
     void *xs = nullptr;   // the convolved query input (Trick 4)
     float *dacc = nullptr;   // backward: dL/dacc [B][E*D_v]
-    __nv_bfloat16 *bwd_t = nullptr;   // backward (tensor cores): acc^T [E*D_v][B], g^T [D'_v][B]
+    __nv_bfloat16 *bwd_t = nullptr;   // backward (tensor cores): acc^T [E*D_v][2 B] (two
+                                      // bf16 terms), g^T [D'_v][B]
     __nv_bfloat16 *qs = nullptr, *acc_bf = nullptr, *w_pt = nullptr;   // tensor path
 };
 
@@ -398,10 +399,12 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
         return ULTRAMEM_ECUDA;
     if (!um::tc_encode(&mp.qs, L->ws.qs, 3ull * c.d_k, (uint64_t)Bmax, 2ull * d.H,
                        (uint32_t)nt1, 3) ||
-        !um::tc_encode(&mp.acc, L->ws.acc_bf, (uint64_t)d.E * d.d_v, (uint64_t)Bmax, 1,
+        !um::tc_encode(&mp.acc, L->ws.acc_bf, 2ull * d.E * d.d_v, (uint64_t)Bmax, 1,
                        (uint32_t)nt1, 2))
         return ULTRAMEM_ECUDA;
+    // the projection reads the pooled rows as two bf16 terms hi + lo
     p.acc_bf = c.has_proj ? L->ws.acc_bf : nullptr;
+    p.acc_terms = 2;
     cudaError_t e;
     mark(L, 0, st);
     // Every kernel after the first is a programmatic dependent launch of its
@@ -644,8 +647,8 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
         // tensor path: split queries, bf16 acc, K-major copy of the projectors
         e = dalloc(&ws.qs, (size_t)2 * H * Bm * 3 * cfg->d_k);
         if (e == cudaSuccess) e = cudaMemset(ws.qs, 0, sizeof(__nv_bfloat16) * 2 * H * Bm * 3 * cfg->d_k);
-        if (e == cudaSuccess) e = dalloc(&ws.acc_bf, Bm * kd);
-        if (e == cudaSuccess) e = cudaMemset(ws.acc_bf, 0, sizeof(__nv_bfloat16) * Bm * kd);
+        if (e == cudaSuccess) e = dalloc(&ws.acc_bf, 2 * Bm * kd);   // hi, lo terms
+        if (e == cudaSuccess) e = cudaMemset(ws.acc_bf, 0, sizeof(__nv_bfloat16) * 2 * Bm * kd);
         if (e == cudaSuccess && cfg->has_proj) {
             e = dalloc(&ws.w_pt, kd * cfg->d_out);
             if (e == cudaSuccess) e = um::launch_transpose_bf16(w->w_proj, ws.w_pt, (int)kd, cfg->d_out, 0);
@@ -679,7 +682,7 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     if (e == cudaSuccess && L->backward_ok) e = um::configure_backward(d);
     if (e == cudaSuccess && L->backward_ok && cfg->has_proj) e = dalloc(&ws.dacc, Bm * d.E * d.d_v);
     if (e == cudaSuccess && L->backward_ok && cfg->has_proj && L->tc)
-        e = dalloc(&ws.bwd_t, Bm * ((size_t)d.E * d.d_v + cfg->d_out));
+        e = dalloc(&ws.bwd_t, Bm * (2 * (size_t)d.E * d.d_v + cfg->d_out));
     if (e == cudaSuccess && L->exact_ok) e = um::configure_exact(d);
     if (e == cudaSuccess) e = um::configure_select(d);
     if (e == cudaSuccess) e = um::configure_gather(d);
@@ -825,23 +828,31 @@ ultramem_status ultramem_lookup_reduce_backward(ultramem_layer *L, const int64_t
         // tensor cores from 256 tokens on (below, the transposes and extra
         // launches cost more than the CUDA-core contraction over few tokens,
         // measured: 65 against 51 us at 64 tokens, 112 against 143 us at 256):
-        // the pooled rows in bf16 (as the forward's projection reads them) and
-        // both operands transposed to put the tokens on K
+        // the pooled rows as two bf16 terms (as the forward's projection reads
+        // them), both operands transposed to put the tokens on K
         bool tc_dw = L->tc && L->ws.bwd_t && B >= 256 && B % 8 == 0 && L->cfg.d_out % 8 == 0;
         CUtensorMap am, gm;
-        __nv_bfloat16 *acc_t = L->ws.bwd_t, *g_t = L->ws.bwd_t + (size_t)B * kd;
-        tc_dw = tc_dw && um::tc_encode(&am, acc_t, (uint64_t)B, (uint64_t)kd, 1, 128, 2) &&
-                um::tc_encode(&gm, g_t, (uint64_t)B, (uint64_t)L->cfg.d_out, 1,
-                              (uint32_t)um::tc_n_tile(L->cfg.d_out, 1), 2);
+        // acc_t2 [E D_v][2 B] (hi terms in columns [0, B), lo in [B, 2 B)), g_t [D'_v][B]
+        __nv_bfloat16 *acc_t2 = L->ws.bwd_t, *g_t = L->ws.bwd_t + (size_t)2 * B * kd;
+        tc_dw = tc_dw &&
+                um::tc_encode(&am, acc_t2, 2ull * B, (uint64_t)kd, 1,
+                              (uint32_t)um::tc_n_tile(kd, 1), 2) &&
+                um::tc_encode(&gm, g_t, (uint64_t)B, (uint64_t)L->cfg.d_out, 1, 128, 2);
         Ptrs pg = p;
-        if (tc_dw) pg.acc_bf = L->ws.acc_bf;
+        if (tc_dw) {
+            pg.acc_bf = L->ws.acc_bf;   // [B][2][E D_v]
+            pg.acc_terms = 2;
+        }
         if ((e = um::launch_gather(d, pg, st)) != cudaSuccess) return from_cuda(e);
         if (tc_dw) {
-            if ((e = um::launch_transpose_bf16(L->ws.acc_bf, acc_t, B, kd, st)) != cudaSuccess ||
-                (e = um::launch_transpose_bf16(g, g_t, B, L->cfg.d_out, st)) != cudaSuccess ||
-                (e = um::launch_dw_tc(d, am, gm, dw_proj, L->ws.err, st)) != cudaSuccess)
+            for (int j = 0; j < 2; ++j)
+                if ((e = um::launch_transpose_bf16(L->ws.acc_bf + (size_t)j * kd, acc_t2 + (size_t)j * B,
+                                                   B, kd, st, 2 * kd, 2 * B)) != cudaSuccess)
+                    return from_cuda(e);
+            if ((e = um::launch_transpose_bf16(g, g_t, B, L->cfg.d_out, st)) != cudaSuccess ||
+                (e = um::launch_dw_tc(d, gm, am, dw_proj, L->ws.err, st)) != cudaSuccess)
                 return from_cuda(e);
-            n += 5;
+            n += 6;
         } else {
             if ((e = um::launch_backward_proj(d, L->ws.acc, g, dw_proj, st)) != cudaSuccess)
                 return from_cuda(e);

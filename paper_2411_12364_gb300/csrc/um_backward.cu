@@ -9,7 +9,9 @@
 // forward gather (one more read of the selected rows).  dV is accumulated
 // with fp32 vector atomics (rows repeat across tokens and heads; their
 // summation order is not fixed), and so is dacc over its split-K slices.
-// dacc and dW_p are CUDA-core tiled contractions.
+// dacc and dW_p are CUDA-core tiled contractions; with fp32 storage they
+// are compensated dot products (Dot2) and dacc is unsplit, so that the
+// fp32 mode's gradients carry the working precision.
 #include "um_internal.cuh"
 
 namespace um {
@@ -33,7 +35,10 @@ __global__ void __launch_bounds__(kThreads) dacc_kernel(Dims d, const T *g, cons
     __shared__ float gs[32][33];   // [o][token]
     __shared__ float wsm[32][65];  // [o][row c]
     const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+    // fp32 storage: compensated sums (Dot2) over the whole of D'_v (one slice)
+    constexpr bool kExact = std::is_same<T, float>::value;
     float acc[2][4] = {};
+    Dot2 ex[kExact ? 2 : 1][kExact ? 4 : 1];
     for (int k0 = kb; k0 < Kd; k0 += 32) {
         for (int e = tid; e < 32 * 32; e += kThreads) {
             const int bb = e / 32, kk = e % 32, b = b0 + bb, k = k0 + kk;
@@ -50,8 +55,13 @@ __global__ void __launch_bounds__(kThreads) dacc_kernel(Dims d, const T *g, cons
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const float wv = wsm[kk][tx * 4 + j];
-                acc[0][j] = fmaf(g0, wv, acc[0][j]);
-                acc[1][j] = fmaf(g1, wv, acc[1][j]);
+                if constexpr (kExact) {
+                    ex[0][j].add(g0, wv);
+                    ex[1][j].add(g1, wv);
+                } else {
+                    acc[0][j] = fmaf(g0, wv, acc[0][j]);
+                    acc[1][j] = fmaf(g1, wv, acc[1][j]);
+                }
             }
         }
         __syncthreads();
@@ -59,7 +69,9 @@ __global__ void __launch_bounds__(kThreads) dacc_kernel(Dims d, const T *g, cons
     for (int i = 0; i < 2; ++i)
         for (int j = 0; j < 4; ++j) {
             const int b = b0 + ty * 2 + i, c = c0 + tx * 4 + j;
-            if (b < d.B && c < Mc) atomicAdd(&dacc[(int64_t)b * Mc + c], acc[i][j]);
+            if (b >= d.B || c >= Mc) continue;
+            if constexpr (kExact) dacc[(int64_t)b * Mc + c] = ex[i][j].value();   // one slice
+            else atomicAdd(&dacc[(int64_t)b * Mc + c], acc[i][j]);
         }
 }
 
@@ -73,7 +85,9 @@ __global__ void __launch_bounds__(kThreads) dwp_kernel(Dims d, const float *acc,
     __shared__ float as[32][65];   // [token][c]
     __shared__ float gsm[32][65];  // [token][o]
     const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+    constexpr bool kExact = std::is_same<T, float>::value;   // fp32 storage: Dot2
     float r[4][4] = {};
+    Dot2 ex[kExact ? 4 : 1][kExact ? 4 : 1];
     for (int b0 = 0; b0 < d.B; b0 += 32) {
         for (int e = tid; e < 32 * 64; e += kThreads) {
             const int bb = e / 64, cc = e % 64, b = b0 + bb;
@@ -92,14 +106,19 @@ __global__ void __launch_bounds__(kThreads) dwp_kernel(Dims d, const float *acc,
 #pragma unroll
             for (int i = 0; i < 4; ++i)
 #pragma unroll
-                for (int j = 0; j < 4; ++j) r[i][j] = fmaf(a[i], q[j], r[i][j]);
+                for (int j = 0; j < 4; ++j) {
+                    if constexpr (kExact) ex[i][j].add(a[i], q[j]);
+                    else r[i][j] = fmaf(a[i], q[j], r[i][j]);
+                }
         }
         __syncthreads();
     }
     for (int i = 0; i < 4; ++i)
         for (int j = 0; j < 4; ++j) {
             const int c = c0 + ty * 4 + i, o = o0 + tx * 4 + j;
-            if (c < Mc && o < No) dW[(int64_t)c * No + o] = r[i][j];
+            float v = r[i][j];
+            if constexpr (kExact) v = ex[i][j].value();
+            if (c < Mc && o < No) dW[(int64_t)c * No + o] = v;
         }
 }
 
@@ -142,7 +161,9 @@ __global__ void __launch_bounds__(kThreads) rows_kernel(Dims d, Ptrs p, const vo
     const int pb = (int)(vs / (uint64_t)d.N);
     const int64_t row = (int64_t)(vs - (uint64_t)pb * (uint64_t)d.N);
     const float we = p.w_in[slot * nc + wsel];
-    float part = 0.f;
+    // the slice dot products: fp64 for fp32 storage (one rounding of dw)
+    using A = typename std::conditional<std::is_same<T, float>::value, double, float>::type;
+    A part = 0;
     if (active) {
         float f[8], dac[8];
         unpack16(*reinterpret_cast<const uint4 *>(static_cast<const T *>(p.values) + row * Dv +
@@ -161,7 +182,7 @@ __global__ void __launch_bounds__(kThreads) rows_kernel(Dims d, Ptrs p, const vo
                      T());
         }
 #pragma unroll
-        for (int c = 0; c < EPV; ++c) part = fmaf(dac[c], f[c], part);
+        for (int c = 0; c < EPV; ++c) part += (A)dac[c] * (A)f[c];
         if (dV) {
             float *dst = dV + row * Dv + lane * EPV;
 #pragma unroll
@@ -174,10 +195,10 @@ __global__ void __launch_bounds__(kThreads) rows_kernel(Dims d, Ptrs p, const vo
     // dw: the sum of the slice's lanes (nc <= 8 warp sums, fixed order)
     if (dw)
         for (int i = 0; i < nc; ++i) {
-            float sv = wsel == i && active ? part : 0.f;
+            A sv = wsel == i && active ? part : (A)0;
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) sv += __shfl_xor_sync(kFull, sv, off);
-            if (lane == 0) dw[slot * nc + i] = sv;
+            if (lane == 0) dw[slot * nc + i] = (float)sv;
         }
 }
 
@@ -199,6 +220,7 @@ cudaError_t launch_backward_rows(const Dims &d, const Ptrs &p, const void *g, fl
         const int tiles = ((d.E * d.d_v + 63) / 64) * ((d.B + 31) / 32);
         int ks = (2 * device_sm_count() + tiles - 1) / tiles;
         ks = max(1, min(ks, (d.d_out + 127) / 128));
+        if (!bf) ks = 1;   // fp32 storage: one compensated sum, stored (no atomics)
         dim3 grid((d.E * d.d_v + 63) / 64, (d.B + 31) / 32, ks);
         cudaError_t z = cudaMemsetAsync(dacc, 0, sizeof(float) * d.B * d.E * d.d_v, st);
         if (z != cudaSuccess) return z;

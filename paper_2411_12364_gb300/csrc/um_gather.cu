@@ -1,6 +1,6 @@
 // um_gather.cu -- S8 (weighted gather-sum grouped by virtual block, Eq. 15's
 // inner V^T s^_p) and S9 on CUDA cores (the IVE projection o = sum_p W_p^T
-// acc_p, used for fp32 storage).
+// acc_p, used for fp32 storage; there with compensated sums, Dot2).
 //
 // Gather, one CTA per token.  Random 512-byte rows of a multi-GB table reach
 // the HBM copy rate only with many rows in flight per SM (measured on GB300:
@@ -14,6 +14,11 @@
 //     fixed order at the end (deterministic).
 // Wider rows or more slots take the per-lane multi-block kernels below.  Row
 // loads bypass L1 (read-only path).
+//
+// fp32 storage accumulates in fp64 (products of two fp32 values are exact
+// there): the fp32 mode's outputs carry the working precision element by
+// element (see Dot2 in um_internal.cuh), and its projection reads fp32
+// pooled rows that are rounded once.
 //
 // Multi-Core Scoring (Eq. 17): a slot has nc weights and weight i scales
 // columns [i*D_v/nc, (i+1)*D_v/nc) of the row.  Slices are whole 16-byte
@@ -36,21 +41,32 @@ __device__ __forceinline__ uint4 ld_stream(const void *ptr) {
     return v;
 }
 
+// The accumulator type of a gather: fp64 for fp32 storage, else fp32.
+template <typename T>
+using AccOf = typename std::conditional<std::is_same<T, float>::value, double, float>::type;
+
+__device__ __forceinline__ float mul_add(float w, float v, float acc) { return fmaf(w, v, acc); }
+__device__ __forceinline__ double mul_add(float w, float v, double acc) {
+    return fma((double)w, (double)v, acc);
+}
+
 // add w * (8 bf16 or 4 fp32 packed in 16 bytes) into dst
-__device__ __forceinline__ void fma_vec(float *dst, uint4 v, float w, __nv_bfloat16) {
+template <typename A>
+__device__ __forceinline__ void fma_vec(A *dst, uint4 v, float w, __nv_bfloat16) {
     const uint32_t u[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
         float lo = __uint_as_float(u[q] << 16), hi = __uint_as_float(u[q] & 0xffff0000u);
-        dst[2 * q] = fmaf(w, lo, dst[2 * q]);
-        dst[2 * q + 1] = fmaf(w, hi, dst[2 * q + 1]);
+        dst[2 * q] = mul_add(w, lo, dst[2 * q]);
+        dst[2 * q + 1] = mul_add(w, hi, dst[2 * q + 1]);
     }
 }
-__device__ __forceinline__ void fma_vec(float *dst, uint4 v, float w, float) {
-    dst[0] = fmaf(w, __uint_as_float(v.x), dst[0]);
-    dst[1] = fmaf(w, __uint_as_float(v.y), dst[1]);
-    dst[2] = fmaf(w, __uint_as_float(v.z), dst[2]);
-    dst[3] = fmaf(w, __uint_as_float(v.w), dst[3]);
+template <typename A>
+__device__ __forceinline__ void fma_vec(A *dst, uint4 v, float w, float) {
+    dst[0] = mul_add(w, __uint_as_float(v.x), dst[0]);
+    dst[1] = mul_add(w, __uint_as_float(v.y), dst[1]);
+    dst[2] = mul_add(w, __uint_as_float(v.z), dst[2]);
+    dst[3] = mul_add(w, __uint_as_float(v.w), dst[3]);
 }
 
 template <typename T>
@@ -79,7 +95,9 @@ __device__ __forceinline__ void unpack<float>(uint4 v, float (&f)[4]) {
 // in flight together.
 template <typename T, int EMAX>
 __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
-    extern __shared__ __align__(16) float red[];   // [kWarps][E][D_v]
+    using A = AccOf<T>;
+    extern __shared__ __align__(16) unsigned char red_raw[];
+    A *red = reinterpret_cast<A *>(red_raw);   // [kWarps][E][D_v]
     constexpr int EPV = 16 / sizeof(T);
     const int b = blockIdx.x;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -93,11 +111,11 @@ __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
     const int e_begin = min(hm, warp * per_warp), e_end = min(hm, e_begin + per_warp);
     pdl_wait();
     pdl_trigger();
-    float acc[EMAX][EPV];
+    A acc[EMAX][EPV];
 #pragma unroll
     for (int q = 0; q < EMAX; ++q)
 #pragma unroll
-        for (int c = 0; c < EPV; ++c) acc[q][c] = 0.f;
+        for (int c = 0; c < EPV; ++c) acc[q][c] = 0;
 
     for (int c0 = e_begin; c0 < e_end; c0 += 32) {
         const int n = min(32, e_end - c0);
@@ -128,7 +146,7 @@ __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
                 for (int q = 0; q < EMAX; ++q) {
                     const float wq = blk == q ? w : 0.f;   // branch-free block select
 #pragma unroll
-                    for (int c = 0; c < EPV; ++c) acc[q][c] = fmaf(wq, f[c], acc[q][c]);
+                    for (int c = 0; c < EPV; ++c) acc[q][c] = mul_add(wq, f[c], acc[q][c]);
                 }
             }
         }
@@ -143,25 +161,23 @@ __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
                     red[(size_t)warp * EDv + q * d.d_v + lane * EPV + c] = acc[q][c];
     __syncthreads();
     for (int i = threadIdx.x; i < EDv; i += kThreads) {
-        float s = 0.f;
+        A s = 0;
 #pragma unroll
         for (int wv = 0; wv < kWarps; ++wv) s += red[(size_t)wv * EDv + i];
-        if (p.acc_bf)
-            p.acc_bf[(int64_t)b * EDv + i] = __float2bfloat16_rn(s);
-        else if (d.has_proj)
-            p.acc[(int64_t)b * EDv + i] = s;
-        else
-            static_cast<T *>(p.out)[(int64_t)b * d.d_v + i] = from_f<T>(s);
+        store_pooled<T>(d, p, b, i, (float)s);
     }
 }
 
 constexpr int kBMaxE = 16;
 constexpr int kMaxCores = 8;   // MCS component cores per head
 
+// bytes of one accumulator of the layer's gather (fp64 for fp32 storage)
+size_t acc_bytes(const Dims &d) { return d.dtype == ULTRAMEM_F32 ? 8 : 4; }
+
 size_t bucket_smem_bytes(const Dims &d, int warps) {
     const int hm = d.H * d.m;
-    return sizeof(int) * (size_t)hm + sizeof(float) * (size_t)hm * d.nc +
-           sizeof(float) * (size_t)warps * d.d_v;
+    return acc_bytes(d) * (size_t)warps * d.d_v + sizeof(int) * (size_t)hm +
+           sizeof(float) * (size_t)hm * d.nc;
 }
 
 // THREADS = 512 (2 CTAs per SM) for batches up to about two CTAs per SM,
@@ -176,10 +192,11 @@ __global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(
     __shared__ int wcnt[kBWarps][kBMaxE];   // per warp and block: count, then offset
     __shared__ int tot[kBMaxE], start[kBMaxE];
     constexpr int EPV = 16 / sizeof(T);
+    using A = AccOf<T>;
     const int b = blockIdx.x, E = d.E, hm = d.H * d.m, Dv = d.d_v;
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
     const int64_t base = (int64_t)b * hm;
-    float *red = reinterpret_cast<float *>(gsm);                 // [kBWarps][D_v]
+    A *red = reinterpret_cast<A *>(gsm);                         // [kBWarps][D_v]
     int *row_s = reinterpret_cast<int *>(red + kBWarps * Dv);    // [hm] bucketed rows
     float *w_s = reinterpret_cast<float *>(row_s + hm);          // [hm][nc] their weights
     const int nc = d.nc;
@@ -239,9 +256,9 @@ __global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(
     const bool active = lane * EPV < Dv;
     const int wsel = nc == 1 || !active ? 0 : (lane * EPV) / (Dv / nc);   // this lane's slice
     const T *V = static_cast<const T *>(p.values) + lane * EPV;
-    float acc[EPV];
+    A acc[EPV];
 #pragma unroll
-    for (int c = 0; c < EPV; ++c) acc[c] = 0.f;
+    for (int c = 0; c < EPV; ++c) acc[c] = 0;
     if (q < E) {
         const int n = tot[q], per = (n + wpb - 1) / wpb;
         const int lo = start[q] + min(n, sub * per), hi = start[q] + min(n, (sub + 1) * per);
@@ -261,7 +278,7 @@ __global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(
                 float f[EPV];
                 unpack<T>(val[u], f);
 #pragma unroll
-                for (int c = 0; c < EPV; ++c) acc[c] = fmaf(wu[u], f[c], acc[c]);
+                for (int c = 0; c < EPV; ++c) acc[c] = mul_add(wu[u], f[c], acc[c]);
             }
         }
         if (active)
@@ -272,28 +289,25 @@ __global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(
     const int EDv = E * Dv;
     for (int i = t; i < EDv; i += kBThreads) {
         const int qq = i / Dv, c = i - qq * Dv;
-        float sum = 0.f;
+        A sum = 0;
         for (int sb = 0; sb < wpb; ++sb) sum += red[(qq * wpb + sb) * Dv + c];
-        if (p.acc_bf)
-            p.acc_bf[(int64_t)b * EDv + i] = __float2bfloat16_rn(sum);
-        else if (d.has_proj)
-            p.acc[(int64_t)b * EDv + i] = sum;
-        else
-            static_cast<T *>(p.out)[(int64_t)b * Dv + i] = from_f<T>(sum);
+        store_pooled<T>(d, p, b, i, (float)sum);
     }
 }
 
-// Shared-memory-accumulating gather for any E and row width.
-template <typename T>
+// Shared-memory-accumulating gather for any E and row width (A: the
+// accumulator, fp64 for fp32 storage while [kWarps][E][D_v] of it fits).
+template <typename T, typename A>
 __global__ void __launch_bounds__(kThreads) gather_kernel(Dims d, Ptrs p) {
-    extern __shared__ __align__(16) float acc_w[];   // [kWarps][E][D_v]
+    extern __shared__ __align__(16) unsigned char acc_raw[];
+    A *acc_w = reinterpret_cast<A *>(acc_raw);   // [kWarps][E][D_v]
     const int b = blockIdx.x;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int EDv = d.E * d.d_v;
     pdl_wait();
     pdl_trigger();
-    float *mine = acc_w + (size_t)warp * EDv;
-    for (int i = lane; i < EDv; i += 32) mine[i] = 0.f;
+    A *mine = acc_w + (size_t)warp * EDv;
+    for (int i = lane; i < EDv; i += 32) mine[i] = 0;
     __syncwarp();
 
     constexpr int EPV = 16 / sizeof(T);   // elements per 16-byte vector
@@ -331,15 +345,10 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Dims d, Ptrs p) {
     }
     __syncthreads();
     for (int i = threadIdx.x; i < EDv; i += kThreads) {
-        float s = 0.f;
+        A s = 0;
 #pragma unroll
         for (int wv = 0; wv < kWarps; ++wv) s += acc_w[(size_t)wv * EDv + i];
-        if (p.acc_bf)
-            p.acc_bf[(int64_t)b * EDv + i] = __float2bfloat16_rn(s);
-        else if (d.has_proj)
-            p.acc[(int64_t)b * EDv + i] = s;
-        else
-            static_cast<T *>(p.out)[(int64_t)b * d.d_v + i] = from_f<T>(s);
+        store_pooled<T>(d, p, b, i, (float)s);
     }
 }
 
@@ -356,7 +365,10 @@ __global__ void __launch_bounds__(kThreads) proj_kernel(Dims d, Ptrs p) {
     __shared__ float as[32][33];   // [c][token]
     __shared__ float ws[32][65];   // [c][output]
     const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+    // fp32 storage: compensated sums (Dot2), each partial to the working precision
+    constexpr bool kExact = std::is_same<T, float>::value;
     float acc[2][4] = {};
+    Dot2 ex[kExact ? 2 : 1][kExact ? 4 : 1];
     for (int k0 = kb; k0 < ke; k0 += 32) {
         for (int e = tid; e < 32 * 32; e += kThreads) {
             int bb = e / 32, kk = e % 32, b = b0 + bb, c = k0 + kk;
@@ -373,8 +385,13 @@ __global__ void __launch_bounds__(kThreads) proj_kernel(Dims d, Ptrs p) {
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 float wv = ws[kk][tx * 4 + j];
-                acc[0][j] = fmaf(a0, wv, acc[0][j]);
-                acc[1][j] = fmaf(a1, wv, acc[1][j]);
+                if constexpr (kExact) {
+                    ex[0][j].add(a0, wv);
+                    ex[1][j].add(a1, wv);
+                } else {
+                    acc[0][j] = fmaf(a0, wv, acc[0][j]);
+                    acc[1][j] = fmaf(a1, wv, acc[1][j]);
+                }
             }
         }
         __syncthreads();
@@ -382,44 +399,54 @@ __global__ void __launch_bounds__(kThreads) proj_kernel(Dims d, Ptrs p) {
     for (int i = 0; i < 2; ++i)
         for (int j = 0; j < 4; ++j) {
             int b = b0 + ty * 2 + i, o = o0 + tx * 4 + j;
+            float v = acc[i][j];
+            if constexpr (kExact) v = ex[i][j].value();
             if (b < d.B && o < d.d_out)
-                p.proj_part[((int64_t)split * d.B + b) * d.d_out + o] = acc[i][j];
+                p.proj_part[((int64_t)split * d.B + b) * d.d_out + o] = v;
         }
 }
 
+// out = the sum of the split-K partials (in fp64 with fp32 storage: one
+// rounding of the output)
 template <typename T>
 __global__ void proj_reduce_kernel(Dims d, Ptrs p) {
     pdl_wait();
     pdl_trigger();
+    using A = AccOf<T>;
     const int64_t total = (int64_t)d.B * d.d_out;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
          i += (int64_t)gridDim.x * blockDim.x) {
-        float s = 0.f;
-        for (int sp = 0; sp < d.p_splits; ++sp) s += p.proj_part[(int64_t)sp * total + i];
-        static_cast<T *>(p.out)[i] = from_f<T>(s);
+        A s = 0;
+        for (int sp = 0; sp < d.p_splits; ++sp) s += (A)p.proj_part[(int64_t)sp * total + i];
+        static_cast<T *>(p.out)[i] = from_f<T>((float)s);
     }
 }
 
 }  // namespace
 
-size_t gather_smem_bytes(const Dims &d) { return sizeof(float) * kWarps * d.E * d.d_v; }
+size_t gather_smem_bytes(const Dims &d) { return acc_bytes(d) * kWarps * d.E * d.d_v; }
 
 template <typename K> static cudaError_t allow(K kern, size_t bytes) {
     return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
+// the per-CTA maximum of dynamic shared memory next to the kernel's static share
 template <auto K> static cudaError_t allow_padded() {
     return allow(K, kSmemPerCta - static_smem_of<K>());
 }
 
-cudaError_t configure_gather(const Dims &d) {
-    const size_t bytes = gather_smem_bytes(d);
-    cudaError_t e = allow(gather_kernel<float>, bytes);
-    if (e == cudaSuccess) e = allow(gather_kernel<__nv_bfloat16>, bytes);
-    if (e == cudaSuccess) e = allow(gather_reg_kernel<float, 1>, bytes);
-    if (e == cudaSuccess) e = allow(gather_reg_kernel<float, 4>, bytes);
-    if (e == cudaSuccess) e = allow(gather_reg_kernel<__nv_bfloat16, 1>, bytes);
-    if (e == cudaSuccess) e = allow(gather_reg_kernel<__nv_bfloat16, 4>, bytes);
-    // the bucketed kernels may be padded up to a whole SM's share (spread_smem)
+// Every gather kernel may use up to the per-CTA maximum of dynamic shared
+// memory: a kernel's limit is a process-wide attribute, so it is only ever
+// raised (set once to the maximum), never set to one layer's need, which
+// would fail a later launch for a larger layer created earlier.
+cudaError_t configure_gather(const Dims &) {
+    cudaError_t e = allow_padded<gather_kernel<float, double>>();
+    if (e == cudaSuccess) e = allow_padded<gather_kernel<float, float>>();
+    if (e == cudaSuccess) e = allow_padded<gather_kernel<__nv_bfloat16, float>>();
+    if (e == cudaSuccess) e = allow_padded<gather_reg_kernel<float, 1>>();
+    if (e == cudaSuccess) e = allow_padded<gather_reg_kernel<float, 4>>();
+    if (e == cudaSuccess) e = allow_padded<gather_reg_kernel<__nv_bfloat16, 1>>();
+    if (e == cudaSuccess) e = allow_padded<gather_reg_kernel<__nv_bfloat16, 4>>();
+    // the bucketed kernels may also be padded up to a whole SM's share (spread_smem)
     if (e == cudaSuccess) e = allow_padded<gather_bucket_kernel<float, 512>>();
     if (e == cudaSuccess) e = allow_padded<gather_bucket_kernel<__nv_bfloat16, 512>>();
     if (e == cudaSuccess) e = allow_padded<gather_bucket_kernel<float, 256>>();
@@ -446,13 +473,22 @@ static cudaError_t launch_gather_t(const Dims &d, const Ptrs &p, cudaStream_t st
                                  st, d, p);
         }
     }
+    // the shared-memory-accumulating kernel: fp64 accumulators (fp32 storage)
+    // while they fit, else fp32 ones
+    auto general = [&]() {
+        if (std::is_same<T, float>::value && bytes <= kSmemPerCta)
+            return launch_kernel(d.pdl, gather_kernel<T, AccOf<T>>, d.B, kThreads, bytes, st, d,
+                                 p);
+        return launch_kernel(d.pdl, gather_kernel<T, float>, d.B, kThreads,
+                             sizeof(float) * kWarps * d.E * d.d_v, st, d, p);
+    };
     if (d.nc > 1)   // MCS beyond the bucketed kernel's range
-        return launch_kernel(d.pdl, gather_kernel<T>, d.B, kThreads, bytes, st, d, p);
+        return general();
     if (fits_lanes && d.E == 1)
         return launch_kernel(d.pdl, gather_reg_kernel<T, 1>, d.B, kThreads, bytes, st, d, p);
     if (fits_lanes && d.E <= 4)
         return launch_kernel(d.pdl, gather_reg_kernel<T, 4>, d.B, kThreads, bytes, st, d, p);
-    return launch_kernel(d.pdl, gather_kernel<T>, d.B, kThreads, bytes, st, d, p);
+    return general();
 }
 
 cudaError_t launch_gather(const Dims &d, const Ptrs &p, cudaStream_t st) {

@@ -11,6 +11,9 @@
 //   sel_w    [B][H][m][nc]             weights of each selected slot (nc > 1:
 //                                      one per value slice, Multi-Core Scoring)
 //   acc      [B][E*D_v]                per-block pooled rows, Eq. 15 inner sum
+//   acc_bf   [B][T][E*D_v] bf16        the same as T bf16 terms (tensor path):
+//                                      T = 2 for the projection, whose B operand
+//                                      is then hi + lo (residual <= 2^-16 |acc|)
 //   proj_part[p_splits][B][D'_v]       split-K partial sums of the projection
 //   xs       the convolved query input x~ (Trick 4): bf16 [B][3][D_i], three
 //            terms per value, for the tensor-core query; fp32 [B][D_i] for
@@ -21,6 +24,8 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+
+#include <type_traits>
 
 #include "../../include/ultramem.h"
 
@@ -63,7 +68,9 @@ struct Ptrs {
     void *out;
     int64_t *idx_out;
     float *w_out;
-    __nv_bfloat16 *acc_bf;       // tensor path: acc rounded to bf16 [B][E*D_v]
+    __nv_bfloat16 *acc_bf;       // tensor path: acc as bf16 terms [B][acc_terms][E*D_v]
+    int acc_terms;               // 2: hi + lo, the pooled value to 2^-16 relative (the
+                                 // projection's operand); 1 (or 0): one rounding
     const int64_t *idx_in;       // lookup_reduce input addresses
     const float *w_in;           // lookup_reduce input weights [B][H][m][nc]
     const float *conv_w, *conv_b;   // [conv_k][D_i], [D_i] or null
@@ -103,11 +110,14 @@ cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaS
 cudaError_t launch_dacc_tc(const Dims &d, const CUtensorMap &w_p, const CUtensorMap &g,
                            float *dacc, int *err, cudaStream_t st);
 // the backward's dW_p = sum_tokens acc g^T on the tensor cores, from the
-// transposed pooled rows [E D_v][B] and gradient rows [D'_v][B] (bf16)
-cudaError_t launch_dw_tc(const Dims &d, const CUtensorMap &acc_t, const CUtensorMap &g_t,
+// transposed gradient rows [D'_v][B] and the transposed pooled rows as two
+// bf16 terms [E D_v][2 B] (hi in columns [0, B), lo in [B, 2 B))
+cudaError_t launch_dw_tc(const Dims &d, const CUtensorMap &g_t, const CUtensorMap &acc_t2,
                          float *dW, int *err, cudaStream_t st);
+// dst[c][r] = src[r][c], rows x cols bf16; row strides ld_src / ld_dst in
+// elements (0: cols / rows, contiguous)
 cudaError_t launch_transpose_bf16(const void *src, void *dst, int rows, int cols,
-                                  cudaStream_t st);
+                                  cudaStream_t st, int64_t ld_src = 0, int64_t ld_dst = 0);
 
 // x_f32: the token rows p.x are fp32 (the convolved input) whatever the storage type
 cudaError_t launch_query(const Dims &d, const Ptrs &p, bool x_f32, cudaStream_t st);
@@ -287,6 +297,60 @@ __device__ __forceinline__ void put_split_query(__nv_bfloat16 *qs, int axis, int
     dst[d_k] = q2;
     dst[2 * d_k] = q3;
 }
+
+// One pooled value acc[b][i] (i < E*D_v) into the buffer the next step
+// reads: the tensor path's bf16 terms (hi = rn(v), lo = rn(v - hi), so that
+// hi + lo equals v to 2^-16 relative), the fp32 acc of the CUDA-core
+// projection, or, without a projector, the output row itself.
+template <typename T>
+__device__ __forceinline__ void store_pooled(const Dims &d, const Ptrs &p, int64_t b, int i,
+                                             float v) {
+    const int EDv = d.E * d.d_v;
+    if (p.acc_bf) {
+        const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+        __nv_bfloat16 *dst = p.acc_bf + b * (p.acc_terms > 1 ? 2 : 1) * EDv + i;
+        dst[0] = hi;
+        if (p.acc_terms > 1) dst[EDv] = __float2bfloat16_rn(v - __bfloat162float(hi));
+    } else if (d.has_proj) {
+        p.acc[b * EDv + i] = v;
+    } else {
+        static_cast<T *>(p.out)[b * d.d_v + i] = from_f<T>(v);
+    }
+}
+
+// ---- fp32 storage: dot products to the working precision ---------------
+// The fp32 mode promises outputs within 1e-4 of the exact result element by
+// element (down to 1e-3 of a row's largest entry), which plain fp32
+// accumulation over hundreds of terms does not reach.  Its CUDA-core
+// contractions therefore accumulate with error-free transformations
+// (Ogita, Rump and Oishi, "Accurate sum and dot product", SIAM J. Sci.
+// Comput. 26(6), 2005, algorithm Dot2): TwoProduct by an FMA and Knuth's
+// TwoSum, the rounding errors summed on the side, so that s + c is as
+// accurate as a dot product computed in twice the working precision.  The
+// intrinsics keep the compiler from contracting or reordering the steps.
+struct Dot2 {
+    float s, c;
+    __device__ __forceinline__ Dot2() : s(0.f), c(0.f) {}
+    // s + p = t + e exactly (TwoSum): s becomes t and e goes to c
+    __device__ __forceinline__ void two_sum_into(float p) {
+        const float t = __fadd_rn(s, p);
+        const float z = __fsub_rn(t, s);
+        const float e = __fadd_rn(__fsub_rn(s, __fsub_rn(t, z)), __fsub_rn(p, z));
+        s = t;
+        c = __fadd_rn(c, e);
+    }
+    __device__ __forceinline__ void add(float a, float b) {
+        const float p = __fmul_rn(a, b);
+        const float pe = __fmaf_rn(a, b, -p);   // a b = p + pe exactly
+        two_sum_into(p);
+        c = __fadd_rn(c, pe);
+    }
+    __device__ __forceinline__ void merge(const Dot2 &o) {   // add another partial sum
+        two_sum_into(o.s);
+        c = __fadd_rn(c, o.c);
+    }
+    __device__ __forceinline__ float value() const { return __fadd_rn(s, c); }
+};
 
 // Barrett's constant for reduction modulo M (P. Barrett, CRYPTO '86).
 inline uint64_t barrett_mu(uint64_t M) { return M ? ~0ull / M : 0; }

@@ -16,7 +16,6 @@
 
 namespace um {
 cudaError_t configure_gather(const Dims &d);
-size_t gather_smem_bytes(const Dims &d);
 void host_shuffle_params(uint64_t seed, uint64_t M, uint64_t *a, uint64_t *c);
 }  // namespace um
 
@@ -29,7 +28,7 @@ static __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
 
 std::mutex g_mu;
 void *g_scratch_addr[kMaxDevices];     // device address of g_scratch per device
-size_t g_gather_smem[kMaxDevices];     // largest gather smem configured per device
+bool g_configured[kMaxDevices];        // the gather kernels' shared memory limit set
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
@@ -124,11 +123,10 @@ extern "C" ultramem_status ultramem_lookup_reduce_noalloc(const ultramem_config 
             if (e != cudaSuccess || !ptr) return status_of(e);
             g_scratch_addr[dev] = ptr;
         }
-        const size_t need = um::gather_smem_bytes(d);
-        if (need > g_gather_smem[dev]) {
+        if (!g_configured[dev]) {   // once per device: the kernels' maximum, never lowered
             cudaError_t e = um::configure_gather(d);
             if (e != cudaSuccess) return status_of(e);
-            g_gather_smem[dev] = need;
+            g_configured[dev] = true;
         }
         base = static_cast<unsigned char *>(g_scratch_addr[dev]);
     }

@@ -45,20 +45,22 @@ __global__ void __launch_bounds__(kThreads) conv_kernel(Dims d, Ptrs p, int spli
     if (c >= d.d_in) return;
     const int row = blockIdx.x;
     if (row < d.B) {
-        float acc = p.conv_b ? p.conv_b[c] : 0.f;
+        // fp32 storage: the taps summed in fp64, one rounding of x~
+        using A = typename std::conditional<std::is_same<T, float>::value, double, float>::type;
+        A acc = p.conv_b ? (A)p.conv_b[c] : (A)0;
         for (int j = 0; j < d.conv_k; ++j)
-            acc = fmaf(p.conv_w[(int64_t)j * d.d_in + c], to_f(input_back<T>(d, p, row, j, c)), acc);
+            acc += (A)p.conv_w[(int64_t)j * d.d_in + c] * (A)to_f(input_back<T>(d, p, row, j, c));
         if (splits) {
             __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(p.xs) + (int64_t)row * 3 * d.d_in + c;
-            const __nv_bfloat16 t1 = __float2bfloat16_rn(acc);
-            const float r1 = acc - __bfloat162float(t1);
+            const __nv_bfloat16 t1 = __float2bfloat16_rn((float)acc);
+            const float r1 = (float)acc - __bfloat162float(t1);
             const __nv_bfloat16 t2 = __float2bfloat16_rn(r1);
             const float r2 = r1 - __bfloat162float(t2);
             dst[0] = t1;
             dst[d.d_in] = t2;
             dst[2 * d.d_in] = __float2bfloat16_rn(r2);
         } else {
-            static_cast<float *>(p.xs)[(int64_t)row * d.d_in + c] = acc;
+            static_cast<float *>(p.xs)[(int64_t)row * d.d_in + c] = (float)acc;
         }
     } else {
         // state row i of sequence s: input seq_len - kk + i of it (a copy)
@@ -107,6 +109,40 @@ __global__ void __launch_bounds__(kThreads) query_ln_kernel(Dims d, Ptrs p, __nv
     if (!live) return;
     const int64_t split_stride = (int64_t)d.A * d.B * HD;
     float *q = p.q_part + ((int64_t)a * d.B + b) * HD + (int64_t)h * d.d_k;
+    if (d.dtype == ULTRAMEM_F32) {
+        // fp32 storage (CUDA-core path, no splits to write): the partial
+        // sums, mean, variance and normalisation in fp64, one rounding
+        double vd[kLnMax];
+        double sum = 0.0;
+#pragma unroll
+        for (int i = 0; i < kLnMax; ++i) {
+            const int c = lane + 32 * i;
+            vd[i] = 0.0;
+            if (c < d.d_k) {
+                for (int s = 0; s < d.q_splits; ++s) vd[i] += (double)q[s * split_stride + c];
+                sum += vd[i];
+            }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(kFull, sum, off);
+        const double mean = sum / (double)d.d_k;
+        double sq = 0.0;
+#pragma unroll
+        for (int i = 0; i < kLnMax; ++i) {
+            const double e = lane + 32 * i < d.d_k ? vd[i] - mean : 0.0;
+            sq += e * e;
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(kFull, sq, off);
+        const double inv = 1.0 / sqrt(sq / (double)d.d_k + (double)d.ln_eps);
+#pragma unroll
+        for (int i = 0; i < kLnMax; ++i) {
+            const int c = lane + 32 * i;
+            if (c >= d.d_k) break;
+            q[c] = (float)((vd[i] - mean) * inv * (double)gv[i] + (double)bv[i]);
+        }
+        return;
+    }
     float v[kLnMax];
     float sum = 0.f;
 #pragma unroll

@@ -1,7 +1,10 @@
 // um_score.cu -- query projection (S1) and row/column scores (S2-S3, Eq. 4
 // and 6) on CUDA cores in fp32, the path of fp32 storage.  The query
 // projection is split over D_i so that enough CTAs stream W_q; the partial
-// sums are added when the score kernel loads the query.
+// sums are added when the score kernel loads the query (and, in fp64, when
+// the selection loads it for the weights).  With fp32 storage each partial
+// is a compensated dot product (Dot2); the scores here only decide which
+// keys survive, and the selection recomputes the survivors' exactly.
 #include "um_internal.cuh"
 
 namespace um {
@@ -28,7 +31,10 @@ __global__ void __launch_bounds__(kThreads) query_kernel(Dims d, Ptrs p) {
     __shared__ float xs[32][33];  // [d][token]
     __shared__ float ws[32][65];  // [d][output]
     const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+    // fp32 storage: compensated sums (Dot2), each partial to the working precision
+    constexpr bool kExact = std::is_same<T, float>::value;
     float acc[2][4] = {};
+    Dot2 ex[kExact ? 2 : 1][kExact ? 4 : 1];
     for (int k0 = kb; k0 < ke; k0 += 32) {
         for (int e = tid; e < 32 * 32; e += kThreads) {
             int bb = e / 32, kk = e % 32, b = b0 + bb, k = k0 + kk;
@@ -45,8 +51,13 @@ __global__ void __launch_bounds__(kThreads) query_kernel(Dims d, Ptrs p) {
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 float wv = ws[kk][tx * 4 + j];
-                acc[0][j] = fmaf(xv0, wv, acc[0][j]);
-                acc[1][j] = fmaf(xv1, wv, acc[1][j]);
+                if constexpr (kExact) {
+                    ex[0][j].add(xv0, wv);
+                    ex[1][j].add(xv1, wv);
+                } else {
+                    acc[0][j] = fmaf(xv0, wv, acc[0][j]);
+                    acc[1][j] = fmaf(xv1, wv, acc[1][j]);
+                }
             }
         }
         __syncthreads();
@@ -54,8 +65,10 @@ __global__ void __launch_bounds__(kThreads) query_kernel(Dims d, Ptrs p) {
     for (int i = 0; i < 2; ++i)
         for (int j = 0; j < 4; ++j) {
             int b = b0 + ty * 2 + i, o = o0 + tx * 4 + j;
+            float v = acc[i][j];
+            if constexpr (kExact) v = ex[i][j].value();
             if (b < d.B && o < HD)
-                p.q_part[(((int64_t)split * d.A + a) * d.B + b) * HD + o] = acc[i][j];
+                p.q_part[(((int64_t)split * d.A + a) * d.B + b) * HD + o] = v;
         }
 }
 

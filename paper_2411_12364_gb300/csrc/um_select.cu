@@ -68,6 +68,7 @@ struct SelShared {
     int warp_tot[kWarps];
     int digit, remaining;
     float scalar;
+    double dscalar;   // fp32 storage: the softmax denominator in fp64
 };
 
 __device__ __forceinline__ u64 comp_of(uint32_t key, uint32_t pos) {
@@ -439,7 +440,7 @@ struct SelLayout {
     uint32_t *key1;     // [K] axis-1 keys (free once the axis winners are ranked)
     int *sel_i, *sel_j; // [k] surviving rows / columns in increasing index
     float *R, *scol;    // [k][r] R = S_row^T C and S_col of the survivors
-    float *srow;        // MCS: [k][r] S_row of the row survivors      } in key1's
+    float *srow;        // MCS, fp32: [k][r] S_row of the row survivors } in key1's
     float *cparts;      // MCS: [nc][r][r] component cores of this head } space
 };
 
@@ -453,10 +454,12 @@ __host__ __device__ inline SelOffsets sel_offsets(const Dims &d) {
     size_t off = 0;
     o.qv = off;    off = up(off + sizeof(float) * 2 * d.d_k);
     o.key0 = off;  off = up(off + sizeof(uint32_t) * (d.K > d.k * d.k ? d.K : d.k * d.k));
-    // with MCS, key1's space later holds S_row of the row survivors and the
-    // component cores (so that the block's shared memory does not grow)
+    // with MCS (and with fp32 storage), key1's space later holds S_row of the
+    // row survivors and the component cores (so that the block's shared
+    // memory does not grow)
     const bool mcs = d.nc > 1;
-    const int mcs_floats = mcs ? d.k * d.r + d.nc * d.r * d.r : 0;
+    const bool keep_srow = mcs || d.dtype == ULTRAMEM_F32;
+    const int mcs_floats = keep_srow ? d.k * d.r + (mcs ? d.nc * d.r * d.r : 0) : 0;
     o.key1 = off;  off = up(off + sizeof(uint32_t) * (d.K > mcs_floats ? d.K : mcs_floats));
     o.srow = o.key1;
     o.cparts = o.key1 + sizeof(float) * d.k * d.r;
@@ -617,6 +620,10 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
     float S[RM];
 #pragma unroll
     for (int a = 0; a < RM; ++a) S[a] = 0.f;
+    // fp32 storage: each chunk score as a compensated dot product (Dot2),
+    // so that the weights carry the working precision (see Dot2)
+    constexpr bool kExact = std::is_same<T, float>::value;
+    Dot2 SX[kExact ? RM : 1];
     if (vec) {
         // 16-byte group iv of the row belongs to chunk iv / cpv
         const int cpv = dk / EPV;
@@ -640,6 +647,25 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
                     unpack16<T>(buf[u], f);
                     // q + iv*EPV is 16-byte aligned: qv is, and D % EPV == 0
                     const float4 *qq = reinterpret_cast<const float4 *>(q + iv * EPV);
+                    if constexpr (kExact) {
+                        // the vector lies in one chunk: add its products there
+                        const int al = RM == 2 ? (iv >= cpv ? RM - 1 : 0)
+                                               : (int)(((float)(iv * EPV) + 0.5f) * inv_dk);
+#pragma unroll
+                        for (int a = 0; a < RM; ++a) {
+                            if (a == al) {
+#pragma unroll
+                                for (int e4 = 0; e4 < EPV / 4; ++e4) {
+                                    const float4 q4 = qq[e4];
+                                    SX[a].add(f[4 * e4], q4.x);
+                                    SX[a].add(f[4 * e4 + 1], q4.y);
+                                    SX[a].add(f[4 * e4 + 2], q4.z);
+                                    SX[a].add(f[4 * e4 + 3], q4.w);
+                                }
+                            }
+                        }
+                        continue;
+                    }
                     float pv = 0.f;
 #pragma unroll
                     for (int e4 = 0; e4 < EPV / 4; ++e4) {
@@ -667,21 +693,41 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
         for (int a = 0; a < RM; ++a) {
             if (a < r && active) {
                 float acc = 0.f;
-                for (int c = a * dk + sub; c < (a + 1) * dk; c += G)
-                    acc = fmaf(to_f(row[c]), q[c], acc);
+                for (int c = a * dk + sub; c < (a + 1) * dk; c += G) {
+                    if constexpr (kExact) SX[a].add(to_f(row[c]), q[c]);
+                    else acc = fmaf(to_f(row[c]), q[c], acc);
+                }
                 S[a] = acc;
             }
         }
     }
+    if constexpr (kExact) {
+        // the group's partial sums merged with their error terms
 #pragma unroll
-    for (int a = 0; a < RM; ++a) {
-        if (a < r)
-            for (int off = G >> 1; off > 0; off >>= 1) S[a] += __shfl_xor_sync(kFull, S[a], off);
+        for (int a = 0; a < RM; ++a) {
+            if (a < r) {
+                for (int off = G >> 1; off > 0; off >>= 1) {
+                    Dot2 o;
+                    o.s = __shfl_xor_sync(kFull, SX[a].s, off);
+                    o.c = __shfl_xor_sync(kFull, SX[a].c, off);
+                    SX[a].merge(o);
+                }
+                S[a] = SX[a].value();
+            }
+        }
+    } else {
+#pragma unroll
+        for (int a = 0; a < RM; ++a) {
+            if (a < r)
+                for (int off = G >> 1; off > 0; off >>= 1) S[a] += __shfl_xor_sync(kFull, S[a], off);
+        }
     }
     if (active && sub == 0) {
         if (s == 0) {
             L.sel_i[ord] = (int)pos;
-            if (d.nc > 1)   // MCS: the individual scores need S_row itself
+            // MCS (the individual scores) and fp32 storage (the weights in
+            // fp64) need S_row itself
+            if (d.nc > 1 || kExact)
 #pragma unroll
                 for (int a = 0; a < RM; ++a)
                     if (a < r) L.srow[ord * r + a] = S[a];
@@ -738,11 +784,19 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
         const int a = (axis == 1 && d.A == 2) ? 1 : 0;
         return p.q_part + ((int64_t)a * d.B + b) * HD + h * d.d_k + c;
     };
+    // the split-K partials of q, summed in fp64 with fp32 storage (one
+    // rounding of the query the weights are computed from)
     auto q_of = [&](int e) {
         const float *src = q_src(e);
-        float q = 0.f;
-        for (int s = 0; s < d.q_splits; ++s) q += src[s * split_stride];
-        return q;
+        if constexpr (std::is_same<T, float>::value) {
+            double q = 0.0;
+            for (int s = 0; s < d.q_splits; ++s) q += (double)src[s * split_stride];
+            return (float)q;
+        } else {
+            float q = 0.f;
+            for (int s = 0; s < d.q_splits; ++s) q += src[s * split_stride];
+            return q;
+        }
     };
     const bool one_split = d.q_splits == 1;
     float q0 = 0.f;
@@ -850,9 +904,51 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     else rank_list(sh.cand[0], cf, m, fwin, threadIdx.x, kThreads);
     __syncthreads();
 
+    // fp32 storage: the weights are the winners' scores recomputed in fp64
+    // from the exact chunk scores (S_row, S_col) and the core, rounded once;
+    // the fp32 scores above only decided the order
+    constexpr bool kExact = std::is_same<T, float>::value;
+    auto exact_g = [&](int ii, int jj, const float *Cm) -> double {
+        if (d.pkm) return (double)L.srow[ii] + (double)L.scol[jj];   // Eq. 2: r = 1
+        double g = 0.0;
+        for (int a = 0; a < r; ++a) {
+            double cs = 0.0;
+            for (int be = 0; be < r; ++be)
+                cs += (double)Cm[a * r + be] * (double)L.scol[jj * r + be];
+            g += (double)L.srow[ii * r + a] * cs;
+        }
+        return g;
+    };
+    auto pair_of = [&](u64 wc, int &ii, int &jj) {
+        int c = (int)pos_of(wc);
+        if ((uint32_t)c >= (uint32_t)k2) c = 0;   // recorded below
+        ii = c / k;
+        jj = c - ii * k;
+    };
+    double gmax_d = 0.0;
+    if constexpr (kExact) {
+        int i0, j0;
+        pair_of(fwin[0], i0, j0);
+        gmax_d = exact_g(i0, j0, sh.core);
+        if (d.act == ULTRAMEM_ACT_SOFTMAX) {
+            if (threadIdx.x < 32) {
+                double z = 0.0;
+                for (int e = threadIdx.x; e < m; e += 32) {
+                    int ii, jj;
+                    pair_of(fwin[e], ii, jj);
+                    z += exp(exact_g(ii, jj, sh.core) - gmax_d);
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(kFull, z, off);
+                if (threadIdx.x == 0) sh.dscalar = z;
+            }
+            __syncthreads();
+        }
+    }
+
     // PKM's softmax over the m selected scores (Eq. 3); Trick 1 skips it
     const float gmax = ord2f(key_of(fwin[0]));
-    if (d.act == ULTRAMEM_ACT_SOFTMAX) {
+    if (!kExact && d.act == ULTRAMEM_ACT_SOFTMAX) {
         if (threadIdx.x < 32) {
             float z = 0.f;
             for (int e = threadIdx.x; e < m; e += 32) z += __expf(ord2f(key_of(fwin[e])) - gmax);
@@ -876,7 +972,13 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
         const int ii = c / k, jj = c - ii * k;
         const uint64_t v = (uint64_t)L.sel_i[ii] * (uint64_t)K + (uint64_t)L.sel_j[jj];
         const float g = ord2f(key_of(wc));
-        const float w = d.act == ULTRAMEM_ACT_SOFTMAX ? __expf(g - gmax) / sh.scalar : g;
+        float w;
+        if constexpr (kExact) {
+            const double gd = exact_g(ii, jj, sh.core);
+            w = (float)(d.act == ULTRAMEM_ACT_SOFTMAX ? exp(gd - gmax_d) / sh.dscalar : gd);
+        } else {
+            w = d.act == ULTRAMEM_ACT_SOFTMAX ? __expf(g - gmax) / sh.scalar : g;
+        }
         const uint32_t vs = (uint32_t)shuffle_address(d, p.perm, v);   // Eq. 14, < M < 2^32
         const uint32_t pb = vs / N;
         const uint32_t prow = vs - pb * N;
@@ -902,6 +1004,12 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
             }
             for (int ci = 0; ci < d.nc; ++ci) {
                 const float *Cc = L.cparts + ci * r * r;
+                if constexpr (kExact) {   // fp32 storage: in fp64, rounded once
+                    const float gx = (float)exact_g(ii, jj, Cc);
+                    p.sel_w[(base + e) * d.nc + ci] = gx;
+                    if (p.w_out) p.w_out[(base + e) * d.nc + ci] = gx;
+                    continue;
+                }
                 float gi = 0.f;
 #pragma unroll
                 for (int a = 0; a < RM; ++a) {
@@ -973,21 +1081,25 @@ cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream
     return cudaGetLastError();
 }
 
-template <typename T, int RM> static cudaError_t allow_select(int bytes) {
+// Each selection kernel may use up to the per-CTA maximum of dynamic shared
+// memory (the decode-grid one is padded to spread its CTAs; see
+// spread_smem).  The limit is a process-wide attribute of the kernel, so it
+// is set once to the maximum, never lowered to one layer's need.
+template <typename T, int RM> static cudaError_t allow_select() {
     const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
-    // the decode-grid kernel may be padded up to a whole SM's share
-    const int pad = (int)(kSmemPerCta - static_smem_of<select_kernel<T, 3, RM>>());
-    cudaError_t e = cudaFuncSetAttribute(select_kernel<T, 3, RM>, a, bytes > pad ? bytes : pad);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<T, 4, RM>, a, bytes);
+    cudaError_t e = cudaFuncSetAttribute(
+        select_kernel<T, 3, RM>, a, (int)(kSmemPerCta - static_smem_of<select_kernel<T, 3, RM>>()));
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(select_kernel<T, 4, RM>, a,
+                                 (int)(kSmemPerCta - static_smem_of<select_kernel<T, 4, RM>>()));
     return e;
 }
 
-cudaError_t configure_select(const Dims &d) {
-    const int bytes = (int)select_smem_bytes(d);
-    cudaError_t e = allow_select<float, 2>(bytes);
-    if (e == cudaSuccess) e = allow_select<float, kMaxR>(bytes);
-    if (e == cudaSuccess) e = allow_select<__nv_bfloat16, 2>(bytes);
-    if (e == cudaSuccess) e = allow_select<__nv_bfloat16, kMaxR>(bytes);
+cudaError_t configure_select(const Dims &) {
+    cudaError_t e = allow_select<float, 2>();
+    if (e == cudaSuccess) e = allow_select<float, kMaxR>();
+    if (e == cudaSuccess) e = allow_select<__nv_bfloat16, 2>();
+    if (e == cudaSuccess) e = allow_select<__nv_bfloat16, kMaxR>();
     return e;
 }
 

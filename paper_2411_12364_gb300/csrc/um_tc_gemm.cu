@@ -2,7 +2,8 @@
 // tensor cores (bf16 storage mode):
 //   S1  q_part = W_q x            M = H*D_k outputs, N = tokens, K = D_i (split-K)
 //   S2  S_alpha = K_chunk q_chunk M = keys, N = tokens, K = D_k in r chunks (Eq. 4)
-//   S9  out = W_p^T acc           M = D'_v outputs, N = tokens, K = E*D_v (Eq. 15)
+//   S9  out = W_p^T acc           M = D'_v outputs, N = tokens, K = E*D_v (Eq. 15),
+//                                 acc entering as two bf16 terms hi + lo
 // Weights fill the 128-row M side ("swap AB"), so a decode batch of B tokens
 // is the N side of one MMA (N = B rounded up to 16).
 //
@@ -663,14 +664,18 @@ struct DaccOp {
     }
 };
 
-// The backward's dW_p = sum_tokens acc_p g^T: A = the pooled rows transposed
-// ([E D_v][B] bf16, K = tokens), B = the gradient rows transposed ([D'_v][B]);
-// fp32 dW [E D_v][D'_v] row-major, unsplit.
+// The backward's dW_p = sum_tokens acc_p g^T, computed transposed: A = the
+// gradient rows transposed ([D'_v][B] bf16, K = tokens), B = the pooled rows
+// transposed as two bf16 terms hi + lo ([E D_v][2 B], the lo term at column
+// offset B), both terms multiplying each A tile into one accumulator (the
+// pooled rows to 2^-16 relative, as in the forward's projection).  Tile
+// rows are outputs o, columns are pooled entries c; fp32 dW [E D_v][D'_v]
+// row-major, unsplit.
 struct DwOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
-    int M, N, kb_total;
-    float *out;   // [M][N]
+    int M, N, kb_total;   // M = D'_v (rows o), N = E D_v (columns c)
+    float *out;           // [N][M]
     __device__ int cluster_splits() const { return 1; }
     int cluster_splits_host() const { return 1; }
     __device__ void store_partial(const Tile &, int, int, float (&)[kMaxAcc][16]) const {}
@@ -689,30 +694,32 @@ struct DwOp {
         return t;
     }
     __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
-        const int m = t.m0 + row;
-        if (m >= M) return;
-        float *dst = out + (int64_t)m * N;
+        const int o = t.m0 + row;
+        if (o >= M) return;
+        // dW[n][o]: a warp's 32 rows o are contiguous for each column n
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
             const int n = t.n0 + c + j;
-            if (n < N) dst[n] = t.nkb ? v[0][j] : 0.f;
+            if (n < N) out[(int64_t)n * M + o] = t.nkb ? v[0][j] : 0.f;
         }
     }
 };
 
-// dst[c][r] = src[r][c] for a rows x cols bf16 matrix (32 x 32 tiles)
+// dst[c][r] = src[r][c] for a rows x cols bf16 matrix (32 x 32 tiles), with
+// row strides ld_src (>= cols) and ld_dst (>= rows) in elements
 __global__ void transpose_kernel(const __nv_bfloat16 *__restrict__ src,
-                                 __nv_bfloat16 *__restrict__ dst, int rows, int cols) {
+                                 __nv_bfloat16 *__restrict__ dst, int rows, int cols,
+                                 int64_t ld_src, int64_t ld_dst) {
     __shared__ __nv_bfloat16 tile[32][33];
     const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
     for (int i = threadIdx.y; i < 32; i += blockDim.y) {
         const int r = r0 + i, c = c0 + threadIdx.x;
-        if (r < rows && c < cols) tile[i][threadIdx.x] = src[(int64_t)r * cols + c];
+        if (r < rows && c < cols) tile[i][threadIdx.x] = src[(int64_t)r * ld_src + c];
     }
     __syncthreads();
     for (int i = threadIdx.y; i < 32; i += blockDim.y) {
         const int c = c0 + i, r = r0 + threadIdx.x;
-        if (r < rows && c < cols) dst[(int64_t)c * rows + r] = tile[threadIdx.x][i];
+        if (r < rows && c < cols) dst[(int64_t)c * ld_dst + r] = tile[threadIdx.x][i];
     }
 }
 
@@ -721,10 +728,12 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 }  // namespace
 
 cudaError_t launch_transpose_bf16(const void *src, void *dst, int rows, int cols,
-                                  cudaStream_t st) {
+                                  cudaStream_t st, int64_t ld_src, int64_t ld_dst) {
     dim3 grid((cols + 31) / 32, (rows + 31) / 32);
     transpose_kernel<<<grid, dim3(32, 8), 0, st>>>(static_cast<const __nv_bfloat16 *>(src),
-                                                   static_cast<__nv_bfloat16 *>(dst), rows, cols);
+                                                   static_cast<__nv_bfloat16 *>(dst), rows, cols,
+                                                   ld_src > 0 ? ld_src : cols,
+                                                   ld_dst > 0 ? ld_dst : rows);
     return cudaGetLastError();
 }
 
@@ -831,26 +840,26 @@ cudaError_t configure_tc() {
     cudaError_t e = allow_smem<1, QueryOp>();
     if (e == cudaSuccess) e = allow_smem<3, QueryOp>();
     if (e == cudaSuccess) e = allow_smem<3, ScoreOp>();
-    if (e == cudaSuccess) e = allow_smem<1, ProjOp>();
+    if (e == cudaSuccess) e = allow_smem<2, ProjOp>();
     if (e == cudaSuccess) e = allow_smem<1, DaccOp>();
-    if (e == cudaSuccess) e = allow_smem<1, DwOp>();
+    if (e == cudaSuccess) e = allow_smem<2, DwOp>();
     return e;
 }
 
-cudaError_t launch_dw_tc(const Dims &d, const CUtensorMap &acc_t, const CUtensorMap &g_t,
+cudaError_t launch_dw_tc(const Dims &d, const CUtensorMap &g_t, const CUtensorMap &acc_t2,
                          float *dW, int *err, cudaStream_t st) {
     DwOp op;
-    op.n_tile = tc_n_tile(d.d_out, 1);
+    op.M = d.d_out;
+    op.N = d.E * d.d_v;
+    op.n_tile = tc_n_tile(op.N, 1);
     op.n_acc = 1;
     op.acc_chunk = 1 << 30;
-    op.b_split_stride = 0;
+    op.b_split_stride = d.B;   // the lo term's columns follow the hi term's
     op.err = err;
-    op.M = d.E * d.d_v;
-    op.N = d.d_out;
     op.kb_total = (d.B + kBlockK - 1) / kBlockK;
     op.out = dW;
     dim3 grid((op.M + kTileM - 1) / kTileM, (op.N + op.n_tile - 1) / op.n_tile, 1);
-    return launch_gemm<1>(grid, acc_t, acc_t, g_t, op, op.kb_total, false, st);
+    return launch_gemm<2>(grid, g_t, g_t, acc_t2, op, op.kb_total, false, st);
 }
 
 cudaError_t launch_dacc_tc(const Dims &d, const CUtensorMap &w_p, const CUtensorMap &g,
@@ -935,7 +944,10 @@ cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaS
     op.n_tile = tc_n_tile(d.B, 1);
     op.n_acc = 1;
     op.acc_chunk = 1 << 30;
-    op.b_split_stride = 0;
+    // the pooled rows are two bf16 terms hi + lo ([B][2][E D_v]): both
+    // multiply each projector tile into one fp32 accumulator, so the operand
+    // carries the pooled value to 2^-16 relative instead of one rounding
+    op.b_split_stride = d.E * d.d_v;
     op.err = p.err;
     op.B = d.B;
     op.d_out = d.d_out;
@@ -945,7 +957,7 @@ cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaS
     op.part = p.proj_part;
     dim3 grid((d.d_out + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, op.splits);
     const int per = (op.kb_total + op.splits - 1) / op.splits;
-    return launch_gemm<1>(grid, mp.w_pt, mp.w_pt, mp.acc, op, per, d.pdl, st);
+    return launch_gemm<2>(grid, mp.w_pt, mp.w_pt, mp.acc, op, per, d.pdl, st);
 }
 
 }  // namespace um

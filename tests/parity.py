@@ -9,10 +9,19 @@ select valid slots (each no worse than the oracle's m-th score within the
 same tolerance), and the token's output is then compared with the oracle's
 lookup-reduce of the GPU's own slots.
 
-Output tolerance: per token, max_e |y - y_ref| / max_e |y_ref| <= 1e-4 in
-fp32 mode and 2e-2 in bf16 mode.  Weights: |w - w_ref| <= 1e-4 * max |w_ref|
-per head (over all h weights of a slot with Multi-Core Scoring).  With MCS
-the selection and the near-tie rule use each head's summed core (Eq. 16).
+Output tolerance, element-wise with a floor: per token,
+max_e |y_e - y_ref_e| / max(|y_ref_e|, 1e-3 max_e' |y_ref_e'|) <= 1e-4 in fp32
+mode and 2e-2 in bf16 mode (the floor keeps the ratio defined for elements
+near 0).  The normwise figure max_e |y - y_ref| / max_e |y_ref| is reported
+beside it.  Weights: |w - w_ref| <= 1e-4 * max |w_ref| per head (over all h
+weights of a slot with Multi-Core Scoring).  With MCS the selection and the
+near-tie rule use each head's summed core (Eq. 16).
+
+A near-tie is a gap of at most 1e-5 relative to the two boundary scores
+themselves.  Boundary scores near 0 come from cancellation, where an fp32
+result is only accurate to the size of the cancelled terms, so a gap within
+1e-5 of 1e-3 times the head's largest score also counts; such heads are
+counted separately (``floor_ties``), and the workload tests require none.
 """
 from __future__ import annotations
 
@@ -24,18 +33,33 @@ from tests import util
 
 TIE_REL = 1e-5
 W_TOL = 1e-4
+OUT_FLOOR = 1e-3     # of the token's largest |y_ref|: the element-wise denominator's floor
 
 
 def out_tol(cfg):
     return 1e-4 if int(cfg["dtype"]) == 0 else 2e-2
 
 
-def _gap_is_tie(vals, kk):
+NO_TIE, TIE, FLOOR_TIE = 0, 1, 2
+
+
+def tie_kind(vals, kk):
+    """Whether the kk-th and (kk+1)-th largest of vals are a near-tie: TIE
+    when their gap is within TIE_REL of the larger of the two, FLOOR_TIE when
+    it is only within TIE_REL of 1e-3 max |vals| (cancellation near 0)."""
     if kk >= vals.size:
-        return False
+        return NO_TIE
     srt = np.sort(vals)[::-1]
-    scale = max(abs(srt[kk - 1]), abs(srt[kk]), 1e-3 * np.abs(vals).max(), 1e-30)
-    return (srt[kk - 1] - srt[kk]) <= TIE_REL * scale
+    gap = srt[kk - 1] - srt[kk]
+    if gap <= TIE_REL * max(abs(srt[kk - 1]), abs(srt[kk]), 1e-30):
+        return TIE
+    if gap <= TIE_REL * 1e-3 * np.abs(vals).max():
+        return FLOOR_TIE
+    return NO_TIE
+
+
+def _gap_is_tie(vals, kk):
+    return tie_kind(vals, kk) != NO_TIE
 
 
 def tucker_core(cfg, t):
@@ -54,14 +78,19 @@ def head_scores(cfg, t, b, h):
 
 
 def near_tie(cfg, t, b, h):
+    """The kind of near-tie (NO_TIE / TIE / FLOOR_TIE) at the head's decision
+    boundaries: either axis' k-th/(k+1)-th rank-1 score, or the survivors'
+    m-th/(m+1)-th grid score."""
     k, m = int(cfg["topk"]), int(cfg["topm"])
     s_row, s_col, a, bb = head_scores(cfg, t, b, h)
-    if _gap_is_tie(a, k) or _gap_is_tie(bb, k):
-        return True
+    kinds = [tie_kind(a, k), tie_kind(bb, k)]
     I = np.argsort(-a, kind="stable")[:k]
     J = np.argsort(-bb, kind="stable")[:k]
     G = grid(cfg, t, h, s_row[:, I], s_col[:, J])
-    return _gap_is_tie(G.ravel(), m)
+    kinds.append(tie_kind(G.ravel(), m))
+    if TIE in kinds:
+        return TIE
+    return FLOOR_TIE if FLOOR_TIE in kinds else NO_TIE
 
 
 def grid(cfg, t, h, s_row, s_col):
@@ -83,12 +112,36 @@ def slot_scores(cfg, t, b, h, v):
     return np.einsum("an,ab,bn->n", s_row[:, i], C, s_col[:, j])
 
 
+def output_errors(got, ref):
+    """Per-token output errors: (element-wise with the floor, normwise)."""
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    peak = np.abs(ref).max(axis=1, keepdims=True)
+    den = np.maximum(np.abs(ref), np.maximum(OUT_FLOOR * peak, 1e-30))
+    diff = np.abs(got - ref)
+    elem = (diff / den).max(axis=1)
+    norm = diff.max(axis=1) / np.maximum(peak[:, 0], 1e-30)
+    return elem, norm
+
+
+class Result(tuple):
+    """(excused heads, element-wise output error), with the normwise error
+    and the count of heads excused only through the floor as attributes."""
+
+    def __new__(cls, excused, err, err_norm, floor_ties):
+        r = super().__new__(cls, (excused, err))
+        r.excused, r.err, r.err_norm, r.floor_ties = excused, err, err_norm, floor_ties
+        return r
+
+
 def compare(cfg, t, tokens, gpu_out, gpu_idx, gpu_w, ora_out, ora_idx, ora_w):
     """Asserts parity for the listed tokens.  gpu_* are indexed by token id,
-    ora_* by position in ``tokens``.  Returns (excused heads, max out error)."""
+    ora_* by position in ``tokens``.  Returns a Result: (excused heads, max
+    element-wise output error), .err_norm, .floor_ties."""
     H = int(cfg["heads"])
     excused_pos = []
     n_excused = 0
+    floor_ties = 0
     for e, b in enumerate(tokens):
         tok_excused = False
         for h in range(H):
@@ -100,8 +153,9 @@ def compare(cfg, t, tokens, gpu_out, gpu_idx, gpu_w, ora_out, ora_idx, ora_w):
                 assert np.abs(gw - ow).max() <= lim, \
                     f"weights differ at token {b} head {h}: {np.abs(gw - ow).max()} > {lim}"
                 continue
-            assert near_tie(cfg, t, b, h), \
-                f"selected slots differ at token {b} head {h} without a near-tie"
+            kind = near_tie(cfg, t, b, h)
+            assert kind != NO_TIE, f"selected slots differ at token {b} head {h} without a near-tie"
+            floor_ties += kind == FLOOR_TIE
             ref = np.sort(slot_scores(cfg, t, b, h, oi))[::-1]
             got = slot_scores(cfg, t, b, h, gi)
             assert len(set(gi.tolist())) == gi.size, "duplicate slot selected"
@@ -117,12 +171,13 @@ def compare(cfg, t, tokens, gpu_out, gpu_idx, gpu_w, ora_out, ora_idx, ora_w):
         tok = np.asarray(tokens)[excused_pos]
         ref[excused_pos] = oracle.lookup_reduce(cfg, t, gpu_idx[tok], gpu_w[tok].astype(np.float64))
     got = np.asarray(gpu_out, np.float64)[np.asarray(tokens)]
-    den = np.maximum(np.abs(ref).max(axis=1), 1e-30)
-    err = (np.abs(got - ref).max(axis=1) / den)
+    err, err_norm = output_errors(got, ref)
     tol = out_tol(cfg)
     worst = int(np.argmax(err))
-    assert err.max() <= tol, f"output error {err.max():.3g} > {tol} at token {tokens[worst]}"
-    return n_excused, float(err.max())
+    assert err.max() <= tol, \
+        f"element-wise output error {err.max():.3g} > {tol} at token {tokens[worst]} " \
+        f"(normwise {err_norm[worst]:.3g})"
+    return Result(n_excused, float(err.max()), float(err_norm.max()), floor_ties)
 
 
 def numpy_inputs(cfg, weights, x):

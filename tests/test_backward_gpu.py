@@ -11,17 +11,21 @@ from tests import parity
 
 pytestmark = pytest.mark.gpu
 
-TOL = 1e-4   # of the largest magnitude of each gradient (fp32 accumulation)
-# dW_p on the tensor cores (bf16 layers) reads the pooled rows rounded to
-# bf16, as the forward's projection does: one rounding, 2^-8 relative
-TOL_DW_BF16 = 2.0 ** -8
+# The rule of the outputs, element-wise with a floor, at the storage's
+# tolerance (1e-4 fp32, 2e-2 bf16); and, for every storage, the normwise
+# error of each gradient within 1e-4 of its largest entry.
+NORM_TOL = 1e-4
 
 
-def _check(got, want, what, tol=TOL):
-    got = np.asarray(got, np.float64)
-    scale = max(np.abs(want).max(), 1e-30)
-    err = np.abs(got - want).max() / scale
-    assert err <= tol, f"{what}: {err:.3g}"
+def _check(got, want, what, cfg):
+    """max_e |got - want| / max(|want_e|, 1e-3 max |want|) over the whole
+    gradient, and max_e |got - want| / max |want|."""
+    got = np.asarray(got, np.float64).reshape(1, -1)
+    want = np.asarray(want, np.float64).reshape(1, -1)
+    err, norm = parity.output_errors(got, want)
+    tol = parity.out_tol(cfg)
+    assert err.max() <= tol, f"{what}: element-wise {err.max():.3g} > {tol}"
+    assert norm.max() <= NORM_TOL, f"{what}: normwise {norm.max():.3g} > {NORM_TOL}"
 
 
 def _run(cfg, B, repeat=False, bad=False):
@@ -53,12 +57,12 @@ def _run(cfg, B, repeat=False, bad=False):
         assert st == 0
     o_dv, o_dw, o_dwp = oracle.lookup_reduce_backward(cfg, t, idx_n, w_n,
                                                       workloads.stored_numpy(g))
-    _check(dv.cpu().numpy(), o_dv, "dV")
+    _check(dv.cpu().numpy(), o_dv, "dV", cfg)
     if bad:   # the skipped slot's dw is 0 on the GPU
         o_dw[B - 1, 0, 1] = 0.0
-    _check(dw.cpu().numpy(), o_dw, "dw")
+    _check(dw.cpu().numpy(), o_dw, "dw", cfg)
     if dwp is not None:
-        _check(dwp.cpu().numpy(), o_dwp, "dW_p", TOL_DW_BF16 if int(cfg["dtype"]) else TOL)
+        _check(dwp.cpu().numpy(), o_dwp, "dW_p", cfg)
     return layer
 
 
@@ -96,6 +100,7 @@ def test_backward_decode_1m(gpu_lib):
 @pytest.mark.parametrize("B", [256, 260])
 def test_backward_many_tokens(B, gpu_lib):
     """256 tokens take the tensor-core dW_p (tokens on K, both operands
-    transposed); 260 (not a multiple of 8) the CUDA-core one."""
+    transposed, the pooled rows as two bf16 terms); 260 (not a multiple of
+    8) the CUDA-core one."""
     layer = _run(workloads.layer_config("decode_1m"), B)
-    assert layer.last_launches() == (7 if B % 8 == 0 else 5)
+    assert layer.last_launches() == (8 if B % 8 == 0 else 5)
