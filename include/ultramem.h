@@ -288,6 +288,29 @@ const char *ultramem_last_error(void);
 /* Human-readable name of a status code. */
 const char *ultramem_status_string(ultramem_status s);
 
+/* Failure-path hooks for tests; they inject failures on the host or behind
+ * a bounded wait, never a device fault.
+ *
+ * ultramem_debug_wait_probe: arms the layer's next forward (tensor-core
+ * path, bf16 storage; ULTRAMEM_EINVAL for other layers) so that its scoring
+ * kernel, after its dependency wait and before it issues any copy or MMA or
+ * takes tensor memory, waits on an mbarrier that nothing signals, with a
+ * limit of a few thousand SM cycles instead of the usual ~1 s.  The wait
+ * gives up, the kernel records ULTRAMEM_ETIMEOUT in the layer's error word
+ * and returns; the rest of that forward runs on stale scores and its output
+ * is meaningless.  ultramem_check then returns ULTRAMEM_ETIMEOUT once; the
+ * hook disarms itself after one forward.
+ *
+ * ultramem_debug_fail_alloc: the nth device allocation (0-based, counted
+ * from this call, over all layers of the process) that the library makes
+ * fails as if the device were out of memory, without calling the allocator;
+ * a negative n disarms.  ultramem_debug_live_allocations returns how many
+ * device allocations the library holds (every live layer's workspace), so a
+ * test can check that a failed create releases everything it took. */
+ultramem_status ultramem_debug_wait_probe(ultramem_layer *layer);
+void ultramem_debug_fail_alloc(int32_t nth);
+int32_t ultramem_debug_live_allocations(void);
+
 /* ABI version, currently 2. */
 int32_t ultramem_version(void);
 

@@ -27,7 +27,9 @@ EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
            "ultramem_profile_read", "ultramem_stage_name", "ultramem_status_string",
            "ultramem_last_error", "ultramem_version", "ultramem_lookup_reduce_noalloc",
            "ultramem_last_launches", "ultramem_forward_seq", "ultramem_key_ln",
-           "ultramem_retrieve_exact", "ultramem_lookup_reduce_backward")
+           "ultramem_retrieve_exact", "ultramem_lookup_reduce_backward",
+           "ultramem_debug_wait_probe", "ultramem_debug_fail_alloc",
+           "ultramem_debug_live_allocations")
 
 
 class Config(C.Structure):
@@ -109,6 +111,12 @@ def load(path: str | None = None) -> C.CDLL:
         lib.ultramem_last_error.restype = C.c_char_p
         lib.ultramem_version.argtypes = []
         lib.ultramem_version.restype = I32
+        lib.ultramem_debug_wait_probe.argtypes = [P]
+        lib.ultramem_debug_wait_probe.restype = I32
+        lib.ultramem_debug_fail_alloc.argtypes = [I32]
+        lib.ultramem_debug_fail_alloc.restype = None
+        lib.ultramem_debug_live_allocations.argtypes = []
+        lib.ultramem_debug_live_allocations.restype = I32
         _lib = lib
         return lib
 

@@ -6,6 +6,7 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <atomic>
 #include <new>
 
 #include "um_internal.cuh"
@@ -64,6 +65,7 @@ struct ultramem_layer {
     int host_graph_next = 0;
     cudaStream_t capture = nullptr;
     bool x_after_copy = false;   // x is written by the copy kernel just before the forward
+    bool probe_armed = false;    // ultramem_debug_wait_probe: the next forward's score probes
     bool dacc_tc = false;        // the backward's dacc may run on the tensor cores
 };
 
@@ -264,9 +266,33 @@ void shuffle_params(uint64_t seed, uint64_t M, uint64_t *a, uint64_t *c) {
     *c = o2 % M;
 }
 
+// Every device allocation of the library goes through lib_malloc / lib_free:
+// they count the live allocations and serve the allocation-failure hook of
+// ultramem_debug_fail_alloc (countdown < 0: disarmed).
+std::atomic<int> g_live_allocs{0};
+std::atomic<int> g_fail_countdown{-1};
+
+cudaError_t lib_malloc(void **p, size_t bytes) {
+    *p = nullptr;
+    int c = g_fail_countdown.load();
+    while (c >= 0 && !g_fail_countdown.compare_exchange_weak(c, c - 1)) {
+    }
+    if (c == 0) return cudaErrorMemoryAllocation;   // the armed allocation fails
+    const cudaError_t e = cudaMalloc(p, bytes);
+    if (e == cudaSuccess) ++g_live_allocs;
+    return e;
+}
+
+void lib_free(void *p) {
+    if (p && cudaFree(p) == cudaSuccess) --g_live_allocs;
+}
+
 template <typename T> cudaError_t dalloc(T **p, size_t n) {
     if (n == 0) n = 1;
-    return cudaMalloc(reinterpret_cast<void **>(p), n * sizeof(T));
+    void *v = nullptr;
+    const cudaError_t e = lib_malloc(&v, n * sizeof(T));
+    *p = static_cast<T *>(v);
+    return e;
 }
 
 void free_workspace(Workspace &ws) {
@@ -274,8 +300,7 @@ void free_workspace(Workspace &ws) {
                     ws.sel_row, ws.sel_p, ws.core,   ws.u,         ws.t,
                     ws.err,    ws.x_stage, ws.out_stage, ws.qs,     ws.acc_bf,
                     ws.w_pt,   ws.cores,   ws.xs,      ws.dacc,    ws.bwd_t};
-    for (void *p : ptrs)
-        if (p) cudaFree(p);
+    for (void *p : ptrs) lib_free(p);
     ws = Workspace();
 }
 
@@ -413,6 +438,8 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     // waits for all earlier work on the stream.
     Dims dd = d;
     dd.pdl = L->profiling ? 0 : 1;
+    dd.probe_wait = L->probe_armed ? 1 : 0;
+    L->probe_armed = false;   // one forward only
     // Trick 4: the convolution runs first and the query projection reads its
     // output (fp32 for the CUDA-core query, three bf16 terms for the tensor
     // cores); with Trick 2 the LayerNorm writes the scaled splits
@@ -626,11 +653,11 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     if (e == cudaSuccess) e = dalloc(&ws.t, (size_t)H * r);
     if (e == cudaSuccess) e = dalloc(&ws.err, 1);
     if (e == cudaSuccess)
-        e = cudaMalloc(&ws.x_stage, Bm * cfg->d_in * elt_size(*cfg));
+        e = lib_malloc(&ws.x_stage, Bm * cfg->d_in * elt_size(*cfg));
     if (e == cudaSuccess)
-        e = cudaMalloc(&ws.out_stage, Bm * cfg->d_out * elt_size(*cfg));
+        e = lib_malloc(&ws.out_stage, Bm * cfg->d_out * elt_size(*cfg));
     // the convolved input: three bf16 terms (tensor path) or fp32, 6 B a value covers both
-    if (e == cudaSuccess && cfg->conv_k > 0) e = cudaMalloc(&ws.xs, Bm * cfg->d_in * 6);
+    if (e == cudaSuccess && cfg->conv_k > 0) e = lib_malloc(&ws.xs, Bm * cfg->d_in * 6);
     if (e == cudaSuccess)
         e = cudaMemcpy(ws.core, hc, sizeof(float) * H * r * r, cudaMemcpyHostToDevice);
     if (e == cudaSuccess && nc > 1)
@@ -973,6 +1000,16 @@ ultramem_status ultramem_check(ultramem_layer *L, void *stream) {
     if (flags & (um::kErrBadIndex | um::kErrInternal)) return ULTRAMEM_EDEVICE;
     return ULTRAMEM_OK;
 }
+
+ultramem_status ultramem_debug_wait_probe(ultramem_layer *L) {
+    if (!L || !L->tc) return ULTRAMEM_EINVAL;
+    L->probe_armed = true;
+    return ULTRAMEM_OK;
+}
+
+void ultramem_debug_fail_alloc(int32_t nth) { g_fail_countdown.store(nth < 0 ? -1 : nth); }
+
+int32_t ultramem_debug_live_allocations(void) { return g_live_allocs.load(); }
 
 ultramem_status ultramem_profile_enable(ultramem_layer *L, int32_t enable) {
     if (!L) return ULTRAMEM_EINVAL;

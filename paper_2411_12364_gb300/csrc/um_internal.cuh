@@ -55,6 +55,8 @@ struct Dims {
     int q_splits, p_splits;
     int pdl;           // host side: launch as a programmatic dependent of the
                        // previous kernel on the stream
+    int probe_wait;    // ultramem_debug_wait_probe: the scoring kernel's
+                       // bounded wait on a barrier nothing signals
 };
 
 struct Ptrs {

@@ -60,15 +60,32 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Waits for the phase of `parity` to complete; gives up after
-// kWaitLimitCycles of this SM's clock and returns false (the caller records
-// the timeout and unwinds).  The SM cycle counter is cheap to read, so a
-// completed phase is noticed at once.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
+// Waits for the phase of `parity` to complete; gives up after `limit`
+// (default kWaitLimitCycles) cycles of this SM's clock and returns false (the
+// caller records the timeout and unwinds).  The SM cycle counter is cheap to
+// read, so a completed phase is noticed at once.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
+                                          long long limit = kWaitLimitCycles) {
     if (mbar_try_wait(bar, parity)) return true;
     const long long start = clock64();
     while (!mbar_try_wait(bar, parity))
-        if (clock64() - start > kWaitLimitCycles) return false;
+        if (clock64() - start > limit) return false;
+    return true;
+}
+
+// The failure-path probe of ultramem_debug_wait_probe: after the dependency
+// wait and before anything is issued, thread 0 waits on a fresh mbarrier
+// that nothing arrives on, with a short limit; it gives up, the kernel's
+// error word records the timeout, and the caller's CTA returns with nothing
+// in flight.  Returns true when the CTA must return.
+constexpr long long kProbeLimitCycles = 4096;
+__device__ __forceinline__ bool probe_timeout(uint64_t *never, int *err, int err_bit) {
+    if (threadIdx.x == 0) {
+        mbar_init(never, 1);
+        fence_mbar_init();
+        if (!mbar_wait(never, 0, kProbeLimitCycles)) atomicOr(err, err_bit);
+    }
+    __syncthreads();
     return true;
 }
 

@@ -67,9 +67,9 @@ template <int NSPLIT, class Op>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0,
                    const __grid_constant__ CUtensorMap mapA1,
-                   const __grid_constant__ CUtensorMap mapB, Op op) {
+                   const __grid_constant__ CUtensorMap mapB, Op op, int probe) {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full[kMaxStages], empty[kMaxStages], accbar;
+    __shared__ __align__(8) uint64_t full[kMaxStages], empty[kMaxStages], accbar, never;
     __shared__ uint32_t tmem_slot;
     uint8_t *ring = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -96,6 +96,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         prefetch_tensormap(&mapB);
     }
     __syncthreads();
+    if (probe) {   // ultramem_debug_wait_probe: a bounded wait that runs out
+        pdl_wait();
+        if (probe_timeout(&never, op.err, kErrTimeout)) return;
+    }
 
     // The A operand is a weight: the first ring stages of it are requested
     // before the dependency wait, so that under programmatic dependent
@@ -275,10 +279,10 @@ __global__ void __launch_bounds__(kPThreads, 1)
     tc_gemm_persistent(const __grid_constant__ CUtensorMap mapA0,
                        const __grid_constant__ CUtensorMap mapA1,
                        const __grid_constant__ CUtensorMap mapB, Op op, int gx, int gy,
-                       int tiles, uint32_t buf_cols) {
+                       int tiles, uint32_t buf_cols, int probe) {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full[kMaxStages], empty[kMaxStages], tfull[2], tempty[2],
-        drained;
+        drained, never;
     __shared__ uint32_t tmem_slot;
     __shared__ volatile int abort_flag;
     uint8_t *ring = reinterpret_cast<uint8_t *>(
@@ -310,6 +314,10 @@ __global__ void __launch_bounds__(kPThreads, 1)
         prefetch_tensormap(&mapB);
     }
     pdl_wait();
+    if (probe) {   // ultramem_debug_wait_probe: a bounded wait that runs out
+        __syncthreads();
+        if (probe_timeout(&never, op.err, kErrTimeout)) return;
+    }
     if (warp == 0) tmem_alloc(&tmem_slot, 2 * buf_cols);
     tc_fence_before();
     __syncthreads();
@@ -800,7 +808,7 @@ static bool persistent_ok(dim3 grid, const Op &op) {
 template <int NSPLIT, class Op>
 static cudaError_t launch_gemm_persistent(dim3 grid, const CUtensorMap &a0, const CUtensorMap &a1,
                                           const CUtensorMap &b, Op op, int nkb, bool pdl,
-                                          cudaStream_t st) {
+                                          cudaStream_t st, int probe) {
     (void)nkb;   // the ring runs across tiles: as many stages as fit
     op.stages = stages_for(NSPLIT, op.n_tile, kMaxStages);
     const size_t smem = 1024 + (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile);
@@ -808,7 +816,7 @@ static cudaError_t launch_gemm_persistent(dim3 grid, const CUtensorMap &a0, cons
     const int ctas = tiles < sm_count() ? tiles : sm_count();
     return launch_kernel(pdl, tc_gemm_persistent<NSPLIT, Op>, dim3(ctas), kPThreads, smem, st, a0,
                          a1, b, op, (int)grid.x, (int)grid.y, tiles,
-                         buf_cols_of(op.n_acc, op.n_tile));
+                         buf_cols_of(op.n_acc, op.n_tile), probe);
 }
 
 // grid.z = the split count (S1, S9; also the cluster's z extent when > 1) or
@@ -816,14 +824,14 @@ static cudaError_t launch_gemm_persistent(dim3 grid, const CUtensorMap &a0, cons
 template <int NSPLIT, class Op>
 static cudaError_t launch_gemm(dim3 grid, const CUtensorMap &a0, const CUtensorMap &a1,
                                const CUtensorMap &b, Op op, int nkb, bool pdl,
-                               cudaStream_t st) {
+                               cudaStream_t st, int probe = 0) {
     if (persistent_ok<NSPLIT>(grid, op))
-        return launch_gemm_persistent<NSPLIT>(grid, a0, a1, b, op, nkb, pdl, st);
+        return launch_gemm_persistent<NSPLIT>(grid, a0, a1, b, op, nkb, pdl, st, probe);
     op.stages = stages_for(NSPLIT, op.n_tile, nkb);
     size_t ring = (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile);
     const size_t smem = 1024 + ring;
     return launch_kernel(pdl, grid.z > 1 ? grid.z : 1u, tc_gemm_kernel<NSPLIT, Op>, grid,
-                         kThreads, smem, st, a0, a1, b, op);
+                         kThreads, smem, st, a0, a1, b, op, probe);
 }
 
 template <int NSPLIT, class Op> static cudaError_t allow_smem() {
@@ -935,7 +943,8 @@ cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cuda
     op.kb_total = (d.d_k + kBlockK - 1) / kBlockK;
     op.akey = p.akey;
     dim3 grid((d.K + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 2 * d.H);
-    return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs, op, op.kb_total, d.pdl, st);
+    return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs, op, op.kb_total, d.pdl, st,
+                          d.probe_wait);
 }
 
 cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
