@@ -61,6 +61,8 @@ def parse():
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true",
+                    help="skip the further workloads (mid_4m, large_20m, prefill_16k)")
     return ap.parse_args()
 
 
@@ -227,7 +229,7 @@ def run_reference(args, cfg, B, wl):
     wn = numpy_weights(w)
     import oracle
     cores = len(os.sched_getaffinity(0))
-    sample = min(B, 8)      # tokens per step: a bounded slice of the batch
+    sample = B              # tokens per step: the whole batch of the workload
     for i in range(args.warmup):
         x = workloads.stored_numpy(workloads.make_tokens(cfg, sample, 2000 + i))
         oracle.forward(cfg, dict(wn, x=x), sample, threads=cores)
@@ -248,7 +250,8 @@ def run_reference(args, cfg, B, wl):
             "data": "synthetic", "config": dict(workload=wl, batch=B, **_cfg_brief(cfg)),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores,
                              "kind": "oracle",
-                             "sample": f"{sample} of the {B} tokens of a batch per step"},
+                             "sample": f"the whole batch ({sample} tokens) of the workload "
+                                       f"per step, fp64, OpenMP over tokens"},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -324,6 +327,178 @@ def _cfg_brief(cfg):
     return d
 
 
+def stage_profile(layer, fwd, stream, flush, K, use_graph, NB):
+    """Device time of each stage (kernels of the stage: first CTA past its
+    dependency wait to last warp done, from the kernels' own global-timer
+    stamps) and the hand-off before it, averaged over K forwards replayed
+    exactly as the timed ones (graphs, programmatic dependent launches, L2
+    flushed between forwards)."""
+    import torch
+    layer.profile(True)
+    graphs = []
+    with torch.cuda.stream(stream):
+        fwd(0)
+        torch.cuda.synchronize()
+        for i in range(NB if use_graph else 0):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                fwd(i)
+            graphs.append(g)
+    torch.cuda.synchronize()
+    times, gaps = {}, {}
+    with torch.cuda.stream(stream):
+        for i in range(K):
+            flush.fill_(float(i))
+            if use_graph:
+                graphs[i % NB].replay()
+            else:
+                fwd(i)
+            torch.cuda.synchronize()
+            t, g = layer.profile_read(gaps=True)
+            for k, v in t.items():
+                times.setdefault(k, []).append(v)
+            for k, v in g.items():
+                gaps.setdefault(k, []).append(v)
+    torch.cuda.synchronize()
+    layer.profile(False)
+    del graphs
+    avg = lambda d: {k: sum(v) / len(v) for k, v in d.items() if min(v) >= 0}
+    return avg(times), avg(gaps)
+
+
+def cold_gather(layer, x, stream, flush, K):
+    """The gather kernel's device time with its value rows in HBM: the
+    forward's slots, pooled through ultramem_lookup_reduce (no selection
+    before it, so no row was prefetched into L2) after an L2 flush."""
+    import torch
+    with torch.cuda.stream(stream):
+        idx, w = layer.retrieve(x)
+        layer.lookup_reduce(idx, w)
+        torch.cuda.synchronize()
+        layer.profile(True)
+        ts = []
+        for i in range(K):
+            flush.fill_(float(i))
+            layer.lookup_reduce(idx, w)
+            torch.cuda.synchronize()
+            ts.append(layer.profile_read()["gather"])
+        layer.profile(False)
+    return sum(ts) / len(ts)
+
+
+def roofline_of(stages, alg, peak, peak_kind):
+    dominant = max(stages, key=stages.get)
+    ach = alg[dominant] / (stages[dominant] * 1e6)
+    return {"kernel": dominant, "bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
+            "frac": ach / peak, "peak_kind": peak_kind, "algorithmic_bytes": alg[dominant],
+            "avg_ms": stages[dominant],
+            "time_source": "kernel global-timer stamps in the replayed forward graph"}
+
+
+def gather_entry(alg, gms, cold_ms, peak):
+    """Gather GB/s: in the forward (its rows were prefetched into L2 by the
+    selection) and cold (rows from HBM after an L2 flush)."""
+    out = {"bytes": alg["gather"]}
+    if gms:
+        gbs = alg["gather"] / (gms * 1e6)
+        out.update(ms=gms, achieved_gbs=gbs, frac_of_measured=gbs / peak,
+                   frac_of_nominal_8tbs=gbs / NOMINAL_HBM_GBS)
+    if cold_ms:
+        cg = alg["gather"] / (cold_ms * 1e6)
+        out.update(cold_ms=cold_ms, cold_gbs=cg, cold_frac_of_measured=cg / peak,
+                   cold_frac_of_nominal_8tbs=cg / NOMINAL_HBM_GBS)
+    return out
+
+
+def time_steps(step, stream, flush, K, dist=None):
+    """K timed steps (CUDA events on the stream, an L2 flush after each,
+    outside the events); returns the mean ms per step."""
+    import torch
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for i in range(K):
+            ev[i][0].record(stream)
+            step(i)
+            ev[i][1].record(stream)
+            flush.fill_(float(i))
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    return sum(a.elapsed_time(b) for a, b in ev) / K
+
+
+def build_layer(cfg, B, rank, NB):
+    import torch
+    from paper_2411_12364_gb300 import workloads
+    from paper_2411_12364_gb300.binding import UltraMemLayer
+    w = workloads.make_weights(cfg, device="cuda")
+    layer = UltraMemLayer(cfg, w, B)
+    xs = [workloads.make_tokens(cfg, B, 100 * rank + i, device="cuda") for i in range(NB)]
+    return w, layer, xs
+
+
+def capture(layer, fwd, stream, NB):
+    import torch
+    graphs = []
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            fwd(0)
+        torch.cuda.synchronize()
+        for i in range(NB):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                fwd(i)
+            graphs.append(g)
+    torch.cuda.synchronize()
+    return graphs
+
+
+SWEEP = [("mid_4m", (128,)), ("large_20m", (64, 256)), ("prefill_16k", (16384,))]
+
+
+def sweep_workload(wl, batches, K, flush, stream, peak, peak_kind):
+    """Further batches of one workload (one table): step time, tokens/s,
+    per-stage device times, the gather's GB/s and the dominant kernel's
+    roofline, measured like the headline line (graph replays, L2 flushed
+    between steps)."""
+    import torch
+    from paper_2411_12364_gb300 import workloads
+    cfg = workloads.layer_config(wl)
+    NB = 2
+    w, layer, xs_all = build_layer(cfg, max(batches), 0, NB)
+    res = []
+    for B in batches:
+        xs = [x[:B].contiguous() for x in xs_all]
+        out = torch.empty((B, cfg["d_out"]), dtype=layer.dtype, device="cuda")
+        fwd = lambda i: layer.forward(xs[i % NB], out=out)
+        graphs = capture(layer, fwd, stream, NB)
+        big = B >= 4096
+        steps, warm = (5, 2) if big else (max(5, min(K, 30)), 3)
+        with torch.cuda.stream(stream):
+            for i in range(warm):
+                graphs[i % NB].replay()
+                flush.fill_(float(i))
+        ms = time_steps(lambda i: graphs[i % NB].replay(), stream, flush, steps)
+        del graphs
+        stages, gaps = stage_profile(layer, fwd, stream, flush, 3 if big else 20, True, NB)
+        cold = cold_gather(layer, xs[0], stream, flush, 3 if big else 10)
+        alg = algorithmic_bytes(cfg, B)
+        res.append({"workload": wl, "batch": B, "steps": steps, "ms_per_step": ms,
+                    "tokens_per_s": B / (ms / 1e3), "stages_ms": stages, "handoff_ms": gaps,
+                    "roofline": roofline_of(stages, alg, peak, peak_kind),
+                    "gather": gather_entry(alg, stages.get("gather"), cold, peak),
+                    "step_hbm_gbs": sum(alg.values()) / (ms * 1e6)})
+        del xs, out
+    layer.close()
+    del layer, w, xs_all
+    torch.cuda.empty_cache()
+    return res
+
+
 def main():
     args = parse()
     from paper_2411_12364_gb300 import workloads
@@ -350,12 +525,9 @@ def main():
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl")
-    from paper_2411_12364_gb300.binding import UltraMemLayer
 
-    w = workloads.make_weights(cfg, device="cuda")
-    layer = UltraMemLayer(cfg, w, B)
     NB = 8     # distinct token batches cycled through (per rank)
-    xs = [workloads.make_tokens(cfg, B, 100 * rank + i, device="cuda") for i in range(NB)]
+    w, layer, xs = build_layer(cfg, B, rank, NB)
     out = torch.empty((B, cfg["d_out"]), dtype=layer.dtype, device="cuda")
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
     kc = int(cfg.get("conv_k", 0))
@@ -372,21 +544,13 @@ def main():
             layer.forward_seq(xs[i % NB], n_seq, states[i % 2], states[(i + 1) % 2], out=out)
 
     stream = torch.cuda.Stream()
-
     use_graph = not args.no_graph
-    graphs = []
     with torch.cuda.stream(stream):
         for i in range(3):
             fwd(0)
         torch.cuda.synchronize()
-        launches = layer.last_launches()   # kernels per forward (and per graph replay)
-        if use_graph:
-            for i in range(NB):
-                g = torch.cuda.CUDAGraph()
-                with torch.cuda.graph(g, stream=stream):
-                    fwd(i)
-                graphs.append(g)
-    torch.cuda.synchronize()
+    launches = layer.last_launches()   # kernels per forward (and per graph replay)
+    graphs = capture(layer, fwd, stream, NB) if use_graph else []
 
     def step(i):
         if use_graph:
@@ -402,71 +566,23 @@ def main():
 
     # ---- timed region ----------------------------------------------------
     K = args.steps
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(K)]
     clocks = Clocks(local, enabled=not args.no_clocks)
     time.sleep(0.3)
-    if dist:
-        dist.barrier()
-    torch.cuda.synchronize()
-    with torch.cuda.stream(stream):
-        for i in range(K):
-            ev[i][0].record(stream)
-            step(i)
-            ev[i][1].record(stream)
-            flush.fill_(float(i))
-    torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
+    step_ms = time_steps(step, stream, flush, K, dist)
     clk = clocks.stop()
-    total_ms = sum(a.elapsed_time(b) for a, b in ev)
-    ms, value = aggregate_step(total_ms / K, B, dist, device="cuda")
+    ms, value = aggregate_step(step_ms, B, dist, device="cuda")
+    del graphs
 
-    # ---- per-stage device times: the forward with the layer's stage events
-    # captured in a graph too, so the events see the kernels back to back ----
-    layer.profile(True)
-    pgraphs = []
-    with torch.cuda.stream(stream):
-        fwd(0)
-        torch.cuda.synchronize()
-        for i in range(NB if use_graph else 0):
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=stream):
-                fwd(i)
-            pgraphs.append(g)
-    torch.cuda.synchronize()
-    stage_ms = {}
-    with torch.cuda.stream(stream):
-        for i in range(K):
-            if use_graph:
-                pgraphs[i % NB].replay()
-            else:
-                fwd(i)
-            torch.cuda.synchronize()
-            for k, v in layer.profile_read().items():
-                stage_ms.setdefault(k, []).append(v)
-            flush.fill_(float(i))
-    torch.cuda.synchronize()
-    layer.profile(False)
-    del pgraphs
-    stage_avg = {k: sum(v) / len(v) for k, v in stage_ms.items()}
+    # ---- per-stage device times from the kernels' own stamps -------------
+    stages, gaps = stage_profile(layer, fwd, stream, flush, min(K, 50), use_graph, NB)
+    cold = cold_gather(layer, xs[0], stream, flush, 10) if states is None else None
     alg = algorithmic_bytes(cfg, B)
     peak, peak_kind = peaks()
-    dominant = max(stage_avg, key=stage_avg.get)
-    dom_bytes = alg[dominant]
-    roof = {"kernel": dominant, "bound": "hbm", "achieved": dom_bytes / (stage_avg[dominant] * 1e6),
-            "peak": peak, "unit": "GB/s", "peak_kind": peak_kind,
-            "traffic": None if int(cfg.get("cores", 0)) > 1 else ncu_traffic(dominant, wl, B),
-            "algorithmic_bytes": dom_bytes,
-            "avg_ms": stage_avg[dominant]}
-    roof["frac"] = roof["achieved"] / peak
-    gms = stage_avg.get("gather")
-    gather = None
-    if gms:
-        gbs = alg["gather"] / (gms * 1e6)
-        gather = {"achieved_gbs": gbs, "ms": gms, "bytes": alg["gather"],
-                  "frac_of_measured": gbs / peak, "frac_of_nominal_8tbs": gbs / NOMINAL_HBM_GBS,
-                  "traffic": ncu_traffic("gather", wl, B)}
+    roof = roofline_of(stages, alg, peak, peak_kind)
+    roof["traffic"] = None if int(cfg.get("cores", 0)) > 1 else \
+        ncu_traffic(roof["kernel"], wl, B)
+    gather = gather_entry(alg, stages.get("gather"), cold, peak)
+    gather["traffic"] = ncu_traffic("gather", wl, B)
 
     # ---- end to end through the public API with host buffers -------------
     xh = [x.cpu().pin_memory() for x in xs]
@@ -492,9 +608,15 @@ def main():
     if args.backward and rank == 0:
         backward = measure_backward(layer, xs[0], cfg, stream, K, flush)
 
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(cfg, numpy_weights(w), B)
+    wn = numpy_weights(w) if rank == 0 and world == 1 and not args.no_cpu_baseline else None
+    sweep = None
+    if world == 1 and not args.no_sweep and args.workload is None and not over:
+        layer.close()
+        del layer, w, xs, xh, out
+        torch.cuda.empty_cache()
+        sweep = [r for swl, bs in SWEEP
+                 for r in sweep_workload(swl, bs, K, flush, stream, peak, peak_kind)]
+    cpu = cpu_baseline(cfg, wn, B) if wn is not None else None
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
@@ -504,9 +626,12 @@ def main():
                 "config": dict(workload=wl, batch=B, **_cfg_brief(cfg), accumulate="f32",
                                l2="flushed between steps (256 MiB write, outside timing)",
                                cuda_graph=use_graph, parallelism=f"replicas x{world}"),
-                "roofline": roof, "gather": gather, "stages_ms": stage_avg,
+                "roofline": roof, "gather": gather, "stages_ms": stages, "handoff_ms": gaps,
+                "step_hbm_gbs": sum(alg.values()) / (ms * 1e6),
                 "gpu_launches": K * launches, "e2e": e2e,
                 "cpu_baseline": cpu, "clocks": clk}
+        if sweep is not None:
+            line["sweep"] = sweep
         if recall is not None:
             line["recall"] = recall
         if backward is not None:

@@ -346,10 +346,17 @@ class UltraMemLayer:
     def profile(self, enable: bool = True):
         _check(self.lib.ultramem_profile_enable(self._h, int(enable)), "profile_enable")
 
-    def profile_read(self) -> dict:
-        buf = (C.c_float * 8)()
-        n = self.lib.ultramem_profile_read(self._h, buf, 8)
-        return {self.lib.ultramem_stage_name(i).decode(): float(buf[i]) for i in range(n)}
+    def profile_read(self, gaps: bool = False):
+        """Device time (ms) of each stage of the most recent profiled
+        forward; with ``gaps`` also the hand-off before each stage."""
+        buf = (C.c_float * 10)()
+        n = self.lib.ultramem_profile_read(self._h, buf, 10)
+        ns = min(n, 5)
+        names = [self.lib.ultramem_stage_name(i).decode() for i in range(ns)]
+        times = {names[i]: float(buf[i]) for i in range(ns)}
+        if not gaps:
+            return times
+        return times, {names[i]: float(buf[5 + i]) for i in range(ns)} if n >= 10 else {}
 
     def close(self):
         if getattr(self, "_h", None):

@@ -32,6 +32,7 @@ struct Workspace {
     __nv_bfloat16 *bwd_t = nullptr;   // backward (tensor cores): acc^T [E*D_v][2 B] (two
                                       // bf16 terms), g^T [D'_v][B]
     __nv_bfloat16 *qs = nullptr, *acc_bf = nullptr, *w_pt = nullptr;   // tensor path
+    unsigned long long *stamps = nullptr;   // profiling: [kStampStages] begins, then ends
 };
 
 }  // namespace
@@ -46,7 +47,6 @@ struct ultramem_layer {
     um::TcMaps maps;     // weight descriptors of the tensor path
     bool profiling = false;
     bool profiled_once = false;
-    cudaEvent_t ev[kStages + 1] = {};
     int launches = 0;    // kernels launched by the most recent successful call
     bool exact_ok = false;   // the brute-force top-m fits this layer's grid
     bool backward_ok = false;   // the lookup-reduce backward fits this layer
@@ -299,7 +299,8 @@ void free_workspace(Workspace &ws) {
     void *ptrs[] = {ws.q_part, ws.akey, ws.sel_w,   ws.acc,       ws.proj_part,
                     ws.sel_row, ws.sel_p, ws.core,   ws.u,         ws.t,
                     ws.err,    ws.x_stage, ws.out_stage, ws.qs,     ws.acc_bf,
-                    ws.w_pt,   ws.cores,   ws.xs,      ws.dacc,    ws.bwd_t};
+                    ws.w_pt,   ws.cores,   ws.xs,      ws.dacc,    ws.bwd_t,
+                    ws.stamps};
     for (void *p : ptrs) lib_free(p);
     ws = Workspace();
 }
@@ -353,16 +354,21 @@ ultramem_status from_cuda(cudaError_t e) {
     return ULTRAMEM_ECUDA;
 }
 
-// Stage events; under stream capture they must be external event nodes so
-// that every replay of the graph records them.
-void mark(ultramem_layer *L, int i, cudaStream_t st) {
-    if (!L->profiling) return;
-    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-    cudaStreamIsCapturing(st, &cs);
-    if (cs == cudaStreamCaptureStatusActive)
-        cudaEventRecordWithFlags(L->ev[i], st, cudaEventRecordExternal);
-    else
-        cudaEventRecord(L->ev[i], st);
+// Profiling: the stage stamps are reset before the forward (begins to the
+// largest value, ends to 0; memset nodes under stream capture) and each
+// kernel gets the pair of its stage.
+cudaError_t reset_stamps(ultramem_layer *L, cudaStream_t st) {
+    if (!L->profiling) return cudaSuccess;
+    unsigned long long *s = L->ws.stamps;
+    cudaError_t e = cudaMemsetAsync(s, 0xff, sizeof(*s) * um::kStampStages, st);
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(s + um::kStampStages, 0, sizeof(*s) * um::kStampStages, st);
+    return e;
+}
+Ptrs stage_ptrs(const ultramem_layer *L, const Ptrs &p, int stage) {
+    Ptrs q = p;
+    q.stamp = L->profiling ? L->ws.stamps + stage : nullptr;
+    return q;
 }
 
 // What a call runs: the whole forward, S1..S6 (retrieval), or S1 and the
@@ -375,35 +381,32 @@ ultramem_status run_cuda_core(ultramem_layer *L, const Dims &d0, Ptrs p, cudaStr
     cudaError_t e;
     Dims d = d0;
     const int extras = (d.conv_k > 0) + d.query_ln;   // convolution, LayerNorm
-    mark(L, 0, st);
-    if (d.conv_k > 0 && (e = um::launch_query_conv(d, p, false, st)) != cudaSuccess)
+    if ((e = reset_stamps(L, st)) != cudaSuccess) return from_cuda(e);
+    const Ptrs p0 = stage_ptrs(L, p, 0);
+    if (d.conv_k > 0 && (e = um::launch_query_conv(d, p0, false, st)) != cudaSuccess)
         return from_cuda(e);
     {
-        Ptrs pq = p;
+        Ptrs pq = p0;
         if (d.conv_k > 0) pq.x = p.xs;   // the fp32 convolved rows
         if ((e = um::launch_query(d, pq, d.conv_k > 0, st)) != cudaSuccess) return from_cuda(e);
     }
     if (d.query_ln) {
-        if ((e = um::launch_query_ln(d, p, nullptr, 0, st)) != cudaSuccess) return from_cuda(e);
+        if ((e = um::launch_query_ln(d, p0, nullptr, 0, st)) != cudaSuccess) return from_cuda(e);
         d.q_splits = 1;   // the normalised query is split 0
     }
-    mark(L, 1, st);
     if (mode == kExact) {
         if ((e = um::launch_exact(d, p, p.idx_out, p.w_out, st)) != cudaSuccess)
             return from_cuda(e);
         *launches = 2 + extras;
         return ULTRAMEM_OK;
     }
-    if ((e = um::launch_score(d, p, st)) != cudaSuccess) return from_cuda(e);
-    mark(L, 2, st);
-    if ((e = um::launch_select(d, p, st)) != cudaSuccess) return from_cuda(e);
-    mark(L, 3, st);
+    if ((e = um::launch_score(d, stage_ptrs(L, p, 1), st)) != cudaSuccess) return from_cuda(e);
+    if ((e = um::launch_select(d, stage_ptrs(L, p, 2), st)) != cudaSuccess) return from_cuda(e);
     *launches = 3 + extras;
     if (mode == kRetrieve) return ULTRAMEM_OK;
-    if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
-    mark(L, 4, st);
-    if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
-    mark(L, 5, st);
+    if ((e = um::launch_gather(d, stage_ptrs(L, p, 3), st)) != cudaSuccess) return from_cuda(e);
+    if (d.has_proj && (e = um::launch_proj(d, stage_ptrs(L, p, 4), st)) != cudaSuccess)
+        return from_cuda(e);
     *launches = 4 + (d.has_proj ? 2 : 0) + extras;   // the projection and its split-K reduce
     if (L->profiling) L->profiled_once = true;
     return ULTRAMEM_OK;
@@ -431,35 +434,35 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     p.acc_bf = c.has_proj ? L->ws.acc_bf : nullptr;
     p.acc_terms = 2;
     cudaError_t e;
-    mark(L, 0, st);
+    if ((e = reset_stamps(L, st)) != cudaSuccess) return from_cuda(e);
     // Every kernel after the first is a programmatic dependent launch of its
-    // predecessor (not while profiling: the stage events sit between the
-    // kernels).  The first (the convolution, else the query projection)
-    // waits for all earlier work on the stream.
+    // predecessor (also while profiling: the stamps are written by the
+    // kernels themselves).  The first (the convolution, else the query
+    // projection) waits for all earlier work on the stream.
     Dims dd = d;
-    dd.pdl = L->profiling ? 0 : 1;
+    dd.pdl = 1;
     dd.probe_wait = L->probe_armed ? 1 : 0;
     L->probe_armed = false;   // one forward only
     // Trick 4: the convolution runs first and the query projection reads its
     // output (fp32 for the CUDA-core query, three bf16 terms for the tensor
     // cores); with Trick 2 the LayerNorm writes the scaled splits
     const bool small = d.B <= kSmallQueryBatch;
-    if (conv && (e = um::launch_query_conv(d, p, !small, st)) != cudaSuccess) return from_cuda(e);
+    const Ptrs p0 = stage_ptrs(L, p, 0);
+    if (conv && (e = um::launch_query_conv(d, p0, !small, st)) != cudaSuccess) return from_cuda(e);
     const bool write_qs = !d.query_ln;
     // a dependent of the convolution, or of the copy kernel that brings x in
     const bool qpdl = (conv || L->x_after_copy) && dd.pdl;
-    if ((e = small ? um::launch_query_small(d, p, L->ws.qs, Bmax, conv, write_qs, qpdl, st)
-                   : um::launch_query_tc(d, p, mp, d.q_splits, L->ws.qs, Bmax, conv, write_qs,
+    if ((e = small ? um::launch_query_small(d, p0, L->ws.qs, Bmax, conv, write_qs, qpdl, st)
+                   : um::launch_query_tc(d, p0, mp, d.q_splits, L->ws.qs, Bmax, conv, write_qs,
                                          qpdl, st)) != cudaSuccess)
         return from_cuda(e);
     if (d.query_ln) {
         Dims dl = dd;
         dl.q_splits = 1;   // the projection left the summed query in split 0
-        if ((e = um::launch_query_ln(dl, p, L->ws.qs, Bmax, st)) != cudaSuccess)
+        if ((e = um::launch_query_ln(dl, p0, L->ws.qs, Bmax, st)) != cudaSuccess)
             return from_cuda(e);
     }
     const int extras = conv + d.query_ln;
-    mark(L, 1, st);
     if (mode == kExact) {
         Dims dx = dd;
         dx.q_splits = 1;   // the summed query is split 0
@@ -468,18 +471,16 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
         *launches = d.A + 1 + extras;
         return ULTRAMEM_OK;
     }
-    if ((e = um::launch_score_tc(dd, p, mp, st)) != cudaSuccess) return from_cuda(e);
-    mark(L, 2, st);
+    if ((e = um::launch_score_tc(dd, stage_ptrs(L, p, 1), mp, st)) != cudaSuccess)
+        return from_cuda(e);
     Dims ds = dd;
     ds.q_splits = 1;   // the query projection wrote the summed query
-    if ((e = um::launch_select(ds, p, st)) != cudaSuccess) return from_cuda(e);
-    mark(L, 3, st);
+    if ((e = um::launch_select(ds, stage_ptrs(L, p, 2), st)) != cudaSuccess) return from_cuda(e);
     *launches = d.A + 2 + extras;   // one query projection per query
     if (mode == kRetrieve) return ULTRAMEM_OK;
-    if ((e = um::launch_gather(dd, p, st)) != cudaSuccess) return from_cuda(e);
-    mark(L, 4, st);
-    if (d.has_proj && (e = um::launch_proj_tc(dd, p, mp, st)) != cudaSuccess) return from_cuda(e);
-    mark(L, 5, st);
+    if ((e = um::launch_gather(dd, stage_ptrs(L, p, 3), st)) != cudaSuccess) return from_cuda(e);
+    if (d.has_proj && (e = um::launch_proj_tc(dd, stage_ptrs(L, p, 4), mp, st)) != cudaSuccess)
+        return from_cuda(e);
     *launches = d.A + 3 + (d.has_proj ? 1 : 0) + extras;
     if (L->profiling) L->profiled_once = true;
     return ULTRAMEM_OK;
@@ -652,6 +653,7 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     if (e == cudaSuccess) e = dalloc(&ws.u, (size_t)H * r);
     if (e == cudaSuccess) e = dalloc(&ws.t, (size_t)H * r);
     if (e == cudaSuccess) e = dalloc(&ws.err, 1);
+    if (e == cudaSuccess) e = dalloc(&ws.stamps, 2 * um::kStampStages);
     if (e == cudaSuccess)
         e = lib_malloc(&ws.x_stage, Bm * cfg->d_in * elt_size(*cfg));
     if (e == cudaSuccess)
@@ -726,8 +728,6 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
 void ultramem_destroy(ultramem_layer *L) {
     if (!L) return;
     cudaDeviceSynchronize();
-    for (auto &ev : L->ev)
-        if (ev) cudaEventDestroy(ev);
     for (auto &g : L->host_graphs)
         if (g.exec) cudaGraphExecDestroy(g.exec);
     if (L->capture) cudaStreamDestroy(L->capture);
@@ -826,10 +826,13 @@ ultramem_status ultramem_lookup_reduce(ultramem_layer *L, const int64_t *idx, co
     cudaStream_t st = (cudaStream_t)stream;
     cudaError_t e;
     cudaGetLastError();
+    if ((e = reset_stamps(L, st)) != cudaSuccess) return from_cuda(e);
     if ((e = um::launch_slots_from_addresses(d, p, st)) != cudaSuccess) return from_cuda(e);
-    if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
-    if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
+    if ((e = um::launch_gather(d, stage_ptrs(L, p, 3), st)) != cudaSuccess) return from_cuda(e);
+    if (d.has_proj && (e = um::launch_proj(d, stage_ptrs(L, p, 4), st)) != cudaSuccess)
+        return from_cuda(e);
     L->launches = 2 + (d.has_proj ? 2 : 0);
+    if (L->profiling) L->profiled_once = true;
     return ULTRAMEM_OK;
 }
 
@@ -1013,9 +1016,6 @@ int32_t ultramem_debug_live_allocations(void) { return g_live_allocs.load(); }
 
 ultramem_status ultramem_profile_enable(ultramem_layer *L, int32_t enable) {
     if (!L) return ULTRAMEM_EINVAL;
-    if (enable && !L->ev[0])
-        for (auto &ev : L->ev)
-            if (cudaEventCreate(&ev) != cudaSuccess) return ULTRAMEM_ECUDA;
     L->profiling = enable != 0;
     L->profiled_once = false;
     return ULTRAMEM_OK;
@@ -1024,17 +1024,25 @@ ultramem_status ultramem_profile_enable(ultramem_layer *L, int32_t enable) {
 int32_t ultramem_last_launches(const ultramem_layer *L) { return L ? L->launches : 0; }
 
 int32_t ultramem_profile_read(ultramem_layer *L, float *ms, int32_t n) {
-    if (!L || !ms || !L->profiled_once) return 0;
-    int cnt = n < kStages ? n : kStages;
-    for (int i = 0; i < cnt; ++i) {
-        float t = 0.f;
-        if (cudaEventElapsedTime(&t, L->ev[i], L->ev[i + 1]) != cudaSuccess) {
-            cudaGetLastError();
-            t = -1.f;
-        }
-        ms[i] = t;
+    if (!L || !ms || !L->profiled_once || n < 1) return 0;
+    unsigned long long st[2 * um::kStampStages];
+    if (cudaMemcpy(st, L->ws.stamps, sizeof st, cudaMemcpyDeviceToHost) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
     }
-    return cnt;
+    const unsigned long long *bg = st, *en = st + um::kStampStages;
+    auto ran = [&](int i) { return bg[i] != ~0ull && en[i] >= bg[i]; };
+    const int cnt = n < kStages ? n : kStages;
+    for (int i = 0; i < cnt; ++i) ms[i] = ran(i) ? (float)((en[i] - bg[i]) * 1e-6) : -1.f;
+    // the hand-offs: from the end of the previous stage to this stage's first
+    // CTA past its dependency wait
+    for (int i = 0; i < kStages && kStages + i < n; ++i) {
+        float g = 0.f;
+        if (i > 0 && ran(i) && ran(i - 1))
+            g = bg[i] > en[i - 1] ? (float)((bg[i] - en[i - 1]) * 1e-6) : 0.f;
+        ms[kStages + i] = g;
+    }
+    return n < 2 * kStages ? cnt : 2 * kStages;
 }
 
 }  // extern "C"

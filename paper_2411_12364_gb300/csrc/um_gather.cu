@@ -110,6 +110,7 @@ __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
     const int per_warp = (hm + kWarps - 1) / kWarps;
     const int e_begin = min(hm, warp * per_warp), e_end = min(hm, e_begin + per_warp);
     pdl_wait();
+    stamp_begin(p.stamp);
     pdl_trigger();
     A acc[EMAX][EPV];
 #pragma unroll
@@ -166,6 +167,7 @@ __global__ void __launch_bounds__(kThreads) gather_reg_kernel(Dims d, Ptrs p) {
         for (int wv = 0; wv < kWarps; ++wv) s += red[(size_t)wv * EDv + i];
         store_pooled<T>(d, p, b, i, (float)s);
     }
+    stamp_end(p.stamp);
 }
 
 constexpr int kBMaxE = 16;
@@ -201,6 +203,7 @@ __global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(
     float *w_s = reinterpret_cast<float *>(row_s + hm);          // [hm][nc] their weights
     const int nc = d.nc;
     pdl_wait();
+    stamp_begin(p.stamp);
     pdl_trigger();
 
     // stable counting sort of the slots by block (slot order kept within a block)
@@ -293,6 +296,7 @@ __global__ void __launch_bounds__(THREADS, 1024 / THREADS) gather_bucket_kernel(
         for (int sb = 0; sb < wpb; ++sb) sum += red[(qq * wpb + sb) * Dv + c];
         store_pooled<T>(d, p, b, i, (float)sum);
     }
+    stamp_end(p.stamp);
 }
 
 // Shared-memory-accumulating gather for any E and row width (A: the
@@ -305,6 +309,7 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Dims d, Ptrs p) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int EDv = d.E * d.d_v;
     pdl_wait();
+    stamp_begin(p.stamp);
     pdl_trigger();
     A *mine = acc_w + (size_t)warp * EDv;
     for (int i = lane; i < EDv; i += 32) mine[i] = 0;
@@ -350,6 +355,7 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Dims d, Ptrs p) {
         for (int wv = 0; wv < kWarps; ++wv) s += acc_w[(size_t)wv * EDv + i];
         store_pooled<T>(d, p, b, i, (float)s);
     }
+    stamp_end(p.stamp);
 }
 
 // proj_part[split][b][o] = sum over this split's slice of E*D_v of acc[b][c] W[c][o]
@@ -362,6 +368,7 @@ __global__ void __launch_bounds__(kThreads) proj_kernel(Dims d, Ptrs p) {
     const int kb = split * chunk, ke = min(Kd, kb + chunk);
     const int o0 = blockIdx.x * 64, b0 = blockIdx.y * 32;
     const T *W = static_cast<const T *>(p.w_proj);
+    stamp_begin(p.stamp);
     __shared__ float as[32][33];   // [c][token]
     __shared__ float ws[32][65];   // [c][output]
     const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
@@ -404,6 +411,7 @@ __global__ void __launch_bounds__(kThreads) proj_kernel(Dims d, Ptrs p) {
             if (b < d.B && o < d.d_out)
                 p.proj_part[((int64_t)split * d.B + b) * d.d_out + o] = v;
         }
+    stamp_end(p.stamp);
 }
 
 // out = the sum of the split-K partials (in fp64 with fp32 storage: one
@@ -411,6 +419,7 @@ __global__ void __launch_bounds__(kThreads) proj_kernel(Dims d, Ptrs p) {
 template <typename T>
 __global__ void proj_reduce_kernel(Dims d, Ptrs p) {
     pdl_wait();
+    stamp_begin(p.stamp);
     pdl_trigger();
     using A = AccOf<T>;
     const int64_t total = (int64_t)d.B * d.d_out;
@@ -420,6 +429,7 @@ __global__ void proj_reduce_kernel(Dims d, Ptrs p) {
         for (int sp = 0; sp < d.p_splits; ++sp) s += (A)p.proj_part[(int64_t)sp * total + i];
         static_cast<T *>(p.out)[i] = from_f<T>((float)s);
     }
+    stamp_end(p.stamp);
 }
 
 }  // namespace

@@ -81,6 +81,7 @@ struct Ptrs {
     void *state_out;             // same shape, or null
     void *xs;                    // the convolved input (layout above)
     int *err;                    // device error word (bit flags above)
+    unsigned long long *stamp;   // profiling: this stage's [begin] (ends kStampStages later)
 };
 
 // TMA descriptors of the tensor-core path: weights (encoded at create) and
@@ -257,6 +258,28 @@ template <auto K> size_t static_smem_of() {
         return (size_t)a.sharedSizeBytes;
     }();
     return bytes;
+}
+
+// ---- profiling stamps -----------------------------------------------------
+// While a layer profiles, each kernel of a forward records, in nanoseconds
+// of the GPU's global timer (32 ns resolution on GB300), the earliest moment
+// one of its CTAs passed its dependency wait (atomicMin into stamp[0]) and
+// the latest moment one of its warps finished (atomicMax into
+// stamp[kStampStages]); the kernels of one stage share the pair.  The
+// forward itself runs unchanged (programmatic dependent launches on), so the
+// stage times are the kernels' own device times in the chain.
+constexpr int kStampStages = 5;
+
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ void stamp_begin(unsigned long long *s) {
+    if (s && threadIdx.x == 0) atomicMin(s, global_ns());
+}
+__device__ __forceinline__ void stamp_end(unsigned long long *s) {
+    if (s && (threadIdx.x & 31) == 0) atomicMax(s + kStampStages, global_ns());
 }
 
 // ---- small device helpers ------------------------------------------------

@@ -40,6 +40,7 @@ __device__ __forceinline__ T input_back(const Dims &d, const Ptrs &p, int b, int
 template <typename T>
 __global__ void __launch_bounds__(kThreads) conv_kernel(Dims d, Ptrs p, int splits) {
     pdl_wait();
+    stamp_begin(p.stamp);
     pdl_trigger();
     const int c = blockIdx.y * kThreads + threadIdx.x;
     if (c >= d.d_in) return;
@@ -68,6 +69,7 @@ __global__ void __launch_bounds__(kThreads) conv_kernel(Dims d, Ptrs p, int spli
         static_cast<T *>(p.state_out)[((int64_t)s * kk + i) * d.d_in + c] =
             input_back<T>(d, p, s * d.seq_len + d.seq_len - 1, kk - 1 - i, c);
     }
+    stamp_end(p.stamp);
 }
 
 __device__ __forceinline__ float warp_sum(float v) {
@@ -105,6 +107,7 @@ __global__ void __launch_bounds__(kThreads) query_ln_kernel(Dims d, Ptrs p, __nv
         tv[i] = in && qs ? p.t[k] : 0.f;
     }
     pdl_wait();
+    stamp_begin(p.stamp);
     pdl_trigger();
     if (!live) return;
     const int64_t split_stride = (int64_t)d.A * d.B * HD;
@@ -141,6 +144,7 @@ __global__ void __launch_bounds__(kThreads) query_ln_kernel(Dims d, Ptrs p, __nv
             if (c >= d.d_k) break;
             q[c] = (float)((vd[i] - mean) * inv * (double)gv[i] + (double)bv[i]);
         }
+        stamp_end(p.stamp);
         return;
     }
     float v[kLnMax];
@@ -174,6 +178,7 @@ __global__ void __launch_bounds__(kThreads) query_ln_kernel(Dims d, Ptrs p, __nv
             if (col_axis) put_split_query(qs, 1, h, c, b, y * tv[i], d.H, Bmax, d.d_k);
         }
     }
+    stamp_end(p.stamp);
 }
 
 // One warp per stored row.

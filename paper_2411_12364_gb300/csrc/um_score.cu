@@ -19,6 +19,7 @@ constexpr int kThreads = 256;
 template <typename T, typename TX>
 __global__ void __launch_bounds__(kThreads) query_kernel(Dims d, Ptrs p) {
     pdl_wait();
+    stamp_begin(p.stamp);
     pdl_trigger();
     const int a = blockIdx.z / d.q_splits, split = blockIdx.z % d.q_splits;
     const TX *X = static_cast<const TX *>(p.x);
@@ -70,6 +71,7 @@ __global__ void __launch_bounds__(kThreads) query_kernel(Dims d, Ptrs p) {
             if (b < d.B && o < HD)
                 p.q_part[(((int64_t)split * d.A + a) * d.B + b) * HD + o] = v;
         }
+    stamp_end(p.stamp);
 }
 
 // For each rank chunk alpha, S_alpha[b][i] = sum_{c < dk} key[h][i][alpha*dk + c]
@@ -80,6 +82,7 @@ __global__ void __launch_bounds__(kThreads) query_kernel(Dims d, Ptrs p) {
 // Tile: 64 keys x 32 tokens; each thread owns 4 keys x 2 tokens.
 template <typename T>
 __global__ void __launch_bounds__(kThreads) score_kernel(Dims d, Ptrs p) {
+    stamp_begin(p.stamp);
     const int h = blockIdx.z >> 1, axis = blockIdx.z & 1;
     const int a = (axis == 1 && d.A == 2) ? 1 : 0;
     const T *keys = static_cast<const T *>(axis == 0 ? p.k_row : p.k_col) +
@@ -134,6 +137,7 @@ __global__ void __launch_bounds__(kThreads) score_kernel(Dims d, Ptrs p) {
             if (i < d.K && b < d.B)
                 p.akey[(((int64_t)b * d.H + h) * 2 + axis) * d.K + i] = f2ord(folded[j][t]);
         }
+    stamp_end(p.stamp);
 }
 
 }  // namespace

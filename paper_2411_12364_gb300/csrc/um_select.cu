@@ -776,6 +776,7 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     const float cp0 = threadIdx.x < ncrr ? cp[threadIdx.x] : 0.f;
     const float cp1 = threadIdx.x + kThreads < ncrr ? cp[threadIdx.x + kThreads] : 0.f;
     pdl_wait();
+    stamp_begin(p.stamp);
     pdl_trigger();
     const int HD = d.H * d.d_k;
     const int64_t split_stride = (int64_t)d.A * d.B * HD;
@@ -1026,6 +1027,7 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
             }
         }
     }
+    stamp_end(p.stamp);
 }
 
 // lookup_reduce input: given virtual addresses and weights -> (row, p, w).

@@ -46,6 +46,7 @@ struct SmallArgs {
     const float *u, *t;          // [H][r] rank-1 coefficients of row / column keys
     int a, A, H, d_k, dk, r, Bmax;
     int write_qs;                // 0: the query LayerNorm writes the splits later
+    unsigned long long *stamp;   // profiling stamps of the stage, or null
 };
 
 // Per output row o: its head, column and the rank-1 coefficients of its
@@ -137,7 +138,10 @@ __global__ void __launch_bounds__(kThreads) small_gemm_kernel(SmallArgs g) {
             for (int r = 0; r < nrows; ++r)
                 bulk_g2s(Ws + r * stride, g.W + (int64_t)(o0 + r) * g.Kd + k0, row_bytes, &bar);
         }
-        if (k0 == 0) pdl_wait();
+        if (k0 == 0) {
+            pdl_wait();
+            stamp_begin(g.stamp);
+        }
         if (threadIdx.x == 0)
             for (int t = 0; t < ntoks; ++t)
                 bulk_g2s(Xs + t * stride, X + (int64_t)(n0 + t) * g.Kd + k0, x_bytes, &bar);
@@ -190,6 +194,7 @@ __global__ void __launch_bounds__(kThreads) small_gemm_kernel(SmallArgs g) {
                 if (r0 + i < nrows && t0 + j < ntoks)
                     Ep::put(g, o0 + r0 + i, n0 + t0 + j, acc[i][j], rs[i]);
     }
+    stamp_end(g.stamp);
 }
 
 template <bool XF> constexpr size_t smem_row_bytes() {   // W row + token row, one element
@@ -243,6 +248,7 @@ cudaError_t launch_query_small(const Dims &d, const Ptrs &p, __nv_bfloat16 *qs, 
         g.r = d.r;
         g.Bmax = Bmax;
         g.write_qs = write_qs ? 1 : 0;
+        g.stamp = p.stamp;
         // the first query waits for all earlier work on the stream, unless it
         // follows this call's convolution
         cudaError_t e = x_f32 ? launch_small<QueryEp, true>(g, pdl && a == 0, st)

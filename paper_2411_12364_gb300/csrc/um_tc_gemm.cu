@@ -129,6 +129,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0)
         for (int it = 0; it < pre; ++it) load_a(it);
     pdl_wait();
+    stamp_begin(op.stamp);
     // TMEM is taken only after the wait: a kernel that waits never holds
     // columns that a CTA of an earlier kernel could still be waiting for
     if (warp == 0) tmem_alloc(&tmem_slot, ncols);
@@ -259,6 +260,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             op.store_sums(t, row, n, sums);
         }
     }
+    stamp_end(op.stamp);
 }
 
 // ---- persistent variant (many tiles, no split-K) ----------------------------
@@ -318,6 +320,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
         __syncthreads();
         if (probe_timeout(&never, op.err, kErrTimeout)) return;
     }
+    stamp_begin(op.stamp);
     if (warp == 0) tmem_alloc(&tmem_slot, 2 * buf_cols);
     tc_fence_before();
     __syncthreads();
@@ -460,6 +463,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, 2 * buf_cols);
+    stamp_end(op.stamp);
 }
 
 // ---- S1: query projection, split over D_i --------------------------------
@@ -468,6 +472,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
 struct QueryOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
+    unsigned long long *stamp;   // profiling stamps of the stage, or null
     int B, HD, A, a, splits, kb_total, H, d_k, dk, r, Bmax;
     int write_qs;         // 0: the query LayerNorm writes the splits later
     float *q_part;        // [splits][A][B][HD]; the result is split 0
@@ -543,6 +548,7 @@ struct QueryOp {
 struct ScoreOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
+    unsigned long long *stamp;   // profiling stamps of the stage, or null
     int B, H, K, kb_total;
     uint32_t *akey;       // [B][H][2][K]
     __device__ int cluster_splits() const { return 1; }
@@ -583,6 +589,7 @@ struct ScoreOp {
 struct ProjOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
+    unsigned long long *stamp;   // profiling stamps of the stage, or null
     int B, d_out, kb_total, splits;
     __nv_bfloat16 *out;   // [B][d_out]
     float *part;          // [splits][B][d_out] split-K partials
@@ -641,6 +648,7 @@ struct ProjOp {
 struct DaccOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
+    unsigned long long *stamp;   // profiling stamps of the stage, or null
     int B, M, kb_total;
     float *out;   // [B][M]
     __device__ int cluster_splits() const { return 1; }
@@ -682,6 +690,7 @@ struct DaccOp {
 struct DwOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
+    unsigned long long *stamp;   // profiling stamps of the stage, or null
     int M, N, kb_total;   // M = D'_v (rows o), N = E D_v (columns c)
     float *out;           // [N][M]
     __device__ int cluster_splits() const { return 1; }
@@ -857,6 +866,7 @@ cudaError_t configure_tc() {
 cudaError_t launch_dw_tc(const Dims &d, const CUtensorMap &g_t, const CUtensorMap &acc_t2,
                          float *dW, int *err, cudaStream_t st) {
     DwOp op;
+    op.stamp = nullptr;
     op.M = d.d_out;
     op.N = d.E * d.d_v;
     op.n_tile = tc_n_tile(op.N, 1);
@@ -873,6 +883,7 @@ cudaError_t launch_dw_tc(const Dims &d, const CUtensorMap &g_t, const CUtensorMa
 cudaError_t launch_dacc_tc(const Dims &d, const CUtensorMap &w_p, const CUtensorMap &g,
                            float *dacc, int *err, cudaStream_t st) {
     DaccOp op;
+    op.stamp = nullptr;
     op.n_tile = tc_n_tile(d.B, 1);
     op.n_acc = 1;
     op.acc_chunk = 1 << 30;
@@ -897,6 +908,7 @@ cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int 
     if (splits > kMaxSplits) return cudaErrorInvalidValue;
     for (int a = 0; a < d.A; ++a) {
         QueryOp op;
+    op.stamp = p.stamp;
         op.n_tile = n_tile;
         op.n_acc = 1;
         op.acc_chunk = 1 << 30;
@@ -932,6 +944,7 @@ cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int 
 
 cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
     ScoreOp op;
+    op.stamp = p.stamp;
     op.n_tile = tc_n_tile(d.B, 1);
     op.n_acc = 1;
     op.acc_chunk = 1 << 30;
@@ -950,6 +963,7 @@ cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cuda
 cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
     if (d.p_splits > kMaxSplits) return cudaErrorInvalidValue;
     ProjOp op;
+    op.stamp = p.stamp;
     op.n_tile = tc_n_tile(d.B, 1);
     op.n_acc = 1;
     op.acc_chunk = 1 << 30;
