@@ -103,6 +103,12 @@ typedef struct ultramem_config {
                               (a = 1 + o1 mod (E*N - 1) stepped up to gcd(a, E*N) = 1,
                               c = o2 mod E*N); E*N must be < 2^32                     */
     float ln_eps;        /* query LayerNorm epsilon, >= 0 (inside the square root)   */
+    int64_t shard_rows;  /* 0: `values` holds all N rows.  > 0: number-wise partition
+                            of the table (App. D): `values` holds this rank's shard of
+                            shard_rows (<= N) consecutive rows; the calls that read the
+                            whole table (forward, lookup_reduce and its backward)
+                            return ULTRAMEM_EINVAL, and the ultramem_shard_* calls
+                            below serve the lookup                                   */
 } ultramem_config;
 
 /* The layer's parameters.  Device tensors are in the storage type cfg.dtype
@@ -295,6 +301,44 @@ const char *ultramem_last_error(void);
 
 /* Human-readable name of a status code. */
 const char *ultramem_status_string(ultramem_status s);
+
+/* Number-wise partition of the value table over P ranks (App. D: indices
+ * all-to-all to the rows' owners, lookup there, rows all-to-all back, then
+ * the weighted sum pooling on the requester): rank q holds rows
+ * [q R, min((q + 1) R, N)), R = rows_per_rank = ceil(N / P), and each rank
+ * selects its own tokens' slots (S1-S6 with the keys replicated,
+ * ultramem_retrieve).  Then:
+ *   1. ultramem_shard_route: the S = n*H*m addresses idx [n][H][m] (int64,
+ *      DEVICE) are shuffled (Eq. 14) to physical rows and grouped by owner
+ *      q = row / R: counts [P] (int32, DEVICE) of requests per owner;
+ *      send_rows [S] (int32, DEVICE) the owners' local row indices, owner by
+ *      owner (owner q's block starts at the sum of counts[0..q)); slot_pos [S]
+ *      (int32, DEVICE) the position of slot s in send_rows.  The order inside
+ *      an owner's block is not fixed; every later step reads through slot_pos,
+ *      so the result is.  An address outside [0, E N) is recorded in the error
+ *      word and requested as row 0 of owner 0 (its slot is then skipped).
+ *   2. (caller) all-to-all of counts, then of send_rows: each rank receives
+ *      the local rows the others request from it.
+ *   3. ultramem_shard_lookup: out_rows[i] = the layer's shard row rows[i]
+ *      ([n_rows][D_v], the storage type, DEVICE), a row outside the shard
+ *      recorded in the error word and returned as zeros.
+ *   4. (caller) all-to-all of the looked-up rows back to the requesters, in
+ *      the order of their send_rows (back_rows [S][D_v]).
+ *   5. ultramem_shard_pool: the weighted sum pooling of Eq. 15 and the IVE
+ *      projection on the returned rows: slot s reads back_rows[slot_pos[s]]
+ *      with weight w[s] (w like ultramem_lookup_reduce's) into its block;
+ *      out [n][D'_v] as ultramem_lookup_reduce writes it.
+ * All three are asynchronous on `stream`, work on layers created with or
+ * without shard_rows, and return ULTRAMEM_EINVAL for invalid sizes or null
+ * pointers (P in 1..1024, rows_per_rank * P >= N, n <= max_tokens). */
+ultramem_status ultramem_shard_route(ultramem_layer *layer, const int64_t *idx, int32_t n,
+                                     int32_t P, int64_t rows_per_rank, int32_t *counts,
+                                     int32_t *send_rows, int32_t *slot_pos, void *stream);
+ultramem_status ultramem_shard_lookup(ultramem_layer *layer, const int32_t *rows,
+                                      int64_t n_rows, void *out_rows, void *stream);
+ultramem_status ultramem_shard_pool(ultramem_layer *layer, const int64_t *idx, const float *w,
+                                    int32_t n, const int32_t *slot_pos, const void *back_rows,
+                                    void *out, void *stream);
 
 /* Failure-path hooks for tests; they inject failures on the host or behind
  * a bounded wait, never a device fault.

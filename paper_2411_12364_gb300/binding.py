@@ -29,14 +29,16 @@ EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
            "ultramem_last_launches", "ultramem_forward_seq", "ultramem_key_ln",
            "ultramem_retrieve_exact", "ultramem_lookup_reduce_backward",
            "ultramem_debug_wait_probe", "ultramem_debug_fail_alloc",
-           "ultramem_debug_live_allocations")
+           "ultramem_debug_live_allocations", "ultramem_shard_route", "ultramem_shard_lookup",
+           "ultramem_shard_pool")
 
 
 class Config(C.Structure):
     _fields_ = [(name, C.c_int32) for name in (
         "d_in", "d_k", "heads", "rank", "n", "expand_e", "d_v", "d_out", "topk", "topm",
         "has_proj", "share_query", "act", "dtype", "max_tokens", "cores", "conv_k",
-        "query_ln", "score_mode")] + [("shuffle_seed", C.c_uint64), ("ln_eps", C.c_float)]
+        "query_ln", "score_mode")] + [("shuffle_seed", C.c_uint64), ("ln_eps", C.c_float),
+                                     ("shard_rows", C.c_int64)]
 
 
 class Weights(C.Structure):
@@ -117,6 +119,12 @@ def load(path: str | None = None) -> C.CDLL:
         lib.ultramem_debug_fail_alloc.restype = None
         lib.ultramem_debug_live_allocations.argtypes = []
         lib.ultramem_debug_live_allocations.restype = I32
+        lib.ultramem_shard_route.argtypes = [P, P, I32, I32, I64, P, P, P, P]
+        lib.ultramem_shard_route.restype = I32
+        lib.ultramem_shard_lookup.argtypes = [P, P, I64, P, P]
+        lib.ultramem_shard_lookup.restype = I32
+        lib.ultramem_shard_pool.argtypes = [P, P, P, I32, P, P, P, P]
+        lib.ultramem_shard_pool.restype = I32
         _lib = lib
         return lib
 
@@ -198,6 +206,7 @@ class UltraMemLayer:
         c.ln_eps = float(cfg.get("ln_eps", 1e-5))
         c.score_mode = int(cfg.get("score_mode", 0))
         c.shuffle_seed = int(cfg.get("shuffle_seed", 0))
+        c.shard_rows = int(cfg.get("shard_rows", 0))
         self._c = c
         dev_keys = ("w_q", "w_q_col", "k_row", "k_col", "values", "w_proj", "perm", "conv_w",
                     "conv_b", "ln_g", "ln_b")
@@ -334,6 +343,45 @@ class UltraMemLayer:
             self._h, idx.data_ptr(), w.data_ptr(), g.data_ptr(), B, _ptr(dvalues), _ptr(dw),
             _ptr(dwp), _stream()), "ultramem_lookup_reduce_backward")
         return dvalues, dw, dwp
+
+    # -- number-wise partitioned table (App. D) ---------------------------
+    def shard_route(self, idx: torch.Tensor, P: int, rows_per_rank: int):
+        """Slots idx [n,H,m] grouped by the rank that owns their row:
+        (counts [P], send_rows [S], slot_pos [S]), int32 device tensors."""
+        idx = idx.contiguous().to(torch.int64)
+        S = idx.numel()
+        counts = torch.empty(P, dtype=torch.int32, device=idx.device)
+        send_rows = torch.empty(S, dtype=torch.int32, device=idx.device)
+        slot_pos = torch.empty(S, dtype=torch.int32, device=idx.device)
+        _check(self.lib.ultramem_shard_route(self._h, idx.data_ptr(), idx.shape[0], int(P),
+                                             int(rows_per_rank), counts.data_ptr(),
+                                             send_rows.data_ptr(), slot_pos.data_ptr(),
+                                             _stream()), "ultramem_shard_route")
+        return counts, send_rows, slot_pos
+
+    def shard_lookup(self, rows: torch.Tensor):
+        """Rows of this layer's table (its shard) at local indices ``rows``."""
+        rows = rows.contiguous().to(torch.int32)
+        out = torch.empty((rows.numel(), int(self.cfg["d_v"])), dtype=self.dtype,
+                          device=rows.device)
+        _check(self.lib.ultramem_shard_lookup(self._h, rows.data_ptr(), rows.numel(),
+                                              out.data_ptr(), _stream()),
+               "ultramem_shard_lookup")
+        return out
+
+    def shard_pool(self, idx: torch.Tensor, w: torch.Tensor, slot_pos: torch.Tensor,
+                   back_rows: torch.Tensor):
+        """Eq. 15 pooling and the projection on the rows the owners returned."""
+        idx = idx.contiguous().to(torch.int64)
+        w = w.contiguous().to(torch.float32)
+        back_rows = back_rows.contiguous()
+        out = torch.empty((idx.shape[0], int(self.cfg["d_out"])), dtype=self.dtype,
+                          device=idx.device)
+        _check(self.lib.ultramem_shard_pool(self._h, idx.data_ptr(), w.data_ptr(), idx.shape[0],
+                                            slot_pos.contiguous().data_ptr(),
+                                            back_rows.data_ptr(), out.data_ptr(), _stream()),
+               "ultramem_shard_pool")
+        return out
 
     def check(self) -> int:
         """Syncs the current stream and returns the device error status."""

@@ -33,6 +33,7 @@ struct Workspace {
                                       // bf16 terms), g^T [D'_v][B]
     __nv_bfloat16 *qs = nullptr, *acc_bf = nullptr, *w_pt = nullptr;   // tensor path
     unsigned long long *stamps = nullptr;   // profiling: [kStampStages] begins, then ends
+    int *shard_cursor = nullptr;            // ultramem_shard_route: [1024] per-owner cursors
 };
 
 }  // namespace
@@ -68,6 +69,10 @@ struct ultramem_layer {
     bool probe_armed = false;    // ultramem_debug_wait_probe: the next forward's score probes
     bool dacc_tc = false;        // the backward's dacc may run on the tensor cores
 };
+
+// A layer over a shard of the table (number-wise partition) serves only the
+// calls that do not read the whole table.
+static bool whole_table(const ultramem_layer *L) { return L->cfg.shard_rows == 0; }
 
 namespace {
 
@@ -180,8 +185,10 @@ ultramem_status validate(const ultramem_config *c, const ultramem_weights *w) {
     if (c->has_proj && !w->w_proj) return ULTRAMEM_EINVAL;
     if ((w->u == nullptr) != (w->t == nullptr)) return ULTRAMEM_EINVAL;
     if (((uintptr_t)w->values) % 16) return ULTRAMEM_EINVAL;
+    if (c->shard_rows < 0 || c->shard_rows > (int64_t)c->n * c->n) return ULTRAMEM_EINVAL;
     return ULTRAMEM_OK;
 }
+
 
 // Leading singular triplet by one-sided (Hestenes) Jacobi on the columns of
 // C: rotations orthogonalise the columns of U = C V; the column norms are the
@@ -300,7 +307,7 @@ void free_workspace(Workspace &ws) {
                     ws.sel_row, ws.sel_p, ws.core,   ws.u,         ws.t,
                     ws.err,    ws.x_stage, ws.out_stage, ws.qs,     ws.acc_bf,
                     ws.w_pt,   ws.cores,   ws.xs,      ws.dacc,    ws.bwd_t,
-                    ws.stamps};
+                    ws.stamps, ws.shard_cursor};
     for (void *p : ptrs) lib_free(p);
     ws = Workspace();
 }
@@ -654,6 +661,7 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     if (e == cudaSuccess) e = dalloc(&ws.t, (size_t)H * r);
     if (e == cudaSuccess) e = dalloc(&ws.err, 1);
     if (e == cudaSuccess) e = dalloc(&ws.stamps, 2 * um::kStampStages);
+    if (e == cudaSuccess) e = dalloc(&ws.shard_cursor, 1024);
     if (e == cudaSuccess)
         e = lib_malloc(&ws.x_stage, Bm * cfg->d_in * elt_size(*cfg));
     if (e == cudaSuccess)
@@ -737,7 +745,7 @@ void ultramem_destroy(ultramem_layer *L) {
 
 ultramem_status ultramem_forward(ultramem_layer *L, const void *x, int32_t B, void *out,
                                  int64_t *idx_out, float *w_out, void *stream) {
-    if (!L || B < 0 || B > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (!L || B < 0 || B > L->cfg.max_tokens || !whole_table(L)) return ULTRAMEM_EINVAL;
     if (B == 0) return ULTRAMEM_OK;
     if (!x || !out) return ULTRAMEM_EINVAL;
     Dims d = dims_for(L, B);
@@ -753,7 +761,7 @@ ultramem_status ultramem_forward_seq(ultramem_layer *L, const void *x, int32_t n
                                      int32_t seq_len, const void *conv_state_in,
                                      void *conv_state_out, void *out, int64_t *idx_out,
                                      float *w_out, void *stream) {
-    if (!L || n_seq < 0 || seq_len < 1) return ULTRAMEM_EINVAL;
+    if (!L || n_seq < 0 || seq_len < 1 || !whole_table(L)) return ULTRAMEM_EINVAL;
     if ((int64_t)n_seq * seq_len > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
     const int B = n_seq * seq_len;
     if (B == 0) return ULTRAMEM_OK;
@@ -815,7 +823,7 @@ ultramem_status ultramem_retrieve_exact(ultramem_layer *L, const void *x, int32_
 
 ultramem_status ultramem_lookup_reduce(ultramem_layer *L, const int64_t *idx, const float *w,
                                        int32_t B, void *out, void *stream) {
-    if (!L || B < 0 || B > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (!L || B < 0 || B > L->cfg.max_tokens || !whole_table(L)) return ULTRAMEM_EINVAL;
     if (B == 0) return ULTRAMEM_OK;
     if (!idx || !w || !out) return ULTRAMEM_EINVAL;
     Dims d = dims_for(L, B);
@@ -840,7 +848,7 @@ ultramem_status ultramem_lookup_reduce_backward(ultramem_layer *L, const int64_t
                                                 const float *w, const void *g, int32_t B,
                                                 float *dvalues, float *dw, float *dw_proj,
                                                 void *stream) {
-    if (!L || B < 0 || B > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (!L || B < 0 || B > L->cfg.max_tokens || !whole_table(L)) return ULTRAMEM_EINVAL;
     if (B == 0) return ULTRAMEM_OK;
     if (!idx || !w || !g || !L->backward_ok) return ULTRAMEM_EINVAL;
     Dims d = dims_for(L, B);
@@ -916,7 +924,7 @@ ultramem_status ultramem_lookup_reduce_backward(ultramem_layer *L, const int64_t
 
 ultramem_status ultramem_forward_host(ultramem_layer *L, const void *x_host, int32_t B,
                                       void *out_host, void *stream) {
-    if (!L || B < 0 || B > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (!L || B < 0 || B > L->cfg.max_tokens || !whole_table(L)) return ULTRAMEM_EINVAL;
     if (B == 0) return ULTRAMEM_OK;
     if (!x_host || !out_host) return ULTRAMEM_EINVAL;
     cudaStream_t st = (cudaStream_t)stream;
@@ -1001,6 +1009,59 @@ ultramem_status ultramem_check(ultramem_layer *L, void *stream) {
     if (flags && cudaMemset(L->ws.err, 0, sizeof(int)) != cudaSuccess) return ULTRAMEM_ECUDA;
     if (flags & um::kErrTimeout) return ULTRAMEM_ETIMEOUT;
     if (flags & (um::kErrBadIndex | um::kErrInternal)) return ULTRAMEM_EDEVICE;
+    return ULTRAMEM_OK;
+}
+
+ultramem_status ultramem_shard_route(ultramem_layer *L, const int64_t *idx, int32_t n, int32_t P,
+                                     int64_t rows_per_rank, int32_t *counts, int32_t *send_rows,
+                                     int32_t *slot_pos, void *stream) {
+    if (!L || n < 0 || n > L->cfg.max_tokens || P < 1 || P > 1024 || rows_per_rank < 1)
+        return ULTRAMEM_EINVAL;
+    const int64_t N = (int64_t)L->cfg.n * L->cfg.n;
+    if (rows_per_rank * P < N) return ULTRAMEM_EINVAL;
+    if (n == 0) return ULTRAMEM_OK;
+    if (!idx || !counts || !send_rows || !slot_pos) return ULTRAMEM_EINVAL;
+    Dims d = dims_for(L, n);
+    Ptrs p = make_ptrs(L);
+    p.idx_in = idx;
+    cudaGetLastError();
+    return from_cuda(um::launch_shard_route(d, p, P, rows_per_rank, counts, L->ws.shard_cursor,
+                                            send_rows, slot_pos, (cudaStream_t)stream));
+}
+
+ultramem_status ultramem_shard_lookup(ultramem_layer *L, const int32_t *rows, int64_t n_rows,
+                                      void *out_rows, void *stream) {
+    if (!L || n_rows < 0) return ULTRAMEM_EINVAL;
+    if (n_rows == 0) return ULTRAMEM_OK;
+    if (!rows || !out_rows || ((uintptr_t)out_rows % 16)) return ULTRAMEM_EINVAL;
+    const int64_t rows_held =
+        L->cfg.shard_rows > 0 ? L->cfg.shard_rows : (int64_t)L->cfg.n * L->cfg.n;
+    cudaGetLastError();
+    return from_cuda(um::launch_shard_lookup(L->w.values, rows_held,
+                                             L->cfg.d_v * (int)elt_size(L->cfg), rows, n_rows,
+                                             out_rows, L->ws.err, (cudaStream_t)stream));
+}
+
+ultramem_status ultramem_shard_pool(ultramem_layer *L, const int64_t *idx, const float *w,
+                                    int32_t n, const int32_t *slot_pos, const void *back_rows,
+                                    void *out, void *stream) {
+    if (!L || n < 0 || n > L->cfg.max_tokens) return ULTRAMEM_EINVAL;
+    if (n == 0) return ULTRAMEM_OK;
+    if (!idx || !w || !slot_pos || !back_rows || !out || ((uintptr_t)back_rows % 16))
+        return ULTRAMEM_EINVAL;
+    Dims d = dims_for(L, n);
+    Ptrs p = make_ptrs(L);
+    p.idx_in = idx;
+    p.w_in = w;
+    p.out = out;
+    p.values = back_rows;   // slot s reads returned row slot_pos[s]
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e;
+    cudaGetLastError();
+    if ((e = um::launch_shard_slots(d, p, slot_pos, st)) != cudaSuccess) return from_cuda(e);
+    if ((e = um::launch_gather(d, p, st)) != cudaSuccess) return from_cuda(e);
+    if (d.has_proj && (e = um::launch_proj(d, p, st)) != cudaSuccess) return from_cuda(e);
+    L->launches = 2 + (d.has_proj ? 2 : 0);
     return ULTRAMEM_OK;
 }
 

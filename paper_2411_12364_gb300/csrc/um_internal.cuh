@@ -140,6 +140,18 @@ cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream
 cudaError_t launch_gather(const Dims &d, const Ptrs &p, cudaStream_t st);
 cudaError_t launch_proj(const Dims &d, const Ptrs &p, cudaStream_t st);
 
+// The number-wise partitioned table (App. D): route slots to their rows'
+// owners (counts and cursor: [P] scratch), look rows up in a shard, and the
+// gather's per-slot inputs for the rows the owners returned.
+cudaError_t launch_shard_route(const Dims &d, const Ptrs &p, int P, int64_t rows_per_rank,
+                               int *counts, int *cursor, int32_t *send_rows, int32_t *slot_pos,
+                               cudaStream_t st);
+cudaError_t launch_shard_lookup(const void *values, int64_t shard_rows, int row_bytes,
+                                const int32_t *rows, int64_t n, void *out, int *err,
+                                cudaStream_t st);
+cudaError_t launch_shard_slots(const Dims &d, const Ptrs &p, const int32_t *slot_pos,
+                               cudaStream_t st);
+
 // Eq. 5 by brute force (recall measurement): the exact top-m of every
 // (token, head)'s whole grid into idx_out / w_out [B][H][m]
 bool exact_fits(const Dims &d);
