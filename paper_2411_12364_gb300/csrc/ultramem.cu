@@ -102,29 +102,48 @@ int query_splits(const ultramem_config &c, int B) {
 // it re-reads once per 8 tokens) it is slower.
 constexpr int kSmallQueryBatch = 64;
 
-// Tensor path split-K: about `target` CTAs stream the weight, at most one
-// portable cluster (8) per tile, whole K blocks.
-int tc_splits(int m_rows, int B, int kdim, int target) {
-    int m_tiles = (m_rows + 127) / 128;
+// Tensor path split-K plan: the N tile (tokens per tile) and the split count
+// of a contraction of m_rows weight rows over B tokens and kdim.  About
+// `target` CTAs stream the weight: with one tile of up to 256 tokens, at
+// most one portable cluster (8) of whole K blocks per tile; when that grid
+// is still short of the target, the token tile is halved (down to `nt_min`),
+// so that a batch of 128 tokens over 4 weight tiles runs 128 CTAs instead
+// of 32.
+struct TcPlan {
+    int n_tile, splits;
+};
+TcPlan tc_plan(int m_rows, int B, int kdim, int target, int max_splits, int nt_min) {
+    const int m_tiles = (m_rows + 127) / 128;
+    const int kb = (kdim + 63) / 64;
     int nt = um::tc_n_tile(B, 1);
-    int n_tiles = (B + nt - 1) / nt;
-    int kb = (kdim + 63) / 64;
-    int s = (target + m_tiles * n_tiles - 1) / (m_tiles * n_tiles);
-    if (s > 8) s = 8;
-    if (s > kb) s = kb;
-    return s < 1 ? 1 : s;
+    for (;;) {
+        const int n_tiles = (B + nt - 1) / nt;
+        int s = (target + m_tiles * n_tiles - 1) / (m_tiles * n_tiles);
+        if (s > max_splits) s = max_splits;
+        if (s > kb) s = kb;
+        if (s < 1) s = 1;
+        if (m_tiles * n_tiles * s >= target || nt <= nt_min) return {nt, s};
+        nt = (nt / 2 + 15) / 16 * 16;
+    }
 }
-// Measured on GB300 (per forward, graphs of back-to-back forwards): the
-// query projection is fastest with the most splits; the IVE projection, whose
-// fp32 partials grow with the batch, with about 64 CTAs below 256 tokens and
-// unsplit from 256 tokens on.
-int tc_query_splits(const ultramem_config &c, int B) {
-    return tc_splits(c.heads * c.d_k, B, c.d_in, 128);
+// Measured on GB300 (stage times of graph-replayed forwards; mid_4m at 128
+// tokens, large_20m at 256): the query is fastest with about 128 CTAs, eight
+// splits and token tiles down to 32 (11.1 against 16.6 us with one 128-token
+// tile, 12.2 against 23.0 us at 256 tokens).  The IVE projection, whose B
+// operand (two bf16 terms of the pooled rows) grows with the batch, keeps
+// about 64 CTAs of up to eight splits up to 64 tokens; above, about 128 CTAs
+// of at most four splits with token tiles down to 64 (6.9 against 9.5 us at
+// 128 tokens, 9.6 against 15.4 us at 256).
+TcPlan tc_query_plan(const ultramem_config &c, int B) {
+    return tc_plan(c.heads * c.d_k, B, c.d_in, 128, 8, 32);
 }
-int tc_proj_splits(const ultramem_config &c, int B) {
-    if (!c.has_proj || B >= 256) return 1;
-    return tc_splits(c.d_out, B, c.expand_e * c.d_v, 64);
+TcPlan tc_proj_plan(const ultramem_config &c, int B) {
+    if (!c.has_proj) return {um::tc_n_tile(B, 1), 1};
+    if (B <= 64) return tc_plan(c.d_out, B, c.expand_e * c.d_v, 64, 8, 256);
+    return tc_plan(c.d_out, B, c.expand_e * c.d_v, 128, 4, 64);
 }
+int tc_query_splits(const ultramem_config &c, int B) { return tc_query_plan(c, B).splits; }
+int tc_proj_splits(const ultramem_config &c, int B) { return tc_proj_plan(c, B).splits; }
 
 // The tensor path needs bf16 storage and 16-byte rows for TMA (D_in, D_k and
 // E*D_v multiples of 8 elements).
@@ -348,6 +367,8 @@ Dims dims_for(const ultramem_layer *L, int B) {
     d.seq_len = B;   // one sequence unless the caller says otherwise
     d.q_splits = L->tc ? tc_query_splits(L->cfg, B) : query_splits(L->cfg, B);
     d.p_splits = L->tc ? tc_proj_splits(L->cfg, B) : proj_splits(L->cfg, B);
+    d.q_ntile = L->tc ? tc_query_plan(L->cfg, B).n_tile : 0;
+    d.p_ntile = L->tc ? tc_proj_plan(L->cfg, B).n_tile : 0;
     return d;
 }
 
@@ -427,15 +448,16 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     const int Bmax = c.max_tokens;
     const int nt1 = um::tc_n_tile(d.B, 1);   // N tile of every contraction (one accumulator)
     const bool conv = d.conv_k > 0;
-    if (!conv && !um::tc_encode(&mp.x, p.x, (uint64_t)c.d_in, (uint64_t)d.B, 1, (uint32_t)nt1, 2))
+    if (!conv && !um::tc_encode(&mp.x, p.x, (uint64_t)c.d_in, (uint64_t)d.B, 1,
+                                (uint32_t)d.q_ntile, 2))
         return ULTRAMEM_EINVAL;   // x must be 16-byte aligned
     if (conv && !um::tc_encode(&mp.xs, L->ws.xs, 3ull * c.d_in, (uint64_t)d.B, 1,
-                               (uint32_t)nt1, 2))
+                               (uint32_t)d.q_ntile, 2))
         return ULTRAMEM_ECUDA;
     if (!um::tc_encode(&mp.qs, L->ws.qs, 3ull * c.d_k, (uint64_t)Bmax, 2ull * d.H,
                        (uint32_t)nt1, 3) ||
         !um::tc_encode(&mp.acc, L->ws.acc_bf, 2ull * d.E * d.d_v, (uint64_t)Bmax, 1,
-                       (uint32_t)nt1, 2))
+                       (uint32_t)d.p_ntile, 2))
         return ULTRAMEM_ECUDA;
     // the projection reads the pooled rows as two bf16 terms hi + lo
     p.acc_bf = c.has_proj ? L->ws.acc_bf : nullptr;

@@ -53,6 +53,7 @@ struct Dims {
     uint64_t shuf_a, shuf_c;
     uint64_t shuf_mu;  // floor((2^64 - 1) / M), the Barrett constant of M
     int q_splits, p_splits;
+    int q_ntile, p_ntile;   // tensor path: token tiles of the query and the projection
     int pdl;           // host side: launch as a programmatic dependent of the
                        // previous kernel on the stream
     int probe_wait;    // ultramem_debug_wait_probe: the scoring kernel's

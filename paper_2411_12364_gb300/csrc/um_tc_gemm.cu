@@ -903,7 +903,7 @@ cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int 
                             __nv_bfloat16 *qs, int Bmax, bool x_splits, bool write_qs,
                             bool pdl, cudaStream_t st) {
     const int HD = d.H * d.d_k;
-    const int n_tile = tc_n_tile(d.B, 1);
+    const int n_tile = d.q_ntile ? d.q_ntile : tc_n_tile(d.B, 1);
     const int kb_total = (d.d_in + kBlockK - 1) / kBlockK;
     if (splits > kMaxSplits) return cudaErrorInvalidValue;
     for (int a = 0; a < d.A; ++a) {
@@ -964,7 +964,7 @@ cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaS
     if (d.p_splits > kMaxSplits) return cudaErrorInvalidValue;
     ProjOp op;
     op.stamp = p.stamp;
-    op.n_tile = tc_n_tile(d.B, 1);
+    op.n_tile = d.p_ntile ? d.p_ntile : tc_n_tile(d.B, 1);
     op.n_acc = 1;
     op.acc_chunk = 1 << 30;
     // the pooled rows are two bf16 terms hi + lo ([B][2][E D_v]): both
