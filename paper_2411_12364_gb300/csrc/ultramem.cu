@@ -364,6 +364,12 @@ Ptrs make_ptrs(ultramem_layer *L) {
 Dims dims_for(const ultramem_layer *L, int B) {
     Dims d = L->base;
     d.B = B;
+    // Long grids (more than three selection CTAs per SM) with more than 4096
+    // keys an axis: staging both axes' keys (8 K bytes) would leave room for
+    // fewer than 4 selection CTAs per SM, so the selection reads them from L2
+    // twice instead.  Measured at large_20m (K = 8960) with 256 tokens: select
+    // 71.3 -> 56.4 us (2 -> 4 CTAs per SM); at K = 4096 staging is as fast.
+    d.stream_keys = (int64_t)B * d.H > 3 * 152 && d.K > 4096 && d.K % 4 == 0;
     d.seq_len = B;   // one sequence unless the caller says otherwise
     d.q_splits = L->tc ? tc_query_splits(L->cfg, B) : query_splits(L->cfg, B);
     d.p_splits = L->tc ? tc_proj_splits(L->cfg, B) : proj_splits(L->cfg, B);

@@ -58,6 +58,8 @@ struct Dims {
                        // previous kernel on the stream
     int probe_wait;    // ultramem_debug_wait_probe: the scoring kernel's
                        // bounded wait on a barrier nothing signals
+    int stream_keys;   // the selection reads its rank-1 keys from L2 twice
+                       // instead of staging them in shared memory
 };
 
 struct Ptrs {

@@ -453,14 +453,16 @@ __host__ __device__ inline SelOffsets sel_offsets(const Dims &d) {
     SelOffsets o;
     size_t off = 0;
     o.qv = off;    off = up(off + sizeof(float) * 2 * d.d_k);
-    o.key0 = off;  off = up(off + sizeof(uint32_t) * (d.K > d.k * d.k ? d.K : d.k * d.k));
+    // streamed keys: the axes' keys stay in L2 (read twice), not in shared memory
+    const int Ka = d.stream_keys ? 0 : d.K;
+    o.key0 = off;  off = up(off + sizeof(uint32_t) * (Ka > d.k * d.k ? Ka : d.k * d.k));
     // with MCS (and with fp32 storage), key1's space later holds S_row of the
     // row survivors and the component cores (so that the block's shared
     // memory does not grow)
     const bool mcs = d.nc > 1;
     const bool keep_srow = mcs || d.dtype == ULTRAMEM_F32;
     const int mcs_floats = keep_srow ? d.k * d.r + (mcs ? d.nc * d.r * d.r : 0) : 0;
-    o.key1 = off;  off = up(off + sizeof(uint32_t) * (d.K > mcs_floats ? d.K : mcs_floats));
+    o.key1 = off;  off = up(off + sizeof(uint32_t) * (Ka > mcs_floats ? Ka : mcs_floats));
     o.srow = o.key1;
     o.cparts = o.key1 + sizeof(float) * d.k * d.r;
     o.sel_i = off; off = up(off + sizeof(int) * d.k);
@@ -491,9 +493,18 @@ __device__ SelLayout carve(const Dims &d, unsigned char *base) {
 // axis (padding reads as 0, below every key); all loads of a round are
 // issued before any store.  Each key is read once: the loads are streaming
 // (L2 evict-first), so that a long batch's keys do not push the key rows,
-// which every (token, head) reads again, out of L2.
+// which every (token, head) reads again, out of L2.  With `stream` the keys
+// are not stored (the compaction reads them again from L2) and are loaded
+// with the L2 caching kept.
+__device__ __forceinline__ uint4 ld_key4(const uint4 *p, bool stream) {
+    return stream ? __ldcg(p) : __ldcs(p);
+}
+__device__ __forceinline__ uint32_t ld_key(const uint32_t *p, bool stream) {
+    return stream ? __ldcg(p) : __ldcs(p);
+}
 __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1, int K,
-                                          const SelLayout &L, uint32_t (&top)[2][2]) {
+                                          const SelLayout &L, uint32_t (&top)[2][2],
+                                          bool stream) {
     uint32_t a1 = 0u, a2 = 0u, b1 = 0u, b2 = 0u;
     if ((K & 3) == 0) {
         const uint4 *V0 = reinterpret_cast<const uint4 *>(A0);
@@ -506,13 +517,13 @@ __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int i = v0 + q * kThreads;
-                a[q] = i < nv ? __ldcs(V0 + i) : make_uint4(0, 0, 0, 0);
-                c[q] = i < nv ? __ldcs(V1 + i) : make_uint4(0, 0, 0, 0);
+                a[q] = i < nv ? ld_key4(V0 + i, stream) : make_uint4(0, 0, 0, 0);
+                c[q] = i < nv ? ld_key4(V1 + i, stream) : make_uint4(0, 0, 0, 0);
             }
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int i = v0 + q * kThreads;
-                if (i < nv) {
+                if (i < nv && !stream) {
                     S0[i] = a[q];
                     S1[i] = c[q];
                 }
@@ -533,13 +544,13 @@ __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int i = i0 + q * kThreads;
-                a[q] = i < K ? __ldcs(A0 + i) : 0u;
-                c[q] = i < K ? __ldcs(A1 + i) : 0u;
+                a[q] = i < K ? ld_key(A0 + i, stream) : 0u;
+                c[q] = i < K ? ld_key(A1 + i, stream) : 0u;
             }
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int i = i0 + q * kThreads;
-                if (i < K) {
+                if (i < K && !stream) {
                     L.key0[i] = a[q];
                     L.key1[i] = c[q];
                 }
@@ -803,7 +814,11 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     float q0 = 0.f;
     if (threadIdx.x < 2 * d.d_k) q0 = one_split ? *q_src(threadIdx.x) : q_of(threadIdx.x);
     uint32_t top[2][2];
-    load_keys(A0, A1, K, L, top);
+    const bool stream = d.stream_keys != 0;   // uniform
+    load_keys(A0, A1, K, L, top, stream);
+    // the axes' keys: in shared memory, or (streamed) in L2, where the
+    // compaction reads them a second time
+    const uint32_t *KA = stream ? A0 : L.key0, *KB = stream ? A1 : L.key1;
     if (threadIdx.x < r * r) sh.core[threadIdx.x] = core_e;
     if (threadIdx.x < 2 * d.d_k) L.qv[threadIdx.x] = q0;
     for (int e = threadIdx.x + kThreads; e < 2 * d.d_k; e += kThreads) L.qv[e] = q_of(e);
@@ -811,11 +826,10 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     // Eq. 8-9: top-k of both axes
     warp_bounds(top[0][0], top[0][1], top[1][0], top[1][1], 2, k, sh);
     __syncthreads();
-    compact<2>(L.key0, L.key1, K, block_bound(0, sh), block_bound(1, sh), sh, kCntAxis,
-               kCntAxis + 1);
+    compact<2>(KA, KB, K, block_bound(0, sh), block_bound(1, sh), sh, kCntAxis, kCntAxis + 1);
     __syncthreads();
-    const int c0 = settle(0, L.key0, K, k, kCntAxis, kCntAxisT, sh);
-    const int c1 = settle(1, L.key1, K, k, kCntAxis + 1, kCntAxisT + 1, sh);
+    const int c0 = settle(0, KA, K, k, kCntAxis, kCntAxisT, sh);
+    const int c1 = settle(1, KB, K, k, kCntAxis + 1, kCntAxisT + 1, sh);
     {
         const int s = threadIdx.x >= kThreads / 2, cs = s ? c1 : c0;
         const int tid = threadIdx.x & (kThreads / 2 - 1);

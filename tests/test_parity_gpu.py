@@ -318,6 +318,8 @@ LONG_GRID = [
     dict(dtype=1, topk=32, topm=100),
     dict(dtype=0, n=600, topk=100, topm=128),                # axis lists over 128: counted
     dict(dtype=1, n=600, topk=96, topm=64),                  # k = 96: three S_col columns a lane
+    dict(dtype=1, n=2400, topk=64, topm=64),                 # K = 4800 > 4096: keys streamed from L2
+    dict(dtype=1, n=2049, topk=64, topm=64),                 # K = 4098, not a multiple of 4: staged
 ]
 
 
