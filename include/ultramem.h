@@ -283,8 +283,8 @@ ultramem_status ultramem_rank1(const float *core, int32_t r, float *u, float *t,
  * the previous stage to this stage's start; 0 for the first); it returns
  * the number of values written.  ultramem_stage_name names stage i (0 query
  * with the convolution and LayerNorm, 1 score, 2 select, 3 gather, 4
- * projection).  The timer's resolution is 32 ns on GB300.  Disabled by
- * default. */
+ * projection).  The timer advances in 256 ns steps on GB300, so average
+ * over many forwards.  Disabled by default. */
 ultramem_status ultramem_profile_enable(ultramem_layer *layer, int32_t enable);
 int32_t ultramem_profile_read(ultramem_layer *layer, float *ms, int32_t n);
 const char *ultramem_stage_name(int32_t i);

@@ -122,7 +122,10 @@ TcPlan tc_plan(int m_rows, int B, int kdim, int target, int max_splits, int nt_m
         if (s > max_splits) s = max_splits;
         if (s > kb) s = kb;
         if (s < 1) s = 1;
-        if (m_tiles * n_tiles * s >= target || nt <= nt_min) return {nt, s};
+        // a split tile's partial slices stay within shared memory: at most
+        // 128 tokens when split
+        if ((m_tiles * n_tiles * s >= target || nt <= nt_min) && (s == 1 || nt <= 128))
+            return {nt, s};
         nt = (nt / 2 + 15) / 16 * 16;
     }
 }

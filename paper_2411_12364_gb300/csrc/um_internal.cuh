@@ -277,8 +277,8 @@ template <auto K> size_t static_smem_of() {
 
 // ---- profiling stamps -----------------------------------------------------
 // While a layer profiles, each kernel of a forward records, in nanoseconds
-// of the GPU's global timer (32 ns resolution on GB300), the earliest moment
-// one of its CTAs passed its dependency wait (atomicMin into stamp[0]) and
+// of the GPU's global timer (it advances in 256 ns steps on GB300), the
+// earliest moment one of its CTAs passed its dependency wait (atomicMin into stamp[0]) and
 // the latest moment one of its warps finished (atomicMax into
 // stamp[kStampStages]); the kernels of one stage share the pair.  The
 // forward itself runs unchanged (programmatic dependent launches on), so the
