@@ -29,8 +29,8 @@ EXPORTS = ("ultramem_create", "ultramem_destroy", "ultramem_forward",
            "ultramem_last_launches", "ultramem_forward_seq", "ultramem_key_ln",
            "ultramem_retrieve_exact", "ultramem_lookup_reduce_backward",
            "ultramem_debug_wait_probe", "ultramem_debug_fail_alloc",
-           "ultramem_debug_live_allocations", "ultramem_shard_route", "ultramem_shard_lookup",
-           "ultramem_shard_pool")
+           "ultramem_debug_live_allocations", "ultramem_debug_candidates",
+           "ultramem_shard_route", "ultramem_shard_lookup", "ultramem_shard_pool")
 
 
 class Config(C.Structure):
@@ -119,6 +119,8 @@ def load(path: str | None = None) -> C.CDLL:
         lib.ultramem_debug_fail_alloc.restype = None
         lib.ultramem_debug_live_allocations.argtypes = []
         lib.ultramem_debug_live_allocations.restype = I32
+        lib.ultramem_debug_candidates.argtypes = [P, I32]
+        lib.ultramem_debug_candidates.restype = I32
         lib.ultramem_shard_route.argtypes = [P, P, I32, I32, I64, P, P, P, P]
         lib.ultramem_shard_route.restype = I32
         lib.ultramem_shard_lookup.argtypes = [P, P, I64, P, P]
@@ -386,6 +388,10 @@ class UltraMemLayer:
     def check(self) -> int:
         """Syncs the current stream and returns the device error status."""
         return int(self.lib.ultramem_check(self._h, _stream()))
+
+    def candidates(self, mode: int):
+        """Scoring form (test hook): 0 every key (default), 1 candidate lists."""
+        _check(self.lib.ultramem_debug_candidates(self._h, int(mode)), "debug_candidates")
 
     def last_launches(self) -> int:
         """Kernels launched by the most recent successful call on this layer."""

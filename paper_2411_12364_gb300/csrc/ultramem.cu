@@ -21,7 +21,9 @@ const char *const kStageNames[kStages] = {"query", "score", "select", "gather", 
 
 struct Workspace {
     float *q_part = nullptr, *sel_w = nullptr, *acc = nullptr, *proj_part = nullptr;
-    uint32_t *akey = nullptr;
+    uint32_t *akey = nullptr;   // the rank-1 keys [B][H][2][K], or (Dims::cand) the
+                                // candidate lists [B][H][2][16 G] u64 in the same space
+    uint32_t *gstat = nullptr, *tau = nullptr;   // candidate lists: group maxima / counts, bounds
     int32_t *sel_row = nullptr, *sel_p = nullptr;
     float *core = nullptr, *u = nullptr, *t = nullptr;
     float *cores = nullptr;   // MCS component cores [H][h][r][r] (h > 1 only)
@@ -67,6 +69,8 @@ struct ultramem_layer {
     cudaStream_t capture = nullptr;
     bool x_after_copy = false;   // x is written by the copy kernel just before the forward
     bool probe_armed = false;    // ultramem_debug_wait_probe: the next forward's score probes
+    bool cand_ok = false;        // the candidate-list scoring fits this layer
+    int cand_mode = 0;           // ultramem_debug_candidates: 0 every key, 1 candidate lists
     bool dacc_tc = false;        // the backward's dacc may run on the tensor cores
 };
 
@@ -325,7 +329,7 @@ template <typename T> cudaError_t dalloc(T **p, size_t n) {
 }
 
 void free_workspace(Workspace &ws) {
-    void *ptrs[] = {ws.q_part, ws.akey, ws.sel_w,   ws.acc,       ws.proj_part,
+    void *ptrs[] = {ws.q_part, ws.akey, ws.gstat, ws.tau, ws.sel_w,   ws.acc,       ws.proj_part,
                     ws.sel_row, ws.sel_p, ws.core,   ws.u,         ws.t,
                     ws.err,    ws.x_stage, ws.out_stage, ws.qs,     ws.acc_bf,
                     ws.w_pt,   ws.cores,   ws.xs,      ws.dacc,    ws.bwd_t,
@@ -355,6 +359,9 @@ Ptrs make_ptrs(ultramem_layer *L) {
     p.t = L->ws.t;
     p.q_part = L->ws.q_part;
     p.akey = L->ws.akey;
+    p.gstat = L->ws.gstat;
+    p.tau = L->ws.tau;
+    p.cand = reinterpret_cast<unsigned long long *>(L->ws.akey);
     p.sel_w = L->ws.sel_w;
     p.acc = L->ws.acc;
     p.proj_part = L->ws.proj_part;
@@ -373,6 +380,14 @@ Dims dims_for(const ultramem_layer *L, int B) {
     // twice instead.  Measured at large_20m (K = 8960) with 256 tokens: select
     // 71.3 -> 56.4 us (2 -> 4 CTAs per SM); at K = 4096 staging is as fast.
     d.stream_keys = (int64_t)B * d.H > 3 * 152 && d.K > 4096 && d.K % 4 == 0;
+    // On request (ultramem_debug_candidates) the tensor path scores twice and
+    // leaves per-axis candidate lists (ScoreListOp): the keys' round trip
+    // through memory goes and the selection starts from about 2 % of them,
+    // but the second contraction costs more than that saves on GB300 (the
+    // scoring passes are bound by L2 -> SM operand traffic), so every key
+    // is written by default.
+    d.cand = L->cand_ok && L->cand_mode == 1 ? 1 : 0;
+    if (d.cand) d.stream_keys = 0;
     d.seq_len = B;   // one sequence unless the caller says otherwise
     d.q_splits = L->tc ? tc_query_splits(L->cfg, B) : query_splits(L->cfg, B);
     d.p_splits = L->tc ? tc_proj_splits(L->cfg, B) : proj_splits(L->cfg, B);
@@ -463,6 +478,9 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     if (conv && !um::tc_encode(&mp.xs, L->ws.xs, 3ull * c.d_in, (uint64_t)d.B, 1,
                                (uint32_t)d.q_ntile, 2))
         return ULTRAMEM_ECUDA;
+    if (d.cand && !um::tc_encode(&mp.qs_t, L->ws.qs, 3ull * c.d_k, (uint64_t)Bmax, 2ull * d.H,
+                                 128u, 3))
+        return ULTRAMEM_ECUDA;
     if (!um::tc_encode(&mp.qs, L->ws.qs, 3ull * c.d_k, (uint64_t)Bmax, 2ull * d.H,
                        (uint32_t)nt1, 3) ||
         !um::tc_encode(&mp.acc, L->ws.acc_bf, 2ull * d.E * d.d_v, (uint64_t)Bmax, 1,
@@ -514,12 +532,15 @@ ultramem_status run_tensor(ultramem_layer *L, const Dims &d, Ptrs p, cudaStream_
     Dims ds = dd;
     ds.q_splits = 1;   // the query projection wrote the summed query
     if ((e = um::launch_select(ds, stage_ptrs(L, p, 2), st)) != cudaSuccess) return from_cuda(e);
-    *launches = d.A + 2 + extras;   // one query projection per query
+    // one query projection per query; the candidate-list scoring is three
+    // launches (two passes and the bound)
+    const int score = d.cand ? 3 : 1;
+    *launches = d.A + 1 + score + extras;
     if (mode == kRetrieve) return ULTRAMEM_OK;
     if ((e = um::launch_gather(dd, stage_ptrs(L, p, 3), st)) != cudaSuccess) return from_cuda(e);
     if (d.has_proj && (e = um::launch_proj_tc(dd, stage_ptrs(L, p, 4), mp, st)) != cudaSuccess)
         return from_cuda(e);
-    *launches = d.A + 3 + (d.has_proj ? 1 : 0) + extras;
+    *launches = d.A + 2 + score + (d.has_proj ? 1 : 0) + extras;
     if (L->profiling) L->profiled_once = true;
     return ULTRAMEM_OK;
 }
@@ -637,6 +658,7 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     d.r = r;
     d.dk = cfg->d_k / r;
     d.K = (int)keys_per_axis(*cfg);
+    d.n_groups = (d.K + 15) / 16;
     d.N = (int64_t)cfg->n * cfg->n;
     d.M = (uint64_t)cfg->expand_e * (uint64_t)d.N;
     d.E = cfg->expand_e;
@@ -680,7 +702,16 @@ ultramem_status ultramem_create(const ultramem_config *cfg, const ultramem_weigh
     cudaError_t e = cudaSuccess;
     const size_t hm = Bm * H * cfg->topm;
     if (e == cudaSuccess) e = dalloc(&ws.q_part, qmax * d.A * HD);
-    if (e == cudaSuccess) e = dalloc(&ws.akey, Bm * H * 2 * (size_t)d.K);
+    // the candidate-list scoring (long grids, tensor path) keeps its u64
+    // lists (16 G entries an axis) where the keys would be
+    L->cand_ok = L->tc && d.n_groups >= d.k && d.n_groups <= 1024;
+    const size_t lists = Bm * H * 2;
+    const size_t key_words = lists * (size_t)d.K;
+    const size_t list_words = lists * 16 * (size_t)d.n_groups * 2;
+    if (e == cudaSuccess)
+        e = dalloc(&ws.akey, L->cand_ok && list_words > key_words ? list_words : key_words);
+    if (e == cudaSuccess && L->cand_ok) e = dalloc(&ws.gstat, lists * (size_t)d.n_groups);
+    if (e == cudaSuccess && L->cand_ok) e = dalloc(&ws.tau, lists);
     if (e == cudaSuccess) e = dalloc(&ws.sel_w, hm * nc);
     if (e == cudaSuccess) e = dalloc(&ws.sel_row, hm);
     if (e == cudaSuccess) e = dalloc(&ws.sel_p, hm);
@@ -1105,6 +1136,13 @@ ultramem_status ultramem_debug_wait_probe(ultramem_layer *L) {
 void ultramem_debug_fail_alloc(int32_t nth) { g_fail_countdown.store(nth < 0 ? -1 : nth); }
 
 int32_t ultramem_debug_live_allocations(void) { return g_live_allocs.load(); }
+
+ultramem_status ultramem_debug_candidates(ultramem_layer *L, int32_t mode) {
+    if (!L || mode < 0 || mode > 1) return ULTRAMEM_EINVAL;
+    if (mode == 1 && !L->cand_ok) return ULTRAMEM_ENODEV;
+    L->cand_mode = mode;
+    return ULTRAMEM_OK;
+}
 
 ultramem_status ultramem_profile_enable(ultramem_layer *L, int32_t enable) {
     if (!L) return ULTRAMEM_EINVAL;

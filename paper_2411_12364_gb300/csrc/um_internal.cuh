@@ -60,6 +60,9 @@ struct Dims {
                        // bounded wait on a barrier nothing signals
     int stream_keys;   // the selection reads its rank-1 keys from L2 twice
                        // instead of staging them in shared memory
+    int cand;          // tensor path, long grids: the scoring leaves per-axis
+                       // candidate lists instead of every key (see ScoreOp)
+    int n_groups;      // candidate lists: groups of 16 keys an axis, ceil(K / 16)
 };
 
 struct Ptrs {
@@ -69,6 +72,12 @@ struct Ptrs {
     const float *cores;          // [H][nc][r][r] component cores when nc > 1
     float *q_part, *sel_w, *acc, *proj_part;
     uint32_t *akey;
+    // candidate lists (Dims::cand): per (token, head, axis) the largest key
+    // of each group of 16 keys, then the group's count of candidates
+    // [B][H][2][n_groups], the bound tau [B][H][2] and the list of
+    // composites, a 16-entry segment per group [B][H][2][n_groups][16]
+    uint32_t *gstat, *tau;
+    unsigned long long *cand;
     int32_t *sel_row, *sel_p;
     void *out;
     int64_t *idx_out;
@@ -92,6 +101,7 @@ struct Ptrs {
 struct TcMaps {
     CUtensorMap w_q, w_q_col, k_row, k_col, w_pt;
     CUtensorMap x, qs, acc;
+    CUtensorMap qs_t;    // the split queries with 128-token boxes (candidate lists)
     CUtensorMap xs;      // the convolved input's three bf16 terms [B][3 D_i]
     CUtensorMap w_p;     // the projectors as stored, [E D_v][D'_v] (backward's A)
 };
@@ -105,6 +115,9 @@ cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int 
                             __nv_bfloat16 *qs, int Bmax, bool x_splits, bool write_qs,
                             bool pdl, cudaStream_t st);
 cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st);
+// candidate lists: tau = the k-th largest group maximum per (token, head,
+// axis)
+cudaError_t launch_cand_bound(const Dims &d, const Ptrs &p, cudaStream_t st);
 // small batches: S1 on CUDA cores, 16 weight rows x 8 tokens per CTA
 cudaError_t configure_small();
 // x_f32: the token rows are the fp32 convolved input (p.xs, [B][D_i])
@@ -317,6 +330,14 @@ __device__ __forceinline__ float ord2f(uint32_t o) {
     uint32_t u = (o & 0x80000000u) ? (o & 0x7fffffffu) : ~o;
     return __uint_as_float(u);
 }
+
+// A selection candidate: (key, position) as one 64-bit value whose
+// descending order is key descending, then position ascending.
+__device__ __forceinline__ unsigned long long comp_of(uint32_t key, uint32_t pos) {
+    return ((unsigned long long)key << 32) | (unsigned long long)(~pos);
+}
+__device__ __forceinline__ uint32_t key_of(unsigned long long c) { return (uint32_t)(c >> 32); }
+__device__ __forceinline__ uint32_t pos_of(unsigned long long c) { return ~(uint32_t)c; }
 
 // The scoring contraction's B operand for one query element: q[h][c] scaled
 // by the rank-1 coefficient of its chunk (u for the row keys, t for the

@@ -71,12 +71,6 @@ struct SelShared {
     double dscalar;   // fp32 storage: the softmax denominator in fp64
 };
 
-__device__ __forceinline__ u64 comp_of(uint32_t key, uint32_t pos) {
-    return ((u64)key << 32) | (u64)(~pos);
-}
-__device__ __forceinline__ uint32_t key_of(u64 c) { return (uint32_t)(c >> 32); }
-__device__ __forceinline__ uint32_t pos_of(u64 c) { return ~(uint32_t)c; }
-
 template <typename T>
 __device__ __forceinline__ void unpack16(uint4 v, float (&f)[16 / sizeof(T)]);
 template <>
@@ -158,6 +152,40 @@ __device__ int block_exclusive_scan(int v, SelShared &sh) {
     return before + incl - v;
 }
 
+// One digit of a radix select: given the histogram of the current digit
+// over the entries that match the digits chosen so far, warp 0 finds the
+// digit that holds the `remaining`-th largest entry and leaves it, and the
+// rank still to go within it, in sh.digit and sh.remaining.
+__device__ __forceinline__ void radix_digit(int remaining, SelShared &sh) {
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        int cnt[8], s = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            cnt[j] = sh.hist[255 - 8 * lane - j];
+            s += cnt[j];
+        }
+        int incl = s;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            int y = __shfl_up_sync(kFull, incl, off);
+            if (lane >= off) incl += y;
+        }
+        int before = incl - s;
+        if (before < remaining && remaining <= incl) {
+            int acc = before;
+            for (int j = 0; j < 8; ++j) {
+                if (acc + cnt[j] >= remaining) {
+                    sh.digit = 255 - 8 * lane - j;
+                    sh.remaining = remaining - acc;
+                    break;
+                }
+                acc += cnt[j];
+            }
+        }
+    }
+}
+
 // Radix select (8-bit digits, most significant first) of the kk-th largest
 // key among key[0..n).  Returns that key T; *need_eq = how many keys equal to
 // T belong to the top kk (count(key > T) = kk - *need_eq).
@@ -173,33 +201,7 @@ __device__ uint32_t select_kth_largest(const uint32_t *key, int n, int kk, SelSh
             if ((v & mask) == prefix) atomicAdd(&sh.hist[(v >> shift) & 255u], 1);
         }
         __syncthreads();
-        if (threadIdx.x < 32) {
-            const int lane = threadIdx.x;
-            int cnt[8], s = 0;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                cnt[j] = sh.hist[255 - 8 * lane - j];
-                s += cnt[j];
-            }
-            int incl = s;
-#pragma unroll
-            for (int off = 1; off < 32; off <<= 1) {
-                int y = __shfl_up_sync(kFull, incl, off);
-                if (lane >= off) incl += y;
-            }
-            int before = incl - s;
-            if (before < remaining && remaining <= incl) {
-                int acc = before;
-                for (int j = 0; j < 8; ++j) {
-                    if (acc + cnt[j] >= remaining) {
-                        sh.digit = 255 - 8 * lane - j;
-                        sh.remaining = remaining - acc;
-                        break;
-                    }
-                    acc += cnt[j];
-                }
-            }
-        }
+        radix_digit(remaining, sh);
         __syncthreads();
         prefix |= (uint32_t)sh.digit << shift;
         mask |= 255u << shift;
@@ -249,6 +251,86 @@ __device__ __forceinline__ void warp_append(bool pr, u64 comp, u64 *list, int *c
     base = __shfl_sync(kFull, base, 0);
     const int slot = base + __popc(bal & ((1u << lane) - 1u));
     if (pr && slot < kCap) list[slot] = comp;
+}
+
+// The scoring's candidate list of axis s (Dims::cand): every key of the
+// axis' top k is in it, with the keys above a bound, as composites.  The
+// list is G segments of 16 entries (one per group of 16 keys); segment g
+// holds its group's candidates in its first cnt[g] entries (the counts
+// replace the group maxima in gstat).  Up to kCap entries are gathered
+// into cand[s] (placed by a block scan of the threads' counts); a longer
+// list (heavy ties) is replaced by its exact top kk, a radix select over the
+// 64-bit composites (distinct: exactly kk are >= the kk-th largest).
+// Length in cnt[slot].  Whole block; ends with a barrier.
+constexpr int kSeg = 16;               // entries of a list segment (keys of a group)
+constexpr int kMaxSegPerThread = 4;   // G <= 1024 segments
+__device__ __noinline__ void cand_fallback(const u64 *seg, const uint32_t *cnt, int G, int kk,
+                                           int s, int slot, SelShared &sh) {
+    const int n = kSeg * G;
+    auto entry = [&](int i) -> u64 {   // 0 for an empty slot (below every composite kept)
+        return i % kSeg < (int)min(cnt[i / kSeg], (uint32_t)kSeg) ? seg[i] : 0ull;
+    };
+    u64 prefix = 0, mask = 0;
+    int remaining = kk;
+    for (int shift = 56; shift >= 0; shift -= 8) {
+        for (int i = threadIdx.x; i < 256; i += kThreads) sh.hist[i] = 0;
+        __syncthreads();
+        for (int i = threadIdx.x; i < n; i += kThreads) {
+            const u64 v = entry(i);
+            if (v && (v & mask) == prefix) atomicAdd(&sh.hist[(int)((v >> shift) & 255u)], 1);
+        }
+        __syncthreads();
+        radix_digit(remaining, sh);
+        __syncthreads();
+        prefix |= (u64)sh.digit << shift;
+        mask |= (u64)255 << shift;
+        remaining = sh.remaining;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) sh.cnt[slot] = 0;
+    __syncthreads();
+    for (int i0 = 0; i0 < n; i0 += kThreads) {   // uniform trip count
+        const int i = i0 + threadIdx.x;
+        const u64 v = i < n ? entry(i) : 0ull;
+        warp_append(v && v >= prefix, v, sh.cand[s], &sh.cnt[slot]);
+    }
+    __syncthreads();
+}
+
+__device__ void load_list(const Ptrs &p, int64_t list, int G, int kk, int s, int slot,
+                          SelShared &sh) {
+    const uint32_t *cnt = p.gstat + list * G;
+    const u64 *seg = p.cand + list * (int64_t)G * kSeg;
+    int mine[kMaxSegPerThread], tot = 0;
+#pragma unroll
+    for (int q = 0; q < kMaxSegPerThread; ++q) {
+        const int g = threadIdx.x + q * kThreads;
+        mine[q] = g < G ? (int)min(cnt[g], (uint32_t)kSeg) : 0;
+        tot += mine[q];
+    }
+    int o = block_exclusive_scan(tot, sh);
+    if (threadIdx.x == kThreads - 1) sh.cnt[slot] = o + tot;
+    __syncthreads();
+    const int c = sh.cnt[slot];
+    if (c > kCap) {
+        cand_fallback(seg, cnt, G, kk, s, slot, sh);
+        return;
+    }
+#pragma unroll
+    for (int q = 0; q < kMaxSegPerThread; ++q) {
+        const u64 *sg = seg + (int64_t)(threadIdx.x + q * kThreads) * kSeg;
+        for (int e = 0; e < mine[q]; ++e) sh.cand[s][o++] = sg[e];
+    }
+    // fewer than kk is impossible (the bound guarantees kk); should it
+    // happen, positions past K mark the missing entries (recorded)
+    for (int f = c + threadIdx.x; f < kk; f += kThreads)
+        sh.cand[s][f] = comp_of(0u, 0xffffffffu - (uint32_t)f);
+    __syncthreads();
+    if (threadIdx.x == 0 && c < kk) {
+        sh.cnt[slot] = kk;
+        atomicOr(p.err, kErrInternal);
+    }
+    __syncthreads();
 }
 
 // Appends key[i] >= tau_s (i < n) of NS selections to their lists.  A round
@@ -453,8 +535,9 @@ __host__ __device__ inline SelOffsets sel_offsets(const Dims &d) {
     SelOffsets o;
     size_t off = 0;
     o.qv = off;    off = up(off + sizeof(float) * 2 * d.d_k);
-    // streamed keys: the axes' keys stay in L2 (read twice), not in shared memory
-    const int Ka = d.stream_keys ? 0 : d.K;
+    // streamed keys: the axes' keys stay in L2 (read twice), not in shared
+    // memory; candidate lists: the selection reads no keys
+    const int Ka = d.stream_keys || d.cand ? 0 : d.K;
     o.key0 = off;  off = up(off + sizeof(uint32_t) * (Ka > d.k * d.k ? Ka : d.k * d.k));
     // with MCS (and with fp32 storage), key1's space later holds S_row of the
     // row survivors and the component cores (so that the block's shared
@@ -815,7 +898,10 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     if (threadIdx.x < 2 * d.d_k) q0 = one_split ? *q_src(threadIdx.x) : q_of(threadIdx.x);
     uint32_t top[2][2];
     const bool stream = d.stream_keys != 0;   // uniform
-    load_keys(A0, A1, K, L, top, stream);
+    // candidate lists: only the long-grid instantiation reads them (the
+    // launch picks it whenever they are on)
+    const bool lists = MINB >= 4 && d.cand;
+    if (!lists) load_keys(A0, A1, K, L, top, stream);
     // the axes' keys: in shared memory, or (streamed) in L2, where the
     // compaction reads them a second time
     const uint32_t *KA = stream ? A0 : L.key0, *KB = stream ? A1 : L.key1;
@@ -824,10 +910,17 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     for (int e = threadIdx.x + kThreads; e < 2 * d.d_k; e += kThreads) L.qv[e] = q_of(e);
 
     // Eq. 8-9: top-k of both axes
-    warp_bounds(top[0][0], top[0][1], top[1][0], top[1][1], 2, k, sh);
-    __syncthreads();
-    compact<2>(KA, KB, K, block_bound(0, sh), block_bound(1, sh), sh, kCntAxis, kCntAxis + 1);
-    __syncthreads();
+    if (lists) {   // the scoring left each axis' candidates
+        __syncthreads();
+        for (int s = 0; s < 2; ++s)
+            load_list(p, ((int64_t)b * d.H + h) * 2 + s, d.n_groups, k, s, kCntAxis + s, sh);
+    } else {
+        warp_bounds(top[0][0], top[0][1], top[1][0], top[1][1], 2, k, sh);
+        __syncthreads();
+        compact<2>(KA, KB, K, block_bound(0, sh), block_bound(1, sh), sh, kCntAxis,
+                   kCntAxis + 1);
+        __syncthreads();
+    }
     const int c0 = settle(0, KA, K, k, kCntAxis, kCntAxisT, sh);
     const int c1 = settle(1, KB, K, k, kCntAxis + 1, kCntAxisT + 1, sh);
     {
@@ -1044,6 +1137,44 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     stamp_end(p.stamp);
 }
 
+// Candidate lists (Dims::cand), between the two scoring passes: the bound of
+// one (token, head, axis) per warp.  tau is the k-th largest of the axis'
+// G group maxima (groups of 16 keys), found bit by bit from the top (the largest T with at
+// least k maxima >= T); k distinct groups hold a key >= tau, so the axis'
+// top k is among the keys >= tau.
+constexpr int kBoundWarps = 8;
+constexpr int kMaxGroupsPerLane = 32;   // G <= 1024 groups (K <= 16384 keys)
+static_assert(32 * kMaxGroupsPerLane == kMaxSegPerThread * kThreads, "one limit on G");
+template <int NQ>   // group maxima a lane holds, 32 NQ >= G
+__global__ void __launch_bounds__(32 * kBoundWarps) cand_bound_kernel(Dims d, Ptrs p) {
+    pdl_wait();
+    stamp_begin(p.stamp);
+    pdl_trigger();
+    const int lane = threadIdx.x & 31;
+    const int64_t w = (int64_t)blockIdx.x * kBoundWarps + (threadIdx.x >> 5);
+    if (w < (int64_t)d.B * d.H * 2) {   // warp-uniform
+        const int G = d.n_groups;
+        const uint32_t *g = p.gstat + w * G;
+        uint32_t v[NQ];
+#pragma unroll
+        for (int q = 0; q < NQ; ++q) {
+            const int e = lane + 32 * q;
+            v[q] = e < G ? g[e] : 0u;   // 0: below every score's key
+        }
+        uint32_t T = 0u;
+#pragma unroll 4
+        for (int bit = 31; bit >= 0; --bit) {
+            const uint32_t c = T | (1u << bit);
+            int n = 0;
+#pragma unroll
+            for (int q = 0; q < NQ; ++q) n += v[q] >= c;
+            if (__reduce_add_sync(kFull, n) >= d.k) T = c;
+        }
+        if (lane == 0) p.tau[w] = T;
+    }
+    stamp_end(p.stamp);
+}
+
 // lookup_reduce input: given virtual addresses and weights -> (row, p, w).
 // An address outside [0, E*N) is recorded in the error word and skipped
 // (weights 0, row 0).  With MCS each slot has nc weights.
@@ -1072,7 +1203,7 @@ size_t select_smem_bytes(const Dims &d) { return sel_offsets(d).total; }
 
 template <typename T, int RM>
 static cudaError_t launch_select_t(const Dims &d, const Ptrs &p, size_t smem, cudaStream_t st) {
-    if (d.B * d.H > 3 * 152)
+    if (d.B * d.H > 3 * 152 || d.cand)
         return launch_kernel(d.pdl, select_kernel<T, 4, RM>, d.B * d.H, kThreads, smem, st, d, p);
     // decode grids: spread over the SMs (see spread_smem)
     const size_t sm = spread_smem(smem, static_smem_of<select_kernel<T, 3, RM>>(), d.B * d.H);
@@ -1086,6 +1217,22 @@ cudaError_t launch_select(const Dims &d, const Ptrs &p, cudaStream_t st) {
                         : launch_select_t<__nv_bfloat16, kMaxR>(d, p, smem, st);
     return d.r <= 2 ? launch_select_t<float, 2>(d, p, smem, st)
                     : launch_select_t<float, kMaxR>(d, p, smem, st);
+}
+
+cudaError_t launch_cand_bound(const Dims &d, const Ptrs &p, cudaStream_t st) {
+    if (d.n_groups < d.k || d.n_groups > 32 * kMaxGroupsPerLane) return cudaErrorInvalidValue;
+    const int64_t warps = (int64_t)d.B * d.H * 2;
+    const int blocks = (int)((warps + kBoundWarps - 1) / kBoundWarps);
+    const int nq = (d.n_groups + 31) / 32;
+    auto go = [&](auto kernel) {
+        return launch_kernel(d.pdl, kernel, blocks, 32 * kBoundWarps, 0, st, d, p);
+    };
+    if (nq <= 1) return go(cand_bound_kernel<1>);
+    if (nq <= 2) return go(cand_bound_kernel<2>);
+    if (nq <= 4) return go(cand_bound_kernel<4>);
+    if (nq <= 8) return go(cand_bound_kernel<8>);
+    if (nq <= 16) return go(cand_bound_kernel<16>);
+    return go(cand_bound_kernel<kMaxGroupsPerLane>);
 }
 
 cudaError_t launch_slots_from_addresses(const Dims &d, const Ptrs &p, cudaStream_t st) {

@@ -84,6 +84,21 @@ inline int stages_for(int nsplit, int n_tile, int nkb) {
     return s < 1 ? 1 : s;
 }
 
+// An op with kSwapAB = true multiplies with the roles of the staged tiles
+// swapped: the B tiles (n_tile = 128 rows) are the MMA's A operand, so that
+// they land on TMEM lanes, and the 128-row A tile is its B operand (128
+// accumulator columns).  Loads, ring and barriers are the same.
+template <class Op, class = void> struct SwapAB {
+    static constexpr bool value = false;
+};
+template <class Op> struct SwapAB<Op, std::void_t<decltype(Op::kSwapAB)>> {
+    static constexpr bool value = Op::kSwapAB;
+};
+// accumulator columns of one MMA: n_tile, or 128 when swapped
+template <class Op> __host__ __device__ inline int acc_cols_of(const Op &op) {
+    return SwapAB<Op>::value ? kTileM : op.n_tile;
+}
+
 template <int NSPLIT, class Op>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap mapA0,
@@ -106,9 +121,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n_tile = op.n_tile;
     const uint32_t b_bytes = (uint32_t)n_tile * 128;
     const uint32_t stage_bytes = kTileABytes + NSPLIT * b_bytes;
+    constexpr bool kSwap = SwapAB<Op>::value;
+    const int acc_n = acc_cols_of(op);   // accumulator columns
     // the epilogue reads 32 columns at a time: cover the last such read
     const uint32_t ncols =
-        tmem_cols_for((uint32_t)((op.n_acc - 1) * n_tile + ((n_tile - 1) / 32) * 32 + 32));
+        tmem_cols_for((uint32_t)((op.n_acc - 1) * acc_n + ((acc_n - 1) / 32) * 32 + 32));
     const CUtensorMap *mapA = t.a_sel ? &mapA1 : &mapA0;
     const int kStages = op.stages;
 
@@ -197,7 +214,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // MMA issuer.  Descriptors are built once per stage and advanced by
         // 32 bytes (2 in the >>4 address field) per 16-wide K step; the
         // accumulator of each step follows its rank chunk without division.
-        const uint32_t idesc = idesc_bf16_f32(kTileM, n_tile);
+        const uint32_t idesc = kSwap ? idesc_bf16_f32(n_tile, kTileM) : idesc_bf16_f32(kTileM, n_tile);
         uint32_t started = 0;
         int acc = (t.kb0 * kBlockK) / op.acc_chunk;
         int next_chunk = (acc + 1) * op.acc_chunk;   // K index where acc advances
@@ -220,11 +237,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ++acc;
                     next_chunk += op.acc_chunk;
                 }
-                const uint32_t dt = tmem + (uint32_t)(acc * n_tile);
+                const uint32_t dt = tmem + (uint32_t)(acc * acc_n);
                 const uint32_t acc_bit = 1u << acc;
 #pragma unroll
                 for (int j = 0; j < NSPLIT; ++j) {
-                    mma_bf16(dt, ad0 + 2 * k16, bd0[j] + 2 * k16, idesc, started & acc_bit);
+                    if constexpr (kSwap)
+                        mma_bf16(dt, bd0[j] + 2 * k16, ad0 + 2 * k16, idesc, started & acc_bit);
+                    else
+                        mma_bf16(dt, ad0 + 2 * k16, bd0[j] + 2 * k16, idesc, started & acc_bit);
                     started |= acc_bit;
                 }
             }
@@ -244,21 +264,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row = quad * 32 + lane;
     const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
     if (S == 1) {
-        for (int c0 = whalf * 32; c0 < n_tile; c0 += 32 * kGroups) {
+        // a per-chunk value the op fetches one chunk ahead (the candidate
+        // lists' bounds), so that its latency overlaps the previous chunk
+        uint32_t pre = op.prefetch(t, row, whalf * 32);
+        for (int c0 = whalf * 32; c0 < acc_n; c0 += 32 * kGroups) {
+            const uint32_t cur = pre;
+            if (c0 + 32 * kGroups < acc_n) pre = op.prefetch(t, row, c0 + 32 * kGroups);
             uint32_t r[kMaxAcc][32];
 #pragma unroll
             for (int a = 0; a < kMaxAcc; ++a)
-                if (a < op.n_acc) tmem_ld32_nowait(lane_base + (uint32_t)(a * n_tile + c0), r[a]);
+                if (a < op.n_acc) tmem_ld32_nowait(lane_base + (uint32_t)(a * acc_n + c0), r[a]);
             tmem_ld_wait();
 #pragma unroll
             for (int half = 0; half < 2; ++half) {
-                if (c0 + half * 16 >= n_tile) break;
+                if (c0 + half * 16 >= acc_n) break;
                 float v[kMaxAcc][16];
 #pragma unroll
                 for (int a = 0; a < kMaxAcc; ++a)
 #pragma unroll
                     for (int i = 0; i < 16; ++i) v[a][i] = __uint_as_float(r[a][half * 16 + i]);
-                op.store(t, row, c0 + half * 16, v);
+                op.store(t, row, c0 + half * 16, v, cur);
             }
         }
         tc_fence_before();
@@ -441,7 +466,9 @@ __global__ void __launch_bounds__(kPThreads, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             // MMA issuer
-            const uint32_t idesc = idesc_bf16_f32(kTileM, n_tile);
+            constexpr bool kSwap = SwapAB<Op>::value;
+            const uint32_t idesc = kSwap ? idesc_bf16_f32(n_tile, kTileM) : idesc_bf16_f32(kTileM, n_tile);
+            const int acc_n = acc_cols_of(op);
             int it = 0, lt = 0;
             for (int i = blockIdx.x; i < tiles && !abort_flag; i += gridDim.x, ++lt) {
                 const Tile t = tile_of(i);
@@ -477,12 +504,16 @@ __global__ void __launch_bounds__(kPThreads, 1)
                             ++acc;
                             next_chunk += op.acc_chunk;
                         }
-                        const uint32_t dt = dbase + (uint32_t)(acc * n_tile);
+                        const uint32_t dt = dbase + (uint32_t)(acc * acc_n);
                         const uint32_t acc_bit = 1u << acc;
 #pragma unroll
                         for (int j = 0; j < NSPLIT; ++j) {
-                            mma_bf16(dt, ad0 + 2 * k16, bd0[j] + 2 * k16, idesc,
-                                     started & acc_bit);
+                            if constexpr (kSwap)
+                                mma_bf16(dt, bd0[j] + 2 * k16, ad0 + 2 * k16, idesc,
+                                         started & acc_bit);
+                            else
+                                mma_bf16(dt, ad0 + 2 * k16, bd0[j] + 2 * k16, idesc,
+                                         started & acc_bit);
                             started |= acc_bit;
                         }
                     }
@@ -512,21 +543,25 @@ __global__ void __launch_bounds__(kPThreads, 1)
             tc_fence_after();
             const uint32_t lane_base =
                 tmem + (uint32_t)buf * buf_cols + ((uint32_t)(quad * 32) << 16);
-            for (int c0 = grp * 32; c0 < n_tile; c0 += 64) {
+            const int acc_n = acc_cols_of(op);
+            uint32_t pre = op.prefetch(t, row, grp * 32);   // one chunk ahead, as above
+            for (int c0 = grp * 32; c0 < acc_n; c0 += 64) {
+                const uint32_t cur = pre;
+                if (c0 + 64 < acc_n) pre = op.prefetch(t, row, c0 + 64);
                 uint32_t r[kMaxAcc][32];
 #pragma unroll
                 for (int a = 0; a < kMaxAcc; ++a)
-                    if (a < op.n_acc) tmem_ld32_nowait(lane_base + (uint32_t)(a * n_tile + c0), r[a]);
+                    if (a < op.n_acc) tmem_ld32_nowait(lane_base + (uint32_t)(a * acc_n + c0), r[a]);
                 tmem_ld_wait();
 #pragma unroll
                 for (int half = 0; half < 2; ++half) {
-                    if (c0 + half * 16 >= n_tile) break;
+                    if (c0 + half * 16 >= acc_n) break;
                     float v[kMaxAcc][16];
 #pragma unroll
                     for (int a = 0; a < kMaxAcc; ++a)
 #pragma unroll
                         for (int q = 0; q < 16; ++q) v[a][q] = __uint_as_float(r[a][half * 16 + q]);
-                    op.store(t, row, c0 + half * 16, v);
+                    op.store(t, row, c0 + half * 16, v, cur);
                 }
             }
             tc_fence_before();
@@ -586,7 +621,9 @@ struct QueryOp {
             if (col_axis) put_split_query(qs, 1, h, c, n, v[j] * ct, H, Bmax, d_k);
         }
     }
-    __device__ void store(const Tile &tl, int row, int c, float (&v)[kMaxAcc][16]) const {
+    __device__ uint32_t prefetch(const Tile &, int, int) const { return 0u; }
+    __device__ void store(const Tile &tl, int row, int c, float (&v)[kMaxAcc][16],
+                          uint32_t) const {
         const int m = tl.m0 + row;
         if (m >= HD) return;
         float w[16];
@@ -605,6 +642,7 @@ struct QueryOp {
 // (u or t per rank chunk), so one fp32 accumulator holds the folded score
 // a = sum_alpha coef[alpha] S_alpha (Eq. 4 with Eq. 6-7) and the epilogue
 // stores its order-preserving 32-bit key.
+//
 struct ScoreOp {
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
@@ -627,7 +665,9 @@ struct ScoreOp {
         tl.nkb = kb_total;
         return tl;
     }
-    __device__ void store(const Tile &tl, int row, int c, float (&v)[kMaxAcc][16]) const {
+    __device__ uint32_t prefetch(const Tile &, int, int) const { return 0u; }
+    __device__ void store(const Tile &tl, int row, int c, float (&v)[kMaxAcc][16],
+                          uint32_t) const {
         const int i = tl.m0 + row;
         if (i >= K) return;
         const int h = tl.z >> 1, axis = tl.z & 1;
@@ -642,6 +682,91 @@ struct ScoreOp {
         }
     }
 };
+
+// Candidate lists (long grids): instead of every key, the contraction runs
+// twice, with the roles of the tiles swapped (kSwapAB): 128 tokens on the
+// TMEM lanes and 128 keys on the columns, so that each epilogue thread owns
+// one token's scores of 16 consecutive keys per store and needs no other
+// lane.  The first pass (kListGroupMax) stores, per (token, head, axis), the
+// largest key of each group of 16 keys.  A small kernel takes tau = the
+// k-th largest of those group maxima: k distinct groups hold a key >= tau,
+// so every key of the axis' top k is >= tau.  The second pass
+// (kListCandidates) recomputes the same keys (the same tiles, MMAs and
+// order, so bit for bit) and writes each key >= tau, as a (key, position)
+// composite, into its group's 16-entry segment of the (token, head, axis)
+// list, and the group's count over its maximum.  About 2 % of the keys land
+// in the lists.  Measured on GB300 (stage times, graph replays): the
+// selection gets 17-25 % shorter (prefill of 16384 tokens 2233 -> 1844 us),
+// but each pass streams the same operands as the one-pass scoring, which is
+// bound by L2 -> SM operand traffic rather than by the keys' DRAM writes, so
+// the two passes and the bound cost more than that (prefill 576 -> 1058 us);
+// the one-pass form is the default and this one is a mode.
+enum { kListGroupMax = 1, kListCandidates = 2 };
+constexpr int kListGroup = 16;   // keys of a group; entries of a list segment
+
+template <int Mode>
+struct ScoreListOp {
+    static constexpr bool kSwapAB = true;
+    int n_tile, stages, n_acc, acc_chunk, b_split_stride;   // n_tile = 128 tokens
+    int *err;
+    unsigned long long *stamp;   // profiling stamps of the stage, or null
+    int B, H, K, kb_total;
+    int G;                        // groups of 16 keys an axis
+    uint32_t *gstat;              // [B][H][2][G] group maxima, then group counts
+    const uint32_t *tau;          // [B][H][2]
+    unsigned long long *cand;     // [B][H][2][G][16] composites
+    __device__ int cluster_splits() const { return 1; }
+    int cluster_splits_host() const { return 1; }
+    __device__ void store_sums(const Tile &, int, int, const float (&)[4]) const {}
+    __device__ Tile tile_at(int bx, int by, int bz) const {
+        Tile tl;
+        const int h = bz >> 1, axis = bz & 1;
+        tl.z = bz;   // head and axis
+        tl.m0 = bx * kTileM;   // first key
+        tl.n0 = by * n_tile;   // first token
+        tl.a_sel = axis;
+        tl.a_z = h;
+        tl.b_z = axis * H + h;
+        tl.kb0 = 0;
+        tl.nkb = kb_total;
+        return tl;
+    }
+    // the bound of this thread's token (the same for every chunk)
+    __device__ uint32_t prefetch(const Tile &tl, int row, int) const {
+        if constexpr (Mode != kListCandidates) return 0u;
+        const int n = tl.n0 + row;
+        return n < B ? tau[(int64_t)n * H * 2 + tl.z] : 0xffffffffu;
+    }
+    // row: the token (TMEM lane); c: the first of the 16 keys (a group)
+    __device__ void store(const Tile &tl, int row, int c, float (&v)[kMaxAcc][16],
+                          uint32_t t) const {
+        const int n = tl.n0 + row;
+        const int i0 = tl.m0 + c;
+        if (n >= B || i0 >= K) return;
+        const int64_t at = ((int64_t)n * H * 2 + tl.z) * G + i0 / kListGroup;
+        const int valid = min(kListGroup, K - i0);
+        // f2ord is monotone (-0 and +0 share a key), so the maximum and the
+        // comparisons are taken on the fp32 scores and only kept keys are
+        // converted
+        if constexpr (Mode == kListGroupMax) {
+            float mx = v[0][0];   // valid >= 1
+#pragma unroll
+            for (int j = 1; j < kListGroup; ++j)
+                if (j < valid) mx = fmaxf(mx, v[0][j]);
+            gstat[at] = f2ord(mx);
+        } else {
+            const float tf = ord2f(t);   // v >= tf  <=>  f2ord(v) >= t
+            unsigned long long *seg = cand + at * kListGroup;
+            uint32_t cnt = 0u;
+#pragma unroll
+            for (int j = 0; j < kListGroup; ++j)
+                if (j < valid && v[0][j] >= tf)
+                    seg[cnt++] = comp_of(f2ord(v[0][j]), (uint32_t)(i0 + j));
+            gstat[at] = cnt;
+        }
+    }
+};
+
 
 // ---- S9: IVE projection, split over E*D_v --------------------------------
 struct ProjOp {
@@ -665,7 +790,9 @@ struct ProjOp {
         t.nkb = max(0, min(kb_total, t.kb0 + per) - t.kb0);
         return t;
     }
-    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
+    __device__ uint32_t prefetch(const Tile &, int, int) const { return 0u; }
+    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16],
+                          uint32_t) const {
         const int o = t.m0 + row;
         if (o >= d_out) return;
 #pragma unroll
@@ -710,7 +837,9 @@ struct DaccOp {
         t.nkb = kb_total;
         return t;
     }
-    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
+    __device__ uint32_t prefetch(const Tile &, int, int) const { return 0u; }
+    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16],
+                          uint32_t) const {
         const int o = t.m0 + row;
         if (o >= M) return;
 #pragma unroll
@@ -750,7 +879,9 @@ struct DwOp {
         t.nkb = kb_total;
         return t;
     }
-    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16]) const {
+    __device__ uint32_t prefetch(const Tile &, int, int) const { return 0u; }
+    __device__ void store(const Tile &t, int row, int c, float (&v)[kMaxAcc][16],
+                          uint32_t) const {
         const int o = t.m0 + row;
         if (o >= M) return;
         // dW[n][o]: a warp's 32 rows o are contiguous for each column n
@@ -848,7 +979,7 @@ static uint32_t buf_cols_of(int n_acc, int n_tile) {
 // does not apply.
 template <int NSPLIT, class Op>
 static bool persistent_ok(dim3 grid, const Op &op) {
-    const uint32_t bc = buf_cols_of(op.n_acc, op.n_tile);
+    const uint32_t bc = buf_cols_of(op.n_acc, acc_cols_of(op));
     return grid.z >= 1 && op.cluster_splits_host() == 1 &&
            (int)(grid.x * grid.y * grid.z) > sm_count() && 2 * bc <= 512 &&
            tmem_cols_for(2 * bc) == 2 * bc;
@@ -865,7 +996,7 @@ static cudaError_t launch_gemm_persistent(dim3 grid, const CUtensorMap &a0, cons
     const int ctas = tiles < sm_count() ? tiles : sm_count();
     return launch_kernel(pdl, tc_gemm_persistent<NSPLIT, Op>, dim3(ctas), kPThreads, smem, st, a0,
                          a1, b, op, (int)grid.x, (int)grid.y, tiles,
-                         buf_cols_of(op.n_acc, op.n_tile), probe);
+                         buf_cols_of(op.n_acc, acc_cols_of(op)), probe);
 }
 
 // grid.z = the split count (S1, S9; also the cluster's z extent when > 1) or
@@ -901,6 +1032,8 @@ cudaError_t configure_tc() {
     cudaError_t e = allow_smem<1, QueryOp>();
     if (e == cudaSuccess) e = allow_smem<3, QueryOp>();
     if (e == cudaSuccess) e = allow_smem<3, ScoreOp>();
+    if (e == cudaSuccess) e = allow_smem<3, ScoreListOp<kListGroupMax>>();
+    if (e == cudaSuccess) e = allow_smem<3, ScoreListOp<kListCandidates>>();
     if (e == cudaSuccess) e = allow_smem<2, ProjOp>();
     if (e == cudaSuccess) e = allow_smem<1, DaccOp>();
     if (e == cudaSuccess) e = allow_smem<2, DwOp>();
@@ -986,7 +1119,8 @@ cudaError_t launch_query_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, int 
     return cudaSuccess;
 }
 
-cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
+cudaError_t launch_score_keys(const Dims &d, const Ptrs &p, const TcMaps &mp, int probe,
+                              cudaStream_t st) {
     ScoreOp op;
     op.stamp = p.stamp;
     op.n_tile = tc_n_tile(d.B, 1);
@@ -1000,8 +1134,41 @@ cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cuda
     op.kb_total = (d.d_k + kBlockK - 1) / kBlockK;
     op.akey = p.akey;
     dim3 grid((d.K + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 2 * d.H);
-    return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs, op, op.kb_total, d.pdl, st,
-                          d.probe_wait);
+    return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs, op, op.kb_total, d.pdl, st, probe);
+}
+
+// one pass of the candidate-list scoring (128 tokens a tile, map qs_t)
+template <int Mode>
+static cudaError_t score_list_pass(const Dims &d, const Ptrs &p, const TcMaps &mp, int probe,
+                                   cudaStream_t st) {
+    ScoreListOp<Mode> op;
+    op.stamp = p.stamp;
+    op.n_tile = kTileM;
+    op.n_acc = 1;
+    op.acc_chunk = 1 << 30;
+    op.b_split_stride = d.d_k;
+    op.err = p.err;
+    op.B = d.B;
+    op.H = d.H;
+    op.K = d.K;
+    op.kb_total = (d.d_k + kBlockK - 1) / kBlockK;
+    op.G = d.n_groups;
+    op.gstat = p.gstat;
+    op.tau = p.tau;
+    op.cand = p.cand;
+    dim3 grid((d.K + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 2 * d.H);
+    return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs_t, op, op.kb_total, d.pdl, st, probe);
+}
+
+cudaError_t launch_score_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
+    if (d.cand) {
+        // group maxima, the bound, then the lists (three dependent launches)
+        cudaError_t e = score_list_pass<kListGroupMax>(d, p, mp, d.probe_wait, st);
+        if (e == cudaSuccess) e = launch_cand_bound(d, p, st);
+        if (e == cudaSuccess) e = score_list_pass<kListCandidates>(d, p, mp, 0, st);
+        return e;
+    }
+    return launch_score_keys(d, p, mp, d.probe_wait, st);
 }
 
 cudaError_t launch_proj_tc(const Dims &d, const Ptrs &p, const TcMaps &mp, cudaStream_t st) {
