@@ -174,7 +174,14 @@ def key_ln(keys: torch.Tensor, g: torch.Tensor, b: torch.Tensor | None = None,
     return out
 
 
+# The raw handle of the current stream without building a torch.cuda.Stream
+# object (which costs about 3 us a call, a tenth of a decode step).
+_raw_stream = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+
+
 def _stream():
+    if _raw_stream is not None:
+        return _raw_stream(torch.cuda.current_device())
     return torch.cuda.current_stream().cuda_stream
 
 
