@@ -291,11 +291,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (warp == 0) tmem_dealloc(tmem, ncols);
     } else {
         // Split-K through distributed shared memory (one accumulator): each
-        // CTA stages its partial, then, once every CTA of the cluster has
-        // (so that every ring is drained), sends slice j to CTA j with one
-        // bulk copy into j's receive slot for it (completing bytes of j's
-        // receive barrier), and adds up its own columns over the S partials
-        // in split order (deterministic).
+        // CTA stages its partial; once every CTA of the cluster has staged
+        // its own (so that every ring is drained), it sends slice j to CTA j
+        // with one bulk copy into j's receive slot for it (completing bytes
+        // of j's receive barrier), and adds up its own columns over the S
+        // partials in split order (deterministic).
         uint8_t *recv = ring + (size_t)S * slice;   // slot of CTA q: q - (q > me)
         // column c's slice c / per as floor((c + 1/2) / per) in fp32: exact
         // while c < 2^22 (the rounding error, below 2^-23 c / per, stays under
