@@ -585,6 +585,7 @@ __device__ __forceinline__ uint4 ld_key4(const uint4 *p, bool stream) {
 __device__ __forceinline__ uint32_t ld_key(const uint32_t *p, bool stream) {
     return stream ? __ldcg(p) : __ldcs(p);
 }
+template <int NS = 2>   // axes loaded: both, or (NS = 1) the one in A0
 __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1, int K,
                                           const SelLayout &L, uint32_t (&top)[2][2],
                                           bool stream) {
@@ -601,14 +602,14 @@ __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1
             for (int q = 0; q < 4; ++q) {
                 const int i = v0 + q * kThreads;
                 a[q] = i < nv ? ld_key4(V0 + i, stream) : make_uint4(0, 0, 0, 0);
-                c[q] = i < nv ? ld_key4(V1 + i, stream) : make_uint4(0, 0, 0, 0);
+                c[q] = NS > 1 && i < nv ? ld_key4(V1 + i, stream) : make_uint4(0, 0, 0, 0);
             }
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int i = v0 + q * kThreads;
                 if (i < nv && !stream) {
                     S0[i] = a[q];
-                    S1[i] = c[q];
+                    if (NS > 1) S1[i] = c[q];
                 }
                 top2(a[q].x, a1, a2);
                 top2(a[q].y, a1, a2);
@@ -628,14 +629,14 @@ __device__ __forceinline__ void load_keys(const uint32_t *A0, const uint32_t *A1
             for (int q = 0; q < 4; ++q) {
                 const int i = i0 + q * kThreads;
                 a[q] = i < K ? ld_key(A0 + i, stream) : 0u;
-                c[q] = i < K ? ld_key(A1 + i, stream) : 0u;
+                c[q] = NS > 1 && i < K ? ld_key(A1 + i, stream) : 0u;
             }
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int i = i0 + q * kThreads;
                 if (i < K && !stream) {
                     L.key0[i] = a[q];
-                    L.key1[i] = c[q];
+                    if (NS > 1) L.key1[i] = c[q];
                 }
                 top2(a[q], a1, a2);
                 top2(c[q], b1, b2);
@@ -660,26 +661,48 @@ __device__ __forceinline__ uint4 ld_key_row(const uint4 *ptr) {
     return v;
 }
 
+// The paired decode selection's exchange: a 32-bit store into the same
+// shared-memory location of CTA `rank` of the cluster, and a barrier of all
+// threads of the cluster (release / acquire).
+__device__ __forceinline__ void st_cluster_u32(const void *local, uint32_t rank, uint32_t v) {
+    const uint32_t a = (uint32_t)__cvta_generic_to_shared(local);
+    uint32_t ra;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(a), "r"(rank));
+    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(ra), "r"(v) : "memory");
+}
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile(
+        "barrier.cluster.arrive.release.aligned;\n\t"
+        "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 // The 2k axis survivors, one group of G lanes each: the survivor's place in
 // increasing key index (so that enumerating I x J row-major is increasing
 // v = i*K + j), and its exact chunk scores S_alpha (Eq. 4) from 16-byte
 // loads of its key row split over the group.  Row survivors store
 // R[i][b] = sum_a S_row[a,i] C[a,b], column survivors S_col[j][b].
 // RM >= r bounds the rank at compile time (2 for the common ranks, else 8).
+// gax < 0: both axes (winners of axis s in win[s]); gax = 0 or 1 (the
+// paired decode selection): only axis gax, whose winners are in win[0].
 template <typename T, int RM>
 __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLayout &L,
-                               const SelShared &sh) {
+                               const SelShared &sh, int gax = -1) {
     constexpr int EPV = 16 / sizeof(T);
     const int k = d.k, r = d.r, dk = d.dk, D = d.d_k;
-    int lg = 0;   // G = 2^lg lanes per survivor
+    const int nl = gax < 0 ? 2 : 1;   // lists
+    // G = 2^lg lanes per survivor, sized for two lists in either case: the
+    // lanes' partial sums (and so the scores' roundings) are then the same
+    // whether one CTA takes both axes or a pair one each
+    int lg = 0;
     while (lg < 5 && 2 * k * (2 << lg) <= kThreads) ++lg;
     const int G = 1 << lg;
     const int lane = threadIdx.x & 31, sub = lane & (G - 1);
-    const int sv = threadIdx.x >> lg;   // 2k * G <= kThreads: one pass
-    const bool active = sv < 2 * k;
-    const int s = active && sv >= k ? 1 : 0;
-    const int qi = active ? sv - s * k : 0;
-    uint32_t pos = active ? pos_of(sh.win[s][qi]) : 0u;
+    const int sv = threadIdx.x >> lg;   // 2k G <= kThreads: one pass
+    const bool active = sv < nl * k;
+    const int ls = active && sv >= k ? 1 : 0;   // the list
+    const int s = gax < 0 ? ls : gax;           // its axis
+    const int qi = active ? sv - ls * k : 0;
+    uint32_t pos = active ? pos_of(sh.win[ls][qi]) : 0u;
     if (active && pos >= (uint32_t)d.K) {   // never expected: record and skip
         if (sub == 0) atomicOr(p.err, kErrInternal);
         pos = 0u;
@@ -703,11 +726,11 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
     if (active) {
         int g = sub;
         for (; g + 3 * G < k; g += 4 * G) {
-            const uint32_t a = pos_of(sh.win[s][g]), b = pos_of(sh.win[s][g + G]),
-                           c = pos_of(sh.win[s][g + 2 * G]), e = pos_of(sh.win[s][g + 3 * G]);
+            const uint32_t a = pos_of(sh.win[ls][g]), b = pos_of(sh.win[ls][g + G]),
+                           c = pos_of(sh.win[ls][g + 2 * G]), e = pos_of(sh.win[ls][g + 3 * G]);
             ord += (a < pos) + (b < pos) + (c < pos) + (e < pos);
         }
-        for (; g < k; g += G) ord += pos_of(sh.win[s][g]) < pos;
+        for (; g < k; g += G) ord += pos_of(sh.win[ls][g]) < pos;
     }
     for (int off = G >> 1; off > 0; off >>= 1) ord += __shfl_xor_sync(kFull, ord, off);
 
@@ -849,15 +872,22 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
 // latency matters; 4: 64 registers, for long grids, where occupancy does).
 // RM >= r: the rank bound of the survivor phase (2, or 8 for larger ranks),
 // one per kernel so that each carries a single copy of it.
-template <typename T, int MINB, int RM>
+// PAIR (decode grids of at most one (token, head) per SM): a cluster of two
+// CTAs per (token, head), blockIdx.z = its axis.  Each takes one axis through
+// the key load, bound, compaction, rank and survivors (half the work a warp
+// does in those phases); the column CTA then stores its survivors (indices
+// and S_col) into the row CTA's shared memory, the pair meets at a cluster
+// barrier, and the row CTA goes on alone (Tucker scores, top-m, outputs).
+template <typename T, int MINB, int RM, bool PAIR = false>
 __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ SelShared sh;
     const int b = blockIdx.x / d.H, h = blockIdx.x % d.H;
+    const int ax = PAIR ? (int)blockIdx.z : 0;   // the cluster's rank (cluster 1 x 1 x 2)
     const SelLayout L = carve(d, smem_raw);
     const int r = d.r, K = d.K, k = d.k, m = d.m;
-    const uint32_t *A0 = p.akey + (((int64_t)b * d.H + h) * 2) * (int64_t)K;
-    const uint32_t *A1 = A0 + K;
+    const uint32_t *A0 = p.akey + (((int64_t)b * d.H + h) * 2 + ax) * (int64_t)K;
+    const uint32_t *A1 = A0 + K;   // (not read when PAIR)
 
     if (threadIdx.x < 8) sh.cnt[threadIdx.x] = 0;
     // C of this head (a weight: read before the dependency wait) and the
@@ -894,23 +924,31 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
         }
     };
     const bool one_split = d.q_splits == 1;
+    // the query elements this CTA needs: both axes', or its own axis'
+    const int e0 = PAIR ? ax * d.d_k : 0, ne = PAIR ? d.d_k : 2 * d.d_k;
     float q0 = 0.f;
-    if (threadIdx.x < 2 * d.d_k) q0 = one_split ? *q_src(threadIdx.x) : q_of(threadIdx.x);
+    if (threadIdx.x < ne) q0 = one_split ? *q_src(e0 + threadIdx.x) : q_of(e0 + threadIdx.x);
     uint32_t top[2][2];
     const bool stream = d.stream_keys != 0;   // uniform
     // candidate lists: only the long-grid instantiation reads them (the
     // launch picks it whenever they are on)
     const bool lists = MINB >= 4 && d.cand;
-    if (!lists) load_keys(A0, A1, K, L, top, stream);
+    if constexpr (PAIR) load_keys<1>(A0, A1, K, L, top, stream);
+    else if (!lists) load_keys(A0, A1, K, L, top, stream);
     // the axes' keys: in shared memory, or (streamed) in L2, where the
     // compaction reads them a second time
     const uint32_t *KA = stream ? A0 : L.key0, *KB = stream ? A1 : L.key1;
     if (threadIdx.x < r * r) sh.core[threadIdx.x] = core_e;
-    if (threadIdx.x < 2 * d.d_k) L.qv[threadIdx.x] = q0;
-    for (int e = threadIdx.x + kThreads; e < 2 * d.d_k; e += kThreads) L.qv[e] = q_of(e);
+    if (threadIdx.x < ne) L.qv[e0 + threadIdx.x] = q0;
+    for (int e = threadIdx.x + kThreads; e < ne; e += kThreads) L.qv[e0 + e] = q_of(e0 + e);
 
     // Eq. 8-9: top-k of both axes
-    if (lists) {   // the scoring left each axis' candidates
+    if constexpr (PAIR) {   // this CTA's axis as list 0
+        warp_bounds(top[0][0], top[0][1], 0u, 0u, 1, k, sh);
+        __syncthreads();
+        compact<1>(KA, nullptr, K, block_bound(0, sh), 0u, sh, kCntAxis, kCntAxis);
+        __syncthreads();
+    } else if (lists) {   // the scoring left each axis' candidates
         __syncthreads();
         for (int s = 0; s < 2; ++s)
             load_list(p, ((int64_t)b * d.H + h) * 2 + s, d.n_groups, k, s, kCntAxis + s, sh);
@@ -922,8 +960,10 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
         __syncthreads();
     }
     const int c0 = settle(0, KA, K, k, kCntAxis, kCntAxisT, sh);
-    const int c1 = settle(1, KB, K, k, kCntAxis + 1, kCntAxisT + 1, sh);
-    {
+    const int c1 = PAIR ? 0 : settle(1, KB, K, k, kCntAxis + 1, kCntAxisT + 1, sh);
+    if constexpr (PAIR) {
+        rank_list(sh.cand[0], c0, k, sh.win[0], threadIdx.x, kThreads);
+    } else {
         const int s = threadIdx.x >= kThreads / 2, cs = s ? c1 : c0;
         const int tid = threadIdx.x & (kThreads / 2 - 1);
         // long grids (issue-bound) rank by sorted runs, which execute fewer
@@ -942,8 +982,24 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     if (threadIdx.x < ncrr) L.cparts[threadIdx.x] = cp0;   // key1 is free now
     if (threadIdx.x + kThreads < ncrr) L.cparts[threadIdx.x + kThreads] = cp1;
     // survivors in increasing index with their exact chunk scores (Eq. 4)
-    axis_survivors<T, RM>(d, p, h, L, sh);
+    axis_survivors<T, RM>(d, p, h, L, sh, PAIR ? ax : -1);
     __syncthreads();
+    if constexpr (PAIR) {
+        // the column CTA stores its survivors into the row CTA; the barrier
+        // (release / acquire) makes them visible there, and the column CTA
+        // is done
+        if (ax == 1) {
+            for (int i = threadIdx.x; i < k; i += kThreads)
+                st_cluster_u32(L.sel_j + i, 0u, (uint32_t)L.sel_j[i]);
+            for (int i = threadIdx.x; i < k * r; i += kThreads)
+                st_cluster_u32(L.scol + i, 0u, __float_as_uint(L.scol[i]));
+        }
+        cluster_sync_all();
+        if (ax == 1) {
+            stamp_end(p.stamp);
+            return;
+        }
+    }
 
     u64 *const fwin = sh.cand[1];   // final winners by rank (list 1 is free now)
 
@@ -1205,6 +1261,14 @@ template <typename T, int RM>
 static cudaError_t launch_select_t(const Dims &d, const Ptrs &p, size_t smem, cudaStream_t st) {
     if (d.B * d.H > 3 * 152 || d.cand)
         return launch_kernel(d.pdl, select_kernel<T, 4, RM>, d.B * d.H, kThreads, smem, st, d, p);
+    if (d.B * d.H <= device_sm_count()) {
+        // at most one (token, head) per SM: a CTA pair per (token, head), the
+        // pairs spread over the SMs
+        const size_t sm =
+            spread_smem(smem, static_smem_of<select_kernel<T, 3, RM, true>>(), 2 * d.B * d.H);
+        return launch_kernel(d.pdl, 2u, select_kernel<T, 3, RM, true>, dim3(d.B * d.H, 1, 2),
+                             kThreads, sm, st, d, p);
+    }
     // decode grids: spread over the SMs (see spread_smem)
     const size_t sm = spread_smem(smem, static_smem_of<select_kernel<T, 3, RM>>(), d.B * d.H);
     return launch_kernel(d.pdl, select_kernel<T, 3, RM>, d.B * d.H, kThreads, sm, st, d, p);
@@ -1252,6 +1316,10 @@ template <typename T, int RM> static cudaError_t allow_select() {
     const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
     cudaError_t e = cudaFuncSetAttribute(
         select_kernel<T, 3, RM>, a, (int)(kSmemPerCta - static_smem_of<select_kernel<T, 3, RM>>()));
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(
+            select_kernel<T, 3, RM, true>, a,
+            (int)(kSmemPerCta - static_smem_of<select_kernel<T, 3, RM, true>>()));
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(select_kernel<T, 4, RM>, a,
                                  (int)(kSmemPerCta - static_smem_of<select_kernel<T, 4, RM>>()));
