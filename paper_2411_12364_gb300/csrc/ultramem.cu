@@ -1140,6 +1140,14 @@ int32_t ultramem_debug_live_allocations(void) { return g_live_allocs.load(); }
 ultramem_status ultramem_debug_candidates(ultramem_layer *L, int32_t mode) {
     if (!L || mode < 0 || mode > 1) return ULTRAMEM_EINVAL;
     if (mode == 1 && !L->cand_ok) return ULTRAMEM_ENODEV;
+    if (mode != L->cand_mode) {
+        // the host-buffer calls' cached graphs hold the launches of the
+        // previous form: captured again on their next call
+        for (auto &g : L->host_graphs) {
+            if (g.exec) cudaGraphExecDestroy(g.exec);
+            g.exec = nullptr;
+        }
+    }
     L->cand_mode = mode;
     return ULTRAMEM_OK;
 }
