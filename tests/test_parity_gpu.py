@@ -160,6 +160,28 @@ def test_retrieve_and_host_forward_agree_with_forward(gpu_lib):
     assert torch.equal(op, out.cpu())
 
 
+@pytest.mark.parametrize("B", [64, 65])
+def test_host_forward_at_decode_shape(B, gpu_lib):
+    """The host-buffer call on decode_1m, on both sides of the CUDA-core
+    query's batch limit: a copy kernel reads the pinned tokens over the host
+    link and the projection writes the pinned output; both calls (captured,
+    then replayed) equal the device forward bit for bit."""
+    from paper_2411_12364_gb300.binding import UltraMemLayer
+    cfg = workloads.layer_config("decode_1m")
+    w = workloads.make_weights(cfg, device="cuda")
+    layer = UltraMemLayer(cfg, w, 65)
+    x = workloads.make_tokens(cfg, B, 3, device="cuda")
+    out = layer.forward(x)
+    xh = x.cpu().pin_memory()
+    oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    for _ in range(2):   # captured, then replayed
+        oh.zero_()
+        layer.forward_host(xh, oh)
+        assert layer.check() == 0
+        assert torch.equal(oh, out.cpu())
+    layer.close()
+
+
 def test_forward_is_deterministic(gpu_lib):
     cfg = workloads.small_config(dtype=1, heads=3)
     layer, (w, x, t), (out, idx, wt), _ = _run(cfg, 70, gpu_lib)
