@@ -141,6 +141,8 @@ __global__ void __launch_bounds__(kThreads) small_gemm_kernel(SmallArgs g) {
         if (k0 == 0) {
             pdl_wait();
             stamp_begin(g.stamp);
+            // the scoring kernel's CTAs may now start streaming its keys
+            pdl_trigger();
         }
         if (threadIdx.x == 0)
             for (int t = 0; t < ntoks; ++t)
@@ -178,7 +180,6 @@ __global__ void __launch_bounds__(kThreads) small_gemm_kernel(SmallArgs g) {
         }
         __syncthreads();   // the buffers are refilled by the next round
     }
-    pdl_trigger();
 #pragma unroll
     for (int i = 0; i < 2; ++i)
 #pragma unroll
