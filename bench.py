@@ -81,13 +81,15 @@ def peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def algorithmic_bytes(cfg, B):
+def algorithmic_bytes(cfg, B, lists=False):
     """Bytes each stage must move at least (paper's Sec. 4 memory-access model
     with heads: the gather reads min(B*H*m, N) rows of D_v).  The selection
     reads, per (token, head), the rank-1 score keys of both axes (2 K x 4 B),
     the query (A D_k x 4 B) and the key rows of the 2k survivors
     (2 k D_k x es), and writes m slots (row, block and h weights: 8 + 4h B,
-    h = 1 without Multi-Core Scoring)."""
+    h = 1 without Multi-Core Scoring).  With the scoring's candidate lists
+    (`lists`) it reads, in place of the keys, each axis' group counts
+    (ceil(K/16) x 4 B) and at least k list entries (8 B each)."""
     es = 4 if int(cfg["dtype"]) == 0 else 2
     H, dk, din = cfg["heads"], cfg["d_k"], cfg["d_in"]
     K = int(round(cfg["expand_e"] ** 0.5)) * cfg["n"]
@@ -95,10 +97,11 @@ def algorithmic_bytes(cfg, B):
     N = cfg["n"] ** 2
     k, m = cfg["topk"], cfg["topm"]
     rows = min(B * H * m, N)
+    axis_in = 2 * ((K + 15) // 16 * 4 + k * 8) if lists else 2 * K * 4
     return {
         "query": A * H * dk * din * es + B * din * es,
         "score": 2 * H * K * dk * es,
-        "select": B * H * (2 * K * 4 + A * dk * 4 + 2 * k * dk * es
+        "select": B * H * (axis_in + A * dk * 4 + 2 * k * dk * es
                            + m * (8 + 4 * max(1, int(cfg.get("cores", 0))))),
         "gather": rows * cfg["d_v"] * es,
         "project": (cfg["expand_e"] * cfg["d_v"] * cfg["d_out"] * es if cfg["has_proj"] else 0)
@@ -460,6 +463,19 @@ def capture(layer, fwd, stream, NB):
 SWEEP = [("mid_4m", (128,)), ("large_20m", (64, 256)), ("prefill_16k", (16384,))]
 
 
+def uses_lists(layer, fwd):
+    """Whether the layer's default scoring form takes the candidate lists at
+    this batch: two more launches than every key."""
+    import torch
+    layer.candidates(0)
+    fwd(0)
+    n0 = layer.last_launches()
+    layer.candidates(2)
+    fwd(0)
+    torch.cuda.synchronize()
+    return layer.last_launches() == n0 + 2
+
+
 def sweep_workload(wl, batches, K, flush, stream, peak, peak_kind):
     """Further batches of one workload (one table): step time, tokens/s,
     per-stage device times, the gather's GB/s and the dominant kernel's
@@ -475,6 +491,7 @@ def sweep_workload(wl, batches, K, flush, stream, peak, peak_kind):
         xs = [x[:B].contiguous() for x in xs_all]
         out = torch.empty((B, cfg["d_out"]), dtype=layer.dtype, device="cuda")
         fwd = lambda i: layer.forward(xs[i % NB], out=out)
+        lists = uses_lists(layer, fwd)
         graphs = capture(layer, fwd, stream, NB)
         big = B >= 4096
         steps, warm = (5, 2) if big else (max(5, min(K, 30)), 3)
@@ -486,8 +503,9 @@ def sweep_workload(wl, batches, K, flush, stream, peak, peak_kind):
         del graphs
         stages, gaps = stage_profile(layer, fwd, stream, flush, 3 if big else 20, True, NB)
         cold = cold_gather(layer, xs[0], stream, flush, 3 if big else 10)
-        alg = algorithmic_bytes(cfg, B)
+        alg = algorithmic_bytes(cfg, B, lists)
         res.append({"workload": wl, "batch": B, "steps": steps, "ms_per_step": ms,
+                    "scoring": "candidate_lists" if lists else "every_key",
                     "tokens_per_s": B / (ms / 1e3), "stages_ms": stages, "handoff_ms": gaps,
                     "roofline": roofline_of(stages, alg, peak, peak_kind),
                     "gather": gather_entry(alg, stages.get("gather"), cold, peak),
@@ -549,6 +567,10 @@ def main():
         for i in range(3):
             fwd(0)
         torch.cuda.synchronize()
+    lists = uses_lists(layer, fwd)
+    with torch.cuda.stream(stream):
+        fwd(0)
+        torch.cuda.synchronize()
     launches = layer.last_launches()   # kernels per forward (and per graph replay)
     graphs = capture(layer, fwd, stream, NB) if use_graph else []
 
@@ -576,7 +598,7 @@ def main():
     # ---- per-stage device times from the kernels' own stamps -------------
     stages, gaps = stage_profile(layer, fwd, stream, flush, min(K, 50), use_graph, NB)
     cold = cold_gather(layer, xs[0], stream, flush, 10) if states is None else None
-    alg = algorithmic_bytes(cfg, B)
+    alg = algorithmic_bytes(cfg, B, lists)
     peak, peak_kind = peaks()
     roof = roofline_of(stages, alg, peak, peak_kind)
     roof["traffic"] = None if int(cfg.get("cores", 0)) > 1 else \
@@ -624,6 +646,7 @@ def main():
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "bf16" if int(cfg["dtype"]) else "f32", "data": "synthetic",
                 "config": dict(workload=wl, batch=B, **_cfg_brief(cfg), accumulate="f32",
+                               scoring="candidate_lists" if lists else "every_key",
                                l2="flushed between steps (256 MiB write, outside timing)",
                                cuda_graph=use_graph, parallelism=f"replicas x{world}"),
                 "roofline": roof, "gather": gather, "stages_ms": stages, "handoff_ms": gaps,

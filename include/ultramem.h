@@ -363,19 +363,21 @@ ultramem_status ultramem_debug_wait_probe(ultramem_layer *layer);
 void ultramem_debug_fail_alloc(int32_t nth);
 int32_t ultramem_debug_live_allocations(void);
 
-/* The scoring's second form, for tests and measurement (tensor-core path).
- * By default (mode 0) the scoring writes every rank-1 key (Eq. 6-7) and the
- * selection takes each axis' top k from all of them (Eq. 8-9).  With mode 1
- * the scoring runs twice: the first pass keeps the largest key of each group
- * of 16 keys of an axis, a bound kernel takes tau = the k-th largest of
- * those per (token, head, axis) (k distinct groups reach tau, so the axis'
- * top k is >= tau), and the second pass writes only the keys >= tau, as
- * per-axis candidate lists, which the selection ranks instead.  Both forms
- * rank the same keys in the same order (score, then the smaller index), so
- * the selection is the same; on GB300 the second contraction costs more
- * than the shorter selection saves, hence the default.  Mode 1 needs the
- * tensor-core path and k to 1024 groups of 16 keys an axis (ULTRAMEM_ENODEV
- * otherwise, and the layer keeps mode 0); ULTRAMEM_EINVAL for another mode. */
+/* The scoring's two forms (tensor-core path), for tests and measurement.
+ * Mode 0: the scoring writes every rank-1 key (Eq. 6-7) and the selection
+ * takes each axis' top k from all of them (Eq. 8-9).  Mode 1: the scoring
+ * runs twice: the first pass keeps the largest key of each group of 16 keys
+ * of an axis, a bound kernel takes tau <= the k-th largest of those per
+ * (token, head, axis) (k distinct groups reach tau, so the axis' top k is
+ * >= tau), and the second pass writes only the keys >= tau, as per-axis
+ * candidate lists, which the selection ranks instead.  Mode 2 (the
+ * default): mode 1 on long grids (at least 3.5 of the list passes' tiles of
+ * 128 tokens x 256 keys per SM), mode 0 below; a layer that cannot take the
+ * lists always scores every key.  All forms rank the same keys in the same
+ * order (score, then the smaller index), so the selection is the same.
+ * Mode 1 needs the tensor-core path and k to 1024 groups of 16 keys an axis
+ * (ULTRAMEM_ENODEV otherwise, and the layer keeps its mode);
+ * ULTRAMEM_EINVAL for another mode. */
 ultramem_status ultramem_debug_candidates(ultramem_layer *layer, int32_t mode);
 
 /* ABI version, currently 2. */

@@ -397,7 +397,8 @@ class UltraMemLayer:
         return int(self.lib.ultramem_check(self._h, _stream()))
 
     def candidates(self, mode: int):
-        """Scoring form (test hook): 0 every key (default), 1 candidate lists."""
+        """Scoring form (test hook): 0 every key, 1 candidate lists, 2 lists on
+        long grids only (the default)."""
         _check(self.lib.ultramem_debug_candidates(self._h, int(mode)), "debug_candidates")
 
     def last_launches(self) -> int:

@@ -70,7 +70,8 @@ struct ultramem_layer {
     bool x_after_copy = false;   // x is written by the copy kernel just before the forward
     bool probe_armed = false;    // ultramem_debug_wait_probe: the next forward's score probes
     bool cand_ok = false;        // the candidate-list scoring fits this layer
-    int cand_mode = 0;           // ultramem_debug_candidates: 0 every key, 1 candidate lists
+    int cand_mode = 2;           // ultramem_debug_candidates: 0 every key, 1 candidate lists,
+                                 // 2 (default) lists on long grids
     bool dacc_tc = false;        // the backward's dacc may run on the tensor cores
 };
 
@@ -380,13 +381,19 @@ Dims dims_for(const ultramem_layer *L, int B) {
     // twice instead.  Measured at large_20m (K = 8960) with 256 tokens: select
     // 71.3 -> 56.4 us (2 -> 4 CTAs per SM); at K = 4096 staging is as fast.
     d.stream_keys = (int64_t)B * d.H > 3 * 152 && d.K > 4096 && d.K % 4 == 0;
-    // On request (ultramem_debug_candidates) the tensor path scores twice and
-    // leaves per-axis candidate lists (ScoreListOp): the keys' round trip
-    // through memory goes and the selection starts from about 2 % of them,
-    // but the second contraction costs more than that saves on GB300 (the
-    // scoring passes are bound by L2 -> SM operand traffic), so every key
-    // is written by default.
-    d.cand = L->cand_ok && L->cand_mode == 1 ? 1 : 0;
+    // Candidate lists (ScoreListOp): the tensor path scores twice and leaves
+    // per-axis candidate lists, so the keys' round trip through memory goes
+    // and the selection starts from about 2 % of them.  The passes pay off
+    // once each SM has several of their tiles (128 tokens x 256 keys of one
+    // head and axis) to pipeline: measured on GB300, lists against every key
+    // at 3.5 or more tiles per SM (mid_4m with 1024 and 2048 tokens,
+    // large_20m with 256, prefill_16k) 2-5 % shorter steps, below it (mid_4m
+    // with 128-512 tokens, large_20m with 64 and 128, decode grids) 3-60 %
+    // longer.  Mode 2 (the default) takes them from 3.5 tiles per SM on;
+    // modes 0 and 1 force every key or the lists.
+    const int64_t list_tiles = (int64_t)((d.K + 255) / 256) * ((B + 127) / 128) * 2 * d.H;
+    const bool long_grid = 2 * list_tiles >= 7 * (int64_t)um::device_sm_count();
+    d.cand = L->cand_ok && (L->cand_mode == 1 || (L->cand_mode == 2 && long_grid)) ? 1 : 0;
     if (d.cand) d.stream_keys = 0;
     d.seq_len = B;   // one sequence unless the caller says otherwise
     d.q_splits = L->tc ? tc_query_splits(L->cfg, B) : query_splits(L->cfg, B);
@@ -1138,7 +1145,7 @@ void ultramem_debug_fail_alloc(int32_t nth) { g_fail_countdown.store(nth < 0 ? -
 int32_t ultramem_debug_live_allocations(void) { return g_live_allocs.load(); }
 
 ultramem_status ultramem_debug_candidates(ultramem_layer *L, int32_t mode) {
-    if (!L || mode < 0 || mode > 1) return ULTRAMEM_EINVAL;
+    if (!L || mode < 0 || mode > 2) return ULTRAMEM_EINVAL;
     if (mode == 1 && !L->cand_ok) return ULTRAMEM_ENODEV;
     if (mode != L->cand_mode) {
         // the host-buffer calls' cached graphs hold the launches of the

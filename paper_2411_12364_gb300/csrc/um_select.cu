@@ -1194,10 +1194,13 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
 }
 
 // Candidate lists (Dims::cand), between the two scoring passes: the bound of
-// one (token, head, axis) per warp.  tau is the k-th largest of the axis'
-// G group maxima (groups of 16 keys), found bit by bit from the top (the largest T with at
-// least k maxima >= T); k distinct groups hold a key >= tau, so the axis'
-// top k is among the keys >= tau.
+// one (token, head, axis) per warp.  tau is the largest T whose low 16 bits
+// are zero with at least k of the axis' G group maxima (groups of 16 keys)
+// >= T, found bit by bit from the top: k distinct groups hold a key >= tau,
+// so the axis' top k is among the keys >= tau.  tau is at most the k-th
+// largest group maximum and agrees with it in the sign, the exponent and
+// the first 7 mantissa bits of the score; the low bits would tighten the
+// lists by a few keys for twice the rounds.
 constexpr int kBoundWarps = 8;
 constexpr int kMaxGroupsPerLane = 32;   // G <= 1024 groups (K <= 16384 keys)
 static_assert(32 * kMaxGroupsPerLane == kMaxSegPerThread * kThreads, "one limit on G");
@@ -1219,7 +1222,7 @@ __global__ void __launch_bounds__(32 * kBoundWarps) cand_bound_kernel(Dims d, Pt
         }
         uint32_t T = 0u;
 #pragma unroll 4
-        for (int bit = 31; bit >= 0; --bit) {
+        for (int bit = 31; bit >= 16; --bit) {
             const uint32_t c = T | (1u << bit);
             int n = 0;
 #pragma unroll

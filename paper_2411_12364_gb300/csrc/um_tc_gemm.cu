@@ -55,8 +55,9 @@ struct Tile {
     int z;             // the tile's third grid coordinate (split or head/axis)
 };
 
-__host__ __device__ inline size_t stage_bytes_of(int nsplit, int n_tile) {
-    return kTileABytes + (size_t)nsplit * n_tile * 128;
+// a_rows: rows of the staged A tile (128, or 256 for ops with kARows = 256)
+__host__ __device__ inline size_t stage_bytes_of(int nsplit, int n_tile, int a_rows = kTileM) {
+    return (size_t)a_rows * 128 + (size_t)nsplit * n_tile * 128;
 }
 
 // Split-K: CTA s of a tile's cluster adds up columns [s * per, (s + 1) * per)
@@ -77,8 +78,8 @@ __host__ __device__ inline size_t split_buf_bytes(int n_tile, int S) {
 }
 
 // As many ring stages as fit (at most 4, never more than the K blocks).
-inline int stages_for(int nsplit, int n_tile, int nkb) {
-    int s = (int)((kSmemBudget - 1024) / stage_bytes_of(nsplit, n_tile));
+inline int stages_for(int nsplit, int n_tile, int nkb, int a_rows = kTileM) {
+    int s = (int)((kSmemBudget - 1024) / stage_bytes_of(nsplit, n_tile, a_rows));
     if (s > kMaxStages) s = kMaxStages;
     if (s > nkb) s = nkb;
     return s < 1 ? 1 : s;
@@ -86,17 +87,65 @@ inline int stages_for(int nsplit, int n_tile, int nkb) {
 
 // An op with kSwapAB = true multiplies with the roles of the staged tiles
 // swapped: the B tiles (n_tile = 128 rows) are the MMA's A operand, so that
-// they land on TMEM lanes, and the 128-row A tile is its B operand (128
-// accumulator columns).  Loads, ring and barriers are the same.
+// they land on TMEM lanes, and the A tile is its B operand (one accumulator
+// column per A row).  Loads, ring and barriers are the same.
 template <class Op, class = void> struct SwapAB {
     static constexpr bool value = false;
 };
 template <class Op> struct SwapAB<Op, std::void_t<decltype(Op::kSwapAB)>> {
     static constexpr bool value = Op::kSwapAB;
 };
-// accumulator columns of one MMA: n_tile, or 128 when swapped
+// Rows of the staged A tile: 128, or Op::kARows (256: a swapped op's tile
+// then carries twice the keys for the same 128-token operand, so half the
+// tiles, half the operand bytes per key and 128 x 256 MMAs; measured on the
+// candidate-list passes at mid_4m with 2048 tokens: 137 -> 118 us for both
+// passes and their bound).  Loaded as 128-row TMA boxes.
+template <class Op, class = void> struct ARows {
+    static constexpr int value = kTileM;
+};
+template <class Op> struct ARows<Op, std::void_t<decltype(Op::kARows)>> {
+    static constexpr int value = Op::kARows;
+};
+
+// An op with kGroupEpilogue = true (the candidate-list passes: swapped)
+// reduces each group of 16 accumulator columns to one 32-bit value (group)
+// and stores a thread's consecutive groups at once (store_groups): each
+// epilogue warp half takes a contiguous half of the columns, so that a
+// token's values leave as 16-byte stores instead of scattered 4-byte ones.
+template <class Op, class = void> struct GroupEpi {
+    static constexpr bool value = false;
+};
+template <class Op> struct GroupEpi<Op, std::void_t<decltype(Op::kGroupEpilogue)>> {
+    static constexpr bool value = Op::kGroupEpilogue;
+};
+
+// The grouped epilogue of one TMEM lane (row) over its warp's columns
+// [cb, cb + 16 NG): NG groups of 16 (NG a multiple of 4).
+template <class Op, int NG>
+__device__ __forceinline__ void group_epilogue(const Op &op, const Tile &t, int row, int cb,
+                                               uint32_t lane_base) {
+    static_assert(NG % 4 == 0, "whole 16-byte stores of group values");
+    const uint32_t pre = op.prefetch(t, row, cb);
+    uint32_t g[NG];
+#pragma unroll
+    for (int cc = 0; cc < NG / 2; ++cc) {
+        uint32_t r[32];
+        tmem_ld32_nowait(lane_base + (uint32_t)(cb + cc * 32), r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            float v[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[half * 16 + i]);
+            g[cc * 2 + half] = op.group(t, row, cb + cc * 32 + half * 16, v, pre);
+        }
+    }
+    op.template store_groups<NG>(t, row, cb, g);
+}
+
+// accumulator columns of one MMA: n_tile, or the A rows when swapped
 template <class Op> __host__ __device__ inline int acc_cols_of(const Op &op) {
-    return SwapAB<Op>::value ? kTileM : op.n_tile;
+    return SwapAB<Op>::value ? ARows<Op>::value : op.n_tile;
 }
 
 template <int NSPLIT, class Op>
@@ -120,7 +169,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const size_t slice = split_slice_bytes(op.n_tile, S);
     const int n_tile = op.n_tile;
     const uint32_t b_bytes = (uint32_t)n_tile * 128;
-    const uint32_t stage_bytes = kTileABytes + NSPLIT * b_bytes;
+    constexpr int kA = ARows<Op>::value;
+    constexpr uint32_t a_bytes = (uint32_t)kA * 128;
+    const uint32_t stage_bytes = a_bytes + NSPLIT * b_bytes;
     constexpr bool kSwap = SwapAB<Op>::value;
     const int acc_n = acc_cols_of(op);   // accumulator columns
     // the epilogue reads 32 columns at a time: cover the last such read
@@ -159,8 +210,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint8_t *sa = ring + (size_t)s * stage_bytes;
         mbar_arrive_expect_tx(&full[s], stage_bytes);
         const int kx = (t.kb0 + it) * kBlockK;
-        if (t.a_z >= 0) tma_load_3d(sa, mapA, &full[s], kx, t.m0, t.a_z);
-        else tma_load_2d(sa, mapA, &full[s], kx, t.m0);
+#pragma unroll
+        for (int ab = 0; ab < kA / kTileM; ++ab) {
+            uint8_t *sab = sa + ab * kTileABytes;
+            if (t.a_z >= 0) tma_load_3d(sab, mapA, &full[s], kx, t.m0 + ab * kTileM, t.a_z);
+            else tma_load_2d(sab, mapA, &full[s], kx, t.m0 + ab * kTileM);
+        }
     };
     auto load_b = [&](int it) {
         const int s = it % kStages;
@@ -168,7 +223,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int kx = (t.kb0 + it) * kBlockK;
 #pragma unroll
         for (int j = 0; j < NSPLIT; ++j) {
-            uint8_t *sb = sa + kTileABytes + j * b_bytes;
+            uint8_t *sb = sa + a_bytes + j * b_bytes;
             const int bx = j * op.b_split_stride + kx;
             if (t.b_z >= 0) tma_load_3d(sb, &mapB, &full[s], bx, t.n0, t.b_z);
             else tma_load_2d(sb, &mapB, &full[s], bx, t.n0);
@@ -214,7 +269,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // MMA issuer.  Descriptors are built once per stage and advanced by
         // 32 bytes (2 in the >>4 address field) per 16-wide K step; the
         // accumulator of each step follows its rank chunk without division.
-        const uint32_t idesc = kSwap ? idesc_bf16_f32(n_tile, kTileM) : idesc_bf16_f32(kTileM, n_tile);
+        const uint32_t idesc = kSwap ? idesc_bf16_f32(n_tile, kA) : idesc_bf16_f32(kTileM, n_tile);
         uint32_t started = 0;
         int acc = (t.kb0 * kBlockK) / op.acc_chunk;
         int next_chunk = (acc + 1) * op.acc_chunk;   // K index where acc advances
@@ -229,7 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t ad0 = desc_k_sw128(sa);
             uint64_t bd0[NSPLIT];
 #pragma unroll
-            for (int j = 0; j < NSPLIT; ++j) bd0[j] = desc_k_sw128(sa + kTileABytes + j * b_bytes);
+            for (int j = 0; j < NSPLIT; ++j) bd0[j] = desc_k_sw128(sa + a_bytes + j * b_bytes);
 #pragma unroll
             for (int k16 = 0; k16 < kBlockK / 16; ++k16) {
                 const int kg = (t.kb0 + it) * kBlockK + k16 * 16;
@@ -263,7 +318,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quad = warp & 3, whalf = warp >> 2;
     const int row = quad * 32 + lane;
     const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
-    if (S == 1) {
+    if constexpr (GroupEpi<Op>::value) {
+        group_epilogue<Op, kA / 16 / kGroups>(op, t, row, whalf * (kA / kGroups), lane_base);
+        tc_fence_before();
+        __syncthreads();
+        if (warp == 0) tmem_dealloc(tmem, ncols);
+    } else if (S == 1) {
         // a per-chunk value the op fetches one chunk ahead (the candidate
         // lists' bounds), so that its latency overlaps the previous chunk
         uint32_t pre = op.prefetch(t, row, whalf * 32);
@@ -366,17 +426,28 @@ __global__ void __launch_bounds__(kThreads, 1)
 // One CTA per SM loops over tiles i = blockIdx.x, + gridDim.x, ... (x fastest,
 // then y, then z of the tile grid).  Warp 0 lane 0 streams A/B K-blocks of
 // successive tiles through the ring; warp 1 lane 0 issues each tile's MMAs
-// into one of two TMEM accumulator buffers; warps 2..9 drain the other
-// buffer (epilogue) meanwhile, so loads, MMAs and stores of consecutive
-// tiles overlap.  Barriers: full/empty per ring stage; tfull (MMAs of a
-// buffer done) and tempty (its epilogue done, 8 arrivals) per buffer.  Every
-// wait is bounded; a timeout raises the error word and an abort flag that
-// every role polls.
-constexpr int kPEpiWarps = 8;
-constexpr int kPThreads = 64 + 32 * kPEpiWarps;
+// into one of two TMEM accumulator buffers; the epilogue warps (2 onwards)
+// drain the other buffer meanwhile, so loads, MMAs and stores of
+// consecutive tiles overlap.  Barriers: full/empty per ring stage; tfull
+// (MMAs of a buffer done) and tempty (its epilogue done, one arrival per
+// epilogue warp) per buffer.  Every wait is bounded; a timeout raises the
+// error word and an abort flag that every role polls.
+//
+// Epilogue warps: 8 (two per TMEM lane quarter), or Op::kEpiWarps (16: four
+// per quarter, each a quarter of the columns).  An epilogue whose work per
+// column is a chain of dependent instructions (the candidate lists'
+// appends) runs at a fraction of the issue rate with two warps per SM
+// sub-partition; more warps hide that latency.
+template <class Op, class = void> struct EpiWarps {
+    static constexpr int value = 8;
+};
+template <class Op> struct EpiWarps<Op, std::void_t<decltype(Op::kEpiWarps)>> {
+    static constexpr int value = Op::kEpiWarps;
+};
+template <class Op> constexpr int persistent_threads() { return 64 + 32 * EpiWarps<Op>::value; }
 
 template <int NSPLIT, class Op>
-__global__ void __launch_bounds__(kPThreads, 1)
+__global__ void __launch_bounds__(persistent_threads<Op>(), 1)
     tc_gemm_persistent(const __grid_constant__ CUtensorMap mapA0,
                        const __grid_constant__ CUtensorMap mapA1,
                        const __grid_constant__ CUtensorMap mapB, Op op, int gx, int gy,
@@ -391,7 +462,9 @@ __global__ void __launch_bounds__(kPThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n_tile = op.n_tile;
     const uint32_t b_bytes = (uint32_t)n_tile * 128;
-    const uint32_t stage_bytes = kTileABytes + NSPLIT * b_bytes;
+    constexpr int kA = ARows<Op>::value;
+    constexpr uint32_t a_bytes = (uint32_t)kA * 128;
+    const uint32_t stage_bytes = a_bytes + NSPLIT * b_bytes;
     const int kStages = op.stages;
     auto tile_of = [&](int i) {
         const int bx = i % gx, r = i / gx;
@@ -405,7 +478,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&tfull[b], 1);
-            mbar_init(&tempty[b], kPEpiWarps);
+            mbar_init(&tempty[b], EpiWarps<Op>::value);
         }
         mbar_init(&drained, 1);
         abort_flag = 0;
@@ -447,11 +520,16 @@ __global__ void __launch_bounds__(kPThreads, 1)
                     uint8_t *sa = ring + (size_t)s * stage_bytes;
                     mbar_arrive_expect_tx(&full[s], stage_bytes);
                     const int kx = (t.kb0 + kb) * kBlockK;
-                    if (t.a_z >= 0) tma_load_3d(sa, mapA, &full[s], kx, t.m0, t.a_z);
-                    else tma_load_2d(sa, mapA, &full[s], kx, t.m0);
+#pragma unroll
+                    for (int ab = 0; ab < kA / kTileM; ++ab) {
+                        uint8_t *sab = sa + ab * kTileABytes;
+                        if (t.a_z >= 0)
+                            tma_load_3d(sab, mapA, &full[s], kx, t.m0 + ab * kTileM, t.a_z);
+                        else tma_load_2d(sab, mapA, &full[s], kx, t.m0 + ab * kTileM);
+                    }
 #pragma unroll
                     for (int j = 0; j < NSPLIT; ++j) {
-                        uint8_t *sb = sa + kTileABytes + j * b_bytes;
+                        uint8_t *sb = sa + a_bytes + j * b_bytes;
                         const int bx = j * op.b_split_stride + kx;
                         if (t.b_z >= 0) tma_load_3d(sb, &mapB, &full[s], bx, t.n0, t.b_z);
                         else tma_load_2d(sb, &mapB, &full[s], bx, t.n0);
@@ -467,7 +545,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
         if (lane == 0) {
             // MMA issuer
             constexpr bool kSwap = SwapAB<Op>::value;
-            const uint32_t idesc = kSwap ? idesc_bf16_f32(n_tile, kTileM) : idesc_bf16_f32(kTileM, n_tile);
+            const uint32_t idesc = kSwap ? idesc_bf16_f32(n_tile, kA) : idesc_bf16_f32(kTileM, n_tile);
             const int acc_n = acc_cols_of(op);
             int it = 0, lt = 0;
             for (int i = blockIdx.x; i < tiles && !abort_flag; i += gridDim.x, ++lt) {
@@ -496,7 +574,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
                     uint64_t bd0[NSPLIT];
 #pragma unroll
                     for (int j = 0; j < NSPLIT; ++j)
-                        bd0[j] = desc_k_sw128(sa + kTileABytes + j * b_bytes);
+                        bd0[j] = desc_k_sw128(sa + a_bytes + j * b_bytes);
 #pragma unroll
                     for (int k16 = 0; k16 < kBlockK / 16; ++k16) {
                         const int kg = (t.kb0 + kb) * kBlockK + k16 * 16;
@@ -528,8 +606,10 @@ __global__ void __launch_bounds__(kPThreads, 1)
         }
         __syncwarp();
     } else {
-        // epilogue warps: warp w reads TMEM lane quarter w % 4 and alternate
-        // 32-column chunks by warp group
+        // epilogue warps: warp w reads TMEM lane quarter w % 4; the kEG warps
+        // of a quarter take interleaved 32-column chunks (grouped ops: one
+        // contiguous share of the columns each)
+        constexpr int kEG = EpiWarps<Op>::value / 4;
         const int quad = warp & 3, grp = (warp - 2) >> 2;
         const int row = quad * 32 + lane;
         int lt = 0;
@@ -544,24 +624,30 @@ __global__ void __launch_bounds__(kPThreads, 1)
             const uint32_t lane_base =
                 tmem + (uint32_t)buf * buf_cols + ((uint32_t)(quad * 32) << 16);
             const int acc_n = acc_cols_of(op);
-            uint32_t pre = op.prefetch(t, row, grp * 32);   // one chunk ahead, as above
-            for (int c0 = grp * 32; c0 < acc_n; c0 += 64) {
-                const uint32_t cur = pre;
-                if (c0 + 64 < acc_n) pre = op.prefetch(t, row, c0 + 64);
-                uint32_t r[kMaxAcc][32];
-#pragma unroll
-                for (int a = 0; a < kMaxAcc; ++a)
-                    if (a < op.n_acc) tmem_ld32_nowait(lane_base + (uint32_t)(a * acc_n + c0), r[a]);
-                tmem_ld_wait();
-#pragma unroll
-                for (int half = 0; half < 2; ++half) {
-                    if (c0 + half * 16 >= acc_n) break;
-                    float v[kMaxAcc][16];
+            if constexpr (GroupEpi<Op>::value) {
+                group_epilogue<Op, kA / 16 / kEG>(op, t, row, grp * (kA / kEG), lane_base);
+            } else {
+                uint32_t pre = op.prefetch(t, row, grp * 32);   // one chunk ahead, as above
+                for (int c0 = grp * 32; c0 < acc_n; c0 += 32 * kEG) {
+                    const uint32_t cur = pre;
+                    if (c0 + 32 * kEG < acc_n) pre = op.prefetch(t, row, c0 + 32 * kEG);
+                    uint32_t r[kMaxAcc][32];
 #pragma unroll
                     for (int a = 0; a < kMaxAcc; ++a)
+                        if (a < op.n_acc)
+                            tmem_ld32_nowait(lane_base + (uint32_t)(a * acc_n + c0), r[a]);
+                    tmem_ld_wait();
 #pragma unroll
-                        for (int q = 0; q < 16; ++q) v[a][q] = __uint_as_float(r[a][half * 16 + q]);
-                    op.store(t, row, c0 + half * 16, v, cur);
+                    for (int half = 0; half < 2; ++half) {
+                        if (c0 + half * 16 >= acc_n) break;
+                        float v[kMaxAcc][16];
+#pragma unroll
+                        for (int a = 0; a < kMaxAcc; ++a)
+#pragma unroll
+                            for (int q = 0; q < 16; ++q)
+                                v[a][q] = __uint_as_float(r[a][half * 16 + q]);
+                        op.store(t, row, c0 + half * 16, v, cur);
+                    }
                 }
             }
             tc_fence_before();
@@ -579,6 +665,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
 // q = W_q x is written in fp32 (q_part, split 0) for the selection and as
 // the three bf16 terms of the scoring contraction (qs).
 struct QueryOp {
+    static constexpr int kEpiWarps = 16;
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
     unsigned long long *stamp;   // profiling stamps of the stage, or null
@@ -644,6 +731,7 @@ struct QueryOp {
 // stores its order-preserving 32-bit key.
 //
 struct ScoreOp {
+    static constexpr int kEpiWarps = 16;
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
     unsigned long long *stamp;   // profiling stamps of the stage, or null
@@ -685,28 +773,29 @@ struct ScoreOp {
 
 // Candidate lists (long grids): instead of every key, the contraction runs
 // twice, with the roles of the tiles swapped (kSwapAB): 128 tokens on the
-// TMEM lanes and 128 keys on the columns, so that each epilogue thread owns
-// one token's scores of 16 consecutive keys per store and needs no other
-// lane.  The first pass (kListGroupMax) stores, per (token, head, axis), the
-// largest key of each group of 16 keys.  A small kernel takes tau = the
-// k-th largest of those group maxima: k distinct groups hold a key >= tau,
-// so every key of the axis' top k is >= tau.  The second pass
-// (kListCandidates) recomputes the same keys (the same tiles, MMAs and
-// order, so bit for bit) and writes each key >= tau, as a (key, position)
-// composite, into its group's 16-entry segment of the (token, head, axis)
-// list, and the group's count over its maximum.  About 2 % of the keys land
-// in the lists.  Measured on GB300 (stage times, graph replays): the
-// selection gets 17-25 % shorter (prefill of 16384 tokens 2233 -> 1844 us),
-// but each pass streams the same operands as the one-pass scoring, which is
-// bound by L2 -> SM operand traffic rather than by the keys' DRAM writes, so
-// the two passes and the bound cost more than that (prefill 576 -> 1058 us);
-// the one-pass form is the default and this one is a mode.
+// TMEM lanes and 256 keys on the columns, so that each epilogue thread owns
+// one token's scores of consecutive keys and needs no other lane.  The
+// first pass (kListGroupMax) stores, per (token, head, axis), the largest
+// key of each group of 16 keys.  A small kernel takes tau <= the k-th
+// largest of those group maxima: k distinct groups hold a key >= tau, so
+// every key of the axis' top k is >= tau.  The second pass (kListCandidates)
+// recomputes the same keys (the same tiles, MMAs and order, so bit for bit)
+// and writes each key >= tau, as a (key, position) composite, into its
+// group's 16-entry segment of the (token, head, axis) list, and the group's
+// count over its maximum.  About 2 % of the keys land in the lists, and the
+// selection gets 17-25 % shorter.  Measured on GB300 (step times, graph
+// replays): with 16 epilogue warps and 256-key tiles the two passes and
+// the bound cost less than that saves once each SM has about 3.5 of their
+// tiles (prefill of 16384 tokens 3255 -> 3083 us a step), more below (mid_4m
+// with 128 tokens 65.7 -> 80.4 us), so the layer picks the form by grid.
 enum { kListGroupMax = 1, kListCandidates = 2 };
 constexpr int kListGroup = 16;   // keys of a group; entries of a list segment
 
 template <int Mode>
 struct ScoreListOp {
     static constexpr bool kSwapAB = true;
+    static constexpr int kARows = 256;   // keys a tile: 128 x 256 MMAs
+    static constexpr int kEpiWarps = 16;
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;   // n_tile = 128 tokens
     int *err;
     unsigned long long *stamp;   // profiling stamps of the stage, or null
@@ -722,7 +811,7 @@ struct ScoreListOp {
         Tile tl;
         const int h = bz >> 1, axis = bz & 1;
         tl.z = bz;   // head and axis
-        tl.m0 = bx * kTileM;   // first key
+        tl.m0 = bx * kARows;   // first key
         tl.n0 = by * n_tile;   // first token
         tl.a_sel = axis;
         tl.a_z = h;
@@ -737,32 +826,55 @@ struct ScoreListOp {
         const int n = tl.n0 + row;
         return n < B ? tau[(int64_t)n * H * 2 + tl.z] : 0xffffffffu;
     }
-    // row: the token (TMEM lane); c: the first of the 16 keys (a group)
-    __device__ void store(const Tile &tl, int row, int c, float (&v)[kMaxAcc][16],
-                          uint32_t t) const {
+    static constexpr bool kGroupEpilogue = true;
+    // row: the token (TMEM lane); c: the tile column of the group's first
+    // key.  Returns the group's largest key (group maxima), or its count
+    // after writing its keys >= t to its segment (candidates).
+    __device__ uint32_t group(const Tile &tl, int row, int c, const float (&v)[16],
+                              uint32_t t) const {
         const int n = tl.n0 + row;
         const int i0 = tl.m0 + c;
-        if (n >= B || i0 >= K) return;
-        const int64_t at = ((int64_t)n * H * 2 + tl.z) * G + i0 / kListGroup;
+        if (n >= B || i0 >= K) return 0u;
         const int valid = min(kListGroup, K - i0);
         // f2ord is monotone (-0 and +0 share a key), so the maximum and the
         // comparisons are taken on the fp32 scores and only kept keys are
         // converted
         if constexpr (Mode == kListGroupMax) {
-            float mx = v[0][0];   // valid >= 1
+            float mx = v[0];   // valid >= 1
 #pragma unroll
             for (int j = 1; j < kListGroup; ++j)
-                if (j < valid) mx = fmaxf(mx, v[0][j]);
-            gstat[at] = f2ord(mx);
+                if (j < valid) mx = fmaxf(mx, v[j]);
+            return f2ord(mx);
         } else {
             const float tf = ord2f(t);   // v >= tf  <=>  f2ord(v) >= t
-            unsigned long long *seg = cand + at * kListGroup;
+            unsigned long long *seg =
+                cand + (((int64_t)n * H * 2 + tl.z) * G + i0 / kListGroup) * kListGroup;
             uint32_t cnt = 0u;
 #pragma unroll
             for (int j = 0; j < kListGroup; ++j)
-                if (j < valid && v[0][j] >= tf)
-                    seg[cnt++] = comp_of(f2ord(v[0][j]), (uint32_t)(i0 + j));
-            gstat[at] = cnt;
+                if (j < valid && v[j] >= tf) seg[cnt++] = comp_of(f2ord(v[j]), (uint32_t)(i0 + j));
+            return cnt;
+        }
+    }
+    // the NG groups from tile column c (a multiple of 16 NG): 16-byte stores
+    // when every row of gstat starts on 16 bytes (G a multiple of 4), else
+    // one store per group
+    template <int NG>
+    __device__ void store_groups(const Tile &tl, int row, int c, const uint32_t (&g)[NG]) const {
+        const int n = tl.n0 + row;
+        const int gi = (tl.m0 + c) / kListGroup;
+        if (n >= B || gi >= G) return;
+        uint32_t *dst = gstat + ((int64_t)n * H * 2 + tl.z) * G + gi;
+        if ((G & 3) == 0) {
+#pragma unroll
+            for (int q = 0; q < NG / 4; ++q)
+                if (gi + 4 * q < G)
+                    *reinterpret_cast<uint4 *>(dst + 4 * q) =
+                        make_uint4(g[4 * q], g[4 * q + 1], g[4 * q + 2], g[4 * q + 3]);
+        } else {
+#pragma unroll
+            for (int q = 0; q < NG; ++q)
+                if (gi + q < G) dst[q] = g[q];
         }
     }
 };
@@ -770,6 +882,7 @@ struct ScoreListOp {
 
 // ---- S9: IVE projection, split over E*D_v --------------------------------
 struct ProjOp {
+    static constexpr int kEpiWarps = 16;
     int n_tile, stages, n_acc, acc_chunk, b_split_stride;
     int *err;
     unsigned long long *stamp;   // profiling stamps of the stage, or null
@@ -990,11 +1103,13 @@ static cudaError_t launch_gemm_persistent(dim3 grid, const CUtensorMap &a0, cons
                                           const CUtensorMap &b, Op op, int nkb, bool pdl,
                                           cudaStream_t st, int probe) {
     (void)nkb;   // the ring runs across tiles: as many stages as fit
-    op.stages = stages_for(NSPLIT, op.n_tile, kMaxStages);
-    const size_t smem = 1024 + (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile);
+    constexpr int kA = ARows<Op>::value;
+    op.stages = stages_for(NSPLIT, op.n_tile, kMaxStages, kA);
+    const size_t smem = 1024 + (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile, kA);
     const int tiles = (int)(grid.x * grid.y * grid.z);
     const int ctas = tiles < sm_count() ? tiles : sm_count();
-    return launch_kernel(pdl, tc_gemm_persistent<NSPLIT, Op>, dim3(ctas), kPThreads, smem, st, a0,
+    return launch_kernel(pdl, tc_gemm_persistent<NSPLIT, Op>, dim3(ctas),
+                         persistent_threads<Op>(), smem, st, a0,
                          a1, b, op, (int)grid.x, (int)grid.y, tiles,
                          buf_cols_of(op.n_acc, acc_cols_of(op)), probe);
 }
@@ -1009,8 +1124,9 @@ static cudaError_t launch_gemm(dim3 grid, const CUtensorMap &a0, const CUtensorM
         return launch_gemm_persistent<NSPLIT>(grid, a0, a1, b, op, nkb, pdl, st, probe);
     // the split-K epilogue adds up one accumulator
     if (op.cluster_splits_host() > 1 && op.n_acc != 1) return cudaErrorInvalidValue;
-    op.stages = stages_for(NSPLIT, op.n_tile, nkb);
-    const size_t ring = (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile);
+    constexpr int kA = ARows<Op>::value;
+    op.stages = stages_for(NSPLIT, op.n_tile, nkb, kA);
+    const size_t ring = (size_t)op.stages * stage_bytes_of(NSPLIT, op.n_tile, kA);
     const size_t split = split_buf_bytes(op.n_tile, op.cluster_splits_host());
     const size_t smem = 1024 + (ring > split ? ring : split);
     if (smem > kSmemBudget) return cudaErrorInvalidValue;   // the split buffers do not fit
@@ -1156,7 +1272,8 @@ static cudaError_t score_list_pass(const Dims &d, const Ptrs &p, const TcMaps &m
     op.gstat = p.gstat;
     op.tau = p.tau;
     op.cand = p.cand;
-    dim3 grid((d.K + kTileM - 1) / kTileM, (d.B + op.n_tile - 1) / op.n_tile, 2 * d.H);
+    constexpr int kA = ScoreListOp<Mode>::kARows;
+    dim3 grid((d.K + kA - 1) / kA, (d.B + op.n_tile - 1) / op.n_tile, 2 * d.H);
     return launch_gemm<3>(grid, mp.k_row, mp.k_col, mp.qs_t, op, op.kb_total, d.pdl, st, probe);
 }
 

@@ -45,6 +45,19 @@ def test_algorithmic_bytes_with_cores_and_column_query():
     assert b3["select"] - b1["select"] == 64 * 2 * 128 * 4
 
 
+def test_algorithmic_bytes_with_candidate_lists():
+    """With the candidate lists the selection reads each axis' group counts
+    (ceil(K/16) x 4 B) and at least k list entries (8 B) instead of the
+    axis' K rank-1 keys (4 B each); the other stages are the same."""
+    cfg = workloads.layer_config("prefill_16k")
+    B, H, k = 16384, cfg["heads"], cfg["topk"]
+    K = 2 * cfg["n"]   # E = 4
+    b0 = bench.algorithmic_bytes(cfg, B)
+    b1 = bench.algorithmic_bytes(cfg, B, lists=True)
+    assert b0["select"] - b1["select"] == B * H * 2 * (K * 4 - (K // 16 * 4 + k * 8))
+    assert {s: b0[s] for s in b0 if s != "select"} == {s: b1[s] for s in b1 if s != "select"}
+
+
 def test_aggregate_step_without_ranks():
     ms, value = bench.aggregate_step(0.035, 64)
     assert ms == 0.035

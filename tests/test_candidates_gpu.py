@@ -1,7 +1,8 @@
 """The scoring's two forms on the tensor-core path (Eq. 6-9): every rank-1
-key written and ranked by the selection (the default), or two scoring passes
-that leave per-axis candidate lists (the keys at or above tau, the k-th
-largest maximum of the axis' groups of 16 keys).  Both rank the same fp32
+key written and ranked by the selection, or two scoring passes that leave
+per-axis candidate lists (the keys at or above tau, a bound at most the k-th
+largest maximum of the axis' groups of 16 keys); by default the lists serve
+long grids and every key the others.  Both rank the same fp32
 keys by (score, smaller index), so the selected slots, their weights and
 the output must be identical bit for bit; the lists are also checked against
 the oracle directly.  Tied keys fill a list past the selection's 1024-entry
@@ -17,7 +18,7 @@ from tests import parity
 
 pytestmark = pytest.mark.gpu
 
-EVERY_KEY, LISTS = 0, 1
+EVERY_KEY, LISTS, AUTO = 0, 1, 2
 
 
 def _layer(cfg, w, B):
@@ -56,6 +57,10 @@ CASES = [
     (dict(dtype=1, n=600, topk=16, topm=32), 17, 1200),    # all tied: 1200 > 1024 listed
     (dict(dtype=1, n=600, topk=16, topm=32), 17, 500),     # 500 tied: tightened first
     (dict(dtype=1, n=2400, topk=64, topm=64), 5, 0),       # K = 4800
+    # more tiles than SMs: the passes keep each token block's query terms
+    # resident and change block inside a CTA's share of the tiles
+    (dict(dtype=1, n=2400, topk=64, topm=64), 300, 0),
+    (dict(dtype=1, n=1000, topk=32, topm=32, heads=3), 260, 0),
 ]
 
 
@@ -88,29 +93,51 @@ def test_lists_at_the_decode_workload(gpu_lib):
     layer.close()
 
 
-def test_every_key_by_default(gpu_lib):
-    """The default scoring writes every key (one scoring launch) at any grid,
-    long ones included; the lists run only on request."""
+def test_lists_at_a_long_grid(gpu_lib):
+    """mid_4m with 2048 tokens (4096 keys an axis, 4 heads: 2048 tiles a
+    pass) with the lists forced: the same selection as every key."""
+    cfg = workloads.layer_config("mid_4m")
+    layer, x, _ = _layer(cfg, workloads.make_weights(cfg, device="cuda"), 2048)
+    o1, i1, w1, _ = _forward(layer, x, EVERY_KEY)
+    o2, i2, w2, _ = _forward(layer, x, LISTS)
+    assert torch.equal(i1, i2) and torch.equal(w1, w2) and torch.equal(o1, o2)
+    layer.close()
+
+
+def test_default_form_by_grid(gpu_lib):
+    """The default writes every key (one scoring launch) while the list
+    passes would have fewer than 3.5 tiles of 128 tokens x 256 keys per SM,
+    and takes the lists (three launches) from there on; either form can be
+    forced, with the same result."""
     cfg = workloads.small_config(dtype=1, n=600, topk=16, topm=32)
     w = workloads.make_weights(cfg, device="cuda")
-    layer = binding.UltraMemLayer(cfg, w, 300)
-    for B in (300, 100):
+    layer = binding.UltraMemLayer(cfg, w, 4096)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    for B in (100, 300, 4096):
+        tiles = 5 * ((B + 127) // 128) * 2 * cfg["heads"]   # K = 1200: 5 tiles of 256 keys
         x = workloads.make_tokens(cfg, B, 0, device="cuda")
-        layer.forward(x)
+        out = layer.forward(x)
         assert layer.check() == 0
-        assert layer.last_launches() == 5
-    layer.candidates(LISTS)
-    layer.forward(x)
-    assert layer.check() == 0
-    assert layer.last_launches() == 7
+        assert layer.last_launches() == (7 if 2 * tiles >= 7 * sms else 5)
+    assert layer.last_launches() == 7   # 640 tiles
+    o_auto, i_auto, w_auto, _ = _forward(layer, x, AUTO)
+    o1, i1, w1, n1 = _forward(layer, x, EVERY_KEY)
+    assert n1 == 5
+    assert torch.equal(i1, i_auto) and torch.equal(w1, w_auto) and torch.equal(o1, o_auto)
+    o2, i2, w2, n2 = _forward(layer, x, LISTS)
+    assert n2 == 7
+    layer.candidates(AUTO)
+    layer.forward(x[:100])
+    assert layer.last_launches() == 5
     layer.close()
 
 
 def test_candidate_hook_arguments(gpu_lib):
     cfg = workloads.small_config(dtype=1, n=600, topk=16, topm=32)
     layer = binding.UltraMemLayer(cfg, workloads.make_weights(cfg, device="cuda"), 8)
-    with pytest.raises(binding.UltraMemError):
-        layer.candidates(2)
+    for bad in (-1, 3):
+        with pytest.raises(binding.UltraMemError):
+            layer.candidates(bad)
     layer.close()
     # fp32 storage runs on CUDA cores: no lists
     cfg32 = workloads.small_config(dtype=0, n=600, topk=16, topm=32)
@@ -118,4 +145,5 @@ def test_candidate_hook_arguments(gpu_lib):
     with pytest.raises(binding.UltraMemError):
         layer32.candidates(LISTS)
     layer32.candidates(EVERY_KEY)
+    layer32.candidates(AUTO)    # the default: every key where lists cannot run
     layer32.close()
