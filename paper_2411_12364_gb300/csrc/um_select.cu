@@ -297,38 +297,69 @@ __device__ __noinline__ void cand_fallback(const u64 *seg, const uint32_t *cnt, 
     __syncthreads();
 }
 
-__device__ void load_list(const Ptrs &p, int64_t list, int G, int kk, int s, int slot,
-                          SelShared &sh) {
-    const uint32_t *cnt = p.gstat + list * G;
-    const u64 *seg = p.cand + list * (int64_t)G * kSeg;
-    int mine[kMaxSegPerThread], tot = 0;
+// Both axes' lists of one (token, head) (lists `list0` and `list0 + 1`)
+// into cand[0] and cand[1], lengths in cnt[kCntAxis + s].  One block scan
+// places both (the two axes' counts packed in the low and high 16 bits:
+// each total is at most 16 G <= 16384), and each thread loads the first
+// entry of all its segments before it stores any, so that the copies cost
+// one round trip to memory, not one per segment.  Whole block; ends with a
+// barrier.
+__device__ void load_lists(const Ptrs &p, int64_t list0, int G, int kk, SelShared &sh) {
+    const uint32_t *cnt[2] = {p.gstat + list0 * G, p.gstat + (list0 + 1) * G};
+    const u64 *seg[2] = {p.cand + list0 * (int64_t)G * kSeg, p.cand + (list0 + 1) * (int64_t)G * kSeg};
+    int mine[2][kMaxSegPerThread], tot = 0;
 #pragma unroll
-    for (int q = 0; q < kMaxSegPerThread; ++q) {
-        const int g = threadIdx.x + q * kThreads;
-        mine[q] = g < G ? (int)min(cnt[g], (uint32_t)kSeg) : 0;
-        tot += mine[q];
-    }
-    int o = block_exclusive_scan(tot, sh);
-    if (threadIdx.x == kThreads - 1) sh.cnt[slot] = o + tot;
-    __syncthreads();
-    const int c = sh.cnt[slot];
-    if (c > kCap) {
-        cand_fallback(seg, cnt, G, kk, s, slot, sh);
-        return;
-    }
+    for (int s = 0; s < 2; ++s) {
 #pragma unroll
-    for (int q = 0; q < kMaxSegPerThread; ++q) {
-        const u64 *sg = seg + (int64_t)(threadIdx.x + q * kThreads) * kSeg;
-        for (int e = 0; e < mine[q]; ++e) sh.cand[s][o++] = sg[e];
+        for (int q = 0; q < kMaxSegPerThread; ++q) {
+            const int g = threadIdx.x + q * kThreads;
+            mine[s][q] = g < G ? (int)min(cnt[s][g], (uint32_t)kSeg) : 0;
+            tot += mine[s][q] << (16 * s);
+        }
     }
-    // fewer than kk is impossible (the bound guarantees kk); should it
-    // happen, positions past K mark the missing entries (recorded)
-    for (int f = c + threadIdx.x; f < kk; f += kThreads)
-        sh.cand[s][f] = comp_of(0u, 0xffffffffu - (uint32_t)f);
+    const int o = block_exclusive_scan(tot, sh);
+    if (threadIdx.x == kThreads - 1) {
+        sh.cnt[kCntAxis] = (o + tot) & 0xffff;
+        sh.cnt[kCntAxis + 1] = (o + tot) >> 16;
+    }
     __syncthreads();
-    if (threadIdx.x == 0 && c < kk) {
-        sh.cnt[slot] = kk;
-        atomicOr(p.err, kErrInternal);
+    const int c[2] = {sh.cnt[kCntAxis], sh.cnt[kCntAxis + 1]};
+    // the first entry of every segment of this thread, then the rest
+    u64 first[2][kMaxSegPerThread];
+#pragma unroll
+    for (int s = 0; s < 2; ++s)
+#pragma unroll
+        for (int q = 0; q < kMaxSegPerThread; ++q)
+            first[s][q] = mine[s][q] > 0 && c[s] <= kCap
+                              ? seg[s][(int64_t)(threadIdx.x + q * kThreads) * kSeg]
+                              : 0ull;
+#pragma unroll
+    for (int s = 0; s < 2; ++s) {
+        if (c[s] > kCap) continue;   // uniform: the radix select below replaces it
+        int at = (o >> (16 * s)) & 0xffff;
+#pragma unroll
+        for (int q = 0; q < kMaxSegPerThread; ++q) {
+            if (mine[s][q] == 0) continue;
+            const u64 *sg = seg[s] + (int64_t)(threadIdx.x + q * kThreads) * kSeg;
+            sh.cand[s][at++] = first[s][q];
+            for (int e = 1; e < mine[s][q]; ++e) sh.cand[s][at++] = sg[e];
+        }
+        // fewer than kk is impossible (the bound guarantees kk); should it
+        // happen, positions past K mark the missing entries (recorded)
+        for (int f = c[s] + threadIdx.x; f < kk; f += kThreads)
+            sh.cand[s][f] = comp_of(0u, 0xffffffffu - (uint32_t)f);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int s = 0; s < 2; ++s) {
+        if (c[s] > kCap) {
+            cand_fallback(seg[s], cnt[s], G, kk, s, kCntAxis + s, sh);
+        } else if (c[s] < kk) {
+            if (threadIdx.x == 0) {
+                sh.cnt[kCntAxis + s] = kk;
+                atomicOr(p.err, kErrInternal);
+            }
+        }
     }
     __syncthreads();
 }
@@ -950,8 +981,7 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
         __syncthreads();
     } else if (lists) {   // the scoring left each axis' candidates
         __syncthreads();
-        for (int s = 0; s < 2; ++s)
-            load_list(p, ((int64_t)b * d.H + h) * 2 + s, d.n_groups, k, s, kCntAxis + s, sh);
+        load_lists(p, ((int64_t)b * d.H + h) * 2, d.n_groups, k, sh);
     } else {
         warp_bounds(top[0][0], top[0][1], top[1][0], top[1][1], 2, k, sh);
         __syncthreads();
