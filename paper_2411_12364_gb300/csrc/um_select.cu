@@ -69,6 +69,7 @@ struct SelShared {
     int digit, remaining;
     float scalar;
     double dscalar;   // fp32 storage: the softmax denominator in fp64
+    unsigned long long xbar;   // paired selection: the row CTA's exchange mbarrier
 };
 
 template <typename T>
@@ -692,19 +693,55 @@ __device__ __forceinline__ uint4 ld_key_row(const uint4 *ptr) {
     return v;
 }
 
-// The paired decode selection's exchange: a 32-bit store into the same
-// shared-memory location of CTA `rank` of the cluster, and a barrier of all
-// threads of the cluster (release / acquire).
-__device__ __forceinline__ void st_cluster_u32(const void *local, uint32_t rank, uint32_t v) {
-    const uint32_t a = (uint32_t)__cvta_generic_to_shared(local);
-    uint32_t ra;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(a), "r"(rank));
-    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(ra), "r"(v) : "memory");
+// The paired decode selection's cluster barrier (arrive, then wait).
+__device__ __forceinline__ void cl_arrive_relaxed() {
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
-__device__ __forceinline__ void cluster_sync_all() {
-    asm volatile(
-        "barrier.cluster.arrive.release.aligned;\n\t"
-        "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+__device__ __forceinline__ void cl_wait() {
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// The exchange mbarrier of the paired selection (in the row CTA): one
+// arrival, which also expects the column CTA's survivors' bytes; the init is
+// published to the pair by a release fence and the pair's first cluster
+// barrier.
+__device__ __forceinline__ void xbar_init(unsigned long long *bar, uint32_t bytes) {
+    const uint32_t a = (uint32_t)__cvta_generic_to_shared(bar);
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes)
+                 : "memory");
+}
+// A 32-bit store into the same shared-memory location of CTA `rank`, which
+// completes 4 bytes of that CTA's mbarrier at the same offset as `bar`.
+__device__ __forceinline__ void st_async_u32(const void *local, uint32_t rank, uint32_t v,
+                                             const unsigned long long *bar) {
+    const uint32_t a = (uint32_t)__cvta_generic_to_shared(local);
+    const uint32_t b = (uint32_t)__cvta_generic_to_shared(bar);
+    uint32_t ra, rb;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(a), "r"(rank));
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(rb) : "r"(b), "r"(rank));
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(ra),
+                 "r"(v), "r"(rb)
+                 : "memory");
+}
+// Bounded wait (about a second of SM cycles) for phase 0 of the exchange
+// mbarrier, with cluster-scope acquire: the column CTA's stores are then
+// visible.  Returns false when it gave up.
+__device__ __forceinline__ bool xbar_wait(unsigned long long *bar) {
+    const uint32_t a = (uint32_t)__cvta_generic_to_shared(bar);
+    const long long start = clock64();
+    for (;;) {
+        uint32_t ok;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], 0;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(ok)
+            : "r"(a)
+            : "memory");
+        if (ok) return true;
+        if (clock64() - start > (1ll << 31)) return false;
+    }
 }
 
 // The 2k axis survivors, one group of G lanes each: the survivor's place in
@@ -906,9 +943,10 @@ __device__ void axis_survivors(const Dims &d, const Ptrs &p, int h, const SelLay
 // PAIR (decode grids of at most one (token, head) per SM): a cluster of two
 // CTAs per (token, head), blockIdx.z = its axis.  Each takes one axis through
 // the key load, bound, compaction, rank and survivors (half the work a warp
-// does in those phases); the column CTA then stores its survivors (indices
-// and S_col) into the row CTA's shared memory, the pair meets at a cluster
-// barrier, and the row CTA goes on alone (Tucker scores, top-m, outputs).
+// does in those phases); the column CTA then sends its survivors (indices
+// and S_col) into the row CTA's shared memory with asynchronous stores that
+// complete bytes of the row CTA's exchange mbarrier, and the row CTA, once
+// that barrier completes, goes on alone (Tucker scores, top-m, outputs).
 template <typename T, int MINB, int RM, bool PAIR = false>
 __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -921,6 +959,13 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     const uint32_t *A1 = A0 + K;   // (not read when PAIR)
 
     if (threadIdx.x < 8) sh.cnt[threadIdx.x] = 0;
+    if constexpr (PAIR) {
+        // the row CTA's exchange barrier, expecting the column CTA's
+        // survivors (k indices and k r scores); the pair's cluster barrier
+        // arrival publishes it, its wait comes just before the exchange
+        if (ax == 0 && threadIdx.x == 0) xbar_init(&sh.xbar, (uint32_t)(d.k + d.k * d.r) * 4u);
+        cl_arrive_relaxed();
+    }
     // C of this head (a weight: read before the dependency wait) and the
     // row/column query of this (token, head), summed over its D_i splits:
     // loaded before the keys, stored after them
@@ -1015,20 +1060,19 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
     axis_survivors<T, RM>(d, p, h, L, sh, PAIR ? ax : -1);
     __syncthreads();
     if constexpr (PAIR) {
-        // the column CTA stores its survivors into the row CTA; the barrier
-        // (release / acquire) makes them visible there, and the column CTA
-        // is done
+        // the column CTA sends its survivors into the row CTA with
+        // asynchronous stores that complete bytes of the row CTA's exchange
+        // mbarrier, and is done; the row CTA waits on that barrier
+        cl_wait();   // the exchange barrier is initialised
         if (ax == 1) {
             for (int i = threadIdx.x; i < k; i += kThreads)
-                st_cluster_u32(L.sel_j + i, 0u, (uint32_t)L.sel_j[i]);
+                st_async_u32(L.sel_j + i, 0u, (uint32_t)L.sel_j[i], &sh.xbar);
             for (int i = threadIdx.x; i < k * r; i += kThreads)
-                st_cluster_u32(L.scol + i, 0u, __float_as_uint(L.scol[i]));
-        }
-        cluster_sync_all();
-        if (ax == 1) {
+                st_async_u32(L.scol + i, 0u, __float_as_uint(L.scol[i]), &sh.xbar);
             stamp_end(p.stamp);
             return;
         }
+        if (!xbar_wait(&sh.xbar) && threadIdx.x == 0) atomicOr(p.err, kErrTimeout);
     }
 
     u64 *const fwin = sh.cand[1];   // final winners by rank (list 1 is free now)
