@@ -1220,11 +1220,6 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
         const uint32_t vs = (uint32_t)shuffle_address(d, p.perm, v);   // Eq. 14, < M < 2^32
         const uint32_t pb = vs / N;
         const uint32_t prow = vs - pb * N;
-        // the gather will read this value row: start moving it into L2,
-        // unless the batch's rows would not stay there until then
-        if (prefetch)
-            prefetch_l2(static_cast<const unsigned char *>(p.values) + (size_t)prow * row_bytes,
-                        row_bytes);
         p.sel_row[base + e] = (int32_t)prow;
         p.sel_p[base + e] = (int32_t)pb;
         if (p.idx_out) p.idx_out[base + e] = (int64_t)v;
@@ -1262,6 +1257,27 @@ __global__ void __launch_bounds__(kThreads, MINB) select_kernel(Dims d, Ptrs p) 
                 p.sel_w[(base + e) * d.nc + ci] = gi;
                 if (p.w_out) p.w_out[(base + e) * d.nc + ci] = gi;
             }
+        }
+    }
+    // The gather will read the winners' value rows: start moving them into
+    // L2 (unless the batch's rows would not stay there until then).  Winner
+    // e's row is fetched by a thread of the warps after those that stored
+    // the slots (for m <= 128), which works out the slot again: a prefetch
+    // holds its warp for about 1300 cycles (the row's address translation,
+    // measured at decode), and this way the stores above do not wait behind
+    // it.
+    if (prefetch) {
+        const int sw = (m + 31) / 32;   // warps that stored slots
+        const int shift = 2 * sw * 32 <= kThreads ? 32 * sw : 32;
+        for (int e = (threadIdx.x + kThreads - shift) % kThreads; e < m; e += kThreads) {
+            int c = (int)pos_of(fwin[e]);
+            if ((uint32_t)c >= (uint32_t)k2) c = 0;   // recorded above
+            const int ii = c / k, jj = c - ii * k;
+            const uint64_t v = (uint64_t)L.sel_i[ii] * (uint64_t)K + (uint64_t)L.sel_j[jj];
+            const uint32_t vs = (uint32_t)shuffle_address(d, p.perm, v);
+            const uint32_t prow = vs - (vs / N) * N;
+            prefetch_l2(static_cast<const unsigned char *>(p.values) + (size_t)prow * row_bytes,
+                        row_bytes);
         }
     }
     stamp_end(p.stamp);
