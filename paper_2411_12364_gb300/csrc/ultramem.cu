@@ -103,8 +103,9 @@ int query_splits(const ultramem_config &c, int B) {
 // cores (16 weight rows x 8 tokens per CTA, no split-K); larger ones, and
 // the IVE projection at every batch, on tcgen05.  Measured on GB300: at 64
 // tokens the CUDA-core query takes 3.3 us against 8.5 us for the split-K
-// tensor-core one; at 128 tokens (and for the projection, whose weight rows
-// it re-reads once per 8 tokens) it is slower.
+// tensor-core one; above that (and for the projection, whose weight rows
+// it re-reads once per 8 tokens) it is slower: 12.4 against 9.6 us at 96
+// tokens of the 4M-slot layer (D_i 2048), 15.4 against 9.7 us at 128.
 constexpr int kSmallQueryBatch = 64;
 
 // Tensor path split-K plan: the N tile (tokens per tile) and the split count
